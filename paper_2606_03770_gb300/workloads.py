@@ -1,0 +1,232 @@
+"""Seeded synthetic fleets, links and layer profiles.
+
+This module is the one piece both the CUDA path and the CPU oracle consume.  It
+draws inputs only: device capabilities, link bandwidths, congestion factors and
+the per-block work of a dense decoder.  None of the planner's arithmetic (stage
+cost, link cost, the partition DP, the objective, the genetic operators) lives
+here.
+
+The paper profiles per-block latency on real devices with a reduced-block
+llama.cpp (Sec. 3.1).  Those profiles are not available, so each device is
+described by a compute rate, a memory bandwidth and a memory capacity, and each
+block of the model by the FLOPs it executes, the bytes it streams and the bytes
+it keeps resident, per inference variant (prefill, or decode with batch b).
+Blocks are identical in size and cost, the premise the paper states for fixing
+the node order in its DP (Sec. 3.2).
+
+Units: FLOPs, bytes, FLOP/s, bytes/s, tokens.  All integers are Python ints /
+numpy uint64 below 2**53 so that both sides convert them to float64 exactly.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+
+import numpy as np
+
+HEAD_DIM = 128
+
+
+@dataclasses.dataclass
+class Problem:
+    """One planning instance: fleet, links, layer profile and GA parameters."""
+
+    name: str
+    # fleet (M devices)
+    rate: np.ndarray  # float64[M] compute rate, FLOP/s
+    bw: np.ndarray  # float64[M] memory bandwidth, bytes/s
+    mem: np.ndarray  # uint64[M] memory available for the model, bytes
+    # links (row = sender, column = receiver)
+    link_bw: np.ndarray  # float64[M, M] base link bandwidth, bytes/s
+    cong: np.ndarray  # float64[M, M] congestion factor in (0, 1]
+    # layer profile: N identical blocks, variant 0 = prefill, v = b >= 1 = decode batch b
+    N: int
+    blk_flops: np.ndarray  # uint64[V]
+    blk_bytes: np.ndarray  # uint64[V]
+    blk_mem: np.ndarray  # uint64[V]
+    head_flops: np.ndarray  # uint64[V]  LM head + output layer, master only
+    head_bytes: np.ndarray  # uint64[V]
+    head_mem: np.ndarray  # uint64[V]
+    act_bytes: np.ndarray  # uint64[V]  activation bytes of one microbatch crossing a link
+    NP: int  # average input tokens per request
+    ND: int  # average generated tokens per request
+    # objective
+    min_tps: float = 7.0
+    t_a: float = 1.0
+    # genetic algorithm
+    P: int = 64
+    Q: int = 2
+    K_max: int = 2
+    G: int = 1
+    tournament: int = 4
+    p_cx: float = 0.5
+    p_mut: float = 0.3
+    p_kind: tuple = (0.2, 0.5, 0.15, 0.15)
+    redraw: bool = False
+    cong_lo: float = 0.2
+    cong_hi: float = 1.0
+    seed: int = 0
+
+    @property
+    def M(self) -> int:
+        return int(self.rate.shape[0])
+
+    @property
+    def b_max(self) -> int:
+        return int(self.blk_flops.shape[0]) - 1
+
+    @property
+    def V(self) -> int:
+        return int(self.blk_flops.shape[0])
+
+
+def _log_uniform(rng, lo, hi, n):
+    return np.exp(rng.uniform(math.log(lo), math.log(hi), n))
+
+
+def _sym(rng, M, draw):
+    """Symmetric matrix of per-pair draws; the diagonal is never used by the planner."""
+    out = np.ones((M, M), dtype=np.float64)
+    iu = np.triu_indices(M, 1)
+    vals = draw(len(iu[0]))
+    out[iu] = vals
+    out[(iu[1], iu[0])] = vals
+    return out
+
+
+def dense_profile(N, d, ffn, kv_heads, vocab, NP, ND, b_max, wbits=16):
+    """Per-block work of a dense decoder with ``wbits``-bit weights and fp16 KV cache.
+
+    Block parameters P_l = 2 d^2 + 2 d d_kv + 3 d ffn (q/o, k/v with grouped KV
+    heads, gated MLP).  Prefill runs one request of NP tokens; decode variant b
+    runs b requests, one token each, against a context of NP + ND tokens.
+    """
+    d_kv = d if kv_heads is None else kv_heads * HEAD_DIM
+    P_l = 2 * d * d + 2 * d * d_kv + 3 * d * ffn
+    wbytes = P_l * wbits // 8
+    assert wbytes * 8 == P_l * wbits
+    ctx = NP + ND
+    V = 1 + b_max
+    f = np.zeros(V, np.uint64)
+    y = np.zeros(V, np.uint64)
+    s = np.zeros(V, np.uint64)
+    hf = np.zeros(V, np.uint64)
+    hy = np.zeros(V, np.uint64)
+    hs = np.zeros(V, np.uint64)
+    a = np.zeros(V, np.uint64)
+    head_params = 2 * d * vocab  # embedding + output projection
+    for v in range(V):
+        tokens = NP if v == 0 else v
+        slots, kv_ctx = (1, NP) if v == 0 else (v, ctx)
+        if v == 0:
+            f[v] = 2 * P_l * NP + 4 * NP * NP * d
+            y[v] = wbytes + NP * 2 * d_kv * 2
+        else:
+            f[v] = 2 * P_l * v + 4 * v * ctx * d
+            y[v] = wbytes + v * ctx * 2 * d_kv * 2
+        s[v] = wbytes + slots * kv_ctx * 2 * d_kv * 2
+        hf[v] = 2 * d * vocab * tokens
+        hy[v] = head_params * wbits // 8
+        hs[v] = head_params * wbits // 8
+        a[v] = tokens * d * 2
+    return dict(blk_flops=f, blk_bytes=y, blk_mem=s, head_flops=hf, head_bytes=hy,
+                head_mem=hs, act_bytes=a)
+
+
+# Fleet and model shapes of the five workloads the planner is measured on.  The
+# 32-block model keeps fp16 weights; the 80- and 126-block models carry 4-bit
+# weights, the precision of the models the paper deploys (Q4_K_M, MXFP4), without
+# which no decode replica of these fleets reaches the 7 tokens/s floor.
+CONFIGS = {
+    "c1_tiny": dict(M=8, tflops=("log", 2, 30), mem_gb=(4, 16), link=("uniform", 0.1, 10),
+                    cong=(0.3, 1.0), model=dict(N=32, d=4096, ffn=11008, kv_heads=None, vocab=32000, wbits=16),
+                    prompt=("fixed", 512), K_max=2, P=64, G=1),
+    "c2": dict(M=32, tflops=("log", 2, 30), mem_gb=(4, 32), link=("uniform", 0.1, 10),
+               cong=(0.3, 1.0), model=dict(N=80, d=8192, ffn=28672, kv_heads=8, vocab=128256, wbits=4),
+               prompt=("mean", 256, 2048), K_max=8, P=1024, G=10),
+    "c3": dict(M=128, tflops=("log", 2, 30), mem_gb=(4, 32), link=("uniform", 0.1, 10),
+               cong=(0.3, 1.0), model=dict(N=80, d=8192, ffn=28672, kv_heads=8, vocab=128256, wbits=4),
+               prompt=("mean", 256, 2048), K_max=16, P=4096, G=50, redraw=(0.2, 1.0)),
+    "c4": dict(M=512, tflops=("log", 1, 60), mem_gb=(2, 64), link=("log", 0.05, 25),
+               cong=(0.3, 1.0), model=dict(N=126, d=16384, ffn=53248, kv_heads=8, vocab=128256, wbits=4),
+               prompt=("mean", 256, 4096), K_max=64, P=16384, G=1),
+    "c5": dict(M=256, tflops=("log", 2, 30), mem_gb=(4, 32), link=("uniform", 0.1, 10),
+               cong=(0.3, 1.0), model=dict(N=80, d=8192, ffn=28672, kv_heads=8, vocab=128256, wbits=4),
+               prompt=("mean", 256, 2048), K_max=32, P=8192, G=200, p_mut=0.01),
+}
+
+DEVICE_BW_GBS = (50.0, 800.0)  # device memory bandwidth, log-uniform (not given by the configs)
+B_MAX = 8
+
+
+def make_config(name: str, seed: int = 0, P: int | None = None) -> Problem:
+    """Draw the named workload with a numpy Philox generator keyed by ``seed``."""
+    c = CONFIGS[name]
+    rng = np.random.Generator(np.random.Philox(key=seed))
+    M = c["M"]
+    kind, lo, hi = c["tflops"]
+    tflops = _log_uniform(rng, lo, hi, M) if kind == "log" else rng.uniform(lo, hi, M)
+    rate = tflops * 1e12
+    bw = _log_uniform(rng, DEVICE_BW_GBS[0], DEVICE_BW_GBS[1], M) * 1e9
+    mem = np.array([int(round(x * 1e9)) for x in rng.uniform(c["mem_gb"][0], c["mem_gb"][1], M)],
+                   dtype=np.uint64)
+    lk, llo, lhi = c["link"]
+    if lk == "log":
+        gbps = _sym(rng, M, lambda n: _log_uniform(rng, llo, lhi, n))
+    else:
+        gbps = _sym(rng, M, lambda n: rng.uniform(llo, lhi, n))
+    link_bw = gbps * 1.25e8
+    np.fill_diagonal(link_bw, np.inf)
+    cong = _sym(rng, M, lambda n: rng.uniform(c["cong"][0], c["cong"][1], n))
+    pk = c["prompt"]
+    if pk[0] == "fixed":
+        NP = int(pk[1])
+    else:
+        NP = int(round(float(np.mean(rng.integers(pk[1], pk[2] + 1, 1000)))))
+    ND = NP  # generated tokens: input/generated ratios of 0.77-1.65 are reported, take 1
+    prof = dense_profile(NP=NP, ND=ND, b_max=B_MAX, **c["model"])
+    P_ = int(P if P is not None else c["P"])
+    redraw = c.get("redraw")
+    return Problem(
+        name=name, rate=rate, bw=bw, mem=mem, link_bw=link_bw, cong=cong,
+        N=c["model"]["N"], NP=NP, ND=ND, P=P_, Q=int(math.ceil(P_ / 32)), K_max=c["K_max"],
+        G=c["G"], p_mut=c.get("p_mut", 0.3), redraw=redraw is not None,
+        cong_lo=(redraw or (0.2, 1.0))[0], cong_hi=(redraw or (0.2, 1.0))[1], seed=seed,
+        **prof)
+
+
+def make_problem(rate, bw, mem, link_bw, cong, N, blk_flops, blk_bytes, blk_mem, head_flops,
+                 head_bytes, head_mem, act_bytes, NP, ND, name="custom", **kw) -> Problem:
+    """Build a Problem from explicit arrays (hand-made cases, edge cases)."""
+    f64 = lambda x: np.ascontiguousarray(np.asarray(x, dtype=np.float64))
+    u64 = lambda x: np.ascontiguousarray(np.asarray(x, dtype=np.uint64))
+    return Problem(name=name, rate=f64(rate), bw=f64(bw), mem=u64(mem), link_bw=f64(link_bw),
+                   cong=f64(cong), N=int(N), blk_flops=u64(blk_flops), blk_bytes=u64(blk_bytes),
+                   blk_mem=u64(blk_mem), head_flops=u64(head_flops), head_bytes=u64(head_bytes),
+                   head_mem=u64(head_mem), act_bytes=u64(act_bytes), NP=int(NP), ND=int(ND), **kw)
+
+
+def random_genomes(M: int, K_max: int, P: int, seed: int, max_clusters: int | None = None):
+    """Valid random genomes (uniform permutation, random composition, random roles).
+
+    Used to feed both sides the same population for evaluation-only parity; the
+    GA's own initialisation is part of the method and is not drawn here.
+    """
+    rng = np.random.Generator(np.random.Philox(key=seed + 7919))
+    kmax = min(K_max, M) if max_clusters is None else min(max_clusters, K_max, M)
+    perm = np.zeros((P, M), np.uint16)
+    sizes = np.zeros((P, K_max), np.uint16)
+    nclus = np.zeros(P, np.uint8)
+    roles = np.zeros(P, np.uint64)
+    for g in range(P):
+        perm[g] = rng.permutation(M)
+        R = int(rng.integers(1, kmax + 1))
+        cuts = np.sort(rng.choice(np.arange(1, M), R - 1, replace=False)) if R > 1 else np.array([], int)
+        edges = np.concatenate([[0], cuts, [M]])
+        sizes[g, :R] = np.diff(edges)
+        nclus[g] = R
+        bits = int(rng.integers(0, 1 << min(R, 62)))
+        if R > 62:
+            bits |= int(rng.integers(0, 1 << (R - 62))) << 62
+        roles[g] = np.uint64(bits)
+    return dict(perm=perm, sizes=sizes, nclus=nclus, roles=roles)

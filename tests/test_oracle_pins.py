@@ -1,0 +1,577 @@
+"""Pins for the CPU oracle: it is checked against what the paper and the
+mathematics fix, never against itself.
+
+* brute force over every composition of the blocks and every master (DP value,
+  master, partition under the smallest-split tie rule);
+* closed forms (identical devices, free links: ceil(N/m) blocks on the slowest
+  stage; the canonical split 3,3,4 of 10 blocks on 3 devices);
+* the paper's worked examples (20 kB over 100 Mbps = 1.6 ms; the gene
+  [(0..5),(3,1,2)]);
+* hand-computed stage costs and objective values (Eq. 3-5);
+* invariants of the formulation (blocks sum to N, >= 1 per device, memory fits,
+  the bottleneck recomputed from the partition equals the DP value);
+* exact metamorphic scaling by powers of two;
+* Philox-4x32-10 known-answer vectors; GA operator validity and frequencies.
+"""
+import itertools
+import math
+import os
+
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_2606_03770_gb300 import workloads as W
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+INF = math.inf
+
+
+# ---------------------------------------------------------------------------
+# helpers
+# ---------------------------------------------------------------------------
+def tiny_problem(rng, M, N, V=3, integer=True, tight_mem=True, head=True):
+    """Small problem whose costs are small integers / simple ratios, so that
+    the DP has many exact ties, memory walls and links that dominate."""
+    if integer:
+        rate = rng.choice([1.0, 2.0, 4.0, 0.5], M)
+        bw = rng.choice([1.0, 2.0, 8.0], M)
+        blk_flops = rng.integers(1, 4, V)
+        blk_bytes = rng.integers(0, 4, V)
+    else:
+        rate = rng.uniform(0.5, 3.0, M)
+        bw = rng.uniform(0.5, 3.0, M)
+        blk_flops = rng.integers(1, 1000, V)
+        blk_bytes = rng.integers(0, 1000, V)
+    blk_mem = rng.integers(1, 3, V)
+    mem = rng.integers(N // 2 if tight_mem else 4 * N, 4 * N + 3, M) if tight_mem else np.full(M, 10 * N)
+    head_flops = rng.integers(0, 6, V) if head else np.zeros(V, int)
+    head_bytes = rng.integers(0, 6, V) if head else np.zeros(V, int)
+    head_mem = rng.integers(0, 3, V) if head else np.zeros(V, int)
+    act = rng.integers(0, 4, V)
+    link_bw = rng.choice([0.5, 1.0, 2.0, np.inf], (M, M))
+    cong = rng.choice([0.5, 1.0], (M, M))
+    return W.make_problem(rate, bw, mem, link_bw, cong, N, blk_flops, blk_bytes, blk_mem,
+                          head_flops, head_bytes, head_mem, act, NP=64, ND=64)
+
+
+def compositions(total, parts):
+    """All (n_1..n_parts), n_t >= 1, sum = total."""
+    for cuts in itertools.combinations(range(1, total), parts - 1):
+        edges = (0,) + cuts + (total,)
+        yield tuple(edges[t + 1] - edges[t] for t in range(parts))
+
+
+def bf_value(op, v, devs, layers_total, k, mu):
+    """min over compositions of layers_total blocks on devs[0..k) with master mu
+    (0-based, may be >= k meaning 'not among them') of the largest stage or link."""
+    best = INF
+    for comp in compositions(layers_total, k):
+        worst = 0.0
+        for t in range(k):
+            worst = max(worst, op.stage_cost(v, int(devs[t]), comp[t], t == mu))
+            if t >= 1:
+                worst = max(worst, op.link_cost(v, int(devs[t - 1]), int(devs[t])))
+        best = min(best, worst)
+    return best
+
+
+def bf_dp(op, v, devs, N):
+    """Brute-force DP_Pipe: value, first optimal master, and the partition the
+    smallest-split tie rule selects (walk back from the last device; at each
+    step the smallest start j that keeps the optimum, where the optimum of the
+    prefix is again found by enumeration)."""
+    m = len(devs)
+    if m > N:
+        return None
+    vals = [bf_value(op, v, devs, N, m, mu) for mu in range(m)]
+    V = min(vals)
+    if V == INF:
+        return None
+    mu = vals.index(V)
+    layers = [0] * m
+    i = N - 1
+    for k in range(m, 1, -1):
+        target = bf_value(op, v, devs, i + 1, k, mu)
+        tau = op.link_cost(v, int(devs[k - 2]), int(devs[k - 1]))
+        for j in range(k - 1, i + 1):
+            prev = bf_value(op, v, devs, j, k - 1, mu)
+            c = max(prev, op.stage_cost(v, int(devs[k - 1]), i - j + 1, mu == k - 1), tau)
+            if c == target:
+                break
+        layers[k - 1] = i - j + 1
+        i = j - 1
+    layers[0] = i + 1
+    return V, mu, layers
+
+
+# ---------------------------------------------------------------------------
+# Philox
+# ---------------------------------------------------------------------------
+def test_philox_known_answers():
+    rows = [l.split() for l in open(os.path.join(GOLDEN, "philox4x32_10_kat.txt"))
+            if l.strip() and not l.startswith("#")]
+    assert len(rows) == 3
+    for r in rows:
+        v = [int(x, 16) for x in r]
+        out = O.philox(v[0:4], v[4:6])
+        assert [int(x) for x in out] == v[6:10]
+
+
+def test_philox_stream_layout_and_uniformity():
+    # word t of a stream is word t%4 of block t//4
+    seed = 0x123456789ABCDEF
+    blk = O.philox([5, 7, 3, 4], [seed & 0xFFFFFFFF, seed >> 32])
+    assert [O.word(seed, 3, 7, 4, 20 + t) for t in range(4)] == [int(x) for x in blk]
+    w = np.array([O.word(1, 0, 0, 0, t) for t in range(40000)], dtype=np.float64)
+    u = w / 2.0 ** 32
+    assert abs(u.mean() - 0.5) < 0.01 and abs(u.var() - 1 / 12) < 0.005
+
+
+def test_threshold():
+    assert O.threshold(0.0) == 0 and O.threshold(1.0) == 2 ** 32 and O.threshold(0.5) == 2 ** 31
+    assert O.threshold(0.3) == math.floor(0.3 * 2 ** 32)
+
+
+# ---------------------------------------------------------------------------
+# cost model: hand values and the paper's worked example
+# ---------------------------------------------------------------------------
+def test_stage_cost_hand_values():
+    # one device: 2e12 FLOP/s, 1e11 B/s, 10e9 B; block = 1e12 FLOP, 1e10 B streamed,
+    # 4e9 B resident; head = 1e12 FLOP, 5e11 B streamed, 3e9 B resident.
+    p = W.make_problem([2e12], [1e11], [10_000_000_000], [[np.inf]], [[1.0]], 4,
+                       [10 ** 12], [10 ** 10], [4 * 10 ** 9], [10 ** 12], [5 * 10 ** 11],
+                       [3 * 10 ** 9], [0], NP=1, ND=1)
+    op = O.OracleProblem(p)
+    assert op.stage_cost(0, 0, 1, 0) == 0.5          # 1e12/2e12 vs 1e10/1e11=0.1
+    assert op.stage_cost(0, 0, 2, 0) == 1.0          # 2e12/2e12 vs 0.2
+    assert op.stage_cost(0, 0, 3, 0) == INF          # 12e9 B > 10e9 B
+    assert op.stage_cost(0, 0, 1, 1) == 5.1          # master: 2e12/2e12=1 vs 5.1e11/1e11=5.1
+    assert op.stage_cost(0, 0, 2, 1) == INF          # 8e9 + 3e9 > 10e9
+
+
+def test_link_cost_paper_example():
+    row = [l for l in open(os.path.join(GOLDEN, "paper_worked_examples.txt")) if l.startswith("link_cost")][0]
+    _, A, bits, expect = row.split()
+    bw = float(bits) / 8.0  # bytes/s
+    p = W.make_problem([1.0, 1.0], [1.0, 1.0], [1, 1], [[np.inf, bw], [bw, np.inf]],
+                       [[1.0, 1.0], [1.0, 1.0]], 2, [1], [1], [1], [0], [0], [0], [int(A)], NP=1, ND=1)
+    op = O.OracleProblem(p)
+    assert op.link_cost(0, 0, 1) == pytest.approx(float(expect), rel=1e-15)
+
+
+def test_link_cost_congestion_scales_bandwidth():
+    p = W.make_problem([1.0, 1.0], [1.0, 1.0], [1, 1], [[np.inf, 1000.0], [1000.0, np.inf]],
+                       [[1.0, 0.25], [0.25, 1.0]], 2, [1], [1], [1], [0], [0], [0], [500], NP=1, ND=1)
+    assert O.OracleProblem(p).link_cost(0, 1, 0) == 2.0   # 500 B / (1000 B/s * 0.25)
+
+
+# ---------------------------------------------------------------------------
+# DP_Pipe against brute force
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("seed", range(40))
+def test_dp_matches_brute_force(seed):
+    rng = np.random.default_rng(seed)
+    N = int(rng.integers(1, 11))
+    M = 6
+    prob = tiny_problem(rng, M, N, integer=seed % 4 != 3, head=seed % 5 != 0)
+    op = O.OracleProblem(prob)
+    for trial in range(4):
+        m = int(rng.integers(1, M + 1))
+        devs = rng.permutation(M)[:m]
+        v = int(rng.integers(0, prob.V))
+        got = op.dp_pipe(v, devs)
+        bf = bf_dp(op, v, devs, N)
+        if bf is None:
+            assert not got["ok"] and got["V"] == INF and got["mu"] == -1
+            continue
+        V, mu, layers = bf
+        assert got["ok"]
+        assert got["V"] == V, (devs, v)
+        assert got["mu"] == mu
+        assert list(got["layers"]) == layers
+
+
+def test_dp_more_devices_than_blocks_is_infeasible():
+    rng = np.random.default_rng(0)
+    prob = tiny_problem(rng, 6, 4, tight_mem=False)
+    r = O.OracleProblem(prob).dp_pipe(0, [0, 1, 2, 3, 4])
+    assert not r["ok"] and r["V"] == INF and list(r["layers"]) == [-1] * 5
+
+
+def test_dp_closed_form_identical_devices():
+    # identical devices, free links, no head, ample memory: the optimum is the
+    # cost of ceil(N/m) blocks, and the smallest-split rule puts the short
+    # stages first (10 blocks on 3 devices -> 3,3,4)
+    for N, m in [(10, 3), (7, 2), (12, 5), (9, 9), (1, 1), (13, 4)]:
+        M = m
+        p = W.make_problem(np.full(M, 3.0), np.full(M, 1.0), np.full(M, 10 ** 6),
+                           np.full((M, M), np.inf), np.ones((M, M)), N, [7], [1], [1], [0], [0], [0],
+                           [5], NP=1, ND=1)
+        op = O.OracleProblem(p)
+        r = op.dp_pipe(0, list(range(m)))
+        q = math.ceil(N / m)
+        assert r["V"] == (7 * q) / 3.0
+        assert sum(r["layers"]) == N and max(r["layers"]) == q
+        if (N, m) == (10, 3):
+            assert list(r["layers"]) == [3, 3, 4]
+        assert r["mu"] == 0
+
+
+def test_dp_candidate_count_is_quadratic():
+    # the recurrence examines N candidates for device 1 and sum_{i} (i-k+2) for
+    # device k, for each of the m masters: O(m^2 N^2) as the paper states
+    rng = np.random.default_rng(1)
+    for N, m in [(10, 3), (20, 5), (32, 8)]:
+        prob = tiny_problem(rng, 8, N, tight_mem=False)
+        r = O.OracleProblem(prob).dp_pipe(0, list(range(m)))
+        per_mu = N + sum((N - k + 1) * (N - k + 2) // 2 for k in range(2, m + 1))
+        assert r["cand"] == m * per_mu
+
+
+def _invariants(op, prob, v, devs, r):
+    N = prob.N
+    lay = [int(x) for x in r["layers"]]
+    assert sum(lay) == N and min(lay) >= 1
+    mu = r["mu"]
+    worst = 0.0
+    for k, d in enumerate(devs):
+        c = op.stage_cost(v, int(d), lay[k], k == mu)
+        assert c < INF  # memory fits
+        worst = max(worst, c)
+        if k:
+            t = op.link_cost(v, int(devs[k - 1]), int(d))
+            assert r["V"] >= t
+            worst = max(worst, t)
+    assert worst == r["V"]
+
+
+def test_dp_invariants_on_tiny_workload():
+    prob = W.make_config("c1_tiny")
+    op = O.OracleProblem(prob)
+    rng = np.random.default_rng(3)
+    checked = 0
+    for _ in range(60):
+        m = int(rng.integers(1, prob.M + 1))
+        devs = rng.permutation(prob.M)[:m]
+        for v in (0, 1, prob.b_max):
+            r = op.dp_pipe(v, devs)
+            if r["ok"]:
+                _invariants(op, prob, v, devs, r)
+                checked += 1
+                if m == 1:
+                    assert r["V"] == op.stage_cost(v, int(devs[0]), prob.N, True)
+    assert checked > 20
+
+
+def test_dp_brute_force_on_tiny_workload_clusters():
+    # real tiny-config costs, a shortened model so that enumeration stays cheap
+    prob = W.make_config("c1_tiny")
+    prob.N = 10
+    op = O.OracleProblem(prob)
+    rng = np.random.default_rng(4)
+    for _ in range(12):
+        m = int(rng.integers(1, 5))
+        devs = rng.permutation(prob.M)[:m]
+        for v in (0, prob.b_max):
+            got = op.dp_pipe(v, devs)
+            bf = bf_dp(op, v, devs, prob.N)
+            if bf is None:
+                assert not got["ok"]
+            else:
+                assert (got["V"], got["mu"], list(got["layers"])) == bf
+
+
+# ---------------------------------------------------------------------------
+# metamorphic: doubling every rate, bandwidth and link speed halves all times
+# exactly (division by a power of two is exact), leaves partitions unchanged
+# ---------------------------------------------------------------------------
+def test_metamorphic_power_of_two_scaling():
+    prob = W.make_config("c1_tiny")
+    fast = W.make_config("c1_tiny")
+    fast.rate = prob.rate * 2
+    fast.bw = prob.bw * 2
+    fast.link_bw = prob.link_bw * 2
+    fast.t_a = prob.t_a / 2
+    fast.min_tps = prob.min_tps * 2
+    g = W.random_genomes(prob.M, prob.K_max, 48, seed=5)
+    a = O.OracleProblem(prob).eval_population(g, prob.K_max)
+    b = O.OracleProblem(fast).eval_population(g, prob.K_max)
+    for k in ("layers", "master", "bsel"):
+        assert np.array_equal(a[k], b[k])
+    assert np.array_equal(a["T"] / 2, b["T"])
+    assert np.array_equal(a["L"] / 2, b["L"])
+    assert np.array_equal(a["fitness"][:, :2] / 2, b["fitness"][:, :2])
+    assert np.array_equal(a["fitness"][:, 2:] * 2, b["fitness"][:, 2:])
+
+
+# ---------------------------------------------------------------------------
+# gene decoding (paper example) and the objective (Eq. 3-5)
+# ---------------------------------------------------------------------------
+def test_gene_decoding_paper_example():
+    row = [l for l in open(os.path.join(GOLDEN, "paper_worked_examples.txt")) if l.startswith("gene")][0]
+    _, body = row.split(" ", 1)
+    order_s, group_s, reps_s = [x.strip() for x in body.split("|")]
+    order = [int(x) for x in order_s.split(",")]
+    groups = [int(x) for x in group_s.split(",")]
+    reps = [[int(x) for x in r.split(",")] for r in reps_s.split(";")]
+    M = len(order)
+    rng = np.random.default_rng(8)
+    prob = tiny_problem(rng, M, 6, tight_mem=False)
+    op = O.OracleProblem(prob)
+    K = 4
+    sizes = np.zeros((1, K), np.uint16)
+    sizes[0, :3] = groups
+    g = dict(perm=np.array([order], np.uint16), sizes=sizes, nclus=np.array([3], np.uint8),
+             roles=np.array([0b010], np.uint64))
+    out = op.eval_population(g, K)
+    off = 0
+    for c, rep in enumerate(reps):
+        r = op.eval_cluster(rep, decode=(c == 1))
+        assert out["T"][0, c] == r["T"] and out["bsel"][0, c] == r["b"]
+        assert list(out["layers"][0, off:off + len(rep)]) == list(r["layers"])
+        off += len(rep)
+
+
+def _objective_problem(NP, ND, t_a):
+    return W.make_problem([1.0], [1.0], [1], [[np.inf]], [[1.0]], 1, [1], [1], [1], [0], [0], [0],
+                          [0], NP=NP, ND=ND, t_a=t_a)
+
+
+def test_objective_hand_cases():
+    op = O.OracleProblem(_objective_problem(100, 100, 1.0))
+    # prefill T=1 s -> PS = 100 tok/s; decode b=2 at T=0.5 s -> DS = 4 tok/s
+    # Eq.3: phase = max(100/100, 100/4) = 25; Eq.4: 25 - 1 = 24; Eq.5: 1 + 24 = 25
+    f = op.score(0b10, [1.0, 0.5], [0, 2])
+    assert list(f) == [25.0, 25.0, 100.0, 4.0]
+    # two prefill replicas aggregate (Sec. 3.3): PS = 100/1 + 100/0.5 = 300
+    f = op.score(0b100, [1.0, 0.5, 0.25], [0, 0, 8])
+    assert f[2] == 300.0 and f[3] == 32.0
+    # phase = max(1/3, 3.125) = 3.125 -> w = 1/3 + 2.125
+    assert f[1] == 3.125 and f[0] == 100.0 / 300.0 + 2.125
+    # no congestion: phase below the arrival interval -> w = 0
+    f = op.score(0b10, [0.01, 0.01], [0, 8])
+    assert f[0] == 0.0 and f[1] == max(100 / (100 / 0.01), 100 / (8 / 0.01))
+    # phase exactly T_a: bottleneck = 0, strict > in Eq. 5 -> w = 0
+    f = op.score(0b10, [1.0, 0.01], [0, 1])   # PS=100 -> NP/PS = 1.0 = T_a
+    assert f[1] == 1.0 and f[0] == 0.0
+    # no prefill capacity, or no decode capacity -> infinite waiting
+    assert op.score(0b11, [1.0, 1.0], [1, 1])[0] == INF
+    assert op.score(0b00, [1.0, 1.0], [0, 0])[0] == INF
+    # an infeasible replica contributes nothing
+    f = op.score(0b10, [1.0, INF], [0, -1])
+    assert f[0] == INF and f[2] == 100.0 and f[3] == 0.0
+
+
+def test_decode_picks_highest_feasible_batch():
+    prob = W.make_config("c1_tiny")
+    op = O.OracleProblem(prob)
+    rng = np.random.default_rng(9)
+    seen_mid = 0
+    for _ in range(80):
+        m = int(rng.integers(1, 5))
+        devs = rng.permutation(prob.M)[:m]
+        r = op.eval_cluster(devs, decode=True)
+        b = r["b"] if r["ok"] else 0
+        for bb in range(b + 1, prob.b_max + 1):       # every larger batch fails
+            d = op.dp_pipe(bb, devs)
+            if d["ok"]:
+                assert 1.0 / op.latency(bb, devs, d["mu"], d["layers"]) < prob.min_tps
+        if r["ok"]:
+            d = op.dp_pipe(b, devs)
+            assert d["V"] == r["T"] and 1.0 / r["L"] >= prob.min_tps
+            seen_mid += 0 < b < prob.b_max
+    assert seen_mid >= 0
+
+
+# ---------------------------------------------------------------------------
+# genetic operators
+# ---------------------------------------------------------------------------
+def _valid(g, M, K):
+    for s in range(len(g["nclus"])):
+        assert sorted(g["perm"][s]) == list(range(M))
+        R = int(g["nclus"][s])
+        assert 1 <= R <= min(K, M)
+        sz = g["sizes"][s]
+        assert all(sz[:R] >= 1) and int(sz[:R].sum()) == M and all(sz[R:] == 0)
+        assert int(g["roles"][s]) >> R == 0
+
+
+def test_init_population_valid_and_spread():
+    ga = O._ga_struct(400, 12, 5, 13, 4, 0.5, 0.3, (0.2, 0.5, 0.15, 0.15))
+    g = O.init_population(ga, 77)
+    _valid(g, 12, 5)
+    counts = np.bincount(g["nclus"], minlength=6)[1:]
+    assert all(counts > 50)                      # R uniform over 1..5
+    assert len({tuple(p) for p in g["perm"]}) > 390
+
+
+def test_repair_hand_example():
+    # A = 0 1 2 3 4, B = 4 3 2 1 0, B taken at positions 0 and 3 -> 4 1 2 1 4;
+    # position 3 repeats 1 and position 4 repeats 4, the missing 0 and 3 fill them
+    assert list(O.repair([4, 1, 2, 1, 4])) == [4, 1, 2, 0, 3]
+    assert list(O.repair([2, 2, 2, 2])) == [2, 0, 1, 3]
+    assert list(O.repair([3, 1, 0, 2])) == [3, 1, 0, 2]
+
+
+def test_mutation_kind_frequencies():
+    # kinds drawn from word 1 of the mutation stream against cumulative
+    # thresholds: 20% swap, 50% regroup-from-position, 15% regroup, 15% both
+    t = [O.threshold(x) for x in (0.2, 0.2 + 0.5, 0.2 + 0.5 + 0.15)]
+    n = 200000
+    w = np.array([O.word(11, 3, s, O.PURPOSE["MUTATE"], 1) for s in range(n)], dtype=np.uint64)
+    kinds = np.searchsorted(np.array(t, dtype=np.uint64), w, side="right")
+    freq = np.bincount(kinds, minlength=4) / n
+    assert np.allclose(freq, [0.2, 0.5, 0.15, 0.15], atol=0.004)
+
+
+def _ga_problem(P=200, M=10, K=4, Q=7, p_mut=0.3, kinds=(0.2, 0.5, 0.15, 0.15)):
+    return O._ga_struct(P, M, K, Q, 4, 0.5, p_mut, kinds)
+
+
+def _fitness_for(g, rng):
+    P = len(g["nclus"])
+    f = np.zeros((P, 4))
+    f[:, 0] = rng.choice([0.0, 1.0, 2.5, INF], P)
+    f[:, 1] = rng.uniform(0, 3, P)
+    return f
+
+
+def test_ga_children_valid_and_elites_copied():
+    rng = np.random.default_rng(12)
+    ga = _ga_problem()
+    g = O.init_population(ga, 5)
+    f = _fitness_for(g, rng)
+    e = O.elites(ga, g, f)
+    nxt = O.ga_step(ga, 5, 1, g, f, e)
+    _valid(nxt, ga.M, ga.K)
+    for q in range(ga.Q):
+        for k in ("perm", "sizes"):
+            assert np.array_equal(nxt[k][q], g[k][e[q]])
+        assert nxt["nclus"][q] == g["nclus"][e[q]] and nxt["roles"][q] == g["roles"][e[q]]
+
+
+def test_ga_mutation_kinds_act_as_described():
+    rng = np.random.default_rng(13)
+    base = _ga_problem(p_mut=0.0)
+    g = O.init_population(base, 9)
+    f = _fitness_for(g, rng)
+    e = O.elites(base, g, f)
+    plain = O.ga_step(base, 9, 2, g, f, e)       # crossover + repair only
+    Q = base.Q
+    # swap only: the ordering differs from the unmutated child by one transposition
+    sw = O.ga_step(_ga_problem(p_mut=1.0, kinds=(1.0, 0, 0, 0)), 9, 2, g, f, e)
+    for s in range(Q, base.P):
+        diff = np.nonzero(sw["perm"][s] != plain["perm"][s])[0]
+        assert len(diff) in (0, 2)
+        assert np.array_equal(sw["sizes"][s], plain["sizes"][s])
+    # regroup from a position: ordering untouched, a prefix of the grouping kept
+    rg = O.ga_step(_ga_problem(p_mut=1.0, kinds=(0, 1.0, 0, 0)), 9, 2, g, f, e)
+    _valid(rg, base.M, base.K)
+    for s in range(Q, base.P):
+        assert np.array_equal(rg["perm"][s], plain["perm"][s])
+    # regenerate both: orderings change (almost surely)
+    bo = O.ga_step(_ga_problem(p_mut=1.0, kinds=(0, 0, 0, 1.0)), 9, 2, g, f, e)
+    _valid(bo, base.M, base.K)
+    changed = sum(not np.array_equal(bo["perm"][s], plain["perm"][s]) for s in range(Q, base.P))
+    assert changed > (base.P - Q) * 0.9
+
+
+def test_crossover_mixes_both_parents_evenly():
+    # with identical fitness everywhere the tournament picks by index; check the
+    # per-position source statistics of a uniform crossover at p = 0.5
+    n = 100000
+    w = np.array([O.word(21, 1, s, O.PURPOSE["CROSS"], 3) for s in range(n)], dtype=np.uint64)
+    assert abs(np.mean(w < O.threshold(0.5)) - 0.5) < 0.005
+
+
+def test_elites_distinct_and_ordered():
+    ga = _ga_problem(P=12, M=5, K=3, Q=6)
+    g = O.init_population(ga, 3)
+    # make genomes 4 and 9 copies of genome 1, genome 7 a copy of 2
+    for dst, src in [(4, 1), (9, 1), (7, 2)]:
+        for k in ("perm", "sizes", "nclus", "roles"):
+            g[k][dst] = g[k][src]
+    f = np.zeros((12, 4))
+    f[:, 0] = [5, 1, 2, 9, 1, 0.5, 7, 2, 8, 1, 3, 4]
+    f[:, 1] = 0
+    e = list(O.elites(ga, g, f))
+    # distinct genomes by (w, index): 5(0.5) 1(1) 2(2) 10(3) 11(4) 0(5)
+    assert e == [5, 1, 2, 10, 11, 0]
+    ga2 = _ga_problem(P=12, M=5, K=3, Q=11)
+    e2 = list(O.elites(ga2, g, f))
+    # 9 distinct genomes, then duplicates by key: 4 (w=1), 9 (w=1)
+    assert e2 == [5, 1, 2, 10, 11, 0, 6, 8, 3, 4, 9]
+
+
+def test_ga_best_is_monotone_and_bounded_by_exhaustive_optimum():
+    # 5 devices, at most 2 replicas: enumerate every genome for the optimum
+    rng = np.random.default_rng(21)
+    M, K, N = 5, 2, 6
+    prob = tiny_problem(rng, M, N, integer=False, tight_mem=False)
+    prob.t_a = 0.0
+    op = O.OracleProblem(prob)
+    allg = []
+    for perm in itertools.permutations(range(M)):
+        for R in (1, 2):
+            for comp in compositions(M, R):
+                for roles in range(1 << R):
+                    allg.append((perm, comp, R, roles))
+    P_all = len(allg)
+    G = dict(perm=np.array([a[0] for a in allg], np.uint16),
+             sizes=np.array([list(a[1]) + [0] * (K - a[2]) for a in allg], np.uint16),
+             nclus=np.array([a[2] for a in allg], np.uint8),
+             roles=np.array([a[3] for a in allg], np.uint64))
+    opt = op.eval_population(G, K, nthreads=4)["fitness"][:, 0].min()
+    ga = O._ga_struct(32, M, K, 2, 4, 0.5, 0.3, (0.2, 0.5, 0.15, 0.15))
+    g = O.init_population(ga, 1)
+    best = INF
+    for gen in range(1, 12):
+        f = op.eval_population(g, K)["fitness"]
+        cur = f[:, 0].min()
+        assert cur >= opt
+        assert cur <= best
+        best = cur
+        e = O.elites(ga, g, f)
+        g = O.ga_step(ga, 1, gen, g, f, e)
+    assert P_all == 120 * (2 + 4 * 4)
+
+
+def test_congestion_redraw_range_and_symmetry():
+    c = O.redraw_congestion(64, 3, 5, 0.2, 1.0)
+    off = c[~np.eye(64, dtype=bool)]
+    assert np.array_equal(c, c.T) and np.all(np.diag(c) == 1.0)
+    assert off.min() >= 0.2 and off.max() < 1.0
+    assert abs(off.mean() - 0.6) < 0.01
+    c2 = O.redraw_congestion(64, 3, 6, 0.2, 1.0)
+    assert not np.array_equal(c, c2)
+    assert np.array_equal(c, O.redraw_congestion(64, 3, 5, 0.2, 1.0))
+
+
+def test_memory_boundary_fits_exactly():
+    # a stage that needs exactly the device's memory fits (infeasible only if it exceeds)
+    p = W.make_problem([1.0], [1.0], [12], [[np.inf]], [[1.0]], 4, [1], [1], [4], [0], [0], [4],
+                       [0], NP=1, ND=1)
+    op = O.OracleProblem(p)
+    assert op.stage_cost(0, 0, 3, 0) == 3.0
+    assert op.stage_cost(0, 0, 2, 1) == 2.0     # 2*4 + 4 = 12 bytes = memory
+    assert op.stage_cost(0, 0, 3, 1) == INF
+
+
+def test_latency_hand_value_and_tps_boundary():
+    # decode b=1: a block is 1 FLOP on 4 FLOP/s devices (0.25 s), the activation
+    # 1 byte over a 4 B/s link (0.25 s): two devices, one block each ->
+    # Lambda = 0.25 + 0.25 + 0.25 = 0.75 s, bottleneck T = 0.25 s.
+    # Sec. 3.2: a per-request rate 1/Lambda that equals Min_TPS is accepted.
+    link = [[np.inf, 4.0], [4.0, np.inf]]
+    mk = lambda tps: W.make_problem([4.0, 4.0], [1.0, 1.0], [10, 10], link, np.ones((2, 2)), 2,
+                                    [1, 1], [0, 0], [1, 1], [0, 0], [0, 0], [0, 0], [1, 1],
+                                    NP=1, ND=1, min_tps=tps)
+    op = O.OracleProblem(mk(1.0 / 0.75))
+    d = op.dp_pipe(1, [0, 1])
+    assert d["V"] == 0.25 and list(d["layers"]) == [1, 1]
+    assert op.latency(1, [0, 1], d["mu"], d["layers"]) == 0.75
+    r = op.eval_cluster([0, 1], decode=True)
+    assert r["ok"] and r["b"] == 1 and r["T"] == 0.25 and r["L"] == 0.75
+    r = O.OracleProblem(mk(np.nextafter(1.0 / 0.75, 2.0))).eval_cluster([0, 1], decode=True)
+    assert not r["ok"] and r["b"] == -1
