@@ -1,0 +1,322 @@
+"""Benchmark: one GA generation of the E2LLM deployment search per step.
+
+A step is the whole hot path over one population: DP_Pipe for every replica
+and variant with the decode batch sweep, the objective, the elites and the
+generation step (tournament, crossover + repair, mutation).  The default
+workload is the 32-device fleet / 80-block model / 8-replica / population
+1024 configuration.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+value: genome evaluations per second over the timed steps, device time with
+CUDA events on the engine's stream, L2 flushed (256 MB write) between steps.
+e2e: the same metric through the C ABI with pinned host buffers: each step
+uploads the population, evaluates, steps, and reads fitness and the next
+population back.  --impl reference times the CPU oracle on the host cores.
+Under torchrun each rank runs an independent replica search (its own seed) on
+its own GPU; value is the sum over ranks divided by the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2606_03770_gb300 import workloads as W  # noqa: E402
+
+METRIC = "genome evaluations/sec (GA generations on device)"
+UNIT = "genomes/s"
+WORKLOAD = "c2"
+L2_FLUSH_BYTES = 256 << 20
+# algorithmic int32 ALU operations: per bisection probe (two key loads, a 64-bit
+# compare = 2 ops, midpoint = 2 ops, index = 1 op, interval update = 1 op) and
+# per DP cell to finish it (two 64-bit min/max = 4 ops, two guards = 2 ops)
+OPS_PER_PROBE = 6
+OPS_PER_CELL = 6
+SM_COUNT = 152
+INT32_LANES_PER_SM = 128
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default=WORKLOAD)
+    ap.add_argument("--seed", type=int, default=2026)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    return ap.parse_args()
+
+
+def dist_info():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            p = [x.strip() for x in line.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                sm.append(float(p[1]))
+                mx.append(float(p[2]))
+            except ValueError:
+                continue
+            for n, val in zip(names, p[5:9]):
+                if val.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def cpu_baseline(prob, seed, sample=None):
+    """The oracle, as it is, on this host's cores: evaluate a bounded sample of
+    one generation's genomes, plus the elites and the full generation step."""
+    from oracle import oracle as O
+    ga = O.ga_of(prob)
+    pop = O.init_population(ga, seed)
+    nt = O.num_threads()
+    sample = sample or min(prob.P, 64 * nt)
+    sub = {k: np.ascontiguousarray(v[:sample]) for k, v in pop.items()}
+    op = O.OracleProblem(prob)
+    t0 = time.perf_counter()
+    op.eval_population(sub, prob.K_max, nthreads=nt)
+    t_eval = time.perf_counter() - t0
+    full_fit = np.zeros((prob.P, 4))
+    full_fit[:, 0] = np.arange(prob.P, dtype=np.float64)      # any order; only timing matters here
+    t0 = time.perf_counter()
+    e = O.elites(ga, pop, full_fit)
+    O.ga_step(ga, seed, 1, pop, full_fit, e)
+    t_ga = time.perf_counter() - t0
+    t_gen = t_eval * prob.P / sample + t_ga
+    return {"value": prob.P / t_gen, "unit": UNIT, "cores": nt, "kind": "oracle",
+            "sample": f"{sample} of {prob.P} genomes of one generation evaluated on {nt} threads "
+                      f"({t_eval:.2f} s), scaled to the population, plus the elites and generation "
+                      f"step of the full population ({t_ga:.3f} s)"}
+
+
+def run_reference(args):
+    rank, world, _ = dist_info()
+    if rank != 0:
+        return
+    prob = W.make_config(args.config)
+    from oracle import oracle as O
+    nt = O.num_threads()
+    sample = min(prob.P, 16 * nt)
+    ga = O.ga_of(prob)
+    pop = O.init_population(ga, args.seed)
+    op = O.OracleProblem(prob)
+    times = []
+    for step in range(args.warmup + args.steps):
+        sub = {k: np.ascontiguousarray(v[(step * sample) % prob.P:][:sample]) for k, v in pop.items()}
+        t0 = time.perf_counter()
+        out = op.eval_population(sub, prob.K_max, nthreads=nt)
+        dt = time.perf_counter() - t0
+        if step >= args.warmup:
+            times.append(dt)
+    t = sum(times)
+    value = sample * len(times) / t
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / len(times),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded fleet, links and dense-decoder profile)",
+            "config": {"workload": f"{prob.name}: M={prob.M} devices, N={prob.N} blocks, K_max={prob.K_max}, "
+                                   f"P={prob.P}", "sample_genomes_per_step": sample},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": nt, "kind": "oracle",
+                             "sample": f"{sample} genomes per step evaluated by the oracle on {nt} threads"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    rank, world, local = dist_info()
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    import __graft_entry__ as ge
+    ge.build()
+    from paper_2606_03770_gb300.e2ga import Engine
+
+    prob = W.make_config(args.config)
+    seed = args.seed + 1000 * rank
+    eng = Engine(prob)
+    stream = eng.stream
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+
+    def sync_all():
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+
+    # ---- device-resident search: eval + elites + generation step per step
+    eng.init_population(seed)
+    gen = 0
+    for _ in range(args.warmup):
+        gen += 1
+        eng.eval(parts=False)
+        eng.ga_step(seed, gen)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    stats = []
+    clocks = Clocks(local)
+    sync_all()
+    clocks.start()
+    for i in range(args.steps):
+        with torch.cuda.stream(stream):
+            flush.fill_(i & 0xFF)
+        gen += 1
+        a, b, c = ev[i]
+        a.record(stream)
+        eng.eval(parts=False)
+        b.record(stream)
+        eng.ga_step(seed, gen)
+        c.record(stream)
+        stats.append(eng.stats())
+    sync_all()
+    clk = clocks.stop()
+    step_ms = [a.elapsed_time(c) for a, b, c in ev]
+    eval_ms = [a.elapsed_time(b) for a, b, c in ev]
+    t_local = sum(step_ms) / 1e3
+    t = torch.tensor([t_local], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    t_max = float(t.item())
+    value = prob.P * args.steps * world / t_max
+
+    # ---- roofline of the dominant kernel (DP_Pipe evaluation)
+    probes = sum(s["dp_probes"] for s in stats) / args.steps
+    cells = sum(s["dp_cells"] for s in stats) / args.steps
+    eval_s = sum(eval_ms) / 1e3 / args.steps
+    ops = OPS_PER_PROBE * probes + OPS_PER_CELL * cells
+    achieved = ops / eval_s / 1e12
+    peaks_path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    sm_max = 2070.0
+    if os.path.exists(peaks_path):
+        sm_max = float(json.load(open(peaks_path)).get("sm_max_mhz", sm_max))
+    peak = SM_COUNT * INT32_LANES_PER_SM * sm_max * 1e6 / 1e12
+    paper = sum(s["paper_candidates"] for s in stats) / args.steps
+
+    # ---- end to end through the C ABI with pinned host buffers
+    e2e = None
+    if not args.no_e2e:
+        P, M, K = prob.P, prob.M, prob.K_max
+        host = dict(perm=torch.empty((P, M), dtype=torch.int16).pin_memory(),
+                    sizes=torch.empty((P, K), dtype=torch.int16).pin_memory(),
+                    nclus=torch.empty(P, dtype=torch.uint8).pin_memory(),
+                    roles=torch.empty(P, dtype=torch.int64).pin_memory())
+        hfit = torch.empty((P, 4), dtype=torch.float64).pin_memory()
+        eng.get_population(host)
+        bytes_pop = P * (2 * M + 2 * K + 1 + 8)
+
+        def e2e_step(g):
+            eng.set_population(host)                 # host -> device, validated
+            eng.eval(fitness=hfit, parts=False)      # fitness -> host
+            eng.ga_step(seed, g)
+            eng.get_population(host)                 # next population -> host
+
+        for _ in range(2):
+            gen += 1
+            e2e_step(gen)
+        sync_all()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            gen += 1
+            e2e_step(gen)
+        torch.cuda.synchronize()
+        te = torch.tensor([time.perf_counter() - t0], dtype=torch.float64, device="cuda")
+        if world > 1:
+            dist.all_reduce(te, op=dist.ReduceOp.MAX)
+        e2e = {"value": P * args.steps * world / float(te.item()), "unit": UNIT,
+               "h2d_bytes_per_step": bytes_pop, "d2h_bytes_per_step": bytes_pop + 32 * P}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * t_max / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded fleet, links and dense-decoder profile; no paper data)",
+            "config": {"workload": f"{prob.name}: M={prob.M} devices, N={prob.N} blocks (d=8192, ffn=28672, "
+                                   f"GQA 8 KV heads, 4-bit weights), K_max={prob.K_max} replicas, "
+                                   f"P={prob.P}, Q={prob.Q}, b_max={prob.b_max}, one generation per step",
+                       "l2": "flushed (256 MB write) between timed steps",
+                       "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+            "gpu_launches": 5 * args.steps,
+            "dp_cells_per_s": cells * args.steps * world / t_max,
+            "paper_candidates_per_s": paper * args.steps * world / t_max,
+            "eval_ms_per_step": 1e3 * eval_s,
+            "served_replicas_per_step": sum(s["served"] for s in stats) / args.steps,
+            "replicas_per_step": sum(s["replicas"] for s in stats) / args.steps,
+            "roofline": {"bound": "alu", "kernel": "dp_eval_kernel + score_kernel (e2_eval_population)",
+                         "achieved": achieved, "peak": peak, "unit": "Tops/s (int32)",
+                         "frac": achieved / peak, "traffic": None,
+                         "per_unit": f"{OPS_PER_PROBE} int32 ops per bisection probe + {OPS_PER_CELL} per DP cell",
+                         "peak_source": f"{SM_COUNT} SMs x {INT32_LANES_PER_SM} int32 lanes x {sm_max:.0f} MHz"},
+            "e2e": e2e,
+            "clocks": clk,
+        }
+        if not args.no_cpu and world == 1:
+            line["cpu_baseline"] = cpu_baseline(prob, seed)
+        print(json.dumps(line), flush=True)
+    eng.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

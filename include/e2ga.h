@@ -1,0 +1,232 @@
+/*
+ * e2ga.h -- C ABI of the GB300 (sm_103a) batched fitness engine for the E2LLM
+ * deployment search (arxiv 2606.03770).
+ *
+ * The library evaluates a whole genetic-algorithm population on one GPU.  A
+ * genome (Sec. 3.4, App. A "Gene definition") is an ordering of the M devices
+ * plus a grouping of that ordering into R <= K_max replicas, each replica
+ * tagged prefill (role bit 0) or decode (role bit 1).  For every replica the
+ * library runs DP_Pipe (Alg. 1, Eq. 1-2): the min-max partition of N identical
+ * transformer blocks into contiguous stages on the replica's devices, in
+ * genome order, with the master (the device holding the LM head and output
+ * layer, Sec. 3.1) enumerated, links as pipeline stages and memory-infeasible
+ * stages at +inf.  Prefill replicas use the prefill profile; decode replicas
+ * take the largest batch b <= b_max whose partition exists and meets
+ * 1/Lambda >= Min_TPS (Alg. 2).  The genome is scored with the bottleneck
+ * phase, backlog and waiting time of Eq. 3-5.  Selection, crossover with
+ * repair, mutation and elites (App. A) run on the device, driven by
+ * Philox-4x32-10 streams keyed by (seed, generation, slot, purpose).
+ *
+ * Conventions
+ *  - Every function returns an e2_status.  Nothing aborts, traps or throws.
+ *  - Device work is enqueued on the stream given to e2_create and is
+ *    asynchronous, except where a function says it synchronises.
+ *  - Pointers marked "host or device" may point at host memory (pageable or
+ *    pinned) or at device memory of the current device; the library copies
+ *    with cudaMemcpyDefault.  When an OUTPUT pointer is host memory the call
+ *    synchronises the stream before it returns, so the data is ready.
+ *  - Device memory: the library allocates none.  The caller provides one
+ *    device workspace of e2_workspace_bytes() bytes (for example a byte
+ *    tensor from PyTorch's allocator), 256-byte aligned, that outlives the
+ *    context.
+ *  - Layouts are row-major.  Genome arrays: perm [P][M] u16, sizes [P][K_max]
+ *    u16 (entries >= R are zero), nclus [P] u8, roles [P] u64 (bit c = role of
+ *    replica c, no bits at or above R).
+ *  - Times are seconds, rates FLOP/s or bytes/s, sizes bytes, all float64
+ *    unless stated.  Integer inputs must stay below 2^53 after the library's
+ *    sums (N blocks plus the head); e2_create checks this.
+ */
+#ifndef E2GA_H
+#define E2GA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    E2_OK = 0,
+    E2_EINVAL = 1,    /* invalid argument (null pointer, size, value, genome) */
+    E2_ENOMEM = 2,    /* workspace smaller than e2_workspace_bytes()          */
+    E2_ECUDA = 3,     /* a CUDA runtime call failed                           */
+    E2_ETIMEOUT = 4,  /* a bounded device wait expired                        */
+    E2_EDEVICE = 5,   /* a device-side check failed (see e2_strerror)         */
+    E2_ESTATE = 6     /* call order: e.g. e2_ga_step before any evaluation    */
+} e2_status;
+
+/* Fleet (Sec. 3.1: profiled devices).  M >= 1, M <= E2_MAX_DEVICES. */
+typedef struct {
+    int32_t M;
+    const double *rate;     /* [M] compute rate, FLOP/s, finite > 0   (host)  */
+    const double *bw;       /* [M] memory bandwidth, bytes/s, finite > 0      */
+    const uint64_t *mem;    /* [M] memory available to the model, bytes       */
+} e2_devices;
+
+/* Links (Sec. 3.2: tau(k-1,k) = A / B(k-1,k)).  Row = sender.  The effective
+ * bandwidth is bw[a][b] * cong[a][b]; bw may be +inf (a free link).  The
+ * diagonal is never read. */
+typedef struct {
+    const double *bw;       /* [M][M] base link bandwidth, bytes/s, > 0 (host) */
+    const double *cong;     /* [M][M] congestion factor, finite > 0     (host) */
+    double cong_lo, cong_hi;/* range of e2_redraw_congestion's factors         */
+} e2_links;
+
+/* Layer profile of one model (Sec. 3.1, Alg. 2 inputs l_P, l_D(b)).  N
+ * identical blocks; V = 1 + b_max variants: v = 0 prefill (one request of NP
+ * tokens), v = b decode with b requests in flight.  The stage time of n
+ * blocks on device d is max(flops/rate_d, bytes/bw_d) with
+ * flops = n*blk_flops[v] (+ head_flops[v] on the master), likewise bytes;
+ * it is +inf when n*blk_mem[v] (+ head_mem[v]) exceeds mem_d. */
+typedef struct {
+    int32_t N;                      /* blocks, 1..E2_MAX_BLOCKS               */
+    int32_t b_max;                  /* 1..E2_MAX_BATCH                        */
+    const uint64_t *blk_flops;      /* [V] (host) */
+    const uint64_t *blk_bytes;      /* [V] */
+    const uint64_t *blk_mem;        /* [V] */
+    const uint64_t *head_flops;     /* [V] LM head + output layer (master)    */
+    const uint64_t *head_bytes;     /* [V] */
+    const uint64_t *head_mem;       /* [V] */
+    const uint64_t *act_bytes;      /* [V] activation bytes per link crossing */
+    uint64_t NP;                    /* mean input tokens per request, >= 1    */
+    uint64_t ND;                    /* mean generated tokens per request, >= 1*/
+} e2_layer_profile;
+
+/* Search parameters (Alg. 2 inputs P, G, Q, Min_TPS; App. A mutation mix). */
+typedef struct {
+    int32_t P;              /* population, 1..E2_MAX_POP                        */
+    int32_t Q;              /* elites, 0..P                                     */
+    int32_t K_max;          /* replicas per genome, 1..E2_MAX_CLUSTERS          */
+    int32_t tournament;     /* tournament size, >= 1                            */
+    double min_tps;         /* per-request tokens/s floor, >= 0 (Sec. 3.5)      */
+    double t_a;             /* request inter-arrival time T_a, s, >= 0 (Eq. 4)  */
+    double p_cx;            /* per-position probability of taking parent B      */
+    double p_mut;           /* probability that a child mutates                 */
+    double p_swap;          /* mutation kinds, App. A: swap two positions       */
+    double p_regroup;       /*   regroup from a random replica onward           */
+    double p_regroup_all;   /*   regroup everything; the rest: regenerate both  */
+} e2_params;
+
+/* A population in the layout above; "host or device" pointers. */
+typedef struct {
+    uint16_t *perm;
+    uint16_t *sizes;
+    uint8_t *nclus;
+    uint64_t *roles;
+} e2_genomes;
+
+/* Per-replica results of an evaluation; "host or device" pointers, any may be
+ * NULL (not returned).  Slot-aligned with the genome:
+ *   layers [P][M]  blocks placed on the device at ordering position p, or -1
+ *                  when its replica cannot serve;
+ *   master [P][K_max]  master position inside the replica (0-based) or -1;
+ *   bsel   [P][K_max]  0 prefill, b >= 1 chosen decode batch, -1 no service
+ *                      (or replica index >= R);
+ *   T      [P][K_max]  bottleneck stage time of the chosen variant (+inf if none);
+ *   lambda [P][K_max]  per-request latency Lambda of the chosen variant (+inf). */
+typedef struct {
+    int16_t *layers;
+    int16_t *master;
+    int16_t *bsel;
+    double *T;
+    double *lambda;
+} e2_partitions;
+
+/* Counters of the last e2_eval_population (device-side tallies). */
+typedef struct {
+    uint64_t genomes;           /* genomes evaluated                           */
+    uint64_t replicas;          /* replicas evaluated (sum of R)                */
+    uint64_t dp_runs;           /* DP_Pipe runs that reached the recurrence     */
+    uint64_t dp_cells;          /* DP cells D_mu(i,k) computed                  */
+    uint64_t dp_probes;         /* split-point probes over all cells            */
+    uint64_t paper_candidates;  /* (mu,k,i,j) candidates Alg. 1 would examine   */
+    uint64_t prechecked;        /* variants rejected by the memory count check  */
+    uint64_t served;            /* replicas that can serve                      */
+} e2_stats;
+
+typedef struct e2_ctx e2_ctx;
+
+#define E2_MAX_DEVICES 4096
+#define E2_MAX_BLOCKS 1024
+#define E2_MAX_BATCH 64
+#define E2_MAX_CLUSTERS 64
+#define E2_MAX_POP (1 << 22)
+
+/* Bytes of device workspace a context with these sizes needs.  Returns 0 on
+ * invalid sizes.  Reads only M, N, b_max, P, Q, K_max. */
+size_t e2_workspace_bytes(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_t Q,
+                          int32_t K_max);
+
+/* Validate and copy the inputs (host pointers), lay out the workspace, build
+ * the stage-cost and link-cost tables on the device (Sec. 3.2 cost model) and
+ * return a context bound to `stream` (a cudaStream_t; NULL = legacy default)
+ * and to the current device.  The caller keeps ownership of every input and
+ * of the workspace.  Synchronises the stream.  Errors: E2_EINVAL for any
+ * invalid value, E2_ENOMEM for a short workspace, E2_ECUDA. */
+int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_profile *prof,
+              const e2_params *prm, void *workspace, size_t workspace_bytes, void *stream,
+              e2_ctx **out);
+
+/* Release the context (host memory only; the workspace stays the caller's).
+ * Synchronises the stream.  NULL is accepted. */
+int e2_destroy(e2_ctx *ctx);
+
+/* Copy a population (host or device pointers) into the context's current
+ * population and validate it (each ordering a permutation, 1 <= R <= K_max,
+ * sizes >= 1 summing to M, zero sizes beyond R, no role bits at or above R).
+ * Synchronises.  E2_EINVAL names the first bad genome via e2_last_error. */
+int e2_set_population(e2_ctx *ctx, const e2_genomes *g);
+
+/* Copy the context's current population out (host or device pointers). */
+int e2_get_population(e2_ctx *ctx, const e2_genomes *g);
+
+/* Random initial population (Alg. 2, first step) from Philox streams of
+ * generation 0: Fisher-Yates orderings, a uniform replica count in
+ * 1..min(K_max, M), uniform cut points, random roles. */
+int e2_init_population(e2_ctx *ctx, uint64_t seed);
+
+/* Evaluate a population: DP_Pipe per replica and variant, the decode batch
+ * sweep, and the objective of Eq. 3-5.  `genomes` (host or device) replaces
+ * the current population when not NULL (validated like e2_set_population);
+ * NULL evaluates the current one.  fitness_out [P][4] = {w, phase, PS, DS}
+ * (host or device, may be NULL); `parts` may be NULL.  The results also stay
+ * in the context for e2_ga_step. */
+int e2_eval_population(e2_ctx *ctx, const e2_genomes *genomes, double *fitness_out,
+                       const e2_partitions *parts);
+
+/* One generation (Alg. 2 population update, App. A): elites = the Q best
+ * distinct genomes of the evaluated population by (w, phase, index); slots
+ * [0, Q) of the next population take them in that order, slots [Q, P) take
+ * children (tournament selection, uniform crossover with repair, grouping and
+ * roles from one parent, mutation), all drawn from the streams of
+ * (seed, generation).  The next population becomes current.  E2_ESTATE if the
+ * current population has not been evaluated. */
+int e2_ga_step(e2_ctx *ctx, uint64_t seed, uint32_t generation);
+
+/* Redraw every link's congestion factor uniformly in [cong_lo, cong_hi) from
+ * the stream of (seed, generation) and rebuild the link-cost tables.  The
+ * population's results are stale afterwards (E2_ESTATE for e2_ga_step until
+ * the next evaluation). */
+int e2_redraw_congestion(e2_ctx *ctx, uint64_t seed, uint32_t generation);
+
+/* Copy the current congestion matrix [M][M] out (host or device pointer). */
+int e2_get_congestion(e2_ctx *ctx, double *cong_out);
+
+/* Elite indices [Q] (into the population that was evaluated before the last
+ * e2_ga_step) and their fitness [Q][4]; either may be NULL. */
+int e2_get_elites(e2_ctx *ctx, int32_t *idx_out, double *fitness_out);
+
+/* Counters of the last evaluation.  Synchronises. */
+int e2_get_stats(e2_ctx *ctx, e2_stats *out);
+
+/* Text of a status code, and the context's last detailed error message.  With
+ * ctx == NULL: the message of the calling thread's last failed e2_create ("" if
+ * none). */
+const char *e2_strerror(int status);
+const char *e2_last_error(const e2_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* E2GA_H */

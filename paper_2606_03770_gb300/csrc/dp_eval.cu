@@ -1,0 +1,385 @@
+// dp_eval.cu -- population fitness: DP_Pipe per replica (Alg. 1, Eq. 1-2),
+// the decode batch sweep (Alg. 2), and the objective (Eq. 3-5).
+//
+// One CTA evaluates one (genome, replica slot).  With identical blocks
+// (Sec. 3.2: the premise that lets the paper fix the node order) a stage's time
+// depends only on its device, its block count n and whether it is the master,
+// so the replica's costs fit in two rows per device, l_k(n) and l_k^head(n),
+// staged in shared memory as 64-bit keys (non-negative doubles order like their
+// bit patterns).
+//
+// Band form of Eq. 1.  Device k can take at most W = N - m + 1 blocks.  Let
+// D_k[r] = DP(i = r + k - 1, k), r in [0, W).  Then
+//     D_1[r] = l_1(r + 1)                                         (Eq. 2)
+//     D_k[r] = min_{s in [0, r]} max(D_{k-1}[s], l_k(r - s + 1), tau_k)   (Eq. 1)
+// where s = j - (k - 1) indexes the split.  D_{k-1}[s] is non-decreasing in s
+// (one more block never lowers the best bottleneck when blocks are identical)
+// and l_k(r - s + 1) is non-increasing in s, so max(D_{k-1}[s], l_k(.)) falls
+// then rises: its minimum sits at the crossover s0 = first s with
+// D_{k-1}[s] >= l_k(r - s + 1) and equals min(l_k(r - s0 + 2), D_{k-1}[s0]).
+// A bisection over s finds s0, so a cell costs O(log W) probes instead of the
+// O(W) scan, with bit-identical values (min and max are exact).
+//
+// Tie rule.  The oracle keeps the smallest split j attaining the minimum.  The
+// set of minimisers is {s : D_{k-1}[s] <= D and l_k(r-s+1) <= D} (tau <= D
+// always), an interval whose first element is the first s with
+// l_k(r-s+1) <= D.  So the traceback needs only the cell value D and the cost
+// row: n_k = largest n <= r + 1 with l_k(n) <= D.
+//
+// Masters.  Columns k < mu do not involve the master and are shared by every
+// mu (computed once by the CTA).  Warps take masters mu = w+1, w+1+NW, ... and
+// run columns mu..m in private ping-pong buffers; the last column needs only
+// its final cell.  mu* = the smallest mu with the least bottleneck (the
+// oracle's first-wins argmin).  The CTA then recomputes mu*'s columns into the
+// shared column store for the traceback.
+#include "e2ga_internal.cuh"
+
+namespace e2 {
+
+namespace {
+
+// D_k[r] for one cell (see the header comment).
+__device__ __forceinline__ uint64_t dp_cell(const uint64_t *__restrict__ prev,
+                                            const uint64_t *__restrict__ row, uint64_t tau, int r)
+{
+    int lo = 0, hi = r + 1;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (prev[mid] >= row[r - mid]) hi = mid;
+        else lo = mid + 1;
+    }
+    uint64_t h = kInfKey;
+    if (lo <= r) h = prev[lo];
+    if (lo >= 1) h = umin64(h, row[r - lo + 1]);
+    return umax64(h, tau);
+}
+
+// Number of finite entries of a non-decreasing row (memory grows with n, so
+// the +inf entries form a suffix).
+__device__ __forceinline__ int finite_prefix(const uint64_t *row, int W)
+{
+    int lo = 0, hi = W;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (row[mid] < kInfKey) lo = mid + 1;
+        else hi = mid;
+    }
+    return lo;
+}
+
+__device__ __forceinline__ int warp_sum(int x)
+{
+#pragma unroll
+    for (int o = 16; o; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
+    return x;
+}
+
+// Candidates (mu, k, i, j) the plain recurrence examines for one DP run:
+// m * (N + sum_{k=2..m} (N-k+1)(N-k+2)/2).
+__device__ __forceinline__ unsigned long long paper_candidates(int m, int N)
+{
+    const unsigned long long a = (unsigned long long)(N - m + 1), b = (unsigned long long)(N - 1);
+    unsigned long long s = 0;
+    if (m >= 2) s = (b * (b + 1) * (b + 2) - (a - 1) * a * (a + 1)) / 6;
+    return (unsigned long long)m * ((unsigned long long)N + s);
+}
+
+// Bisection probes of one full column of W cells: sum_{n=1..W} (floor(log2 n) + 1).
+__device__ __forceinline__ unsigned long long column_probes(int W)
+{
+    const int L = 31 - __clz(W);
+    return (unsigned long long)W + (unsigned long long)(W + 1) * L - (2ull << L) + 2ull;
+}
+
+}  // namespace
+
+// Shared-memory bytes for the largest replica the problem allows.
+size_t dp_smem_bytes(int M, int N, int threads)
+{
+    const int NW = threads / 32;
+    size_t best = 0;
+    const int mmax = M < N ? M : N;
+    for (int m = 1; m <= mmax; ++m) {
+        const size_t W = (size_t)(N - m + 1);
+        size_t u64s = 3 * (size_t)m * W + 2 * (size_t)NW * W + (size_t)m;
+        size_t bytes = u64s * 8 + (size_t)m * (3 * sizeof(int)) + (size_t)m * sizeof(uint16_t) + 16;
+        if (bytes > best) best = bytes;
+    }
+    return (best + 15) & ~(size_t)15;
+}
+
+__global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    __shared__ int s_off, s_m, s_role, s_S0, s_Z, s_any, s_mu, s_done;
+    __shared__ uint64_t s_V;
+    __shared__ double s_L;
+    __shared__ uint64_t s_wV[4];
+    __shared__ int s_wMu[4];
+
+    const int K = dm.K, M = dm.M, N = dm.N;
+    const int g = blockIdx.x / K, c = blockIdx.x - g * K;
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
+    const size_t gk = (size_t)g * K + c;
+    const int R = pop.nclus[g];
+    if (c >= R) {
+        if (tid == 0) {
+            out.master[gk] = -1; out.bsel[gk] = -1;
+            out.T[gk] = keyd(kInfKey); out.L[gk] = keyd(kInfKey);
+        }
+        return;
+    }
+    if (tid == 0) {
+        int off = 0;
+        for (int q = 0; q < c; ++q) off += pop.sizes[(size_t)g * K + q];
+        s_off = off;
+        s_m = pop.sizes[gk];
+        s_role = (int)((pop.roles[g] >> c) & 1ull);
+    }
+    __syncthreads();
+    const int off = s_off, m = s_m, role = s_role;
+    int16_t *lay_out = out.layers + (size_t)g * M + off;
+
+    unsigned long long st_runs = 0, st_cells = 0, st_probes = 0, st_paper = 0, st_pre = 0;
+    bool served = false;
+
+    if (m <= N) {
+        const int W = N - m + 1;
+        uint64_t *leaf0 = reinterpret_cast<uint64_t *>(smem);   // [m][W] l_k(n)
+        uint64_t *leaf1 = leaf0 + (size_t)m * W;                // [m][W] l_k^head(n)
+        uint64_t *Fst = leaf1 + (size_t)m * W;                  // [m][W] column store
+        uint64_t *pp = Fst + (size_t)m * W;                     // [NW][2][W]
+        uint64_t *tauk = pp + (size_t)NW * 2 * W;               // [m]
+        int *cnt0 = reinterpret_cast<int *>(tauk + m);          // [m]
+        int *cnt1 = cnt0 + m;                                   // [m]
+        int *nk = cnt1 + m;                                     // [m]
+        uint16_t *devs = reinterpret_cast<uint16_t *>(nk + m);  // [m]
+
+        for (int k = tid; k < m; k += blockDim.x) devs[k] = pop.perm[(size_t)g * M + off + k];
+        __syncthreads();
+
+        const int nvar = role ? dm.b_max : 1;
+        const unsigned long long pc = paper_candidates(m, N);
+        const unsigned long long cprobe = column_probes(W);
+        for (int vi = 0; vi < nvar && !served; ++vi) {
+            const int v = role ? dm.b_max - vi : 0;
+            // ---- stage the cost rows and link times of this variant
+            for (int e = tid; e < m * W; e += blockDim.x) {
+                const int k = e / W, n = e - k * W;
+                const double *base = tb.leaf + ((size_t)v * M + devs[k]) * 2 * dm.LS;
+                leaf0[e] = dkey(base[n]);
+                leaf1[e] = dkey(base[dm.LS + n]);
+            }
+            for (int k = tid; k < m; k += blockDim.x)
+                tauk[k] = k ? dkey(tb.tau[((size_t)v * M + devs[k - 1]) * M + devs[k]]) : 0ull;
+            __syncthreads();
+            // ---- exact memory check: with identical blocks a partition with
+            // master mu exists iff every device holds >= 1 block and the block
+            // capacities (capped at W) add up to N
+            for (int k = tid; k < m; k += blockDim.x) {
+                cnt0[k] = finite_prefix(leaf0 + (size_t)k * W, W);
+                cnt1[k] = finite_prefix(leaf1 + (size_t)k * W, W);
+            }
+            __syncthreads();
+            if (wid == 0) {
+                int s = 0, z = 0;
+                for (int k = lane; k < m; k += 32) { s += cnt0[k]; z += cnt0[k] == 0; }
+                s = warp_sum(s); z = warp_sum(z);
+                if (lane == 0) { s_S0 = s; s_Z = z; }
+            }
+            __syncthreads();
+            const int S0 = s_S0, Z = s_Z;
+            auto mu_ok = [&](int mu) {
+                const int k = mu - 1;
+                return (Z - (cnt0[k] == 0)) == 0 && cnt1[k] >= 1 && S0 - cnt0[k] + cnt1[k] >= N;
+            };
+            int any = 0;
+            for (int mu = tid + 1; mu <= m; mu += blockDim.x) any |= mu_ok(mu);
+            any = __syncthreads_or(any);
+            st_paper += pc;
+            if (!any) { ++st_pre; continue; }
+            ++st_runs;
+            auto colF = [&](int k) -> const uint64_t * { return k == 1 ? leaf0 : Fst + (size_t)(k - 1) * W; };
+            // ---- shared columns 2..m-1 without the master
+            for (int k = 2; k <= m - 1; ++k) {
+                const uint64_t *prev = colF(k - 1), *row = leaf0 + (size_t)(k - 1) * W;
+                const uint64_t t = tauk[k - 1];
+                uint64_t *cur = Fst + (size_t)(k - 1) * W;
+                for (int r = tid; r < W; r += blockDim.x) cur[r] = dp_cell(prev, row, t, r);
+                __syncthreads();
+            }
+            if (tid == 0 && m >= 3) { st_cells += (unsigned long long)(m - 2) * W; st_probes += (m - 2) * cprobe; }
+            // ---- one master per warp at a time
+            uint64_t bestV = kInfKey;
+            int bestMu = 0x7FFFFFFF;
+            unsigned long long w_cells = 0, w_probes = 0;
+            for (int mu = wid + 1; mu <= m; mu += NW) {
+                if (!mu_ok(mu)) continue;
+                uint64_t V;
+                if (m == 1) {
+                    V = leaf1[W - 1];
+                } else {
+                    uint64_t *buf0 = pp + (size_t)wid * 2 * W, *buf1 = buf0 + W;
+                    const uint64_t *prev = mu == 1 ? leaf1 : colF(mu - 1);
+                    int which = 0;
+                    V = kInfKey;
+                    for (int k = (mu == 1 ? 2 : mu); k <= m; ++k) {
+                        const uint64_t *row = (k == mu ? leaf1 : leaf0) + (size_t)(k - 1) * W;
+                        const uint64_t t = tauk[k - 1];
+                        if (k == m) { V = dp_cell(prev, row, t, W - 1); w_cells += 1; w_probes += 32 - __clz(W); break; }
+                        uint64_t *cur = which ? buf1 : buf0;
+                        which ^= 1;
+                        for (int r = lane; r < W; r += 32) cur[r] = dp_cell(prev, row, t, r);
+                        __syncwarp();
+                        prev = cur;
+                        w_cells += W; w_probes += cprobe;
+                    }
+                }
+                if (V < bestV) { bestV = V; bestMu = mu; }
+            }
+            if (lane == 0) { s_wV[wid] = bestV; s_wMu[wid] = bestMu; }
+            __syncthreads();
+            if (tid == 0) {
+                uint64_t V = kInfKey;
+                int mu = 0x7FFFFFFF;
+                for (int w = 0; w < NW; ++w)
+                    if (s_wV[w] < V || (s_wV[w] == V && s_wMu[w] < mu)) { V = s_wV[w]; mu = s_wMu[w]; }
+                s_V = V; s_mu = mu;
+            }
+            if (lane == 0) { st_cells += w_cells; st_probes += w_probes; }
+            __syncthreads();
+            const uint64_t V = s_V;
+            const int mus = s_mu;
+            if (V >= kInfKey) continue;      // cannot happen after the exact memory check
+            // ---- mu*'s own columns, for the traceback
+            auto rowk = [&](int k) -> const uint64_t * { return (k == mus ? leaf1 : leaf0) + (size_t)(k - 1) * W; };
+            auto colD = [&](int k) -> const uint64_t * {
+                if (k == 1) return mus == 1 ? leaf1 : leaf0;
+                return Fst + (size_t)(k - 1) * W;
+            };
+            for (int k = (mus > 2 ? mus : 2); k <= m - 1; ++k) {
+                const uint64_t *prev = colD(k - 1), *row = rowk(k);
+                const uint64_t t = tauk[k - 1];
+                uint64_t *cur = Fst + (size_t)(k - 1) * W;
+                for (int r = tid; r < W; r += blockDim.x) cur[r] = dp_cell(prev, row, t, r);
+                __syncthreads();
+                if (tid == 0) { st_cells += W; st_probes += cprobe; }
+            }
+            // ---- traceback (smallest split on ties) and Lambda in pipeline order
+            if (tid == 0) {
+                int r = W - 1;
+                uint64_t D = V;
+                for (int k = m; k >= 2; --k) {
+                    const uint64_t *row = rowk(k);
+                    int lo = 1, hi = r + 1;                    // largest n <= r+1 with l_k(n) <= D
+                    while (lo < hi) {
+                        const int mid = (lo + hi + 1) >> 1;
+                        if (row[mid - 1] <= D) lo = mid;
+                        else hi = mid - 1;
+                    }
+                    nk[k - 1] = lo;
+                    r = r + 1 - lo;
+                    D = colD(k - 1)[r];
+                }
+                nk[0] = r + 1;
+                double lam = keyd(rowk(1)[nk[0] - 1]);
+                for (int k = 2; k <= m; ++k) {
+                    lam = lam + keyd(tauk[k - 1]);
+                    lam = lam + keyd(rowk(k)[nk[k - 1] - 1]);
+                }
+                s_L = lam;
+                s_done = (!role) || (1.0 / lam >= dm.min_tps);
+            }
+            __syncthreads();
+            if (s_done) {
+                for (int k = tid; k < m; k += blockDim.x) lay_out[k] = (int16_t)nk[k];
+                if (tid == 0) {
+                    out.master[gk] = (int16_t)(mus - 1);
+                    out.bsel[gk] = (int16_t)v;
+                    out.T[gk] = keyd(V);
+                    out.L[gk] = s_L;
+                }
+                served = true;
+            }
+            __syncthreads();
+        }
+    }
+    if (!served) {
+        for (int k = tid; k < m; k += blockDim.x) lay_out[k] = -1;
+        if (tid == 0) {
+            out.master[gk] = -1; out.bsel[gk] = -1;
+            out.T[gk] = keyd(kInfKey); out.L[gk] = keyd(kInfKey);
+        }
+    }
+    // per-CTA tallies
+    if (lane == 0 && (st_cells | st_probes)) {
+        atomicAdd(&out.stats[kStCells], st_cells);
+        atomicAdd(&out.stats[kStProbes], st_probes);
+    }
+    if (tid == 0) {
+        atomicAdd(&out.stats[kStReplicas], 1ull);
+        if (st_runs) atomicAdd(&out.stats[kStDpRuns], st_runs);
+        if (st_paper) atomicAdd(&out.stats[kStPaper], st_paper);
+        if (st_pre) atomicAdd(&out.stats[kStPrecheck], st_pre);
+        if (served) atomicAdd(&out.stats[kStServed], 1ull);
+    }
+}
+
+// Objective, one thread per genome (Sec. 3.3).  PS and DS are summed over the
+// serving replicas of each role in ascending replica order, then Eq. 3
+// (bottleneck phase), Eq. 4 (backlog) and Eq. 5 (waiting time).  Also a
+// 64-bit fingerprint of the genome for the elites' duplicate test.
+__global__ void __launch_bounds__(256) score_kernel(Dims dm, DevPop pop, EvalOut out)
+{
+    const int g = blockIdx.x * blockDim.x + threadIdx.x;
+    if (g >= dm.P) return;
+    const int K = dm.K, M = dm.M;
+    const int R = pop.nclus[g];
+    const uint64_t roles = pop.roles[g];
+    double PS = 0.0, DS = 0.0;
+    for (int c = 0; c < R; ++c) {
+        const int b = out.bsel[(size_t)g * K + c];
+        if (b < 0) continue;
+        const double T = out.T[(size_t)g * K + c];
+        if (((roles >> c) & 1ull) == 0) PS = PS + (double)dm.NP / T;
+        else DS = DS + (double)b / T;
+    }
+    double w = keyd(kInfKey), phase = keyd(kInfKey);
+    if (PS != 0.0 && DS != 0.0) {
+        const double tp = (double)dm.NP / PS, td = (double)dm.ND / DS;
+        phase = tp >= td ? tp : td;                 // Eq. 3
+        const double x = phase - dm.t_a;
+        const double bn = x > 0.0 ? x : 0.0;        // Eq. 4
+        w = bn > 0.0 ? tp + bn : 0.0;               // Eq. 5
+    }
+    double *f = out.fit + (size_t)g * 4;
+    f[0] = w; f[1] = phase; f[2] = PS; f[3] = DS;
+    // fingerprint: ordering, grouping, replica count, roles
+    uint64_t h = 0x9E3779B97F4A7C15ull;
+    auto mix = [&](uint64_t x) { h = (h ^ x) * 0xBF58476D1CE4E5B9ull; h ^= h >> 31; };
+    const uint16_t *pp = pop.perm + (size_t)g * M;
+    for (int i = 0; i < M; ++i) mix(pp[i]);
+    const uint16_t *ss = pop.sizes + (size_t)g * K;
+    for (int i = 0; i < R; ++i) mix((uint64_t)ss[i] << 16);
+    mix((uint64_t)R << 40);
+    mix(roles);
+    out.hash[g] = h;
+    atomicAdd(&out.stats[kStGenomes], 1ull);
+}
+
+cudaError_t configure_eval(size_t smem)
+{
+    return cudaFuncSetAttribute(dp_eval_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+}
+
+cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
+{
+    Tables tb{c->rate, c->bw, c->mem, c->prof, c->leaf, c->tau};
+    EvalOut out{c->fit, c->layers, c->master, c->bsel, c->T, c->L, c->hash, c->stats};
+    const long long blocks = (long long)c->dm.P * c->dm.K;
+    dp_eval_kernel<<<(unsigned)blocks, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out);
+    score_kernel<<<(c->dm.P + 255) / 256, 256, 0, c->stream>>>(c->dm, p, out);
+    return cudaGetLastError();
+}
+
+}  // namespace e2

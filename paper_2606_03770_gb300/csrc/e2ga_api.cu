@@ -1,0 +1,457 @@
+// e2ga_api.cu -- the C ABI (include/e2ga.h): input validation, workspace
+// layout, table construction and the call sequence of a search.
+#include <math.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <new>
+
+#include "e2ga_internal.cuh"
+
+using namespace e2;
+
+namespace {
+
+constexpr uint64_t kTwo53 = 1ull << 53;
+
+// Message of the last failed e2_create on this thread (no context exists then).
+thread_local char g_create_error[256] = "";
+
+size_t align_up(size_t x, size_t a = 256) { return (x + a - 1) / a * a; }
+
+struct Layout {
+    size_t rate, bw, mem, link_bw, cong, prof, leaf, tau;
+    size_t perm[2], sizes[2], nclus[2], roles[2];
+    size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, stats, err, total;
+    int LS;
+};
+
+bool dims_ok(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_t Q, int32_t K)
+{
+    return M >= 1 && M <= E2_MAX_DEVICES && N >= 1 && N <= E2_MAX_BLOCKS && b_max >= 1 &&
+           b_max <= E2_MAX_BATCH && P >= 1 && P <= E2_MAX_POP && Q >= 0 && Q <= P && K >= 1 &&
+           K <= E2_MAX_CLUSTERS;
+}
+
+Layout layout(int M, int N, int b_max, int P, int Q, int K)
+{
+    Layout l{};
+    const size_t V = (size_t)b_max + 1, MM = (size_t)M * M;
+    l.LS = (N + 1) & ~1;
+    size_t o = 0;
+    auto take = [&](size_t bytes) { size_t at = o; o = align_up(o + bytes); return at; };
+    l.rate = take(8 * (size_t)M);
+    l.bw = take(8 * (size_t)M);
+    l.mem = take(8 * (size_t)M);
+    l.link_bw = take(8 * MM);
+    l.cong = take(8 * MM);
+    l.prof = take(8 * kNumProf * V);
+    l.leaf = take(8 * V * M * 2 * (size_t)l.LS);
+    l.tau = take(8 * V * MM);
+    for (int b = 0; b < 2; ++b) {
+        l.perm[b] = take(2 * (size_t)P * M);
+        l.sizes[b] = take(2 * (size_t)P * K);
+        l.nclus[b] = take((size_t)P);
+        l.roles[b] = take(8 * (size_t)P);
+    }
+    l.fit = take(32 * (size_t)P);
+    l.layers = take(2 * (size_t)P * M);
+    l.master = take(2 * (size_t)P * K);
+    l.bsel = take(2 * (size_t)P * K);
+    l.T = take(8 * (size_t)P * K);
+    l.L = take(8 * (size_t)P * K);
+    l.hash = take(8 * (size_t)P);
+    l.dup = take(4 * (size_t)P);
+    l.elite = take(4 * (size_t)(Q > 0 ? Q : 1));
+    l.elite_fit = take(32 * (size_t)(Q > 0 ? Q : 1));
+    l.stats = take(8 * kNumStats);
+    l.err = take(4);
+    l.total = o;
+    return l;
+}
+
+uint64_t threshold(double p)
+{
+    if (!(p > 0.0)) return 0;
+    if (p >= 1.0) return 4294967296ull;
+    return (uint64_t)floor(p * 4294967296.0);
+}
+
+int fail(e2_ctx *c, int status, const char *msg)
+{
+    if (c) c->last_error = msg;
+    return status;
+}
+
+int cuda_fail(e2_ctx *c, cudaError_t e, const char *where)
+{
+    char buf[256];
+    snprintf(buf, sizeof buf, "%s: %s", where, cudaGetErrorString(e));
+    if (c) c->last_error = buf;
+    return E2_ECUDA;
+}
+
+#define E2_CUDA(ctx, call)                                   \
+    do {                                                     \
+        cudaError_t e2_err_ = (call);                        \
+        if (e2_err_ != cudaSuccess) return cuda_fail((ctx), e2_err_, #call); \
+    } while (0)
+
+bool is_host(const void *p)
+{
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        cudaGetLastError();
+        return true;
+    }
+    return a.type == cudaMemoryTypeHost || a.type == cudaMemoryTypeUnregistered;
+}
+
+bool finite_pos(double x) { return isfinite(x) && x > 0.0; }
+
+// Host-side validation of everything e2_create receives (no CUDA call).
+int validate_inputs(const e2_devices *d, const e2_links *l, const e2_layer_profile *pf, const e2_params *p,
+                    char *msg, size_t n)
+{
+    if (!d || !l || !pf || !p) { snprintf(msg, n, "null descriptor"); return E2_EINVAL; }
+    if (!dims_ok(d->M, pf->N, pf->b_max, p->P, p->Q, p->K_max)) {
+        snprintf(msg, n, "sizes out of range (M=%d N=%d b_max=%d P=%d Q=%d K_max=%d)", d->M, pf->N,
+                 pf->b_max, p->P, p->Q, p->K_max);
+        return E2_EINVAL;
+    }
+    const int M = d->M, V = pf->b_max + 1;
+    if (!d->rate || !d->bw || !d->mem || !l->bw || !l->cong) { snprintf(msg, n, "null array"); return E2_EINVAL; }
+    const uint64_t *arr[kNumProf] = {pf->blk_flops, pf->blk_bytes, pf->blk_mem, pf->head_flops,
+                                     pf->head_bytes, pf->head_mem, pf->act_bytes};
+    for (int a = 0; a < kNumProf; ++a)
+        if (!arr[a]) { snprintf(msg, n, "null profile array %d", a); return E2_EINVAL; }
+    for (int i = 0; i < M; ++i) {
+        if (!finite_pos(d->rate[i]) || !finite_pos(d->bw[i])) {
+            snprintf(msg, n, "device %d: rate and bandwidth must be finite and > 0", i);
+            return E2_EINVAL;
+        }
+    }
+    for (int a = 0; a < M; ++a)
+        for (int b = 0; b < M; ++b) {
+            if (a == b) continue;
+            const double bw = l->bw[(size_t)a * M + b], cg = l->cong[(size_t)a * M + b];
+            if (!(bw > 0.0) || !finite_pos(cg)) {
+                snprintf(msg, n, "link %d->%d: bandwidth must be > 0, congestion finite and > 0", a, b);
+                return E2_EINVAL;
+            }
+        }
+    if (!finite_pos(l->cong_lo) || !finite_pos(l->cong_hi) || l->cong_lo > l->cong_hi) {
+        snprintf(msg, n, "congestion range must satisfy 0 < lo <= hi < inf");
+        return E2_EINVAL;
+    }
+    for (int v = 0; v < V; ++v) {
+        for (int a = 0; a < 3; ++a) {   // n * block + head must stay below 2^53
+            const uint64_t blk = arr[a][v], head = arr[a + 3][v];
+            if (head >= kTwo53 || blk > (kTwo53 - head) / (uint64_t)pf->N) {
+                snprintf(msg, n, "profile variant %d: N*block + head reaches 2^53", v);
+                return E2_EINVAL;
+            }
+        }
+        if (pf->act_bytes[v] >= kTwo53) { snprintf(msg, n, "activation bytes reach 2^53"); return E2_EINVAL; }
+    }
+    if (pf->NP < 1 || pf->ND < 1 || pf->NP >= kTwo53 || pf->ND >= kTwo53) {
+        snprintf(msg, n, "NP and ND must be in [1, 2^53)");
+        return E2_EINVAL;
+    }
+    if (!(isfinite(p->min_tps) && p->min_tps >= 0) || !(isfinite(p->t_a) && p->t_a >= 0)) {
+        snprintf(msg, n, "min_tps and t_a must be finite and >= 0");
+        return E2_EINVAL;
+    }
+    const double probs[5] = {p->p_cx, p->p_mut, p->p_swap, p->p_regroup, p->p_regroup_all};
+    for (double q : probs)
+        if (!(q >= 0.0 && q <= 1.0)) { snprintf(msg, n, "probabilities must lie in [0, 1]"); return E2_EINVAL; }
+    if (p->tournament < 1) { snprintf(msg, n, "tournament size must be >= 1"); return E2_EINVAL; }
+    return E2_OK;
+}
+
+DevPop pop_at(unsigned char *ws, const Layout &l, int b)
+{
+    return DevPop{reinterpret_cast<uint16_t *>(ws + l.perm[b]), reinterpret_cast<uint16_t *>(ws + l.sizes[b]),
+                  ws + l.nclus[b], reinterpret_cast<uint64_t *>(ws + l.roles[b])};
+}
+
+int copy_pop(e2_ctx *c, const DevPop &dst, const e2_genomes *g, bool out)
+{
+    const size_t P = c->dm.P, M = c->dm.M, K = c->dm.K;
+    if (!g || !g->perm || !g->sizes || !g->nclus || !g->roles) return fail(c, E2_EINVAL, "null genome array");
+    const cudaMemcpyKind k = cudaMemcpyDefault;
+    if (!out) {
+        E2_CUDA(c, cudaMemcpyAsync(dst.perm, g->perm, 2 * P * M, k, c->stream));
+        E2_CUDA(c, cudaMemcpyAsync(dst.sizes, g->sizes, 2 * P * K, k, c->stream));
+        E2_CUDA(c, cudaMemcpyAsync(dst.nclus, g->nclus, P, k, c->stream));
+        E2_CUDA(c, cudaMemcpyAsync(dst.roles, g->roles, 8 * P, k, c->stream));
+    } else {
+        E2_CUDA(c, cudaMemcpyAsync(g->perm, dst.perm, 2 * P * M, k, c->stream));
+        E2_CUDA(c, cudaMemcpyAsync(g->sizes, dst.sizes, 2 * P * K, k, c->stream));
+        E2_CUDA(c, cudaMemcpyAsync(g->nclus, dst.nclus, P, k, c->stream));
+        E2_CUDA(c, cudaMemcpyAsync(g->roles, dst.roles, 8 * P, k, c->stream));
+        if (is_host(g->perm) || is_host(g->sizes) || is_host(g->nclus) || is_host(g->roles))
+            E2_CUDA(c, cudaStreamSynchronize(c->stream));
+    }
+    return E2_OK;
+}
+
+int set_and_validate(e2_ctx *c, const e2_genomes *g)
+{
+    int st = copy_pop(c, c->pop[c->cur], g, false);
+    if (st) return st;
+    const int32_t big = 0x7FFFFFFF;
+    E2_CUDA(c, cudaMemcpyAsync(c->err, &big, 4, cudaMemcpyHostToDevice, c->stream));
+    E2_CUDA(c, launch_validate(c, c->pop[c->cur]));
+    int32_t bad = big;
+    E2_CUDA(c, cudaMemcpyAsync(&bad, c->err, 4, cudaMemcpyDeviceToHost, c->stream));
+    E2_CUDA(c, cudaStreamSynchronize(c->stream));
+    c->evaluated = false;
+    if (bad != big) {
+        char buf[128];
+        snprintf(buf, sizeof buf, "genome %d is not a valid gene (ordering, grouping or roles)", bad);
+        return fail(c, E2_EINVAL, buf);
+    }
+    return E2_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t e2_workspace_bytes(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_t Q, int32_t K_max)
+{
+    if (!dims_ok(M, N, b_max, P, Q, K_max)) return 0;
+    return layout(M, N, b_max, P, Q, K_max).total;
+}
+
+int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_profile *prof,
+              const e2_params *prm, void *workspace, size_t workspace_bytes, void *stream, e2_ctx **out)
+{
+    g_create_error[0] = 0;
+    auto reject = [&](int code, const char *why) {
+        snprintf(g_create_error, sizeof g_create_error, "%s", why);
+        return code;
+    };
+    if (!out) return reject(E2_EINVAL, "null output pointer");
+    *out = nullptr;
+    char msg[256];
+    int st = validate_inputs(devs, links, prof, prm, msg, sizeof msg);
+    if (st) return reject(st, msg);
+    const int M = devs->M, N = prof->N, b_max = prof->b_max, P = prm->P, Q = prm->Q, K = prm->K_max;
+    const Layout l = layout(M, N, b_max, P, Q, K);
+    if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255))
+        return reject(E2_EINVAL, "workspace must be non-null and 256-byte aligned");
+    if (workspace_bytes < l.total) return reject(E2_ENOMEM, "workspace smaller than e2_workspace_bytes()");
+
+    e2_ctx *c = new (std::nothrow) e2_ctx();
+    if (!c) return E2_ENOMEM;
+    c->stream = static_cast<cudaStream_t>(stream);
+    c->dm = Dims{M, N, b_max + 1, b_max, P, Q, K, l.LS, prm->tournament, prof->NP, prof->ND,
+                 prm->min_tps, prm->t_a};
+    c->cong_lo = links->cong_lo;
+    c->cong_hi = links->cong_hi;
+    c->thr_cx = threshold(prm->p_cx);
+    c->thr_half = threshold(0.5);
+    c->thr_mut = threshold(prm->p_mut);
+    const double s1 = prm->p_swap, s2 = s1 + prm->p_regroup, s3 = s2 + prm->p_regroup_all;
+    c->thr_k1 = threshold(s1);
+    c->thr_k2 = threshold(s2);
+    c->thr_k3 = threshold(s3);
+
+    auto fail_free = [&](int code, const char *why) { delete c; return reject(code, why); };
+    if (cudaGetDevice(&c->device) != cudaSuccess) return fail_free(E2_ECUDA, "no CUDA device");
+    int smem_optin = 0;
+    if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, c->device) != cudaSuccess)
+        return fail_free(E2_ECUDA, "cudaDeviceGetAttribute failed");
+    c->dp_threads = 128;
+    c->dp_smem = dp_smem_bytes(M, N, c->dp_threads);
+    if (c->dp_smem + 1024 > (size_t)smem_optin)
+        return fail_free(E2_EINVAL, "the largest replica's DP does not fit in shared memory (N too large)");
+    if (configure_eval(c->dp_smem) != cudaSuccess) return fail_free(E2_ECUDA, "cudaFuncSetAttribute failed");
+
+    unsigned char *ws = static_cast<unsigned char *>(workspace);
+    c->rate = reinterpret_cast<double *>(ws + l.rate);
+    c->bw = reinterpret_cast<double *>(ws + l.bw);
+    c->mem = reinterpret_cast<uint64_t *>(ws + l.mem);
+    c->link_bw = reinterpret_cast<double *>(ws + l.link_bw);
+    c->cong = reinterpret_cast<double *>(ws + l.cong);
+    c->prof = reinterpret_cast<uint64_t *>(ws + l.prof);
+    c->leaf = reinterpret_cast<double *>(ws + l.leaf);
+    c->tau = reinterpret_cast<double *>(ws + l.tau);
+    for (int b = 0; b < 2; ++b) c->pop[b] = pop_at(ws, l, b);
+    c->fit = reinterpret_cast<double *>(ws + l.fit);
+    c->layers = reinterpret_cast<int16_t *>(ws + l.layers);
+    c->master = reinterpret_cast<int16_t *>(ws + l.master);
+    c->bsel = reinterpret_cast<int16_t *>(ws + l.bsel);
+    c->T = reinterpret_cast<double *>(ws + l.T);
+    c->L = reinterpret_cast<double *>(ws + l.L);
+    c->hash = reinterpret_cast<uint64_t *>(ws + l.hash);
+    c->dup = reinterpret_cast<int32_t *>(ws + l.dup);
+    c->elite = reinterpret_cast<int32_t *>(ws + l.elite);
+    c->elite_fit = reinterpret_cast<double *>(ws + l.elite_fit);
+    c->stats = reinterpret_cast<unsigned long long *>(ws + l.stats);
+    c->err = reinterpret_cast<int32_t *>(ws + l.err);
+
+    const size_t V = (size_t)b_max + 1, MM = (size_t)M * M;
+    uint64_t *prof_h = new (std::nothrow) uint64_t[kNumProf * V];
+    if (!prof_h) return fail_free(E2_ENOMEM, "host allocation failed");
+    const uint64_t *arr[kNumProf] = {prof->blk_flops, prof->blk_bytes, prof->blk_mem, prof->head_flops,
+                                     prof->head_bytes, prof->head_mem, prof->act_bytes};
+    for (int a = 0; a < kNumProf; ++a) memcpy(prof_h + a * V, arr[a], 8 * V);
+    cudaError_t e = cudaSuccess;
+    auto chk = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
+    chk(cudaMemsetAsync(ws, 0, l.total, c->stream));
+    chk(cudaMemcpyAsync(c->rate, devs->rate, 8 * (size_t)M, cudaMemcpyHostToDevice, c->stream));
+    chk(cudaMemcpyAsync(c->bw, devs->bw, 8 * (size_t)M, cudaMemcpyHostToDevice, c->stream));
+    chk(cudaMemcpyAsync(c->mem, devs->mem, 8 * (size_t)M, cudaMemcpyHostToDevice, c->stream));
+    chk(cudaMemcpyAsync(c->link_bw, links->bw, 8 * MM, cudaMemcpyHostToDevice, c->stream));
+    chk(cudaMemcpyAsync(c->cong, links->cong, 8 * MM, cudaMemcpyHostToDevice, c->stream));
+    chk(cudaMemcpyAsync(c->prof, prof_h, 8 * kNumProf * V, cudaMemcpyHostToDevice, c->stream));
+    if (e == cudaSuccess) e = launch_tables(c);
+    if (e == cudaSuccess) e = launch_tau(c);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+    delete[] prof_h;
+    if (e != cudaSuccess) return fail_free(E2_ECUDA, cudaGetErrorString(e));
+    *out = c;
+    return E2_OK;
+}
+
+int e2_destroy(e2_ctx *c)
+{
+    if (!c) return E2_OK;
+    cudaError_t e = cudaStreamSynchronize(c->stream);
+    delete c;
+    return e == cudaSuccess ? E2_OK : E2_ECUDA;
+}
+
+int e2_set_population(e2_ctx *c, const e2_genomes *g)
+{
+    if (!c) return E2_EINVAL;
+    return set_and_validate(c, g);
+}
+
+int e2_get_population(e2_ctx *c, const e2_genomes *g)
+{
+    if (!c) return E2_EINVAL;
+    return copy_pop(c, c->pop[c->cur], g, true);
+}
+
+int e2_init_population(e2_ctx *c, uint64_t seed)
+{
+    if (!c) return E2_EINVAL;
+    E2_CUDA(c, launch_init(c, c->pop[c->cur], seed));
+    c->evaluated = false;
+    return E2_OK;
+}
+
+int e2_eval_population(e2_ctx *c, const e2_genomes *genomes, double *fitness_out, const e2_partitions *parts)
+{
+    if (!c) return E2_EINVAL;
+    if (genomes) {
+        int st = set_and_validate(c, genomes);
+        if (st) return st;
+    }
+    E2_CUDA(c, cudaMemsetAsync(c->stats, 0, 8 * kNumStats, c->stream));
+    E2_CUDA(c, launch_eval(c, c->pop[c->cur]));
+    c->evaluated = true;
+    const size_t P = c->dm.P, M = c->dm.M, K = c->dm.K;
+    bool host = false;
+    auto out = [&](void *dst, const void *src, size_t bytes) -> cudaError_t {
+        if (!dst) return cudaSuccess;
+        host = host || is_host(dst);
+        return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, c->stream);
+    };
+    E2_CUDA(c, out(fitness_out, c->fit, 32 * P));
+    if (parts) {
+        E2_CUDA(c, out(parts->layers, c->layers, 2 * P * M));
+        E2_CUDA(c, out(parts->master, c->master, 2 * P * K));
+        E2_CUDA(c, out(parts->bsel, c->bsel, 2 * P * K));
+        E2_CUDA(c, out(parts->T, c->T, 8 * P * K));
+        E2_CUDA(c, out(parts->lambda, c->L, 8 * P * K));
+    }
+    if (host) E2_CUDA(c, cudaStreamSynchronize(c->stream));
+    return E2_OK;
+}
+
+int e2_ga_step(e2_ctx *c, uint64_t seed, uint32_t generation)
+{
+    if (!c) return E2_EINVAL;
+    if (!c->evaluated) return fail(c, E2_ESTATE, "the current population has not been evaluated");
+    E2_CUDA(c, launch_elites(c, c->pop[c->cur]));
+    E2_CUDA(c, launch_ga(c, c->pop[c->cur], c->pop[c->cur ^ 1], seed, generation));
+    c->cur ^= 1;
+    c->evaluated = false;
+    c->have_elites = true;
+    return E2_OK;
+}
+
+int e2_redraw_congestion(e2_ctx *c, uint64_t seed, uint32_t generation)
+{
+    if (!c) return E2_EINVAL;
+    E2_CUDA(c, launch_redraw(c, seed, generation));
+    E2_CUDA(c, launch_tau(c));
+    c->evaluated = false;
+    return E2_OK;
+}
+
+int e2_get_congestion(e2_ctx *c, double *cong_out)
+{
+    if (!c || !cong_out) return E2_EINVAL;
+    E2_CUDA(c, cudaMemcpyAsync(cong_out, c->cong, 8 * (size_t)c->dm.M * c->dm.M, cudaMemcpyDefault, c->stream));
+    if (is_host(cong_out)) E2_CUDA(c, cudaStreamSynchronize(c->stream));
+    return E2_OK;
+}
+
+int e2_get_elites(e2_ctx *c, int32_t *idx_out, double *fitness_out)
+{
+    if (!c) return E2_EINVAL;
+    if (!c->have_elites) return fail(c, E2_ESTATE, "no generation step has run");
+    const size_t Q = c->dm.Q;
+    bool host = false;
+    if (idx_out && Q) {
+        E2_CUDA(c, cudaMemcpyAsync(idx_out, c->elite, 4 * Q, cudaMemcpyDefault, c->stream));
+        host = host || is_host(idx_out);
+    }
+    if (fitness_out && Q) {
+        E2_CUDA(c, cudaMemcpyAsync(fitness_out, c->elite_fit, 32 * Q, cudaMemcpyDefault, c->stream));
+        host = host || is_host(fitness_out);
+    }
+    if (host) E2_CUDA(c, cudaStreamSynchronize(c->stream));
+    return E2_OK;
+}
+
+int e2_get_stats(e2_ctx *c, e2_stats *out)
+{
+    if (!c || !out) return E2_EINVAL;
+    unsigned long long s[kNumStats];
+    E2_CUDA(c, cudaMemcpyAsync(s, c->stats, sizeof s, cudaMemcpyDeviceToHost, c->stream));
+    E2_CUDA(c, cudaStreamSynchronize(c->stream));
+    out->genomes = s[kStGenomes];
+    out->replicas = s[kStReplicas];
+    out->dp_runs = s[kStDpRuns];
+    out->dp_cells = s[kStCells];
+    out->dp_probes = s[kStProbes];
+    out->paper_candidates = s[kStPaper];
+    out->prechecked = s[kStPrecheck];
+    out->served = s[kStServed];
+    return E2_OK;
+}
+
+const char *e2_strerror(int s)
+{
+    switch (s) {
+    case E2_OK: return "ok";
+    case E2_EINVAL: return "invalid argument";
+    case E2_ENOMEM: return "workspace too small";
+    case E2_ECUDA: return "CUDA runtime error";
+    case E2_ETIMEOUT: return "bounded device wait expired";
+    case E2_EDEVICE: return "device-side check failed";
+    case E2_ESTATE: return "call out of order";
+    default: return "unknown status";
+    }
+}
+
+const char *e2_last_error(const e2_ctx *c) { return c ? c->last_error.c_str() : g_create_error; }
+
+}  // extern "C"

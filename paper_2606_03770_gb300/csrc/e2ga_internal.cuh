@@ -1,0 +1,159 @@
+// e2ga_internal.cuh -- device-side layout and helpers shared by the library's
+// translation units.  Not part of the public ABI (see include/e2ga.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+#include "e2ga.h"
+
+namespace e2 {
+
+// +inf as a 64-bit key.  Every time in the planner is a non-negative float64
+// (or +inf), and non-negative IEEE-754 doubles order exactly like their bit
+// patterns read as unsigned integers, so the DP compares 64-bit integer keys.
+constexpr uint64_t kInfKey = 0x7FF0000000000000ull;
+
+// Philox stream purposes (counter word 3).
+enum Purpose : uint32_t {
+    kInitPerm = 0, kInitGroup = 1, kInitRoles = 2, kSelect = 3, kCross = 4, kMutate = 5,
+    kMutPerm = 6, kMutGroup = 7, kMutRoles = 8, kCong = 9
+};
+
+// Profile arrays in the workspace: kProf* index the 7 arrays of length V.
+enum ProfArray { kBlkFlops = 0, kBlkBytes, kBlkMem, kHeadFlops, kHeadBytes, kHeadMem, kAct, kNumProf };
+
+struct DevPop {
+    uint16_t *perm;    // [P][M]
+    uint16_t *sizes;   // [P][K]
+    uint8_t *nclus;    // [P]
+    uint64_t *roles;   // [P]
+};
+
+// Stats slots (unsigned long long, atomically accumulated).
+enum StatSlot { kStGenomes = 0, kStReplicas, kStDpRuns, kStCells, kStProbes, kStPaper, kStPrecheck,
+                kStServed, kNumStats };
+
+// Everything a kernel needs, passed by value.
+struct Dims {
+    int M, N, V, b_max, P, Q, K;
+    int LS;              // leaf row stride (>= N, even)
+    int tournament;
+    uint64_t NP, ND;
+    double min_tps, t_a;
+};
+
+struct Tables {
+    const double *rate, *bw;
+    const uint64_t *mem;
+    const uint64_t *prof;      // [kNumProf][V]
+    const double *leaf;        // [V][M][2][LS]: leaf[((v*M+d)*2+mf)*LS + n-1] = l_d(n blocks, master mf)
+    const double *tau;         // [V][M][M]
+};
+
+struct EvalOut {
+    double *fit;               // [P][4]
+    int16_t *layers;           // [P][M]
+    int16_t *master, *bsel;    // [P][K]
+    double *T, *L;             // [P][K]
+    uint64_t *hash;            // [P]
+    unsigned long long *stats; // [kNumStats]
+};
+
+// ---------------------------------------------------------------------------
+// Philox-4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two
+// 32x32->64 multiplies of counter words 0 and 2, the high halves xored with
+// the other words and the key, the key advanced by the Weyl increments
+// between rounds.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1)
+{
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        if (r) { k0 += 0x9E3779B9u; k1 += 0xBB67AE85u; }
+        const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+        const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+        c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+    }
+    return c;
+}
+
+// A stream (seed, generation, slot, purpose) of 32-bit words; word t is
+// component t%4 of the block with counter (t/4, slot, generation, purpose).
+struct Stream {
+    uint32_t k0, k1, gen, slot, purpose;
+    uint32_t blk;
+    uint4 cache;
+    __device__ Stream(uint64_t seed, uint32_t g, uint32_t s, uint32_t p)
+        : k0((uint32_t)seed), k1((uint32_t)(seed >> 32)), gen(g), slot(s), purpose(p), blk(0xFFFFFFFFu) {}
+    __device__ __forceinline__ uint32_t word(uint32_t t)
+    {
+        const uint32_t b = t >> 2;
+        if (b != blk) {
+            cache = philox4x32_10(make_uint4(b, slot, gen, purpose), k0, k1);
+            blk = b;
+        }
+        const uint32_t q = t & 3u;
+        return q == 0 ? cache.x : q == 1 ? cache.y : q == 2 ? cache.z : cache.w;
+    }
+};
+
+// Integer in [0, n): multiply-shift of one word (Lemire, no rejection).
+__device__ __forceinline__ uint32_t below(uint32_t x, uint32_t n)
+{
+    return (uint32_t)(((uint64_t)x * n) >> 32);
+}
+
+__device__ __forceinline__ uint64_t dkey(double x) { return (uint64_t)__double_as_longlong(x); }
+__device__ __forceinline__ double keyd(uint64_t k) { return __longlong_as_double((long long)k); }
+__device__ __forceinline__ uint64_t umin64(uint64_t a, uint64_t b) { return a < b ? a : b; }
+__device__ __forceinline__ uint64_t umax64(uint64_t a, uint64_t b) { return a > b ? a : b; }
+
+}  // namespace e2
+
+// Host-side context (opaque to callers).
+struct e2_ctx {
+    int device = 0;
+    cudaStream_t stream = nullptr;
+    e2::Dims dm{};
+    double cong_lo = 0, cong_hi = 0;
+    uint64_t thr_cx = 0, thr_half = 0, thr_mut = 0, thr_k1 = 0, thr_k2 = 0, thr_k3 = 0;
+    // device pointers (all inside the caller's workspace)
+    double *rate = nullptr, *bw = nullptr;
+    uint64_t *mem = nullptr;
+    double *link_bw = nullptr, *cong = nullptr;
+    uint64_t *prof = nullptr;
+    double *leaf = nullptr, *tau = nullptr;
+    e2::DevPop pop[2]{};
+    int cur = 0;
+    double *fit = nullptr;
+    int16_t *layers = nullptr, *master = nullptr, *bsel = nullptr;
+    double *T = nullptr, *L = nullptr;
+    uint64_t *hash = nullptr;
+    int32_t *dup = nullptr, *elite = nullptr;
+    double *elite_fit = nullptr;
+    unsigned long long *stats = nullptr;
+    int32_t *err = nullptr;
+    // launch shapes
+    int dp_threads = 128;
+    size_t dp_smem = 0;
+    bool evaluated = false;
+    bool have_elites = false;
+    std::string last_error;
+};
+
+namespace e2 {
+// launchers (defined in the .cu files); return cudaGetLastError()
+cudaError_t launch_tables(const e2_ctx *c);
+cudaError_t launch_tau(const e2_ctx *c);
+cudaError_t launch_redraw(const e2_ctx *c, uint64_t seed, uint32_t gen);
+cudaError_t launch_validate(const e2_ctx *c, const DevPop &p);
+cudaError_t launch_eval(const e2_ctx *c, const DevPop &p);
+cudaError_t launch_init(const e2_ctx *c, const DevPop &p, uint64_t seed);
+cudaError_t launch_elites(const e2_ctx *c, const DevPop &p);
+cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen);
+size_t dp_smem_bytes(int M, int N, int threads);
+cudaError_t configure_eval(size_t smem);
+}  // namespace e2

@@ -1,0 +1,393 @@
+// ga.cu -- cost tables, congestion redraw, population validation, the random
+// initial population, elites and the generation step (Sec. 3.2 cost model,
+// Sec. 3.4 and App. A genetic algorithm).  All randomness comes from
+// Philox-4x32-10 streams keyed by (seed, generation, slot, purpose), so a
+// generation replays bit for bit whatever the thread mapping.
+#include "e2ga_internal.cuh"
+
+namespace e2 {
+
+namespace {
+
+constexpr int kBitmapWords = E2_MAX_DEVICES / 32;
+
+// l_d(n, master): the larger of compute time and streaming time of n identical
+// blocks (plus the LM head and output layer on the master), +inf when the
+// resident bytes exceed the device memory (Sec. 3.2).
+__global__ void tables_kernel(Dims dm, const double *rate, const double *bw, const uint64_t *mem,
+                              const uint64_t *prof, double *leaf)
+{
+    const size_t total = (size_t)dm.V * dm.M * 2 * dm.LS;
+    for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < total;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        const int n = (int)(idx % dm.LS);
+        size_t rest = idx / dm.LS;
+        const int mf = (int)(rest & 1);
+        rest >>= 1;
+        const int d = (int)(rest % dm.M);
+        const int v = (int)(rest / dm.M);
+        double out = keyd(kInfKey);
+        if (n < dm.N) {
+            const uint64_t nb = (uint64_t)n + 1;
+            const int V = dm.V;
+            const uint64_t need = nb * prof[kBlkMem * V + v] + (mf ? prof[kHeadMem * V + v] : 0ull);
+            if (need <= mem[d]) {
+                const uint64_t fl = nb * prof[kBlkFlops * V + v] + (mf ? prof[kHeadFlops * V + v] : 0ull);
+                const uint64_t by = nb * prof[kBlkBytes * V + v] + (mf ? prof[kHeadBytes * V + v] : 0ull);
+                const double tc = __ull2double_rn(fl) / rate[d];
+                const double tm = __ull2double_rn(by) / bw[d];
+                out = tc >= tm ? tc : tm;
+            }
+        }
+        leaf[idx] = out;
+    }
+}
+
+// tau_v(a, b) = A_v / (B(a,b) * congestion(a,b)) (Sec. 3.2).
+__global__ void tau_kernel(Dims dm, const double *link_bw, const double *cong, const uint64_t *prof,
+                           double *tau)
+{
+    const size_t MM = (size_t)dm.M * dm.M, total = (size_t)dm.V * MM;
+    for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < total;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        const int v = (int)(idx / MM);
+        const size_t ab = idx - (size_t)v * MM;
+        const double beff = link_bw[ab] * cong[ab];
+        tau[idx] = __ull2double_rn(prof[kAct * dm.V + v]) / beff;
+    }
+}
+
+// Congestion factor of each unordered pair a < b: lo + (hi - lo) u, with u a
+// 53-bit uniform from words 2(aM+b), 2(aM+b)+1 of the stream (seed, gen, 0, CONG).
+__global__ void redraw_kernel(int M, uint64_t seed, uint32_t gen, double lo, double hi, double *cong)
+{
+    const size_t MM = (size_t)M * M;
+    for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < MM;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        const int a = (int)(idx / M), b = (int)(idx - (size_t)a * M);
+        if (a == b) { cong[idx] = 1.0; continue; }
+        if (a > b) continue;
+        Stream st(seed, gen, 0, kCong);
+        const uint32_t w0 = st.word(2u * (uint32_t)idx), w1 = st.word(2u * (uint32_t)idx + 1u);
+        const uint64_t u53 = ((uint64_t)(w0 >> 5) << 26) | (uint64_t)(w1 >> 6);
+        const double u = (double)u53 * (1.0 / 9007199254740992.0);
+        const double span = hi - lo;
+        const double t = span * u;
+        const double f = lo + t;
+        cong[idx] = f;
+        cong[(size_t)b * M + a] = f;
+    }
+}
+
+__global__ void validate_kernel(Dims dm, DevPop p, int32_t *err)
+{
+    const int g = blockIdx.x * blockDim.x + threadIdx.x;
+    if (g >= dm.P) return;
+    const int M = dm.M, K = dm.K;
+    const int R = p.nclus[g];
+    bool ok = R >= 1 && R <= K && R <= M;
+    int sum = 0;
+    for (int c = 0; c < K && ok; ++c) {
+        const int s = p.sizes[(size_t)g * K + c];
+        if (c < R) { ok = s >= 1; sum += s; }
+        else ok = s == 0;
+    }
+    ok = ok && sum == M;
+    if (ok && R < 64) ok = (p.roles[g] >> R) == 0ull;
+    uint32_t seen[kBitmapWords];
+    const int words = (M + 31) >> 5;
+    for (int w = 0; w < words; ++w) seen[w] = 0;
+    for (int i = 0; i < M && ok; ++i) {
+        const int d = p.perm[(size_t)g * M + i];
+        if (d >= M || ((seen[d >> 5] >> (d & 31)) & 1u)) ok = false;
+        else seen[d >> 5] |= 1u << (d & 31);
+    }
+    if (!ok) atomicMin(err, g);
+}
+
+// Fisher-Yates shuffle of the identity ordering (word M-1-t draws position t).
+__device__ void random_perm(Stream &st, int M, uint16_t *perm)
+{
+    for (int i = 0; i < M; ++i) perm[i] = (uint16_t)i;
+    for (int t = M - 1; t >= 1; --t) {
+        const uint32_t j = below(st.word((uint32_t)(M - 1 - t)), (uint32_t)t + 1);
+        const uint16_t x = perm[t];
+        perm[t] = perm[j];
+        perm[j] = x;
+    }
+}
+
+// Grouping of Mr devices: replica count 1 + uniform(min(Kr, Mr)) from word 0;
+// the R-1 cut points by sequential selection sampling (candidate cut t taken
+// with probability needed/remaining, word t); one role bit per replica from
+// two words of the roles stream.  Returns R.
+__device__ int random_grouping(Stream &sg, Stream &sr, int Mr, int Kr, uint16_t *sizes, uint64_t *roles)
+{
+    const int cap = Kr < Mr ? Kr : Mr;
+    const int R = 1 + (int)below(sg.word(0), (uint32_t)cap);
+    int need = R - 1, prev = 0, c = 0;
+    for (int t = 1; t <= Mr - 1 && need > 0; ++t) {
+        if (below(sg.word((uint32_t)t), (uint32_t)(Mr - t)) < (uint32_t)need) {
+            sizes[c++] = (uint16_t)(t - prev);
+            prev = t;
+            --need;
+        }
+    }
+    sizes[c] = (uint16_t)(Mr - prev);
+    const uint64_t bits = (uint64_t)sr.word(0) | ((uint64_t)sr.word(1) << 32);
+    *roles = R >= 64 ? bits : (bits & ((1ull << R) - 1ull));
+    return R;
+}
+
+__global__ void init_kernel(Dims dm, DevPop p, uint64_t seed)
+{
+    const int s = blockIdx.x * blockDim.x + threadIdx.x;
+    if (s >= dm.P) return;
+    const int M = dm.M, K = dm.K;
+    uint16_t *perm = p.perm + (size_t)s * M;
+    uint16_t *sizes = p.sizes + (size_t)s * K;
+    Stream sp(seed, 0, (uint32_t)s, kInitPerm);
+    random_perm(sp, M, perm);
+    for (int c = 0; c < K; ++c) sizes[c] = 0;
+    Stream sg(seed, 0, (uint32_t)s, kInitGroup), sr(seed, 0, (uint32_t)s, kInitRoles);
+    uint64_t roles;
+    p.nclus[s] = (uint8_t)random_grouping(sg, sr, M, K, sizes, &roles);
+    p.roles[s] = roles;
+}
+
+// Total order of the elites: distinct genomes before duplicates, then lower w,
+// lower bottleneck phase, lower index.
+__device__ __forceinline__ bool elite_before(int da, double wa, double pa, int a, int db, double wb,
+                                             double pb, int b)
+{
+    if (da != db) return da < db;
+    if (wa != wb) return wa < wb;
+    if (pa != pb) return pa < pb;
+    return a < b;
+}
+
+// A genome equal to a lower-indexed one is a duplicate.  Equal genomes have
+// equal fitness (the evaluation is deterministic) and equal fingerprints, so
+// only those pairs are compared in full.
+__global__ void __launch_bounds__(256) dup_kernel(Dims dm, DevPop p, const double *fit,
+                                                  const uint64_t *hash, int32_t *dup)
+{
+    __shared__ double s_w[256], s_p[256];
+    __shared__ uint64_t s_h[256];
+    const int g = blockIdx.x * blockDim.x + threadIdx.x;
+    const bool live = g < dm.P;
+    const double w = live ? fit[(size_t)g * 4] : 0.0, ph = live ? fit[(size_t)g * 4 + 1] : 0.0;
+    const uint64_t h = live ? hash[g] : 0ull;
+    int d = 0;
+    const int gmax = min(dm.P, (int)(blockIdx.x + 1) * (int)blockDim.x);
+    for (int base = 0; base < gmax; base += blockDim.x) {
+        const int hidx = base + threadIdx.x;
+        if (hidx < dm.P) {
+            s_w[threadIdx.x] = fit[(size_t)hidx * 4];
+            s_p[threadIdx.x] = fit[(size_t)hidx * 4 + 1];
+            s_h[threadIdx.x] = hash[hidx];
+        }
+        __syncthreads();
+        if (live && !d) {
+            const int lim = min((int)blockDim.x, g - base);
+            for (int t = 0; t < lim && !d; ++t) {
+                if (s_h[t] != h || s_w[t] != w || s_p[t] != ph) continue;
+                const int o = base + t;
+                bool eq = p.nclus[o] == p.nclus[g] && p.roles[o] == p.roles[g];
+                for (int i = 0; i < dm.M && eq; ++i) eq = p.perm[(size_t)o * dm.M + i] == p.perm[(size_t)g * dm.M + i];
+                for (int i = 0; i < dm.K && eq; ++i) eq = p.sizes[(size_t)o * dm.K + i] == p.sizes[(size_t)g * dm.K + i];
+                d = eq;
+            }
+        }
+        __syncthreads();
+    }
+    if (live) dup[g] = d;
+}
+
+// rank(g) = number of genomes before g in the elite order; the first Q ranks
+// are the elites.
+__global__ void __launch_bounds__(256) rank_kernel(Dims dm, const double *fit, const int32_t *dup,
+                                                   int32_t *elite, double *elite_fit)
+{
+    __shared__ double s_w[256], s_p[256];
+    __shared__ int s_d[256];
+    const int g = blockIdx.x * blockDim.x + threadIdx.x;
+    const bool live = g < dm.P;
+    const double w = live ? fit[(size_t)g * 4] : 0.0, ph = live ? fit[(size_t)g * 4 + 1] : 0.0;
+    const int dg = live ? dup[g] : 0;
+    int rank = 0;
+    for (int base = 0; base < dm.P; base += blockDim.x) {
+        const int hidx = base + threadIdx.x;
+        if (hidx < dm.P) {
+            s_w[threadIdx.x] = fit[(size_t)hidx * 4];
+            s_p[threadIdx.x] = fit[(size_t)hidx * 4 + 1];
+            s_d[threadIdx.x] = dup[hidx];
+        }
+        __syncthreads();
+        const int lim = min((int)blockDim.x, dm.P - base);
+        if (live)
+            for (int t = 0; t < lim; ++t) rank += elite_before(s_d[t], s_w[t], s_p[t], base + t, dg, w, ph, g);
+        __syncthreads();
+    }
+    if (live && rank < dm.Q) {
+        elite[rank] = g;
+        for (int q = 0; q < 4; ++q) elite_fit[(size_t)rank * 4 + q] = fit[(size_t)g * 4 + q];
+    }
+}
+
+struct GaThr {
+    uint64_t cx, half, mut, k1, k2, k3;
+};
+
+__device__ __forceinline__ bool key_less(const double *fit, int a, int b)
+{
+    const double wa = fit[(size_t)a * 4], wb = fit[(size_t)b * 4];
+    if (wa != wb) return wa < wb;
+    const double pa = fit[(size_t)a * 4 + 1], pb = fit[(size_t)b * 4 + 1];
+    if (pa != pb) return pa < pb;
+    return a < b;
+}
+
+// One child per thread (App. A): tournament selection of two parents, uniform
+// crossover of the ordering chromosome, repair, grouping and roles from one
+// parent, then at most one mutation.  Slots [0, Q) copy the elites.
+__global__ void ga_kernel(Dims dm, DevPop src, DevPop dst, const double *fit, const int32_t *elite,
+                          uint64_t seed, uint32_t gen, GaThr thr)
+{
+    const int s = blockIdx.x * blockDim.x + threadIdx.x;
+    if (s >= dm.P) return;
+    const int M = dm.M, K = dm.K, P = dm.P;
+    uint16_t *cp = dst.perm + (size_t)s * M;
+    uint16_t *cs = dst.sizes + (size_t)s * K;
+    if (s < dm.Q) {
+        const int e = elite[s];
+        for (int i = 0; i < M; ++i) cp[i] = src.perm[(size_t)e * M + i];
+        for (int i = 0; i < K; ++i) cs[i] = src.sizes[(size_t)e * K + i];
+        dst.nclus[s] = src.nclus[e];
+        dst.roles[s] = src.roles[e];
+        return;
+    }
+    Stream sel(seed, gen, (uint32_t)s, kSelect);
+    int par[2];
+    for (int q = 0; q < 2; ++q) {
+        int best = (int)below(sel.word((uint32_t)(q * dm.tournament)), (uint32_t)P);
+        for (int t = 1; t < dm.tournament; ++t) {
+            const int c = (int)below(sel.word((uint32_t)(q * dm.tournament + t)), (uint32_t)P);
+            if (key_less(fit, c, best)) best = c;
+        }
+        par[q] = best;
+    }
+    const uint16_t *pa = src.perm + (size_t)par[0] * M, *pb = src.perm + (size_t)par[1] * M;
+    Stream cx(seed, gen, (uint32_t)s, kCross);
+    for (int i = 0; i < M; ++i) cp[i] = (uint64_t)cx.word((uint32_t)i) < thr.cx ? pb[i] : pa[i];
+    // repair: a repeated device leaves a hole; holes take the missing devices in order
+    uint32_t seen[kBitmapWords];
+    const int words = (M + 31) >> 5;
+    for (int w = 0; w < words; ++w) seen[w] = 0;
+    for (int i = 0; i < M; ++i) {
+        const int d = cp[i];
+        if ((seen[d >> 5] >> (d & 31)) & 1u) cp[i] = 0xFFFFu;
+        else seen[d >> 5] |= 1u << (d & 31);
+    }
+    int miss = 0;
+    for (int i = 0; i < M; ++i) {
+        if (cp[i] != 0xFFFFu) continue;
+        while ((seen[miss >> 5] >> (miss & 31)) & 1u) ++miss;
+        cp[i] = (uint16_t)miss;
+        seen[miss >> 5] |= 1u << (miss & 31);
+    }
+    const int from = (uint64_t)cx.word((uint32_t)M) < thr.half ? par[1] : par[0];
+    for (int i = 0; i < K; ++i) cs[i] = src.sizes[(size_t)from * K + i];
+    int R = src.nclus[from];
+    uint64_t rl = src.roles[from];
+
+    Stream mt(seed, gen, (uint32_t)s, kMutate);
+    if ((uint64_t)mt.word(0) < thr.mut) {
+        const uint64_t kind = mt.word(1);
+        if (kind < thr.k1) {                                   // swap two positions
+            const uint32_t x = below(mt.word(2), (uint32_t)M), y = below(mt.word(3), (uint32_t)M);
+            const uint16_t t = cp[x];
+            cp[x] = cp[y];
+            cp[y] = t;
+        } else {
+            int r = 0;
+            if (kind < thr.k2) {                               // regroup from a random replica
+                r = (int)below(mt.word(2), (uint32_t)R);
+            } else if (kind >= thr.k3) {                       // regenerate both chromosomes
+                Stream sp(seed, gen, (uint32_t)s, kMutPerm);
+                random_perm(sp, M, cp);
+            }
+            int kept = 0;
+            for (int c = 0; c < r; ++c) kept += cs[c];
+            for (int c = r; c < K; ++c) cs[c] = 0;
+            Stream sg(seed, gen, (uint32_t)s, kMutGroup), sr(seed, gen, (uint32_t)s, kMutRoles);
+            uint64_t nr;
+            const int Rn = random_grouping(sg, sr, M - kept, K - r, cs + r, &nr);
+            const uint64_t keep = r >= 64 ? ~0ull : ((1ull << r) - 1ull);
+            rl = (rl & keep) | (r >= 64 ? 0ull : (nr << r));
+            R = r + Rn;
+        }
+    }
+    dst.nclus[s] = (uint8_t)R;
+    dst.roles[s] = rl;
+}
+
+// 1D launch helpers
+inline unsigned grid_for(size_t n, int threads, size_t cap = 152 * 32)
+{
+    size_t b = (n + threads - 1) / threads;
+    if (b > cap) b = cap;
+    return (unsigned)(b ? b : 1);
+}
+
+}  // namespace
+
+cudaError_t launch_tables(const e2_ctx *c)
+{
+    const size_t total = (size_t)c->dm.V * c->dm.M * 2 * c->dm.LS;
+    tables_kernel<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm, c->rate, c->bw, c->mem, c->prof, c->leaf);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_tau(const e2_ctx *c)
+{
+    const size_t total = (size_t)c->dm.V * c->dm.M * c->dm.M;
+    tau_kernel<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm, c->link_bw, c->cong, c->prof, c->tau);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_redraw(const e2_ctx *c, uint64_t seed, uint32_t gen)
+{
+    const size_t total = (size_t)c->dm.M * c->dm.M;
+    redraw_kernel<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm.M, seed, gen, c->cong_lo, c->cong_hi, c->cong);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_validate(const e2_ctx *c, const DevPop &p)
+{
+    validate_kernel<<<(c->dm.P + 127) / 128, 128, 0, c->stream>>>(c->dm, p, c->err);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_init(const e2_ctx *c, const DevPop &p, uint64_t seed)
+{
+    init_kernel<<<(c->dm.P + 127) / 128, 128, 0, c->stream>>>(c->dm, p, seed);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_elites(const e2_ctx *c, const DevPop &p)
+{
+    const unsigned blocks = (c->dm.P + 255) / 256;
+    dup_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, p, c->fit, c->hash, c->dup);
+    if (c->dm.Q > 0) rank_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, c->fit, c->dup, c->elite, c->elite_fit);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen)
+{
+    GaThr thr{c->thr_cx, c->thr_half, c->thr_mut, c->thr_k1, c->thr_k2, c->thr_k3};
+    ga_kernel<<<(c->dm.P + 127) / 128, 128, 0, c->stream>>>(c->dm, src, dst, c->fit, c->elite, seed, gen, thr);
+    return cudaGetLastError();
+}
+
+}  // namespace e2
