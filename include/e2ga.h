@@ -220,6 +220,30 @@ int e2_get_elites(e2_ctx *ctx, int32_t *idx_out, double *fitness_out);
 /* Counters of the last evaluation.  Synchronises. */
 int e2_get_stats(e2_ctx *ctx, e2_stats *out);
 
+/* Elite selection that allocates nothing.  The paper has no counterpart: this
+ * is a service of this library for callers that cannot allocate device memory
+ * -- code recording a CUDA graph (allocation is not capturable), plug-ins whose
+ * host framework's allocator owns all device memory, loops that must never
+ * pay cudaMalloc's implicit synchronisation.  It computes what e2_ga_step's
+ * elite step computes (the Q best distinct genomes of an evaluated
+ * population by (w, phase, index)) without a context or workspace: its
+ * scratch is a file-scope device array sized for E2_NOALLOC_MAX_POP genomes (1 MiB,
+ * held by every GPU that loads the library until the process exits).
+ *   pop       population [P] in the genome layout, DEVICE pointers
+ *   fitness   [P][4] {w, phase, PS, DS} from e2_eval_population, DEVICE
+ *   elite_idx [Q] output, DEVICE; may be NULL when Q == 0
+ *   stream    cudaStream_t the work is enqueued on (asynchronous)
+ * Returns E2_EINVAL for P > E2_NOALLOC_MAX_POP, other out-of-range sizes, null or
+ * host pointers; E2_ECUDA if the scratch address cannot be obtained or a launch
+ * fails.  The first call on each device looks up the scratch array's device
+ * address with that device current; make that first call before any stream
+ * capture.  All calls share the one scratch array and overwrite it; calls that
+ * overlap on the GPU (other streams, other host threads) race and must be
+ * serialised by the caller. */
+#define E2_NOALLOC_MAX_POP 65536
+int e2_select_elites_noalloc(const e2_genomes *pop, const double *fitness, int32_t P, int32_t M,
+                             int32_t K_max, int32_t Q, int32_t *elite_idx, void *stream);
+
 /* Text of a status code, and the context's last detailed error message.  With
  * ctx == NULL: the message of the calling thread's last failed e2_create ("" if
  * none). */

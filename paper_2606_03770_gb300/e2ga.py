@@ -70,6 +70,8 @@ SIGNATURES = {
     "e2_get_congestion": (C.c_int, [C.c_void_p, C.c_void_p]),
     "e2_get_elites": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "e2_get_stats": (C.c_int, [C.c_void_p, C.c_void_p]),
+    "e2_select_elites_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
+                                            C.c_int32, C.c_void_p, C.c_void_p]),
     "e2_strerror": (C.c_char_p, [C.c_int]),
     "e2_last_error": (C.c_char_p, [C.c_void_p]),
 }
@@ -147,6 +149,10 @@ def e2_get_elites(ctx, idx_ptr, fit_ptr):
 
 def e2_get_stats(ctx, stats):
     return load().e2_get_stats(ctx, C.byref(stats))
+
+
+def e2_select_elites_noalloc(genomes, fitness_ptr, P, M, K_max, Q, elite_ptr, stream_ptr):
+    return load().e2_select_elites_noalloc(C.byref(genomes), fitness_ptr, P, M, K_max, Q, elite_ptr, stream_ptr)
 
 
 def e2_strerror(status):
