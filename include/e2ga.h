@@ -143,6 +143,8 @@ typedef struct {
     uint64_t paper_candidates;  /* (mu,k,i,j) candidates Alg. 1 would examine   */
     uint64_t prechecked;        /* variants rejected by the memory count check  */
     uint64_t served;            /* replicas that can serve                      */
+    uint64_t tps_pruned;        /* decode variants a latency lower bound proved
+                                   to miss Min_TPS (their DP is skipped)        */
 } e2_stats;
 
 typedef struct e2_ctx e2_ctx;

@@ -54,19 +54,6 @@ __device__ __forceinline__ uint64_t dp_cell(const uint64_t *__restrict__ prev,
     return umax64(h, tau);
 }
 
-// Number of finite entries of a non-decreasing row (memory grows with n, so
-// the +inf entries form a suffix).
-__device__ __forceinline__ int finite_prefix(const uint64_t *row, int W)
-{
-    int lo = 0, hi = W;
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (row[mid] < kInfKey) lo = mid + 1;
-        else hi = mid;
-    }
-    return lo;
-}
-
 __device__ __forceinline__ int warp_sum(int x)
 {
 #pragma unroll
@@ -101,24 +88,101 @@ size_t dp_smem_bytes(int M, int N, int threads)
     const int mmax = M < N ? M : N;
     for (int m = 1; m <= mmax; ++m) {
         const size_t W = (size_t)(N - m + 1);
-        size_t u64s = 3 * (size_t)m * W + 2 * (size_t)NW * W + (size_t)m;
-        size_t bytes = u64s * 8 + (size_t)m * (3 * sizeof(int)) + (size_t)m * sizeof(uint16_t) + 16;
+        const size_t u64s = 4 * (size_t)m * W + (size_t)(NW + 1) * W + 2 * (size_t)m;
+        const size_t bytes = u64s * 8 + (size_t)m * (3 * sizeof(int)) + (size_t)m * sizeof(uint16_t) + 16;
         if (bytes > best) best = bytes;
     }
     return (best + 15) & ~(size_t)15;
 }
 
-__global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out)
+namespace {
+
+__device__ __forceinline__ void bar_named(int id, int nthreads)
+{
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// Estimated work of one (genome, replica slot), for heavy-first ordering:
+// 0 = empty slot, 1 = more devices than blocks, else a log-scale bucket of
+// m * W * (number of variants the replica may sweep).
+__device__ __forceinline__ int work_key(const Dims &dm, const DevPop &pop, int slot)
+{
+    const int g = slot / dm.K, c = slot - g * dm.K;
+    if (c >= pop.nclus[g]) return 0;
+    const int m = pop.sizes[slot];
+    if (m > dm.N) return 1;
+    const int W = dm.N - m + 1;
+    const int nv = ((pop.roles[g] >> c) & 1ull) ? dm.b_max : 1;
+    const float est = (float)m * (float)W * (float)nv;
+    const int key = 2 + (int)(8.0f * __log2f(1.0f + est));
+    return key < kOrderBins - 1 ? key : kOrderBins - 1;
+}
+
+}  // namespace
+
+__global__ void order_hist_kernel(Dims dm, DevPop pop, unsigned *bins)
+{
+    const int total = dm.P * dm.K;
+    for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < total; s += gridDim.x * blockDim.x)
+        atomicAdd(&bins[work_key(dm, pop, s)], 1u);
+}
+
+// Exclusive scan of the bins in descending key order (heaviest first).
+__global__ void order_scan_kernel(unsigned *bins)
+{
+    __shared__ unsigned s[kOrderBins];
+    const int t = threadIdx.x;
+    s[t] = bins[kOrderBins - 1 - t];
+    __syncthreads();
+    for (int o = 1; o < kOrderBins; o <<= 1) {
+        const unsigned v = t >= o ? s[t - o] : 0u;
+        __syncthreads();
+        s[t] += v;
+        __syncthreads();
+    }
+    const unsigned incl = s[t];
+    const unsigned cnt = bins[kOrderBins - 1 - t];
+    __syncthreads();
+    bins[kOrderBins - 1 - t] = incl - cnt;
+}
+
+__global__ void order_scatter_kernel(Dims dm, DevPop pop, unsigned *cursor, int *order)
+{
+    const int total = dm.P * dm.K;
+    for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < total; s += gridDim.x * blockDim.x)
+        order[atomicAdd(&cursor[work_key(dm, pop, s)], 1u)] = s;
+}
+
+// One CTA per (genome, replica slot), heaviest first.  Per variant:
+//  1. stage the cost rows l_k(n), l_k^head(n) and the link times;
+//  2. exact memory check per master;
+//  3. prefix columns F_k (no master, devices 1..k) on warps 0-1 and suffix
+//     columns G_k (no master, devices k..m) on warps 2-3, concurrently:
+//        F_k[r] = min_s max(F_{k-1}[s], l_k(r-s+1), tau_k)
+//        G_k[r] = min_s max(G_{k+1}[s], l_k(r-s+1), tau_{k+1})
+//  4. master mu: the prefix holds a extra blocks, the suffix b, the master
+//     W - a - b, so with H_mu[c] = min_{a+b=c} max(F_{mu-1}[a], G_{mu+1}[b])
+//        V_mu = max(tau_mu, tau_{mu+1}, min_c max(H_mu[c], l_mu^head(W - c)))
+//     (F_0 and G_{m+1} are the empty stage: 0 at index 0, +inf after);
+//  5. mu* = smallest mu with the least V_mu; its prefix columns D_k (master
+//     at mu*) are recomputed for the traceback;
+//  6. traceback with the smallest-split rule (n_k = number of n <= r+1 with
+//     l_k(n) <= D, counted with warp ballots) and Lambda in pipeline order.
+// Every value is a min/max of the same leaf and link times the oracle uses,
+// so V, mu*, the partition and Lambda are bit-identical to Alg. 1.
+__global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out,
+                                                      const int *order)
 {
     extern __shared__ __align__(16) unsigned char smem[];
-    __shared__ int s_off, s_m, s_role, s_S0, s_Z, s_any, s_mu, s_done;
+    __shared__ int s_off, s_m, s_role, s_S0, s_Z, s_mu, s_done;
     __shared__ uint64_t s_V;
     __shared__ double s_L;
     __shared__ uint64_t s_wV[4];
     __shared__ int s_wMu[4];
 
     const int K = dm.K, M = dm.M, N = dm.N;
-    const int g = blockIdx.x / K, c = blockIdx.x - g * K;
+    const int slot = order[blockIdx.x];
+    const int g = slot / K, c = slot - g * K;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
     const size_t gk = (size_t)g * K + c;
     const int R = pop.nclus[g];
@@ -140,47 +204,55 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
     const int off = s_off, m = s_m, role = s_role;
     int16_t *lay_out = out.layers + (size_t)g * M + off;
 
-    unsigned long long st_runs = 0, st_cells = 0, st_probes = 0, st_paper = 0, st_pre = 0;
+    unsigned long long st_runs = 0, st_cells = 0, st_probes = 0, st_paper = 0, st_pre = 0, st_tps = 0;
     bool served = false;
 
     if (m <= N) {
         const int W = N - m + 1;
         uint64_t *leaf0 = reinterpret_cast<uint64_t *>(smem);   // [m][W] l_k(n)
         uint64_t *leaf1 = leaf0 + (size_t)m * W;                // [m][W] l_k^head(n)
-        uint64_t *Fst = leaf1 + (size_t)m * W;                  // [m][W] column store
-        uint64_t *pp = Fst + (size_t)m * W;                     // [NW][2][W]
-        uint64_t *tauk = pp + (size_t)NW * 2 * W;               // [m]
-        int *cnt0 = reinterpret_cast<int *>(tauk + m);          // [m]
+        uint64_t *Fst = leaf1 + (size_t)m * W;                  // [m][W] prefix / traceback columns
+        uint64_t *Gst = Fst + (size_t)m * W;                    // [m][W] suffix columns
+        uint64_t *Hb = Gst + (size_t)m * W;                     // [NW][W] per-warp convolution
+        uint64_t *delta = Hb + (size_t)NW * W;                  // [W] the empty stage
+        uint64_t *tauk = delta + W;                             // [m] tauk[k] = link (k-1) -> k
+        double *cpbk = reinterpret_cast<double *>(tauk + m);    // [m] per-block times
+        int *cnt0 = reinterpret_cast<int *>(cpbk + m);          // [m]
         int *cnt1 = cnt0 + m;                                   // [m]
         int *nk = cnt1 + m;                                     // [m]
         uint16_t *devs = reinterpret_cast<uint16_t *>(nk + m);  // [m]
 
         for (int k = tid; k < m; k += blockDim.x) devs[k] = pop.perm[(size_t)g * M + off + k];
+        for (int r = tid; r < W; r += blockDim.x) delta[r] = r ? kInfKey : 0ull;
         __syncthreads();
+
+        // column accessors (1-based device index k)
+        auto colF = [&](int k) -> const uint64_t * {
+            return k == 0 ? delta : k == 1 ? leaf0 : Fst + (size_t)(k - 1) * W;
+        };
+        auto colG = [&](int k) -> const uint64_t * {
+            return k == m + 1 ? delta : k == m ? leaf0 + (size_t)(m - 1) * W : Gst + (size_t)(k - 1) * W;
+        };
 
         const int nvar = role ? dm.b_max : 1;
         const unsigned long long pc = paper_candidates(m, N);
         const unsigned long long cprobe = column_probes(W);
+        const unsigned long long lprobe = 32 - __clz(W);
         for (int vi = 0; vi < nvar && !served; ++vi) {
             const int v = role ? dm.b_max - vi : 0;
-            // ---- stage the cost rows and link times of this variant
-            for (int e = tid; e < m * W; e += blockDim.x) {
-                const int k = e / W, n = e - k * W;
-                const double *base = tb.leaf + ((size_t)v * M + devs[k]) * 2 * dm.LS;
-                leaf0[e] = dkey(base[n]);
-                leaf1[e] = dkey(base[dm.LS + n]);
-            }
-            for (int k = tid; k < m; k += blockDim.x)
+            // ---- 1. capacities, per-block times and link times of this variant
+            for (int k = tid; k < m; k += blockDim.x) {
+                const size_t vd = (size_t)v * M + devs[k];
+                const int c0 = tb.cap[vd * 2], c1 = tb.cap[vd * 2 + 1];
+                cnt0[k] = c0 < W ? c0 : W;
+                cnt1[k] = c1 < W ? c1 : W;
+                cpbk[k] = tb.cpb[vd];
                 tauk[k] = k ? dkey(tb.tau[((size_t)v * M + devs[k - 1]) * M + devs[k]]) : 0ull;
+            }
             __syncthreads();
-            // ---- exact memory check: with identical blocks a partition with
+            // ---- 2. exact memory check: with identical blocks a partition with
             // master mu exists iff every device holds >= 1 block and the block
             // capacities (capped at W) add up to N
-            for (int k = tid; k < m; k += blockDim.x) {
-                cnt0[k] = finite_prefix(leaf0 + (size_t)k * W, W);
-                cnt1[k] = finite_prefix(leaf1 + (size_t)k * W, W);
-            }
-            __syncthreads();
             if (wid == 0) {
                 int s = 0, z = 0;
                 for (int k = lane; k < m; k += 32) { s += cnt0[k]; z += cnt0[k] == 0; }
@@ -198,46 +270,91 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             any = __syncthreads_or(any);
             st_paper += pc;
             if (!any) { ++st_pre; continue; }
-            ++st_runs;
-            auto colF = [&](int k) -> const uint64_t * { return k == 1 ? leaf0 : Fst + (size_t)(k - 1) * W; };
-            // ---- shared columns 2..m-1 without the master
-            for (int k = 2; k <= m - 1; ++k) {
-                const uint64_t *prev = colF(k - 1), *row = leaf0 + (size_t)(k - 1) * W;
-                const uint64_t t = tauk[k - 1];
-                uint64_t *cur = Fst + (size_t)(k - 1) * W;
-                for (int r = tid; r < W; r += blockDim.x) cur[r] = dp_cell(prev, row, t, r);
+            // ---- 2b. decode: a lower bound on Lambda over every feasible
+            // partition.  Lambda = sum of link times + sum_k l_k(n_k) with
+            // l_k(n) >= n * c_k (c_k the per-block time; the head only adds), and
+            // sum_k n_k c_k is least when each device takes one block and the
+            // other N - m go to the cheapest devices up to their capacity.  If
+            // even that bound misses Min_TPS the variant fails whatever the DP
+            // returns, so its DP is skipped; the 1e-9 margin exceeds the
+            // rounding of every sum involved, so no passing variant is lost.
+            if (role) {
+                if (wid == 0) {
+                    const int Rx = N - m;
+                    double part = 0.0;
+                    for (int k = lane; k < m; k += 32) {
+                        const double ck = cpbk[k];
+                        long long before = 0;
+                        for (int j = 0; j < m; ++j) {
+                            const double cj = cpbk[j];
+                            if (cj < ck || (cj == ck && j < k)) before += cnt0[j] - 1;
+                        }
+                        const long long room = (long long)Rx - before;
+                        const long long take = room <= 0 ? 0 : (room < cnt0[k] - 1 ? room : cnt0[k] - 1);
+                        part += ck * (double)(1 + take);
+                        if (k >= 1) part += keyd(tauk[k]);
+                    }
+#pragma unroll
+                    for (int o = 16; o; o >>= 1) part += __shfl_xor_sync(0xFFFFFFFFu, part, o);
+                    if (lane == 0) {
+                        const double lb = part * (1.0 - 1e-9);
+                        s_done = lb > 0.0 && 1.0 / lb < dm.min_tps;
+                    }
+                }
                 __syncthreads();
+                if (s_done) { ++st_tps; continue; }
             }
-            if (tid == 0 && m >= 3) { st_cells += (unsigned long long)(m - 2) * W; st_probes += (m - 2) * cprobe; }
-            // ---- one master per warp at a time
+            // ---- 2c. stage the cost rows
+            for (int e = tid; e < m * W; e += blockDim.x) {
+                const int k = e / W, n = e - k * W;
+                const double *base = tb.leaf + ((size_t)v * M + devs[k]) * 2 * dm.LS;
+                leaf0[e] = dkey(base[n]);
+                leaf1[e] = dkey(base[dm.LS + n]);
+            }
+            __syncthreads();
+            ++st_runs;
+            // ---- 3. prefix columns (warps 0-1) and suffix columns (warps 2-3)
+            if (wid < 2) {
+                for (int k = 2; k <= m - 1; ++k) {
+                    const uint64_t *prev = colF(k - 1), *row = leaf0 + (size_t)(k - 1) * W;
+                    const uint64_t t = tauk[k - 1];
+                    uint64_t *cur = Fst + (size_t)(k - 1) * W;
+                    for (int r = tid; r < W; r += 64) cur[r] = dp_cell(prev, row, t, r);
+                    bar_named(1, 64);
+                }
+            } else {
+                for (int k = m - 1; k >= 2; --k) {
+                    const uint64_t *prev = colG(k + 1), *row = leaf0 + (size_t)(k - 1) * W;
+                    const uint64_t t = tauk[k];
+                    uint64_t *cur = Gst + (size_t)(k - 1) * W;
+                    for (int r = tid - 64; r < W; r += 64) cur[r] = dp_cell(prev, row, t, r);
+                    bar_named(2, 64);
+                }
+            }
+            if (tid == 0 && m >= 3) {
+                st_cells += 2ull * (m - 2) * W;
+                st_probes += 2ull * (m - 2) * cprobe;
+            }
+            __syncthreads();
+            // ---- 4. one master per warp at a time
             uint64_t bestV = kInfKey;
             int bestMu = 0x7FFFFFFF;
             unsigned long long w_cells = 0, w_probes = 0;
+            uint64_t *H = Hb + (size_t)wid * W;
             for (int mu = wid + 1; mu <= m; mu += NW) {
                 if (!mu_ok(mu)) continue;
-                uint64_t V;
-                if (m == 1) {
-                    V = leaf1[W - 1];
-                } else {
-                    uint64_t *buf0 = pp + (size_t)wid * 2 * W, *buf1 = buf0 + W;
-                    const uint64_t *prev = mu == 1 ? leaf1 : colF(mu - 1);
-                    int which = 0;
-                    V = kInfKey;
-                    for (int k = (mu == 1 ? 2 : mu); k <= m; ++k) {
-                        const uint64_t *row = (k == mu ? leaf1 : leaf0) + (size_t)(k - 1) * W;
-                        const uint64_t t = tauk[k - 1];
-                        if (k == m) { V = dp_cell(prev, row, t, W - 1); w_cells += 1; w_probes += 32 - __clz(W); break; }
-                        uint64_t *cur = which ? buf1 : buf0;
-                        which ^= 1;
-                        for (int r = lane; r < W; r += 32) cur[r] = dp_cell(prev, row, t, r);
-                        __syncwarp();
-                        prev = cur;
-                        w_cells += W; w_probes += cprobe;
-                    }
-                }
+                const uint64_t *P = colF(mu - 1), *S = colG(mu + 1);
+                for (int r = lane; r < W; r += 32) H[r] = dp_cell(P, S, 0ull, r);
+                __syncwarp();
+                uint64_t V = dp_cell(H, leaf1 + (size_t)(mu - 1) * W, 0ull, W - 1);
+                if (mu >= 2) V = umax64(V, tauk[mu - 1]);
+                if (mu <= m - 1) V = umax64(V, tauk[mu]);
+                __syncwarp();
+                w_cells += W + 1;
+                w_probes += cprobe + lprobe;
                 if (V < bestV) { bestV = V; bestMu = mu; }
             }
-            if (lane == 0) { s_wV[wid] = bestV; s_wMu[wid] = bestMu; }
+            if (lane == 0) { s_wV[wid] = bestV; s_wMu[wid] = bestMu; st_cells += w_cells; st_probes += w_probes; }
             __syncthreads();
             if (tid == 0) {
                 uint64_t V = kInfKey;
@@ -246,12 +363,11 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
                     if (s_wV[w] < V || (s_wV[w] == V && s_wMu[w] < mu)) { V = s_wV[w]; mu = s_wMu[w]; }
                 s_V = V; s_mu = mu;
             }
-            if (lane == 0) { st_cells += w_cells; st_probes += w_probes; }
             __syncthreads();
             const uint64_t V = s_V;
             const int mus = s_mu;
             if (V >= kInfKey) continue;      // cannot happen after the exact memory check
-            // ---- mu*'s own columns, for the traceback
+            // ---- 5. mu*'s prefix columns, for the traceback
             auto rowk = [&](int k) -> const uint64_t * { return (k == mus ? leaf1 : leaf0) + (size_t)(k - 1) * W; };
             auto colD = [&](int k) -> const uint64_t * {
                 if (k == 1) return mus == 1 ? leaf1 : leaf0;
@@ -265,30 +381,33 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
                 __syncthreads();
                 if (tid == 0) { st_cells += W; st_probes += cprobe; }
             }
-            // ---- traceback (smallest split on ties) and Lambda in pipeline order
-            if (tid == 0) {
+            // ---- 6. traceback (smallest split on ties) and Lambda in pipeline order
+            if (wid == 0) {
                 int r = W - 1;
                 uint64_t D = V;
                 for (int k = m; k >= 2; --k) {
                     const uint64_t *row = rowk(k);
-                    int lo = 1, hi = r + 1;                    // largest n <= r+1 with l_k(n) <= D
-                    while (lo < hi) {
-                        const int mid = (lo + hi + 1) >> 1;
-                        if (row[mid - 1] <= D) lo = mid;
-                        else hi = mid - 1;
+                    int n = 0;                                    // #{n <= r+1 : l_k(n) <= D}
+                    for (int base = 0; base <= r; base += 32) {
+                        const int p = base + lane;
+                        const unsigned b = __ballot_sync(0xFFFFFFFFu, p <= r && row[p] <= D);
+                        n += __popc(b);
+                        if (b != 0xFFFFFFFFu) break;
                     }
-                    nk[k - 1] = lo;
-                    r = r + 1 - lo;
+                    if (lane == 0) nk[k - 1] = n;
+                    r = r + 1 - n;
                     D = colD(k - 1)[r];
                 }
-                nk[0] = r + 1;
-                double lam = keyd(rowk(1)[nk[0] - 1]);
-                for (int k = 2; k <= m; ++k) {
-                    lam = lam + keyd(tauk[k - 1]);
-                    lam = lam + keyd(rowk(k)[nk[k - 1] - 1]);
+                if (lane == 0) {
+                    nk[0] = r + 1;
+                    double lam = keyd(rowk(1)[nk[0] - 1]);
+                    for (int k = 2; k <= m; ++k) {
+                        lam = lam + keyd(tauk[k - 1]);
+                        lam = lam + keyd(rowk(k)[nk[k - 1] - 1]);
+                    }
+                    s_L = lam;
+                    s_done = (!role) || (1.0 / lam >= dm.min_tps);
                 }
-                s_L = lam;
-                s_done = (!role) || (1.0 / lam >= dm.min_tps);
             }
             __syncthreads();
             if (s_done) {
@@ -321,6 +440,7 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
         if (st_runs) atomicAdd(&out.stats[kStDpRuns], st_runs);
         if (st_paper) atomicAdd(&out.stats[kStPaper], st_paper);
         if (st_pre) atomicAdd(&out.stats[kStPrecheck], st_pre);
+        if (st_tps) atomicAdd(&out.stats[kStTpsPruned], st_tps);
         if (served) atomicAdd(&out.stats[kStServed], 1ull);
     }
 }
@@ -374,10 +494,16 @@ cudaError_t configure_eval(size_t smem)
 
 cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
 {
-    Tables tb{c->rate, c->bw, c->mem, c->prof, c->leaf, c->tau};
+    Tables tb{c->rate, c->bw, c->mem, c->prof, c->leaf, c->tau, c->cap, c->cpb};
     EvalOut out{c->fit, c->layers, c->master, c->bsel, c->T, c->L, c->hash, c->stats};
     const long long blocks = (long long)c->dm.P * c->dm.K;
-    dp_eval_kernel<<<(unsigned)blocks, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out);
+    cudaError_t e = cudaMemsetAsync(c->order_bins, 0, sizeof(unsigned) * kOrderBins, c->stream);
+    if (e != cudaSuccess) return e;
+    const unsigned gb = (unsigned)((blocks + 255) / 256 < 1024 ? (blocks + 255) / 256 : 1024);
+    order_hist_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, c->order_bins);
+    order_scan_kernel<<<1, kOrderBins, 0, c->stream>>>(c->order_bins);
+    order_scatter_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, c->order_bins, c->order);
+    dp_eval_kernel<<<(unsigned)blocks, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, c->order);
     score_kernel<<<(c->dm.P + 255) / 256, 256, 0, c->stream>>>(c->dm, p, out);
     return cudaGetLastError();
 }

@@ -20,9 +20,9 @@ thread_local char g_create_error[256] = "";
 size_t align_up(size_t x, size_t a = 256) { return (x + a - 1) / a * a; }
 
 struct Layout {
-    size_t rate, bw, mem, link_bw, cong, prof, leaf, tau;
+    size_t rate, bw, mem, link_bw, cong, prof, leaf, tau, cap, cpb;
     size_t perm[2], sizes[2], nclus[2], roles[2];
-    size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, stats, err, total;
+    size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, stats, err, order_bins, order, total;
     int LS;
 };
 
@@ -48,6 +48,8 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K)
     l.prof = take(8 * kNumProf * V);
     l.leaf = take(8 * V * M * 2 * (size_t)l.LS);
     l.tau = take(8 * V * MM);
+    l.cap = take(4 * V * M * 2);
+    l.cpb = take(8 * V * M);
     for (int b = 0; b < 2; ++b) {
         l.perm[b] = take(2 * (size_t)P * M);
         l.sizes[b] = take(2 * (size_t)P * K);
@@ -66,6 +68,8 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K)
     l.elite_fit = take(32 * (size_t)(Q > 0 ? Q : 1));
     l.stats = take(8 * kNumStats);
     l.err = take(4);
+    l.order_bins = take(4 * kOrderBins);
+    l.order = take(4 * (size_t)P * K);
     l.total = o;
     return l;
 }
@@ -279,6 +283,8 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->prof = reinterpret_cast<uint64_t *>(ws + l.prof);
     c->leaf = reinterpret_cast<double *>(ws + l.leaf);
     c->tau = reinterpret_cast<double *>(ws + l.tau);
+    c->cap = reinterpret_cast<int32_t *>(ws + l.cap);
+    c->cpb = reinterpret_cast<double *>(ws + l.cpb);
     for (int b = 0; b < 2; ++b) c->pop[b] = pop_at(ws, l, b);
     c->fit = reinterpret_cast<double *>(ws + l.fit);
     c->layers = reinterpret_cast<int16_t *>(ws + l.layers);
@@ -292,6 +298,8 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->elite_fit = reinterpret_cast<double *>(ws + l.elite_fit);
     c->stats = reinterpret_cast<unsigned long long *>(ws + l.stats);
     c->err = reinterpret_cast<int32_t *>(ws + l.err);
+    c->order_bins = reinterpret_cast<unsigned *>(ws + l.order_bins);
+    c->order = reinterpret_cast<int *>(ws + l.order);
 
     const size_t V = (size_t)b_max + 1, MM = (size_t)M * M;
     uint64_t *prof_h = new (std::nothrow) uint64_t[kNumProf * V];
@@ -435,6 +443,7 @@ int e2_get_stats(e2_ctx *c, e2_stats *out)
     out->paper_candidates = s[kStPaper];
     out->prechecked = s[kStPrecheck];
     out->served = s[kStServed];
+    out->tps_pruned = s[kStTpsPruned];
     return E2_OK;
 }
 

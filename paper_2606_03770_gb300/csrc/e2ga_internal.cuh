@@ -32,9 +32,12 @@ struct DevPop {
     uint64_t *roles;   // [P]
 };
 
+// Buckets of the heavy-first work ordering of the evaluation.
+constexpr int kOrderBins = 256;
+
 // Stats slots (unsigned long long, atomically accumulated).
 enum StatSlot { kStGenomes = 0, kStReplicas, kStDpRuns, kStCells, kStProbes, kStPaper, kStPrecheck,
-                kStServed, kNumStats };
+                kStServed, kStTpsPruned, kNumStats };
 
 // Everything a kernel needs, passed by value.
 struct Dims {
@@ -51,6 +54,8 @@ struct Tables {
     const uint64_t *prof;      // [kNumProf][V]
     const double *leaf;        // [V][M][2][LS]: leaf[((v*M+d)*2+mf)*LS + n-1] = l_d(n blocks, master mf)
     const double *tau;         // [V][M][M]
+    const int32_t *cap;        // [V][M][2]: most blocks device d holds (memory), without / with the head
+    const double *cpb;         // [V][M]: per-block time max(blk_flops/rate, blk_bytes/bw)
 };
 
 struct EvalOut {
@@ -126,6 +131,8 @@ struct e2_ctx {
     double *link_bw = nullptr, *cong = nullptr;
     uint64_t *prof = nullptr;
     double *leaf = nullptr, *tau = nullptr;
+    int32_t *cap = nullptr;
+    double *cpb = nullptr;
     e2::DevPop pop[2]{};
     int cur = 0;
     double *fit = nullptr;
@@ -136,6 +143,8 @@ struct e2_ctx {
     double *elite_fit = nullptr;
     unsigned long long *stats = nullptr;
     int32_t *err = nullptr;
+    unsigned *order_bins = nullptr;   // [kOrderBins]
+    int *order = nullptr;             // [P*K] evaluation order of (genome, replica) slots
     // launch shapes
     int dp_threads = 128;
     size_t dp_smem = 0;
@@ -146,7 +155,7 @@ struct e2_ctx {
 
 namespace e2 {
 // launchers (defined in the .cu files); return cudaGetLastError()
-cudaError_t launch_tables(const e2_ctx *c);
+cudaError_t launch_tables(const e2_ctx *c);   // leaf, cap and cpb tables
 cudaError_t launch_tau(const e2_ctx *c);
 cudaError_t launch_redraw(const e2_ctx *c, uint64_t seed, uint32_t gen);
 cudaError_t launch_validate(const e2_ctx *c, const DevPop &p);

@@ -43,6 +43,28 @@ __global__ void tables_kernel(Dims dm, const double *rate, const double *bw, con
     }
 }
 
+// Per (variant, device): the most blocks the device can hold, without and with
+// the LM head (the number of finite entries of its two cost rows), and the
+// per-block time max(blk_flops/rate, blk_bytes/bw) used by the latency bound.
+__global__ void captab_kernel(Dims dm, const double *rate, const double *bw, const uint64_t *mem,
+                              const uint64_t *prof, int32_t *cap, double *cpb)
+{
+    const size_t total = (size_t)dm.V * dm.M;
+    for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < total;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        const int v = (int)(idx / dm.M), d = (int)(idx - (size_t)v * dm.M);
+        const int V = dm.V;
+        const uint64_t bm = prof[kBlkMem * V + v], hm = prof[kHeadMem * V + v], mm = mem[d];
+        const uint64_t c0 = bm ? mm / bm : (uint64_t)dm.N;
+        const uint64_t c1 = mm < hm ? 0ull : (bm ? (mm - hm) / bm : (uint64_t)dm.N);
+        cap[idx * 2] = (int32_t)(c0 < (uint64_t)dm.N ? c0 : (uint64_t)dm.N);
+        cap[idx * 2 + 1] = (int32_t)(c1 < (uint64_t)dm.N ? c1 : (uint64_t)dm.N);
+        const double tc = __ull2double_rn(prof[kBlkFlops * V + v]) / rate[d];
+        const double tm = __ull2double_rn(prof[kBlkBytes * V + v]) / bw[d];
+        cpb[idx] = tc >= tm ? tc : tm;
+    }
+}
+
 // tau_v(a, b) = A_v / (B(a,b) * congestion(a,b)) (Sec. 3.2).
 __global__ void tau_kernel(Dims dm, const double *link_bw, const double *cong, const uint64_t *prof,
                            double *tau)
@@ -168,68 +190,48 @@ __device__ __forceinline__ bool elite_before(int da, double wa, double pa, int a
 
 // A genome equal to a lower-indexed one is a duplicate.  Equal genomes have
 // equal fitness (the evaluation is deterministic) and equal fingerprints, so
-// only those pairs are compared in full.
+// only those pairs are compared in full.  One warp per genome: lanes scan the
+// lower indices 32 at a time and compare candidates' genes lane-parallel.
 __global__ void __launch_bounds__(256) dup_kernel(Dims dm, DevPop p, const double *fit,
                                                   const uint64_t *hash, int32_t *dup)
 {
-    __shared__ double s_w[256], s_p[256];
-    __shared__ uint64_t s_h[256];
-    const int g = blockIdx.x * blockDim.x + threadIdx.x;
-    const bool live = g < dm.P;
-    const double w = live ? fit[(size_t)g * 4] : 0.0, ph = live ? fit[(size_t)g * 4 + 1] : 0.0;
-    const uint64_t h = live ? hash[g] : 0ull;
+    const int g = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    if (g >= dm.P) return;
+    const double w = fit[(size_t)g * 4], ph = fit[(size_t)g * 4 + 1];
+    const uint64_t h = hash[g];
+    const int M = dm.M, K = dm.K;
     int d = 0;
-    const int gmax = min(dm.P, (int)(blockIdx.x + 1) * (int)blockDim.x);
-    for (int base = 0; base < gmax; base += blockDim.x) {
-        const int hidx = base + threadIdx.x;
-        if (hidx < dm.P) {
-            s_w[threadIdx.x] = fit[(size_t)hidx * 4];
-            s_p[threadIdx.x] = fit[(size_t)hidx * 4 + 1];
-            s_h[threadIdx.x] = hash[hidx];
+    for (int base = 0; base < g && !d; base += 32) {
+        const int o = base + lane;
+        const bool cand = o < g && hash[o] == h && fit[(size_t)o * 4] == w && fit[(size_t)o * 4 + 1] == ph;
+        unsigned b = __ballot_sync(0xFFFFFFFFu, cand);
+        while (b && !d) {
+            const int oo = base + __ffs(b) - 1;
+            b &= b - 1;
+            bool diff = p.nclus[oo] != p.nclus[g] || p.roles[oo] != p.roles[g];
+            for (int i = lane; i < M && !diff; i += 32) diff = p.perm[(size_t)oo * M + i] != p.perm[(size_t)g * M + i];
+            for (int i = lane; i < K && !diff; i += 32) diff = p.sizes[(size_t)oo * K + i] != p.sizes[(size_t)g * K + i];
+            d = __ballot_sync(0xFFFFFFFFu, diff) == 0u;
         }
-        __syncthreads();
-        if (live && !d) {
-            const int lim = min((int)blockDim.x, g - base);
-            for (int t = 0; t < lim && !d; ++t) {
-                if (s_h[t] != h || s_w[t] != w || s_p[t] != ph) continue;
-                const int o = base + t;
-                bool eq = p.nclus[o] == p.nclus[g] && p.roles[o] == p.roles[g];
-                for (int i = 0; i < dm.M && eq; ++i) eq = p.perm[(size_t)o * dm.M + i] == p.perm[(size_t)g * dm.M + i];
-                for (int i = 0; i < dm.K && eq; ++i) eq = p.sizes[(size_t)o * dm.K + i] == p.sizes[(size_t)g * dm.K + i];
-                d = eq;
-            }
-        }
-        __syncthreads();
     }
-    if (live) dup[g] = d;
+    if (lane == 0) dup[g] = d;
 }
 
-// rank(g) = number of genomes before g in the elite order; the first Q ranks
-// are the elites.
+// rank(g) = number of genomes before g in the elite order (duplicate flag,
+// w, phase, index); the first Q ranks are the elites.  One warp per genome.
 __global__ void __launch_bounds__(256) rank_kernel(Dims dm, const double *fit, const int32_t *dup,
                                                    int32_t *elite, double *elite_fit)
 {
-    __shared__ double s_w[256], s_p[256];
-    __shared__ int s_d[256];
-    const int g = blockIdx.x * blockDim.x + threadIdx.x;
-    const bool live = g < dm.P;
-    const double w = live ? fit[(size_t)g * 4] : 0.0, ph = live ? fit[(size_t)g * 4 + 1] : 0.0;
-    const int dg = live ? dup[g] : 0;
+    const int g = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    if (g >= dm.P) return;
+    const double w = fit[(size_t)g * 4], ph = fit[(size_t)g * 4 + 1];
+    const int dg = dup[g];
     int rank = 0;
-    for (int base = 0; base < dm.P; base += blockDim.x) {
-        const int hidx = base + threadIdx.x;
-        if (hidx < dm.P) {
-            s_w[threadIdx.x] = fit[(size_t)hidx * 4];
-            s_p[threadIdx.x] = fit[(size_t)hidx * 4 + 1];
-            s_d[threadIdx.x] = dup[hidx];
-        }
-        __syncthreads();
-        const int lim = min((int)blockDim.x, dm.P - base);
-        if (live)
-            for (int t = 0; t < lim; ++t) rank += elite_before(s_d[t], s_w[t], s_p[t], base + t, dg, w, ph, g);
-        __syncthreads();
-    }
-    if (live && rank < dm.Q) {
+    for (int o = lane; o < dm.P; o += 32)
+        rank += elite_before(dup[o], fit[(size_t)o * 4], fit[(size_t)o * 4 + 1], o, dg, w, ph, g);
+#pragma unroll
+    for (int x = 16; x; x >>= 1) rank += __shfl_xor_sync(0xFFFFFFFFu, rank, x);
+    if (lane == 0 && rank < dm.Q) {
         elite[rank] = g;
         for (int q = 0; q < 4; ++q) elite_fit[(size_t)rank * 4 + q] = fit[(size_t)g * 4 + q];
     }
@@ -346,6 +348,8 @@ cudaError_t launch_tables(const e2_ctx *c)
 {
     const size_t total = (size_t)c->dm.V * c->dm.M * 2 * c->dm.LS;
     tables_kernel<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm, c->rate, c->bw, c->mem, c->prof, c->leaf);
+    const size_t vm = (size_t)c->dm.V * c->dm.M;
+    captab_kernel<<<grid_for(vm, 256), 256, 0, c->stream>>>(c->dm, c->rate, c->bw, c->mem, c->prof, c->cap, c->cpb);
     return cudaGetLastError();
 }
 
@@ -377,7 +381,7 @@ cudaError_t launch_init(const e2_ctx *c, const DevPop &p, uint64_t seed)
 
 cudaError_t launch_elites(const e2_ctx *c, const DevPop &p)
 {
-    const unsigned blocks = (c->dm.P + 255) / 256;
+    const unsigned blocks = (unsigned)(((size_t)c->dm.P * 32 + 255) / 256);
     dup_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, p, c->fit, c->hash, c->dup);
     if (c->dm.Q > 0) rank_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, c->fit, c->dup, c->elite, c->elite_fit);
     return cudaGetLastError();

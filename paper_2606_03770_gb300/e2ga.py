@@ -53,7 +53,7 @@ class e2_partitions(C.Structure):
 
 class e2_stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in ("genomes", "replicas", "dp_runs", "dp_cells", "dp_probes",
-                                         "paper_candidates", "prechecked", "served")]
+                                         "paper_candidates", "prechecked", "served", "tps_pruned")]
 
 
 # name -> (restype, argtypes); the exported surface of include/e2ga.h
