@@ -141,7 +141,8 @@ typedef struct {
     uint64_t dp_cells;          /* DP cells D_mu(i,k) computed                  */
     uint64_t dp_probes;         /* split-point probes over all cells            */
     uint64_t paper_candidates;  /* (mu,k,i,j) candidates Alg. 1 would examine   */
-    uint64_t prechecked;        /* variants rejected by the memory count check  */
+    uint64_t prechecked;        /* variants rejected by the memory count check
+                                   (over each replica's whole sweep)            */
     uint64_t served;            /* replicas that can serve                      */
     uint64_t tps_pruned;        /* decode variants a latency lower bound proved
                                    to miss Min_TPS (their DP is skipped)        */
@@ -165,7 +166,9 @@ size_t e2_workspace_bytes(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_
  * return a context bound to `stream` (a cudaStream_t; NULL = legacy default)
  * and to the current device.  The caller keeps ownership of every input and
  * of the workspace.  Synchronises the stream.  Errors: E2_EINVAL for any
- * invalid value, E2_ENOMEM for a short workspace, E2_ECUDA. */
+ * invalid value, for min(M, N) > 256 (a replica's DP holds at most 256
+ * devices) or when the largest replica's DP exceeds shared memory;
+ * E2_ENOMEM for a short workspace; E2_ECUDA. */
 int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_profile *prof,
               const e2_params *prm, void *workspace, size_t workspace_bytes, void *stream,
               e2_ctx **out);

@@ -88,7 +88,7 @@ size_t dp_smem_bytes(int M, int N, int threads)
     const int mmax = M < N ? M : N;
     for (int m = 1; m <= mmax; ++m) {
         const size_t W = (size_t)(N - m + 1);
-        const size_t u64s = 4 * (size_t)m * W + (size_t)(NW + 1) * W + 2 * (size_t)m;
+        const size_t u64s = 4 * (size_t)m * W + (size_t)(NW + 1) * W + (size_t)m;
         const size_t bytes = u64s * 8 + (size_t)m * (3 * sizeof(int)) + (size_t)m * sizeof(uint16_t) + 16;
         if (bytes > best) best = bytes;
     }
@@ -102,29 +102,115 @@ __device__ __forceinline__ void bar_named(int id, int nthreads)
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-// Estimated work of one (genome, replica slot), for heavy-first ordering:
-// 0 = empty slot, 1 = more devices than blocks, else a log-scale bucket of
-// m * W * (number of variants the replica may sweep).
-__device__ __forceinline__ int work_key(const Dims &dm, const DevPop &pop, int slot)
+__device__ __forceinline__ double warp_sum_d(double x)
 {
-    const int g = slot / dm.K, c = slot - g * dm.K;
-    if (c >= pop.nclus[g]) return 0;
-    const int m = pop.sizes[slot];
-    if (m > dm.N) return 1;
-    const int W = dm.N - m + 1;
-    const int nv = ((pop.roles[g] >> c) & 1ull) ? dm.b_max : 1;
-    const float est = (float)m * (float)W * (float)nv;
-    const int key = 2 + (int)(8.0f * __log2f(1.0f + est));
-    return key < kOrderBins - 1 ? key : kOrderBins - 1;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
+    return x;
 }
 
 }  // namespace
 
-__global__ void order_hist_kernel(Dims dm, DevPop pop, unsigned *bins)
+// Pre-pass, one warp per (genome, replica slot): the replica's offset in the
+// ordering chromosome, and the set of variants worth a DP run (bit i = variant
+// 0 for a prefill replica, variant i+1 for a decode replica):
+//  * memory: with identical blocks a partition with master mu exists iff every
+//    device holds >= 1 block and the capacities, capped at W = N - m + 1, add
+//    up to N (exact);
+//  * decode latency: Lambda >= sum of link times + sum_k n_k c_k (c_k the
+//    per-block time, the head only adds), whose least value puts one block on
+//    each device and the other N - m on the cheapest devices up to their
+//    capacity.  A variant whose bound misses Min_TPS fails whatever partition
+//    the DP returns; the 1e-9 margin exceeds the rounding of every sum here.
+// Also a heavy-first ordering key: 0 empty slot, 1 nothing to run, else a
+// log-scale bucket of m * W * (variants to run).
+__global__ void __launch_bounds__(128) variant_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si, unsigned *bins,
+                                                      unsigned long long *stats)
 {
-    const int total = dm.P * dm.K;
-    for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < total; s += gridDim.x * blockDim.x)
-        atomicAdd(&bins[work_key(dm, pop, s)], 1u);
+    __shared__ uint16_t s_dev[4][kMaxReplicaDevices];
+    __shared__ int s_c0[4][kMaxReplicaDevices], s_c1[4][kMaxReplicaDevices];
+    __shared__ uint64_t s_cb[4][kMaxReplicaDevices];
+    const int slot = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    const int K = dm.K, M = dm.M, N = dm.N;
+    if (slot >= dm.P * K) return;
+    const int g = slot / K, c = slot - g * K;
+    const int R = pop.nclus[g];
+    int key = 0, off = 0, n_mem = 0, n_lat = 0;
+    uint64_t mask = 0;
+    if (c < R) {
+        const uint16_t *sz = pop.sizes + (size_t)g * K;
+        off = warp_sum(lane < c ? sz[lane] : 0) + warp_sum(lane + 32 < c ? sz[lane + 32] : 0);
+        const int m = sz[c];
+        const int role = (int)((pop.roles[g] >> c) & 1ull);
+        key = 1;
+        if (m <= N) {
+            const int W = N - m + 1;
+            const int wl = threadIdx.x >> 5;
+            uint16_t *sdev = s_dev[wl];
+            int *sc0 = s_c0[wl], *sc1 = s_c1[wl];
+            uint64_t *scb = s_cb[wl];      // per-block times as order-preserving keys
+            const uint16_t *devs = pop.perm + (size_t)g * M + off;
+            for (int k = lane; k < m; k += 32) sdev[k] = devs[k];
+            __syncwarp();
+            const int nv = role ? dm.b_max : 1;
+            for (int i = 0; i < nv; ++i) {
+                const int v = role ? i + 1 : 0;
+                const int32_t *cap = tb.cap + (size_t)v * M * 2;
+                int s0 = 0, z = 0;
+                for (int k = lane; k < m; k += 32) {
+                    const int d = sdev[k];
+                    const int c0 = min(cap[d * 2], W), c1 = min(cap[d * 2 + 1], W);
+                    sc0[k] = c0;
+                    sc1[k] = c1;
+                    s0 += c0;
+                    z += c0 == 0;
+                }
+                s0 = warp_sum(s0);
+                z = warp_sum(z);
+                __syncwarp();
+                bool ok = false;
+                for (int k = lane; k < m && !ok; k += 32)
+                    ok = (z - (sc0[k] == 0)) == 0 && sc1[k] >= 1 && s0 - sc0[k] + sc1[k] >= N;
+                if (!__any_sync(0xFFFFFFFFu, ok)) { ++n_mem; continue; }
+                if (role && dm.min_tps > 0.0) {
+                    const double *cpb = tb.cpb + (size_t)v * M;
+                    const double *tau = tb.tau + (size_t)v * M * M;
+                    for (int k = lane; k < m; k += 32) scb[k] = dkey(cpb[sdev[k]]);
+                    __syncwarp();
+                    double part = 0.0;
+                    for (int k = lane; k < m; k += 32) {
+                        const uint64_t ck = scb[k];
+                        long long before = 0;            // capacity of the cheaper devices
+                        for (int j = 0; j < m; ++j) {
+                            const uint64_t cj = scb[j];
+                            if (cj < ck || (cj == ck && j < k)) before += sc0[j] - 1;
+                        }
+                        const long long ek = sc0[k] - 1;
+                        const long long room = (long long)(N - m) - before;
+                        const long long take = room <= 0 ? 0 : (room < ek ? room : ek);
+                        part += keyd(ck) * (double)(1 + take);
+                        if (k >= 1) part += tau[(size_t)sdev[k - 1] * M + sdev[k]];
+                    }
+                    const double lb = warp_sum_d(part) * (1.0 - 1e-9);
+                    if (lb > 0.0 && 1.0 / lb < dm.min_tps) { ++n_lat; continue; }
+                }
+                mask |= 1ull << i;
+            }
+            if (mask) {
+                const float est = (float)m * (float)W * (float)__popcll(mask);
+                const int k2 = 2 + (int)(8.0f * __log2f(1.0f + est));
+                key = k2 < kOrderBins - 1 ? k2 : kOrderBins - 1;
+            }
+        }
+    }
+    if (lane == 0) {
+        si.off[slot] = off;
+        si.mask[slot] = mask;
+        si.key[slot] = (uint8_t)key;
+        atomicAdd(&bins[key], 1u);
+        if (n_mem) atomicAdd(&stats[kStPrecheck], (unsigned long long)n_mem);
+        if (n_lat) atomicAdd(&stats[kStTpsPruned], (unsigned long long)n_lat);
+    }
 }
 
 // Exclusive scan of the bins in descending key order (heaviest first).
@@ -146,11 +232,10 @@ __global__ void order_scan_kernel(unsigned *bins)
     bins[kOrderBins - 1 - t] = incl - cnt;
 }
 
-__global__ void order_scatter_kernel(Dims dm, DevPop pop, unsigned *cursor, int *order)
+__global__ void order_scatter_kernel(int total, const uint8_t *keys, unsigned *cursor, int *order)
 {
-    const int total = dm.P * dm.K;
     for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < total; s += gridDim.x * blockDim.x)
-        order[atomicAdd(&cursor[work_key(dm, pop, s)], 1u)] = s;
+        order[atomicAdd(&cursor[keys[s]], 1u)] = s;
 }
 
 // One CTA per (genome, replica slot), heaviest first.  Per variant:
@@ -171,7 +256,7 @@ __global__ void order_scatter_kernel(Dims dm, DevPop pop, unsigned *cursor, int 
 // Every value is a min/max of the same leaf and link times the oracle uses,
 // so V, mu*, the partition and Lambda are bit-identical to Alg. 1.
 __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out,
-                                                      const int *order)
+                                                      const int *order, SlotInfo si)
 {
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ int s_off, s_m, s_role, s_S0, s_Z, s_mu, s_done;
@@ -185,29 +270,23 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
     const int g = slot / K, c = slot - g * K;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
     const size_t gk = (size_t)g * K + c;
-    const int R = pop.nclus[g];
-    if (c >= R) {
+    if (c >= pop.nclus[g]) {
         if (tid == 0) {
             out.master[gk] = -1; out.bsel[gk] = -1;
             out.T[gk] = keyd(kInfKey); out.L[gk] = keyd(kInfKey);
         }
         return;
     }
-    if (tid == 0) {
-        int off = 0;
-        for (int q = 0; q < c; ++q) off += pop.sizes[(size_t)g * K + q];
-        s_off = off;
-        s_m = pop.sizes[gk];
-        s_role = (int)((pop.roles[g] >> c) & 1ull);
-    }
-    __syncthreads();
-    const int off = s_off, m = s_m, role = s_role;
+    const int off = si.off[slot], m = pop.sizes[gk];
+    const int role = (int)((pop.roles[g] >> c) & 1ull);
+    uint64_t vmask = si.mask[slot];
     int16_t *lay_out = out.layers + (size_t)g * M + off;
 
-    unsigned long long st_runs = 0, st_cells = 0, st_probes = 0, st_paper = 0, st_pre = 0, st_tps = 0;
+    unsigned long long st_runs = 0, st_cells = 0, st_probes = 0;
     bool served = false;
+    int served_v = -1;
 
-    if (m <= N) {
+    if (m <= N && vmask) {
         const int W = N - m + 1;
         uint64_t *leaf0 = reinterpret_cast<uint64_t *>(smem);   // [m][W] l_k(n)
         uint64_t *leaf1 = leaf0 + (size_t)m * W;                // [m][W] l_k^head(n)
@@ -216,8 +295,7 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
         uint64_t *Hb = Gst + (size_t)m * W;                     // [NW][W] per-warp convolution
         uint64_t *delta = Hb + (size_t)NW * W;                  // [W] the empty stage
         uint64_t *tauk = delta + W;                             // [m] tauk[k] = link (k-1) -> k
-        double *cpbk = reinterpret_cast<double *>(tauk + m);    // [m] per-block times
-        int *cnt0 = reinterpret_cast<int *>(cpbk + m);          // [m]
+        int *cnt0 = reinterpret_cast<int *>(tauk + m);          // [m]
         int *cnt1 = cnt0 + m;                                   // [m]
         int *nk = cnt1 + m;                                     // [m]
         uint16_t *devs = reinterpret_cast<uint16_t *>(nk + m);  // [m]
@@ -234,25 +312,28 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             return k == m + 1 ? delta : k == m ? leaf0 + (size_t)(m - 1) * W : Gst + (size_t)(k - 1) * W;
         };
 
-        const int nvar = role ? dm.b_max : 1;
-        const unsigned long long pc = paper_candidates(m, N);
         const unsigned long long cprobe = column_probes(W);
         const unsigned long long lprobe = 32 - __clz(W);
-        for (int vi = 0; vi < nvar && !served; ++vi) {
-            const int v = role ? dm.b_max - vi : 0;
-            // ---- 1. capacities, per-block times and link times of this variant
+        while (vmask && !served) {
+            const int bit = 63 - __clzll((long long)vmask);          // highest batch first
+            vmask &= ~(1ull << bit);
+            const int v = role ? bit + 1 : 0;
+            // ---- 1. capacities, link times and cost rows of this variant
             for (int k = tid; k < m; k += blockDim.x) {
                 const size_t vd = (size_t)v * M + devs[k];
                 const int c0 = tb.cap[vd * 2], c1 = tb.cap[vd * 2 + 1];
                 cnt0[k] = c0 < W ? c0 : W;
                 cnt1[k] = c1 < W ? c1 : W;
-                cpbk[k] = tb.cpb[vd];
                 tauk[k] = k ? dkey(tb.tau[((size_t)v * M + devs[k - 1]) * M + devs[k]]) : 0ull;
             }
+            for (int e = tid; e < m * W; e += blockDim.x) {
+                const int k = e / W, n = e - k * W;
+                const double *base = tb.leaf + ((size_t)v * M + devs[k]) * 2 * dm.LS;
+                leaf0[e] = dkey(base[n]);
+                leaf1[e] = dkey(base[dm.LS + n]);
+            }
             __syncthreads();
-            // ---- 2. exact memory check: with identical blocks a partition with
-            // master mu exists iff every device holds >= 1 block and the block
-            // capacities (capped at W) add up to N
+            // ---- 2. masters the memory allows (the pre-pass guarantees one)
             if (wid == 0) {
                 int s = 0, z = 0;
                 for (int k = lane; k < m; k += 32) { s += cnt0[k]; z += cnt0[k] == 0; }
@@ -265,53 +346,6 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
                 const int k = mu - 1;
                 return (Z - (cnt0[k] == 0)) == 0 && cnt1[k] >= 1 && S0 - cnt0[k] + cnt1[k] >= N;
             };
-            int any = 0;
-            for (int mu = tid + 1; mu <= m; mu += blockDim.x) any |= mu_ok(mu);
-            any = __syncthreads_or(any);
-            st_paper += pc;
-            if (!any) { ++st_pre; continue; }
-            // ---- 2b. decode: a lower bound on Lambda over every feasible
-            // partition.  Lambda = sum of link times + sum_k l_k(n_k) with
-            // l_k(n) >= n * c_k (c_k the per-block time; the head only adds), and
-            // sum_k n_k c_k is least when each device takes one block and the
-            // other N - m go to the cheapest devices up to their capacity.  If
-            // even that bound misses Min_TPS the variant fails whatever the DP
-            // returns, so its DP is skipped; the 1e-9 margin exceeds the
-            // rounding of every sum involved, so no passing variant is lost.
-            if (role) {
-                if (wid == 0) {
-                    const int Rx = N - m;
-                    double part = 0.0;
-                    for (int k = lane; k < m; k += 32) {
-                        const double ck = cpbk[k];
-                        long long before = 0;
-                        for (int j = 0; j < m; ++j) {
-                            const double cj = cpbk[j];
-                            if (cj < ck || (cj == ck && j < k)) before += cnt0[j] - 1;
-                        }
-                        const long long room = (long long)Rx - before;
-                        const long long take = room <= 0 ? 0 : (room < cnt0[k] - 1 ? room : cnt0[k] - 1);
-                        part += ck * (double)(1 + take);
-                        if (k >= 1) part += keyd(tauk[k]);
-                    }
-#pragma unroll
-                    for (int o = 16; o; o >>= 1) part += __shfl_xor_sync(0xFFFFFFFFu, part, o);
-                    if (lane == 0) {
-                        const double lb = part * (1.0 - 1e-9);
-                        s_done = lb > 0.0 && 1.0 / lb < dm.min_tps;
-                    }
-                }
-                __syncthreads();
-                if (s_done) { ++st_tps; continue; }
-            }
-            // ---- 2c. stage the cost rows
-            for (int e = tid; e < m * W; e += blockDim.x) {
-                const int k = e / W, n = e - k * W;
-                const double *base = tb.leaf + ((size_t)v * M + devs[k]) * 2 * dm.LS;
-                leaf0[e] = dkey(base[n]);
-                leaf1[e] = dkey(base[dm.LS + n]);
-            }
-            __syncthreads();
             ++st_runs;
             // ---- 3. prefix columns (warps 0-1) and suffix columns (warps 2-3)
             if (wid < 2) {
@@ -419,6 +453,7 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
                     out.L[gk] = s_L;
                 }
                 served = true;
+                served_v = v;
             }
             __syncthreads();
         }
@@ -436,11 +471,14 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
         atomicAdd(&out.stats[kStProbes], st_probes);
     }
     if (tid == 0) {
+        // candidates the plain recurrence examines for the same sweep: every
+        // variant from the top down to the accepted one (all of them if none)
+        unsigned long long nrun = 0;
+        if (m <= N) nrun = served ? (role ? (unsigned long long)(dm.b_max - served_v + 1) : 1ull)
+                                  : (role ? (unsigned long long)dm.b_max : 1ull);
         atomicAdd(&out.stats[kStReplicas], 1ull);
         if (st_runs) atomicAdd(&out.stats[kStDpRuns], st_runs);
-        if (st_paper) atomicAdd(&out.stats[kStPaper], st_paper);
-        if (st_pre) atomicAdd(&out.stats[kStPrecheck], st_pre);
-        if (st_tps) atomicAdd(&out.stats[kStTpsPruned], st_tps);
+        if (nrun) atomicAdd(&out.stats[kStPaper], nrun * paper_candidates(m, N));
         if (served) atomicAdd(&out.stats[kStServed], 1ull);
     }
 }
@@ -449,7 +487,7 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
 // serving replicas of each role in ascending replica order, then Eq. 3
 // (bottleneck phase), Eq. 4 (backlog) and Eq. 5 (waiting time).  Also a
 // 64-bit fingerprint of the genome for the elites' duplicate test.
-__global__ void __launch_bounds__(256) score_kernel(Dims dm, DevPop pop, EvalOut out)
+__global__ void __launch_bounds__(32) score_kernel(Dims dm, DevPop pop, EvalOut out)
 {
     const int g = blockIdx.x * blockDim.x + threadIdx.x;
     if (g >= dm.P) return;
@@ -497,14 +535,15 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     Tables tb{c->rate, c->bw, c->mem, c->prof, c->leaf, c->tau, c->cap, c->cpb};
     EvalOut out{c->fit, c->layers, c->master, c->bsel, c->T, c->L, c->hash, c->stats};
     const long long blocks = (long long)c->dm.P * c->dm.K;
+    SlotInfo si{c->slot_off, c->slot_mask, c->slot_key};
     cudaError_t e = cudaMemsetAsync(c->order_bins, 0, sizeof(unsigned) * kOrderBins, c->stream);
     if (e != cudaSuccess) return e;
     const unsigned gb = (unsigned)((blocks + 255) / 256 < 1024 ? (blocks + 255) / 256 : 1024);
-    order_hist_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, c->order_bins);
+    variant_kernel<<<(unsigned)((blocks * 32 + 127) / 128), 128, 0, c->stream>>>(c->dm, tb, p, si, c->order_bins, c->stats);
     order_scan_kernel<<<1, kOrderBins, 0, c->stream>>>(c->order_bins);
-    order_scatter_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, c->order_bins, c->order);
-    dp_eval_kernel<<<(unsigned)blocks, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, c->order);
-    score_kernel<<<(c->dm.P + 255) / 256, 256, 0, c->stream>>>(c->dm, p, out);
+    order_scatter_kernel<<<gb, 256, 0, c->stream>>>((int)blocks, c->slot_key, c->order_bins, c->order);
+    dp_eval_kernel<<<(unsigned)blocks, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, c->order, si);
+    score_kernel<<<(c->dm.P + 31) / 32, 32, 0, c->stream>>>(c->dm, p, out);
     return cudaGetLastError();
 }
 

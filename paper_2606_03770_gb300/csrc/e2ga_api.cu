@@ -22,7 +22,7 @@ size_t align_up(size_t x, size_t a = 256) { return (x + a - 1) / a * a; }
 struct Layout {
     size_t rate, bw, mem, link_bw, cong, prof, leaf, tau, cap, cpb;
     size_t perm[2], sizes[2], nclus[2], roles[2];
-    size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, stats, err, order_bins, order, total;
+    size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, stats, err, order_bins, order, slot_off, slot_mask, slot_key, total;
     int LS;
 };
 
@@ -70,6 +70,9 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K)
     l.err = take(4);
     l.order_bins = take(4 * kOrderBins);
     l.order = take(4 * (size_t)P * K);
+    l.slot_off = take(4 * (size_t)P * K);
+    l.slot_mask = take(8 * (size_t)P * K);
+    l.slot_key = take((size_t)P * K);
     l.total = o;
     return l;
 }
@@ -270,6 +273,8 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
         return fail_free(E2_ECUDA, "cudaDeviceGetAttribute failed");
     c->dp_threads = 128;
     c->dp_smem = dp_smem_bytes(M, N, c->dp_threads);
+    if ((M < N ? M : N) > kMaxReplicaDevices)
+        return fail_free(E2_EINVAL, "replicas could exceed 256 devices (min(M, N) > 256)");
     if (c->dp_smem + 1024 > (size_t)smem_optin)
         return fail_free(E2_EINVAL, "the largest replica's DP does not fit in shared memory (N too large)");
     if (configure_eval(c->dp_smem) != cudaSuccess) return fail_free(E2_ECUDA, "cudaFuncSetAttribute failed");
@@ -300,6 +305,9 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->err = reinterpret_cast<int32_t *>(ws + l.err);
     c->order_bins = reinterpret_cast<unsigned *>(ws + l.order_bins);
     c->order = reinterpret_cast<int *>(ws + l.order);
+    c->slot_off = reinterpret_cast<int32_t *>(ws + l.slot_off);
+    c->slot_mask = reinterpret_cast<uint64_t *>(ws + l.slot_mask);
+    c->slot_key = ws + l.slot_key;
 
     const size_t V = (size_t)b_max + 1, MM = (size_t)M * M;
     uint64_t *prof_h = new (std::nothrow) uint64_t[kNumProf * V];

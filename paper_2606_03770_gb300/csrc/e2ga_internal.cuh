@@ -32,6 +32,11 @@ struct DevPop {
     uint64_t *roles;   // [P]
 };
 
+// Largest replica (devices) a DP can receive: replicas with more devices than
+// blocks are infeasible, and the evaluation pre-pass stages up to 256 devices
+// of a replica per warp in shared memory.
+constexpr int kMaxReplicaDevices = 256;
+
 // Buckets of the heavy-first work ordering of the evaluation.
 constexpr int kOrderBins = 256;
 
@@ -56,6 +61,13 @@ struct Tables {
     const double *tau;         // [V][M][M]
     const int32_t *cap;        // [V][M][2]: most blocks device d holds (memory), without / with the head
     const double *cpb;         // [V][M]: per-block time max(blk_flops/rate, blk_bytes/bw)
+};
+
+// Per (genome, replica slot) results of the evaluation pre-pass.
+struct SlotInfo {
+    int32_t *off;              // [P*K] offset of the replica in the ordering chromosome
+    uint64_t *mask;            // [P*K] variants to run (bit i: prefill v=0 / decode v=i+1)
+    uint8_t *key;              // [P*K] heavy-first ordering key
 };
 
 struct EvalOut {
@@ -145,6 +157,9 @@ struct e2_ctx {
     int32_t *err = nullptr;
     unsigned *order_bins = nullptr;   // [kOrderBins]
     int *order = nullptr;             // [P*K] evaluation order of (genome, replica) slots
+    int32_t *slot_off = nullptr;      // [P*K]
+    uint64_t *slot_mask = nullptr;    // [P*K]
+    uint8_t *slot_key = nullptr;      // [P*K]
     // launch shapes
     int dp_threads = 128;
     size_t dp_smem = 0;

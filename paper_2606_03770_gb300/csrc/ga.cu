@@ -178,9 +178,10 @@ __global__ void init_kernel(Dims dm, DevPop p, uint64_t seed)
 }
 
 // Total order of the elites: distinct genomes before duplicates, then lower w,
-// lower bottleneck phase, lower index.
-__device__ __forceinline__ bool elite_before(int da, double wa, double pa, int a, int db, double wb,
-                                             double pb, int b)
+// lower bottleneck phase, lower index.  w and phase are non-negative or +inf,
+// so they are compared as their bit patterns (same order, integer pipe).
+__device__ __forceinline__ bool elite_before(int da, uint64_t wa, uint64_t pa, int a, int db, uint64_t wb,
+                                             uint64_t pb, int b)
 {
     if (da != db) return da < db;
     if (wa != wb) return wa < wb;
@@ -197,13 +198,14 @@ __global__ void __launch_bounds__(256) dup_kernel(Dims dm, DevPop p, const doubl
 {
     const int g = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
     if (g >= dm.P) return;
-    const double w = fit[(size_t)g * 4], ph = fit[(size_t)g * 4 + 1];
+    const uint64_t *fk = reinterpret_cast<const uint64_t *>(fit);
+    const uint64_t w = fk[(size_t)g * 4], ph = fk[(size_t)g * 4 + 1];
     const uint64_t h = hash[g];
     const int M = dm.M, K = dm.K;
     int d = 0;
     for (int base = 0; base < g && !d; base += 32) {
         const int o = base + lane;
-        const bool cand = o < g && hash[o] == h && fit[(size_t)o * 4] == w && fit[(size_t)o * 4 + 1] == ph;
+        const bool cand = o < g && hash[o] == h && fk[(size_t)o * 4] == w && fk[(size_t)o * 4 + 1] == ph;
         unsigned b = __ballot_sync(0xFFFFFFFFu, cand);
         while (b && !d) {
             const int oo = base + __ffs(b) - 1;
@@ -224,11 +226,12 @@ __global__ void __launch_bounds__(256) rank_kernel(Dims dm, const double *fit, c
 {
     const int g = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
     if (g >= dm.P) return;
-    const double w = fit[(size_t)g * 4], ph = fit[(size_t)g * 4 + 1];
+    const uint64_t *fk = reinterpret_cast<const uint64_t *>(fit);
+    const uint64_t w = fk[(size_t)g * 4], ph = fk[(size_t)g * 4 + 1];
     const int dg = dup[g];
     int rank = 0;
     for (int o = lane; o < dm.P; o += 32)
-        rank += elite_before(dup[o], fit[(size_t)o * 4], fit[(size_t)o * 4 + 1], o, dg, w, ph, g);
+        rank += elite_before(dup[o], fk[(size_t)o * 4], fk[(size_t)o * 4 + 1], o, dg, w, ph, g);
 #pragma unroll
     for (int x = 16; x; x >>= 1) rank += __shfl_xor_sync(0xFFFFFFFFu, rank, x);
     if (lane == 0 && rank < dm.Q) {
@@ -241,11 +244,14 @@ struct GaThr {
     uint64_t cx, half, mut, k1, k2, k3;
 };
 
+// Fitness order (lower w, lower phase, lower index) on the bit patterns of
+// the non-negative w and phase.
 __device__ __forceinline__ bool key_less(const double *fit, int a, int b)
 {
-    const double wa = fit[(size_t)a * 4], wb = fit[(size_t)b * 4];
+    const uint64_t *fk = reinterpret_cast<const uint64_t *>(fit);
+    const uint64_t wa = fk[(size_t)a * 4], wb = fk[(size_t)b * 4];
     if (wa != wb) return wa < wb;
-    const double pa = fit[(size_t)a * 4 + 1], pb = fit[(size_t)b * 4 + 1];
+    const uint64_t pa = fk[(size_t)a * 4 + 1], pb = fk[(size_t)b * 4 + 1];
     if (pa != pb) return pa < pb;
     return a < b;
 }
@@ -375,7 +381,7 @@ cudaError_t launch_validate(const e2_ctx *c, const DevPop &p)
 
 cudaError_t launch_init(const e2_ctx *c, const DevPop &p, uint64_t seed)
 {
-    init_kernel<<<(c->dm.P + 127) / 128, 128, 0, c->stream>>>(c->dm, p, seed);
+    init_kernel<<<(c->dm.P + 31) / 32, 32, 0, c->stream>>>(c->dm, p, seed);
     return cudaGetLastError();
 }
 
@@ -390,7 +396,7 @@ cudaError_t launch_elites(const e2_ctx *c, const DevPop &p)
 cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen)
 {
     GaThr thr{c->thr_cx, c->thr_half, c->thr_mut, c->thr_k1, c->thr_k2, c->thr_k3};
-    ga_kernel<<<(c->dm.P + 127) / 128, 128, 0, c->stream>>>(c->dm, src, dst, c->fit, c->elite, seed, gen, thr);
+    ga_kernel<<<(c->dm.P + 31) / 32, 32, 0, c->stream>>>(c->dm, src, dst, c->fit, c->elite, seed, gen, thr);
     return cudaGetLastError();
 }
 
