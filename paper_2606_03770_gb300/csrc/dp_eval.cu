@@ -38,9 +38,9 @@ namespace e2 {
 
 namespace {
 
-// D_k[r] for one cell (see the header comment).
-__device__ __forceinline__ uint64_t dp_cell(const uint64_t *__restrict__ prev,
-                                            const uint64_t *__restrict__ row, uint64_t tau, int r)
+// D_k[r] for one cell (see the header comment), on 32-bit order keys.
+__device__ __forceinline__ uint32_t dp_cell(const uint32_t *__restrict__ prev,
+                                            const uint32_t *__restrict__ row, uint32_t tau, int r)
 {
     int lo = 0, hi = r + 1;
     while (lo < hi) {
@@ -48,11 +48,19 @@ __device__ __forceinline__ uint64_t dp_cell(const uint64_t *__restrict__ prev,
         if (prev[mid] >= row[r - mid]) hi = mid;
         else lo = mid + 1;
     }
-    uint64_t h = kInfKey;
+    uint32_t h = 0xFFFFFFFFu;
     if (lo <= r) h = prev[lo];
-    if (lo >= 1) h = umin64(h, row[r - lo + 1]);
-    return umax64(h, tau);
+    if (lo >= 1) h = min(h, row[r - lo + 1]);
+    return max(h, tau);
 }
+
+__device__ __forceinline__ void cp_async4(void *smem_dst, const void *gmem_src)
+{
+    const unsigned sa = (unsigned)__cvta_generic_to_shared(smem_dst);
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(sa), "l"(gmem_src) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
 __device__ __forceinline__ int warp_sum(int x)
 {
@@ -88,8 +96,8 @@ size_t dp_smem_bytes(int M, int N, int threads)
     const int mmax = M < N ? M : N;
     for (int m = 1; m <= mmax; ++m) {
         const size_t W = (size_t)(N - m + 1);
-        const size_t u64s = 4 * (size_t)m * W + (size_t)(NW + 1) * W + (size_t)m;
-        const size_t bytes = u64s * 8 + (size_t)m * (3 * sizeof(int)) + (size_t)m * sizeof(uint16_t) + 16;
+        const size_t u32s = 3 * (size_t)m * W + (size_t)(2 * NW + 2) * W + (size_t)m;
+        const size_t bytes = u32s * 4 + (size_t)m * (3 * sizeof(int)) + (size_t)m * sizeof(uint16_t) + 16;
         if (bytes > best) best = bytes;
     }
     return (best + 15) & ~(size_t)15;
@@ -111,9 +119,9 @@ __device__ __forceinline__ double warp_sum_d(double x)
 
 }  // namespace
 
-// Pre-pass, one warp per (genome, replica slot): the replica's offset in the
-// ordering chromosome, and the set of variants worth a DP run (bit i = variant
-// 0 for a prefill replica, variant i+1 for a decode replica):
+// Pre-pass, one warp per (genome, replica slot, variant): whether the variant
+// is worth a DP run (bit i of the slot's mask: variant 0 of a prefill
+// replica, variant i+1 of a decode replica):
 //  * memory: with identical blocks a partition with master mu exists iff every
 //    device holds >= 1 block and the capacities, capped at W = N - m + 1, add
 //    up to N (exact);
@@ -122,98 +130,135 @@ __device__ __forceinline__ double warp_sum_d(double x)
 //    each device and the other N - m on the cheapest devices up to their
 //    capacity.  A variant whose bound misses Min_TPS fails whatever partition
 //    the DP returns; the 1e-9 margin exceeds the rounding of every sum here.
-// Also a heavy-first ordering key: 0 empty slot, 1 nothing to run, else a
-// log-scale bucket of m * W * (variants to run).
-__global__ void __launch_bounds__(128) variant_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si, unsigned *bins,
+// The variant-0 warp also records the replica's offset in the ordering.
+__global__ void __launch_bounds__(128) variant_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si,
                                                       unsigned long long *stats)
 {
     __shared__ uint16_t s_dev[4][kMaxReplicaDevices];
     __shared__ int s_c0[4][kMaxReplicaDevices], s_c1[4][kMaxReplicaDevices];
     __shared__ uint64_t s_cb[4][kMaxReplicaDevices];
-    const int slot = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    const long long wg = (long long)((blockIdx.x * (size_t)blockDim.x + threadIdx.x) >> 5);
+    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
     const int K = dm.K, M = dm.M, N = dm.N;
-    if (slot >= dm.P * K) return;
+    if (wg >= (long long)dm.P * K * dm.b_max) return;
+    const int slot = (int)(wg / dm.b_max), i = (int)(wg - (long long)slot * dm.b_max);
     const int g = slot / K, c = slot - g * K;
-    const int R = pop.nclus[g];
-    int key = 0, off = 0, n_mem = 0, n_lat = 0;
-    uint64_t mask = 0;
-    if (c < R) {
-        const uint16_t *sz = pop.sizes + (size_t)g * K;
-        off = warp_sum(lane < c ? sz[lane] : 0) + warp_sum(lane + 32 < c ? sz[lane + 32] : 0);
-        const int m = sz[c];
-        const int role = (int)((pop.roles[g] >> c) & 1ull);
-        key = 1;
-        if (m <= N) {
-            const int W = N - m + 1;
-            const int wl = threadIdx.x >> 5;
-            uint16_t *sdev = s_dev[wl];
-            int *sc0 = s_c0[wl], *sc1 = s_c1[wl];
-            uint64_t *scb = s_cb[wl];      // per-block times as order-preserving keys
-            const uint16_t *devs = pop.perm + (size_t)g * M + off;
-            for (int k = lane; k < m; k += 32) sdev[k] = devs[k];
-            __syncwarp();
-            const int nv = role ? dm.b_max : 1;
-            for (int i = 0; i < nv; ++i) {
-                const int v = role ? i + 1 : 0;
-                const int32_t *cap = tb.cap + (size_t)v * M * 2;
-                int s0 = 0, z = 0;
-                for (int k = lane; k < m; k += 32) {
-                    const int d = sdev[k];
-                    const int c0 = min(cap[d * 2], W), c1 = min(cap[d * 2 + 1], W);
-                    sc0[k] = c0;
-                    sc1[k] = c1;
-                    s0 += c0;
-                    z += c0 == 0;
-                }
-                s0 = warp_sum(s0);
-                z = warp_sum(z);
-                __syncwarp();
-                bool ok = false;
-                for (int k = lane; k < m && !ok; k += 32)
-                    ok = (z - (sc0[k] == 0)) == 0 && sc1[k] >= 1 && s0 - sc0[k] + sc1[k] >= N;
-                if (!__any_sync(0xFFFFFFFFu, ok)) { ++n_mem; continue; }
-                if (role && dm.min_tps > 0.0) {
-                    const double *cpb = tb.cpb + (size_t)v * M;
-                    const double *tau = tb.tau + (size_t)v * M * M;
-                    for (int k = lane; k < m; k += 32) scb[k] = dkey(cpb[sdev[k]]);
-                    __syncwarp();
-                    double part = 0.0;
-                    for (int k = lane; k < m; k += 32) {
-                        const uint64_t ck = scb[k];
-                        long long before = 0;            // capacity of the cheaper devices
-                        for (int j = 0; j < m; ++j) {
-                            const uint64_t cj = scb[j];
-                            if (cj < ck || (cj == ck && j < k)) before += sc0[j] - 1;
-                        }
-                        const long long ek = sc0[k] - 1;
-                        const long long room = (long long)(N - m) - before;
-                        const long long take = room <= 0 ? 0 : (room < ek ? room : ek);
-                        part += keyd(ck) * (double)(1 + take);
-                        if (k >= 1) part += tau[(size_t)sdev[k - 1] * M + sdev[k]];
-                    }
-                    const double lb = warp_sum_d(part) * (1.0 - 1e-9);
-                    if (lb > 0.0 && 1.0 / lb < dm.min_tps) { ++n_lat; continue; }
-                }
-                mask |= 1ull << i;
+    if (c >= pop.nclus[g]) return;
+    const uint16_t *sz = pop.sizes + (size_t)g * K;
+    const int m = sz[c];
+    const int role = (int)((pop.roles[g] >> c) & 1ull);
+    if (!role && i > 0) return;
+    const int off = warp_sum(lane < c ? sz[lane] : 0) + warp_sum(lane + 32 < c ? sz[lane + 32] : 0);
+    if (i == 0 && lane == 0) si.off[slot] = off;
+    if (m > N) return;
+    const int W = N - m + 1;
+    const int v = role ? i + 1 : 0;
+    uint16_t *sdev = s_dev[wl];
+    int *sc0 = s_c0[wl], *sc1 = s_c1[wl];
+    uint64_t *scb = s_cb[wl];                                    // per-block times as order keys
+    const uint16_t *devs = pop.perm + (size_t)g * M + off;
+    const int32_t *cap = tb.cap + (size_t)v * M * 2;
+    int s0 = 0, z = 0;
+    for (int k = lane; k < m; k += 32) {
+        const int d = devs[k];
+        sdev[k] = (uint16_t)d;
+        const int c0 = min(cap[d * 2], W), c1 = min(cap[d * 2 + 1], W);
+        sc0[k] = c0;
+        sc1[k] = c1;
+        s0 += c0;
+        z += c0 == 0;
+    }
+    s0 = warp_sum(s0);
+    z = warp_sum(z);
+    __syncwarp();
+    bool ok = false;
+    for (int k = lane; k < m && !ok; k += 32)
+        ok = (z - (sc0[k] == 0)) == 0 && sc1[k] >= 1 && s0 - sc0[k] + sc1[k] >= N;
+    if (!__any_sync(0xFFFFFFFFu, ok)) {
+        if (lane == 0) atomicAdd(&stats[kStPrecheck], 1ull);
+        return;
+    }
+    if (role && dm.min_tps > 0.0) {
+        const double *cpb = tb.cpb + (size_t)v * M;
+        const double *tau = tb.tau + (size_t)v * M * M;
+        for (int k = lane; k < m; k += 32) scb[k] = dkey(cpb[sdev[k]]);
+        __syncwarp();
+        double part = 0.0;
+        for (int k = lane; k < m; k += 32) {
+            const uint64_t ck = scb[k];
+            long long before = 0;            // capacity of the cheaper devices
+            for (int j = 0; j < m; ++j) {
+                const uint64_t cj = scb[j];
+                if (cj < ck || (cj == ck && j < k)) before += sc0[j] - 1;
             }
-            if (mask) {
-                const float est = (float)m * (float)W * (float)__popcll(mask);
-                const int k2 = 2 + (int)(8.0f * __log2f(1.0f + est));
-                key = k2 < kOrderBins - 1 ? k2 : kOrderBins - 1;
-            }
+            const long long ek = sc0[k] - 1;
+            const long long room = (long long)(N - m) - before;
+            const long long take = room <= 0 ? 0 : (room < ek ? room : ek);
+            part += keyd(ck) * (double)(1 + take);
+            if (k >= 1) part += tau[(size_t)sdev[k - 1] * M + sdev[k]];
+        }
+        const double lb = warp_sum_d(part) * (1.0 - 1e-9);
+        if (lb > 0.0 && 1.0 / lb < dm.min_tps) {
+            if (lane == 0) atomicAdd(&stats[kStTpsPruned], 1ull);
+            return;
         }
     }
-    if (lane == 0) {
-        si.off[slot] = off;
-        si.mask[slot] = mask;
-        si.key[slot] = (uint8_t)key;
-        atomicAdd(&bins[key], 1u);
-        if (n_mem) atomicAdd(&stats[kStPrecheck], (unsigned long long)n_mem);
-        if (n_lat) atomicAdd(&stats[kStTpsPruned], (unsigned long long)n_lat);
+    if (lane == 0) atomicOr(reinterpret_cast<unsigned long long *>(&si.mask[slot]), 1ull << i);
+}
+
+// Writes the outputs of a replica that cannot serve.
+__device__ __forceinline__ void write_unserved(const EvalOut &out, size_t gk, int16_t *lay, int m)
+{
+    for (int k = 0; k < m; ++k) lay[k] = -1;
+    out.master[gk] = -1; out.bsel[gk] = -1;
+    out.T[gk] = keyd(kInfKey); out.L[gk] = keyd(kInfKey);
+}
+
+// Per slot: slots with nothing to run get their outputs here (empty slots,
+// more devices than blocks, no variant left by the pre-pass).  Every other
+// slot contributes one work item per variant to run; items are ordered by
+// level (the variant's rank among its replica's variants, largest batch
+// first), then by work size (m * W, log scale), largest first.  A replica's
+// smaller batches thus come after every replica's larger ones, by which time
+// the larger batch has usually been decided: a variant below an accepted one
+// is skipped, as the sequential sweep of Alg. 2 would.
+__device__ __forceinline__ int item_bin(int level, int size)
+{
+    const int lv = level < 63 ? level : 63;
+    return (63 - lv) * kSizeBins + size;
+}
+
+__global__ void key_kernel(Dims dm, DevPop pop, SlotInfo si, EvalOut out, unsigned *bins)
+{
+    const int total = dm.P * dm.K;
+    for (int slot = blockIdx.x * blockDim.x + threadIdx.x; slot < total; slot += gridDim.x * blockDim.x) {
+        const int g = slot / dm.K, c = slot - g * dm.K;
+        si.best[slot] = -1;
+        if (c >= pop.nclus[g]) {
+            out.master[slot] = -1; out.bsel[slot] = -1;
+            out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
+            continue;
+        }
+        const uint64_t mask = si.mask[slot];
+        const int m = pop.sizes[slot];
+        if (!mask) {
+            const int role = (int)((pop.roles[g] >> c) & 1ull);
+            write_unserved(out, slot, out.layers + (size_t)g * dm.M + si.off[slot], m);
+            atomicAdd(&out.stats[kStReplicas], 1ull);
+            if (m <= dm.N) atomicAdd(&out.stats[kStPaper], (role ? dm.b_max : 1) * paper_candidates(m, dm.N));
+            continue;
+        }
+        const int W = dm.N - m + 1;
+        const int sz = (int)(1.0f * __log2f(1.0f + (float)m * (float)W));
+        const int size = sz < kSizeBins - 1 ? sz : kSizeBins - 1;
+        si.size[slot] = (uint8_t)size;
+        const int nv = __popcll(mask);
+        for (int lv = 0; lv < nv; ++lv) atomicAdd(&bins[item_bin(lv, size)], 1u);
     }
 }
 
-// Exclusive scan of the bins in descending key order (heaviest first).
+// Exclusive scan of the bins in descending key order (heaviest first); the
+// total number of work items goes to bins[kOrderBins].
 __global__ void order_scan_kernel(unsigned *bins)
 {
     __shared__ unsigned s[kOrderBins];
@@ -230,17 +275,31 @@ __global__ void order_scan_kernel(unsigned *bins)
     const unsigned cnt = bins[kOrderBins - 1 - t];
     __syncthreads();
     bins[kOrderBins - 1 - t] = incl - cnt;
+    if (t == kOrderBins - 1) { bins[kOrderBins] = incl; bins[kOrderBins + 1] = 0u; }
 }
 
-__global__ void order_scatter_kernel(int total, const uint8_t *keys, unsigned *cursor, int *order)
+__global__ void order_scatter_kernel(Dims dm, DevPop pop, SlotInfo si, WorkList wl)
 {
-    for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < total; s += gridDim.x * blockDim.x)
-        order[atomicAdd(&cursor[keys[s]], 1u)] = s;
+    const int total = dm.P * dm.K;
+    for (int slot = blockIdx.x * blockDim.x + threadIdx.x; slot < total; slot += gridDim.x * blockDim.x) {
+        const int g = slot / dm.K, c = slot - g * dm.K;
+        if (c >= pop.nclus[g]) continue;
+        uint64_t mask = si.mask[slot];
+        const int size = si.size[slot];
+        for (int lv = 0; mask; ++lv) {
+            const int bit = 63 - __clzll((long long)mask);
+            mask &= ~(1ull << bit);
+            wl.items[atomicAdd(&wl.ctrl[item_bin(lv, size)], 1u)] = ((uint64_t)slot << 8) | (uint64_t)bit;
+        }
+    }
 }
 
-// One CTA per (genome, replica slot), heaviest first.  Per variant:
-//  1. stage the cost rows l_k(n), l_k^head(n) and the link times;
-//  2. exact memory check per master;
+// Persistent CTAs; each work item is one (genome, replica slot, variant) the
+// pre-pass kept, skipped if a larger batch of its replica was already
+// accepted.  Per item:
+//  1. stage the master-free cost rows l_k(n) and the link times as 32-bit
+//     order keys (exact ranks, see ranks.cu);
+//  2. masters the memory allows;
 //  3. prefix columns F_k (no master, devices 1..k) on warps 0-1 and suffix
 //     columns G_k (no master, devices k..m) on warps 2-3, concurrently:
 //        F_k[r] = min_s max(F_{k-1}[s], l_k(r-s+1), tau_k)
@@ -248,39 +307,49 @@ __global__ void order_scatter_kernel(int total, const uint8_t *keys, unsigned *c
 //  4. master mu: the prefix holds a extra blocks, the suffix b, the master
 //     W - a - b, so with H_mu[c] = min_{a+b=c} max(F_{mu-1}[a], G_{mu+1}[b])
 //        V_mu = max(tau_mu, tau_{mu+1}, min_c max(H_mu[c], l_mu^head(W - c)))
-//     (F_0 and G_{m+1} are the empty stage: 0 at index 0, +inf after);
-//  5. mu* = smallest mu with the least V_mu; its prefix columns D_k (master
-//     at mu*) are recomputed for the traceback;
+//     (F_0 and G_{m+1} are the empty stage: 0 at index 0, +inf after); the
+//     warp fetches l_mu^head asynchronously while it builds H_mu;
+//  5. mu* = smallest mu with the least V_mu; its prefix columns D_k (master at
+//     mu*) are recomputed for the traceback;
 //  6. traceback with the smallest-split rule (n_k = number of n <= r+1 with
-//     l_k(n) <= D, counted with warp ballots) and Lambda in pipeline order.
-// Every value is a min/max of the same leaf and link times the oracle uses,
-// so V, mu*, the partition and Lambda are bit-identical to Alg. 1.
+//     l_k(n) <= D, counted with warp ballots); the bottleneck T (the largest
+//     stage or link time of the partition, equal to V) and Lambda (summed in
+//     pipeline order) in float64 from the stage and link tables.
+// Every comparison is between ranks of the same stage and link times the
+// oracle compares, so V, mu*, the partition, T and Lambda are bit-identical to
+// Alg. 1.
 __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out,
-                                                      const int *order, SlotInfo si)
+                                                      WorkList wl, SlotInfo si, SplitOut so)
 {
     extern __shared__ __align__(16) unsigned char smem[];
-    __shared__ int s_off, s_m, s_role, s_S0, s_Z, s_mu, s_done;
-    __shared__ uint64_t s_V;
-    __shared__ double s_L;
-    __shared__ uint64_t s_wV[4];
+    __shared__ int s_S0, s_Z, s_mu, s_done;
+    __shared__ uint32_t s_V;
+    __shared__ double s_L, s_T;
+    __shared__ uint32_t s_wV[4];
     __shared__ int s_wMu[4];
+    __shared__ unsigned s_item;
 
     const int K = dm.K, M = dm.M, N = dm.N;
-    const int slot = order[blockIdx.x];
-    const int g = slot / K, c = slot - g * K;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
+    const unsigned n_items = wl.ctrl[kOrderBins];
+  for (;;) {
+    // ---- next work item (heaviest first)
+    if (tid == 0) s_item = atomicAdd(&wl.ctrl[kOrderBins + 1], 1u);
+    __syncthreads();
+    const unsigned idx = s_item;
+    __syncthreads();
+    if (idx >= n_items) break;
+    const uint64_t item = wl.items[idx];
+    const int slot = (int)(item >> 8), code = (int)(item & 0xFFu);
+    if (tid == 0) s_done = *(volatile const int32_t *)&si.best[slot] > code;   // a larger batch won
+    __syncthreads();
+    if (s_done) continue;
+    const int g = slot / K, c = slot - g * K;
     const size_t gk = (size_t)g * K + c;
-    if (c >= pop.nclus[g]) {
-        if (tid == 0) {
-            out.master[gk] = -1; out.bsel[gk] = -1;
-            out.T[gk] = keyd(kInfKey); out.L[gk] = keyd(kInfKey);
-        }
-        return;
-    }
     const int off = si.off[slot], m = pop.sizes[gk];
     const int role = (int)((pop.roles[g] >> c) & 1ull);
-    uint64_t vmask = si.mask[slot];
-    int16_t *lay_out = out.layers + (size_t)g * M + off;
+    uint64_t vmask = 1ull << code;
+    int16_t *lay_out = so.layers + ((size_t)g * dm.b_max + code) * M + off;
 
     unsigned long long st_runs = 0, st_cells = 0, st_probes = 0;
     bool served = false;
@@ -288,27 +357,28 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
 
     if (m <= N && vmask) {
         const int W = N - m + 1;
-        uint64_t *leaf0 = reinterpret_cast<uint64_t *>(smem);   // [m][W] l_k(n)
-        uint64_t *leaf1 = leaf0 + (size_t)m * W;                // [m][W] l_k^head(n)
-        uint64_t *Fst = leaf1 + (size_t)m * W;                  // [m][W] prefix / traceback columns
-        uint64_t *Gst = Fst + (size_t)m * W;                    // [m][W] suffix columns
-        uint64_t *Hb = Gst + (size_t)m * W;                     // [NW][W] per-warp convolution
-        uint64_t *delta = Hb + (size_t)NW * W;                  // [W] the empty stage
-        uint64_t *tauk = delta + W;                             // [m] tauk[k] = link (k-1) -> k
+        uint32_t *leaf0 = reinterpret_cast<uint32_t *>(smem);   // [m][W] l_k(n)
+        uint32_t *Fst = leaf0 + (size_t)m * W;                  // [m][W] prefix / traceback columns
+        uint32_t *Gst = Fst + (size_t)m * W;                    // [m][W] suffix columns
+        uint32_t *Hb = Gst + (size_t)m * W;                     // [NW][W] per-warp convolution
+        uint32_t *Lb = Hb + (size_t)NW * W;                     // [NW][W] per-warp head row
+        uint32_t *row1s = Lb + (size_t)NW * W;                  // [W] head row of mu*
+        uint32_t *delta = row1s + W;                            // [W] the empty stage
+        uint32_t *tauk = delta + W;                             // [m] tauk[k] = link (k-1) -> k
         int *cnt0 = reinterpret_cast<int *>(tauk + m);          // [m]
         int *cnt1 = cnt0 + m;                                   // [m]
         int *nk = cnt1 + m;                                     // [m]
         uint16_t *devs = reinterpret_cast<uint16_t *>(nk + m);  // [m]
 
         for (int k = tid; k < m; k += blockDim.x) devs[k] = pop.perm[(size_t)g * M + off + k];
-        for (int r = tid; r < W; r += blockDim.x) delta[r] = r ? kInfKey : 0ull;
+        for (int r = tid; r < W; r += blockDim.x) delta[r] = r ? 0xFFFFFFFFu : 0u;
         __syncthreads();
 
         // column accessors (1-based device index k)
-        auto colF = [&](int k) -> const uint64_t * {
+        auto colF = [&](int k) -> const uint32_t * {
             return k == 0 ? delta : k == 1 ? leaf0 : Fst + (size_t)(k - 1) * W;
         };
-        auto colG = [&](int k) -> const uint64_t * {
+        auto colG = [&](int k) -> const uint32_t * {
             return k == m + 1 ? delta : k == m ? leaf0 + (size_t)(m - 1) * W : Gst + (size_t)(k - 1) * W;
         };
 
@@ -318,19 +388,18 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             const int bit = 63 - __clzll((long long)vmask);          // highest batch first
             vmask &= ~(1ull << bit);
             const int v = role ? bit + 1 : 0;
-            // ---- 1. capacities, link times and cost rows of this variant
+            const size_t vM = (size_t)v * M;
+            // ---- 1. capacities, link ranks and master-free cost rows
             for (int k = tid; k < m; k += blockDim.x) {
-                const size_t vd = (size_t)v * M + devs[k];
+                const size_t vd = vM + devs[k];
                 const int c0 = tb.cap[vd * 2], c1 = tb.cap[vd * 2 + 1];
                 cnt0[k] = c0 < W ? c0 : W;
                 cnt1[k] = c1 < W ? c1 : W;
-                tauk[k] = k ? dkey(tb.tau[((size_t)v * M + devs[k - 1]) * M + devs[k]]) : 0ull;
+                tauk[k] = k ? tb.tau_rank[(vM + devs[k - 1]) * M + devs[k]] : 0u;
             }
             for (int e = tid; e < m * W; e += blockDim.x) {
                 const int k = e / W, n = e - k * W;
-                const double *base = tb.leaf + ((size_t)v * M + devs[k]) * 2 * dm.LS;
-                leaf0[e] = dkey(base[n]);
-                leaf1[e] = dkey(base[dm.LS + n]);
+                leaf0[e] = tb.leaf_rank[(vM + devs[k]) * 2 * dm.LS + n];
             }
             __syncthreads();
             // ---- 2. masters the memory allows (the pre-pass guarantees one)
@@ -350,17 +419,17 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             // ---- 3. prefix columns (warps 0-1) and suffix columns (warps 2-3)
             if (wid < 2) {
                 for (int k = 2; k <= m - 1; ++k) {
-                    const uint64_t *prev = colF(k - 1), *row = leaf0 + (size_t)(k - 1) * W;
-                    const uint64_t t = tauk[k - 1];
-                    uint64_t *cur = Fst + (size_t)(k - 1) * W;
+                    const uint32_t *prev = colF(k - 1), *row = leaf0 + (size_t)(k - 1) * W;
+                    const uint32_t t = tauk[k - 1];
+                    uint32_t *cur = Fst + (size_t)(k - 1) * W;
                     for (int r = tid; r < W; r += 64) cur[r] = dp_cell(prev, row, t, r);
                     bar_named(1, 64);
                 }
             } else {
                 for (int k = m - 1; k >= 2; --k) {
-                    const uint64_t *prev = colG(k + 1), *row = leaf0 + (size_t)(k - 1) * W;
-                    const uint64_t t = tauk[k];
-                    uint64_t *cur = Gst + (size_t)(k - 1) * W;
+                    const uint32_t *prev = colG(k + 1), *row = leaf0 + (size_t)(k - 1) * W;
+                    const uint32_t t = tauk[k];
+                    uint32_t *cur = Gst + (size_t)(k - 1) * W;
                     for (int r = tid - 64; r < W; r += 64) cur[r] = dp_cell(prev, row, t, r);
                     bar_named(2, 64);
                 }
@@ -371,18 +440,21 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             }
             __syncthreads();
             // ---- 4. one master per warp at a time
-            uint64_t bestV = kInfKey;
+            uint32_t bestV = 0xFFFFFFFFu;
             int bestMu = 0x7FFFFFFF;
             unsigned long long w_cells = 0, w_probes = 0;
-            uint64_t *H = Hb + (size_t)wid * W;
+            uint32_t *H = Hb + (size_t)wid * W, *L1 = Lb + (size_t)wid * W;
             for (int mu = wid + 1; mu <= m; mu += NW) {
                 if (!mu_ok(mu)) continue;
-                const uint64_t *P = colF(mu - 1), *S = colG(mu + 1);
-                for (int r = lane; r < W; r += 32) H[r] = dp_cell(P, S, 0ull, r);
+                const uint32_t *hrow = tb.leaf_rank + ((vM + devs[mu - 1]) * 2 + 1) * dm.LS;
+                for (int r = lane; r < W; r += 32) cp_async4(L1 + r, hrow + r);
+                const uint32_t *P = colF(mu - 1), *S = colG(mu + 1);
+                for (int r = lane; r < W; r += 32) H[r] = dp_cell(P, S, 0u, r);
+                cp_async_wait_all();
                 __syncwarp();
-                uint64_t V = dp_cell(H, leaf1 + (size_t)(mu - 1) * W, 0ull, W - 1);
-                if (mu >= 2) V = umax64(V, tauk[mu - 1]);
-                if (mu <= m - 1) V = umax64(V, tauk[mu]);
+                uint32_t V = dp_cell(H, L1, 0u, W - 1);
+                if (mu >= 2) V = max(V, tauk[mu - 1]);
+                if (mu <= m - 1) V = max(V, tauk[mu]);
                 __syncwarp();
                 w_cells += W + 1;
                 w_probes += cprobe + lprobe;
@@ -391,36 +463,39 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             if (lane == 0) { s_wV[wid] = bestV; s_wMu[wid] = bestMu; st_cells += w_cells; st_probes += w_probes; }
             __syncthreads();
             if (tid == 0) {
-                uint64_t V = kInfKey;
+                uint32_t V = 0xFFFFFFFFu;
                 int mu = 0x7FFFFFFF;
                 for (int w = 0; w < NW; ++w)
                     if (s_wV[w] < V || (s_wV[w] == V && s_wMu[w] < mu)) { V = s_wV[w]; mu = s_wMu[w]; }
                 s_V = V; s_mu = mu;
             }
             __syncthreads();
-            const uint64_t V = s_V;
+            const uint32_t V = s_V;
             const int mus = s_mu;
-            if (V >= kInfKey) continue;      // cannot happen after the exact memory check
+            if (V == 0xFFFFFFFFu) continue;   // cannot happen: the pre-pass checked memory
+            for (int r = tid; r < W; r += blockDim.x)
+                row1s[r] = tb.leaf_rank[((vM + devs[mus - 1]) * 2 + 1) * dm.LS + r];
+            __syncthreads();
             // ---- 5. mu*'s prefix columns, for the traceback
-            auto rowk = [&](int k) -> const uint64_t * { return (k == mus ? leaf1 : leaf0) + (size_t)(k - 1) * W; };
-            auto colD = [&](int k) -> const uint64_t * {
-                if (k == 1) return mus == 1 ? leaf1 : leaf0;
+            auto rowk = [&](int k) -> const uint32_t * { return k == mus ? row1s : leaf0 + (size_t)(k - 1) * W; };
+            auto colD = [&](int k) -> const uint32_t * {
+                if (k == 1) return mus == 1 ? row1s : leaf0;
                 return Fst + (size_t)(k - 1) * W;
             };
             for (int k = (mus > 2 ? mus : 2); k <= m - 1; ++k) {
-                const uint64_t *prev = colD(k - 1), *row = rowk(k);
-                const uint64_t t = tauk[k - 1];
-                uint64_t *cur = Fst + (size_t)(k - 1) * W;
+                const uint32_t *prev = colD(k - 1), *row = rowk(k);
+                const uint32_t t = tauk[k - 1];
+                uint32_t *cur = Fst + (size_t)(k - 1) * W;
                 for (int r = tid; r < W; r += blockDim.x) cur[r] = dp_cell(prev, row, t, r);
                 __syncthreads();
                 if (tid == 0) { st_cells += W; st_probes += cprobe; }
             }
-            // ---- 6. traceback (smallest split on ties) and Lambda in pipeline order
+            // ---- 6. traceback (smallest split on ties), T and Lambda
             if (wid == 0) {
                 int r = W - 1;
-                uint64_t D = V;
+                uint32_t D = V;
                 for (int k = m; k >= 2; --k) {
-                    const uint64_t *row = rowk(k);
+                    const uint32_t *row = rowk(k);
                     int n = 0;                                    // #{n <= r+1 : l_k(n) <= D}
                     for (int base = 0; base <= r; base += 32) {
                         const int p = base + lane;
@@ -432,14 +507,33 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
                     r = r + 1 - n;
                     D = colD(k - 1)[r];
                 }
-                if (lane == 0) {
-                    nk[0] = r + 1;
-                    double lam = keyd(rowk(1)[nk[0] - 1]);
-                    for (int k = 2; k <= m; ++k) {
-                        lam = lam + keyd(tauk[k - 1]);
-                        lam = lam + keyd(rowk(k)[nk[k - 1] - 1]);
+                if (lane == 0) nk[0] = r + 1;
+                __syncwarp();
+                // stage and link times of the partition, lane k holds device k
+                const double *lrow = tb.leaf + vM * 2 * dm.LS;
+                const double *trow = tb.tau + vM * M;
+                double lam = 0.0;
+                uint64_t tmax = 0;
+                for (int base = 0; base < m; base += 32) {
+                    const int k = base + lane;               // 0-based device
+                    double lk = 0.0, tk = 0.0;
+                    if (k < m) {
+                        lk = lrow[((size_t)devs[k] * 2 + (k == mus - 1)) * dm.LS + nk[k] - 1];
+                        if (k >= 1) tk = trow[(size_t)devs[k - 1] * M + devs[k]];
+                        tmax = umax64(tmax, umax64(dkey(lk), dkey(tk)));
                     }
+                    for (int q = 0; q < 32 && base + q < m; ++q) {
+                        const double lq = __shfl_sync(0xFFFFFFFFu, lk, q);
+                        const double tq = __shfl_sync(0xFFFFFFFFu, tk, q);
+                        if (base + q == 0) lam = lq;
+                        else { lam = lam + tq; lam = lam + lq; }
+                    }
+                }
+#pragma unroll
+                for (int o = 16; o; o >>= 1) tmax = umax64(tmax, __shfl_xor_sync(0xFFFFFFFFu, tmax, o));
+                if (lane == 0) {
                     s_L = lam;
+                    s_T = keyd(tmax);
                     s_done = (!role) || (1.0 / lam >= dm.min_tps);
                 }
             }
@@ -447,10 +541,12 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             if (s_done) {
                 for (int k = tid; k < m; k += blockDim.x) lay_out[k] = (int16_t)nk[k];
                 if (tid == 0) {
-                    out.master[gk] = (int16_t)(mus - 1);
-                    out.bsel[gk] = (int16_t)v;
-                    out.T[gk] = keyd(V);
-                    out.L[gk] = s_L;
+                    const size_t sv = gk * dm.b_max + code;
+                    so.mu[sv] = (int16_t)(mus - 1);
+                    so.T[sv] = s_T;
+                    so.L[sv] = s_L;
+                    __threadfence();
+                    atomicMax(&si.best[slot], code);
                 }
                 served = true;
                 served_v = v;
@@ -458,50 +554,92 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             __syncthreads();
         }
     }
-    if (!served) {
-        for (int k = tid; k < m; k += blockDim.x) lay_out[k] = -1;
-        if (tid == 0) {
-            out.master[gk] = -1; out.bsel[gk] = -1;
-            out.T[gk] = keyd(kInfKey); out.L[gk] = keyd(kInfKey);
-        }
-    }
-    // per-CTA tallies
+    __syncthreads();
     if (lane == 0 && (st_cells | st_probes)) {
         atomicAdd(&out.stats[kStCells], st_cells);
         atomicAdd(&out.stats[kStProbes], st_probes);
     }
-    if (tid == 0) {
-        // candidates the plain recurrence examines for the same sweep: every
-        // variant from the top down to the accepted one (all of them if none)
-        unsigned long long nrun = 0;
-        if (m <= N) nrun = served ? (role ? (unsigned long long)(dm.b_max - served_v + 1) : 1ull)
-                                  : (role ? (unsigned long long)dm.b_max : 1ull);
+    if (tid == 0 && st_runs) atomicAdd(&out.stats[kStDpRuns], st_runs);
+    (void)served_v;
+  }
+}
+
+// Per slot with work: the largest accepted variant is the sweep's answer
+// (Alg. 2 keeps the highest feasible batch); its master, batch, times and
+// partition become the outputs.
+__global__ void finalize_kernel(Dims dm, DevPop pop, SlotInfo si, SplitOut so, EvalOut out)
+{
+    const int total = dm.P * dm.K;
+    for (int slot = blockIdx.x * blockDim.x + threadIdx.x; slot < total; slot += gridDim.x * blockDim.x) {
+        const int g = slot / dm.K, c = slot - g * dm.K;
+        if (c >= pop.nclus[g] || !si.mask[slot]) continue;
+        const int m = pop.sizes[slot], off = si.off[slot];
+        const int role = (int)((pop.roles[g] >> c) & 1ull);
+        const int best = si.best[slot];
+        int16_t *lay = out.layers + (size_t)g * dm.M + off;
+        unsigned long long nrun = role ? (unsigned long long)dm.b_max : 1ull;
+        if (best < 0) {
+            write_unserved(out, slot, lay, m);
+        } else {
+            const size_t sv = (size_t)slot * dm.b_max + best;
+            const int16_t *src = so.layers + ((size_t)g * dm.b_max + best) * dm.M + off;
+            for (int k = 0; k < m; ++k) lay[k] = src[k];
+            out.master[slot] = so.mu[sv];
+            out.bsel[slot] = (int16_t)(role ? best + 1 : 0);
+            out.T[slot] = so.T[sv];
+            out.L[slot] = so.L[sv];
+            if (role) nrun = (unsigned long long)(dm.b_max - best);   // variants b_max .. best+1
+            atomicAdd(&out.stats[kStServed], 1ull);
+        }
         atomicAdd(&out.stats[kStReplicas], 1ull);
-        if (st_runs) atomicAdd(&out.stats[kStDpRuns], st_runs);
-        if (nrun) atomicAdd(&out.stats[kStPaper], nrun * paper_candidates(m, N));
-        if (served) atomicAdd(&out.stats[kStServed], 1ull);
+        atomicAdd(&out.stats[kStPaper], nrun * paper_candidates(m, dm.N));
     }
 }
 
-// Objective, one thread per genome (Sec. 3.3).  PS and DS are summed over the
-// serving replicas of each role in ascending replica order, then Eq. 3
+// Objective, one warp per genome (Sec. 3.3).  Each serving replica's rate
+// (NP / T for prefill, b / T for decode) is computed by its own lane; PS and
+// DS are then summed by lane 0 in ascending replica order, then Eq. 3
 // (bottleneck phase), Eq. 4 (backlog) and Eq. 5 (waiting time).  Also a
 // 64-bit fingerprint of the genome for the elites' duplicate test.
-__global__ void __launch_bounds__(32) score_kernel(Dims dm, DevPop pop, EvalOut out)
+__global__ void __launch_bounds__(128) score_kernel(Dims dm, DevPop pop, EvalOut out)
 {
-    const int g = blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
     if (g >= dm.P) return;
     const int K = dm.K, M = dm.M;
     const int R = pop.nclus[g];
     const uint64_t roles = pop.roles[g];
+    double rate[2];
+    int kind[2];                                   // -1 none, 0 prefill, 1 decode
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int c = lane + 32 * h;
+        kind[h] = -1;
+        rate[h] = 0.0;
+        if (c < R) {
+            const int b = out.bsel[(size_t)g * K + c];
+            if (b >= 0) {
+                const double T = out.T[(size_t)g * K + c];
+                kind[h] = (int)((roles >> c) & 1ull);
+                rate[h] = kind[h] ? (double)b / T : (double)dm.NP / T;
+            }
+        }
+    }
     double PS = 0.0, DS = 0.0;
     for (int c = 0; c < R; ++c) {
-        const int b = out.bsel[(size_t)g * K + c];
-        if (b < 0) continue;
-        const double T = out.T[(size_t)g * K + c];
-        if (((roles >> c) & 1ull) == 0) PS = PS + (double)dm.NP / T;
-        else DS = DS + (double)b / T;
+        const int h = c >> 5;
+        const double x = __shfl_sync(0xFFFFFFFFu, h ? rate[1] : rate[0], c & 31);
+        const int k = __shfl_sync(0xFFFFFFFFu, h ? kind[1] : kind[0], c & 31);
+        if (k == 0) PS = PS + x;
+        else if (k == 1) DS = DS + x;
     }
+    // fingerprint: lanes mix interleaved slices of the ordering, lane 0 folds
+    uint64_t hl = 0x9E3779B97F4A7C15ull ^ (uint64_t)lane;
+    auto mix = [](uint64_t h, uint64_t x) { h = (h ^ x) * 0xBF58476D1CE4E5B9ull; return h ^ (h >> 31); };
+    const uint16_t *pp = pop.perm + (size_t)g * M;
+    for (int i = lane; i < M; i += 32) hl = mix(hl, pp[i]);
+    uint64_t h = 0;
+    for (int l = 0; l < 32; ++l) h = mix(h, __shfl_sync(0xFFFFFFFFu, hl, l));
+    if (lane != 0) return;
     double w = keyd(kInfKey), phase = keyd(kInfKey);
     if (PS != 0.0 && DS != 0.0) {
         const double tp = (double)dm.NP / PS, td = (double)dm.ND / DS;
@@ -512,38 +650,47 @@ __global__ void __launch_bounds__(32) score_kernel(Dims dm, DevPop pop, EvalOut 
     }
     double *f = out.fit + (size_t)g * 4;
     f[0] = w; f[1] = phase; f[2] = PS; f[3] = DS;
-    // fingerprint: ordering, grouping, replica count, roles
-    uint64_t h = 0x9E3779B97F4A7C15ull;
-    auto mix = [&](uint64_t x) { h = (h ^ x) * 0xBF58476D1CE4E5B9ull; h ^= h >> 31; };
-    const uint16_t *pp = pop.perm + (size_t)g * M;
-    for (int i = 0; i < M; ++i) mix(pp[i]);
     const uint16_t *ss = pop.sizes + (size_t)g * K;
-    for (int i = 0; i < R; ++i) mix((uint64_t)ss[i] << 16);
-    mix((uint64_t)R << 40);
-    mix(roles);
+    for (int i = 0; i < R; ++i) h = mix(h, (uint64_t)ss[i] << 16);
+    h = mix(h, (uint64_t)R << 40);
+    h = mix(h, roles);
     out.hash[g] = h;
     atomicAdd(&out.stats[kStGenomes], 1ull);
 }
 
-cudaError_t configure_eval(size_t smem)
+cudaError_t configure_eval(e2_ctx *c)
 {
-    return cudaFuncSetAttribute(dp_eval_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = cudaFuncSetAttribute(dp_eval_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c->dp_smem);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0, sms = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, dp_eval_kernel, c->dp_threads, c->dp_smem);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
+    if (e != cudaSuccess) return e;
+    c->dp_grid = (per_sm > 0 ? per_sm : 1) * (sms > 0 ? sms : 1);
+    return cudaSuccess;
 }
 
 cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
 {
-    Tables tb{c->rate, c->bw, c->mem, c->prof, c->leaf, c->tau, c->cap, c->cpb};
+    Tables tb{c->rate, c->bw, c->mem, c->prof, c->leaf, c->tau, c->cap, c->cpb, c->leaf_rank, c->tau_rank};
     EvalOut out{c->fit, c->layers, c->master, c->bsel, c->T, c->L, c->hash, c->stats};
-    const long long blocks = (long long)c->dm.P * c->dm.K;
-    SlotInfo si{c->slot_off, c->slot_mask, c->slot_key};
-    cudaError_t e = cudaMemsetAsync(c->order_bins, 0, sizeof(unsigned) * kOrderBins, c->stream);
+    SlotInfo si{c->slot_off, c->slot_mask, c->slot_size, c->slot_best};
+    WorkList wl{c->items, c->order_bins};
+    SplitOut so{c->split_T, c->split_L, c->split_mu, c->split_layers};
+    const long long slots = (long long)c->dm.P * c->dm.K;
+    cudaError_t e = cudaMemsetAsync(c->order_bins, 0, sizeof(unsigned) * (kOrderBins + 2), c->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->slot_mask, 0, sizeof(uint64_t) * (size_t)slots, c->stream);
     if (e != cudaSuccess) return e;
-    const unsigned gb = (unsigned)((blocks + 255) / 256 < 1024 ? (blocks + 255) / 256 : 1024);
-    variant_kernel<<<(unsigned)((blocks * 32 + 127) / 128), 128, 0, c->stream>>>(c->dm, tb, p, si, c->order_bins, c->stats);
+    const unsigned gb = (unsigned)((slots + 255) / 256 < 1024 ? (slots + 255) / 256 : 1024);
+    const long long vwarps = slots * c->dm.b_max;
+    variant_kernel<<<(unsigned)((vwarps * 32 + 127) / 128), 128, 0, c->stream>>>(c->dm, tb, p, si, c->stats);
+    key_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, out, c->order_bins);
     order_scan_kernel<<<1, kOrderBins, 0, c->stream>>>(c->order_bins);
-    order_scatter_kernel<<<gb, 256, 0, c->stream>>>((int)blocks, c->slot_key, c->order_bins, c->order);
-    dp_eval_kernel<<<(unsigned)blocks, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, c->order, si);
-    score_kernel<<<(c->dm.P + 31) / 32, 32, 0, c->stream>>>(c->dm, p, out);
+    order_scatter_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, wl);
+    dp_eval_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so);
+    finalize_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, so, out);
+    score_kernel<<<(unsigned)(((size_t)c->dm.P * 32 + 127) / 128), 128, 0, c->stream>>>(c->dm, p, out);
     return cudaGetLastError();
 }
 

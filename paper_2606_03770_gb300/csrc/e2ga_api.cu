@@ -20,9 +20,11 @@ thread_local char g_create_error[256] = "";
 size_t align_up(size_t x, size_t a = 256) { return (x + a - 1) / a * a; }
 
 struct Layout {
-    size_t rate, bw, mem, link_bw, cong, prof, leaf, tau, cap, cpb;
+    size_t rate, bw, mem, link_bw, cong, prof, leaf, tau, cap, cpb, leaf_sorted, beff_sorted, tau_sorted,
+        leaf_rank, tau_rank;
     size_t perm[2], sizes[2], nclus[2], roles[2];
-    size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, stats, err, order_bins, order, slot_off, slot_mask, slot_key, total;
+    size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, stats, err, order_bins, items, slot_off, slot_mask, slot_size, slot_best,
+        split_T, split_L, split_mu, split_layers, total;
     int LS;
 };
 
@@ -50,6 +52,11 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K)
     l.tau = take(8 * V * MM);
     l.cap = take(4 * V * M * 2);
     l.cpb = take(8 * V * M);
+    l.leaf_sorted = take(8 * V * rank_pow2((size_t)M * 2 * N));
+    l.beff_sorted = take(8 * rank_pow2(MM));
+    l.tau_sorted = take(8 * V * MM);
+    l.leaf_rank = take(4 * V * M * 2 * (size_t)l.LS);
+    l.tau_rank = take(4 * V * MM);
     for (int b = 0; b < 2; ++b) {
         l.perm[b] = take(2 * (size_t)P * M);
         l.sizes[b] = take(2 * (size_t)P * K);
@@ -68,11 +75,16 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K)
     l.elite_fit = take(32 * (size_t)(Q > 0 ? Q : 1));
     l.stats = take(8 * kNumStats);
     l.err = take(4);
-    l.order_bins = take(4 * kOrderBins);
-    l.order = take(4 * (size_t)P * K);
+    l.order_bins = take(4 * (kOrderBins + 2));
+    l.items = take(8 * (size_t)P * K * b_max);
     l.slot_off = take(4 * (size_t)P * K);
     l.slot_mask = take(8 * (size_t)P * K);
-    l.slot_key = take((size_t)P * K);
+    l.slot_size = take((size_t)P * K);
+    l.slot_best = take(4 * (size_t)P * K);
+    l.split_T = take(8 * (size_t)P * K * b_max);
+    l.split_L = take(8 * (size_t)P * K * b_max);
+    l.split_mu = take(2 * (size_t)P * K * b_max);
+    l.split_layers = take(2 * (size_t)P * b_max * M);
     l.total = o;
     return l;
 }
@@ -277,7 +289,7 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
         return fail_free(E2_EINVAL, "replicas could exceed 256 devices (min(M, N) > 256)");
     if (c->dp_smem + 1024 > (size_t)smem_optin)
         return fail_free(E2_EINVAL, "the largest replica's DP does not fit in shared memory (N too large)");
-    if (configure_eval(c->dp_smem) != cudaSuccess) return fail_free(E2_ECUDA, "cudaFuncSetAttribute failed");
+    if (configure_eval(c) != cudaSuccess) return fail_free(E2_ECUDA, "configuring the DP kernel failed");
 
     unsigned char *ws = static_cast<unsigned char *>(workspace);
     c->rate = reinterpret_cast<double *>(ws + l.rate);
@@ -290,6 +302,11 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->tau = reinterpret_cast<double *>(ws + l.tau);
     c->cap = reinterpret_cast<int32_t *>(ws + l.cap);
     c->cpb = reinterpret_cast<double *>(ws + l.cpb);
+    c->leaf_sorted = reinterpret_cast<uint64_t *>(ws + l.leaf_sorted);
+    c->beff_sorted = reinterpret_cast<uint64_t *>(ws + l.beff_sorted);
+    c->tau_sorted = reinterpret_cast<double *>(ws + l.tau_sorted);
+    c->leaf_rank = reinterpret_cast<uint32_t *>(ws + l.leaf_rank);
+    c->tau_rank = reinterpret_cast<uint32_t *>(ws + l.tau_rank);
     for (int b = 0; b < 2; ++b) c->pop[b] = pop_at(ws, l, b);
     c->fit = reinterpret_cast<double *>(ws + l.fit);
     c->layers = reinterpret_cast<int16_t *>(ws + l.layers);
@@ -304,10 +321,15 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->stats = reinterpret_cast<unsigned long long *>(ws + l.stats);
     c->err = reinterpret_cast<int32_t *>(ws + l.err);
     c->order_bins = reinterpret_cast<unsigned *>(ws + l.order_bins);
-    c->order = reinterpret_cast<int *>(ws + l.order);
+    c->items = reinterpret_cast<uint64_t *>(ws + l.items);
+    c->slot_best = reinterpret_cast<int32_t *>(ws + l.slot_best);
+    c->split_T = reinterpret_cast<double *>(ws + l.split_T);
+    c->split_L = reinterpret_cast<double *>(ws + l.split_L);
+    c->split_mu = reinterpret_cast<int16_t *>(ws + l.split_mu);
+    c->split_layers = reinterpret_cast<int16_t *>(ws + l.split_layers);
     c->slot_off = reinterpret_cast<int32_t *>(ws + l.slot_off);
     c->slot_mask = reinterpret_cast<uint64_t *>(ws + l.slot_mask);
-    c->slot_key = ws + l.slot_key;
+    c->slot_size = ws + l.slot_size;
 
     const size_t V = (size_t)b_max + 1, MM = (size_t)M * M;
     uint64_t *prof_h = new (std::nothrow) uint64_t[kNumProf * V];
@@ -326,6 +348,8 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     chk(cudaMemcpyAsync(c->prof, prof_h, 8 * kNumProf * V, cudaMemcpyHostToDevice, c->stream));
     if (e == cudaSuccess) e = launch_tables(c);
     if (e == cudaSuccess) e = launch_tau(c);
+    if (e == cudaSuccess) e = build_leaf_sorted(c);
+    if (e == cudaSuccess) e = build_ranks(c);
     if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
     delete[] prof_h;
     if (e != cudaSuccess) return fail_free(E2_ECUDA, cudaGetErrorString(e));
@@ -407,6 +431,7 @@ int e2_redraw_congestion(e2_ctx *c, uint64_t seed, uint32_t generation)
     if (!c) return E2_EINVAL;
     E2_CUDA(c, launch_redraw(c, seed, generation));
     E2_CUDA(c, launch_tau(c));
+    E2_CUDA(c, build_ranks(c));
     c->evaluated = false;
     return E2_OK;
 }

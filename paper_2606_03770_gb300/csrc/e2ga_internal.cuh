@@ -37,8 +37,10 @@ struct DevPop {
 // of a replica per warp in shared memory.
 constexpr int kMaxReplicaDevices = 256;
 
-// Buckets of the heavy-first work ordering of the evaluation.
-constexpr int kOrderBins = 256;
+// Buckets of the work ordering of the evaluation: 64 levels (the rank of a
+// variant among its replica's variants, largest batch first) x 16 work sizes.
+constexpr int kOrderBins = 1024;
+constexpr int kSizeBins = 16;
 
 // Stats slots (unsigned long long, atomically accumulated).
 enum StatSlot { kStGenomes = 0, kStReplicas, kStDpRuns, kStCells, kStProbes, kStPaper, kStPrecheck,
@@ -61,13 +63,29 @@ struct Tables {
     const double *tau;         // [V][M][M]
     const int32_t *cap;        // [V][M][2]: most blocks device d holds (memory), without / with the head
     const double *cpb;         // [V][M]: per-block time max(blk_flops/rate, blk_bytes/bw)
+    const uint32_t *leaf_rank; // [V][M][2][LS]: order key of leaf within its variant's value set
+    const uint32_t *tau_rank;  // [V][M][M]
 };
 
 // Per (genome, replica slot) results of the evaluation pre-pass.
 struct SlotInfo {
     int32_t *off;              // [P*K] offset of the replica in the ordering chromosome
     uint64_t *mask;            // [P*K] variants to run (bit i: prefill v=0 / decode v=i+1)
-    uint8_t *key;              // [P*K] heavy-first ordering key
+    uint8_t *size;             // [P*K] log-scale work size of one DP run of the slot
+    int32_t *best;             // [P*K] largest variant bit accepted so far (-1: none)
+};
+
+// Work items of the DP: (slot << 8) | variant bit.
+struct WorkList {
+    uint64_t *items;           // [P*K*b_max]
+    unsigned *ctrl;            // [kOrderBins] bins/cursors, then [kOrderBins] = total, [+1] = next item
+};
+
+// Results of the DP runs, per (slot, variant bit).
+struct SplitOut {
+    double *T, *L;             // [P*K*b_max]
+    int16_t *mu;               // [P*K*b_max]
+    int16_t *layers;           // [P*b_max][M]
 };
 
 struct EvalOut {
@@ -145,6 +163,11 @@ struct e2_ctx {
     double *leaf = nullptr, *tau = nullptr;
     int32_t *cap = nullptr;
     double *cpb = nullptr;
+    uint64_t *leaf_sorted = nullptr;  // [V][pow2(2 M N)] sorted stage-time keys
+    uint64_t *beff_sorted = nullptr;  // [pow2(M M)] sorted effective link bandwidths
+    double *tau_sorted = nullptr;     // [V][M M] sorted link times
+    uint32_t *leaf_rank = nullptr;    // [V][M][2][LS]
+    uint32_t *tau_rank = nullptr;     // [V][M][M]
     e2::DevPop pop[2]{};
     int cur = 0;
     double *fit = nullptr;
@@ -155,11 +178,16 @@ struct e2_ctx {
     double *elite_fit = nullptr;
     unsigned long long *stats = nullptr;
     int32_t *err = nullptr;
-    unsigned *order_bins = nullptr;   // [kOrderBins]
-    int *order = nullptr;             // [P*K] evaluation order of (genome, replica) slots
+    unsigned *order_bins = nullptr;   // [kOrderBins + 2]
+    uint64_t *items = nullptr;        // [P*K*b_max] DP work items, heaviest first
     int32_t *slot_off = nullptr;      // [P*K]
     uint64_t *slot_mask = nullptr;    // [P*K]
-    uint8_t *slot_key = nullptr;      // [P*K]
+    uint8_t *slot_size = nullptr;     // [P*K]
+    int32_t *slot_best = nullptr;     // [P*K]
+    double *split_T = nullptr, *split_L = nullptr;   // [P*K*b_max]
+    int16_t *split_mu = nullptr;                     // [P*K*b_max]
+    int16_t *split_layers = nullptr;                 // [P*b_max*M]
+    int dp_grid = 0;                  // persistent DP CTAs
     // launch shapes
     int dp_threads = 128;
     size_t dp_smem = 0;
@@ -179,5 +207,8 @@ cudaError_t launch_init(const e2_ctx *c, const DevPop &p, uint64_t seed);
 cudaError_t launch_elites(const e2_ctx *c, const DevPop &p);
 cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen);
 size_t dp_smem_bytes(int M, int N, int threads);
-cudaError_t configure_eval(size_t smem);
+cudaError_t configure_eval(e2_ctx *c);   // shared memory limit and persistent grid size
+size_t rank_pow2(size_t n);
+cudaError_t build_leaf_sorted(const e2_ctx *c);   // once per context
+cudaError_t build_ranks(const e2_ctx *c);         // after every change of the link table
 }  // namespace e2

@@ -127,15 +127,17 @@ __global__ void validate_kernel(Dims dm, DevPop p, int32_t *err)
     if (!ok) atomicMin(err, g);
 }
 
-// Fisher-Yates shuffle of the identity ordering (word M-1-t draws position t).
-__device__ void random_perm(Stream &st, int M, uint16_t *perm)
+// Fisher-Yates shuffle of the identity ordering (word M-1-t draws position t);
+// element i of the ordering lives at perm[i * stride].
+template <typename T>
+__device__ void random_perm(Stream &st, int M, T *perm, int stride = 1)
 {
-    for (int i = 0; i < M; ++i) perm[i] = (uint16_t)i;
+    for (int i = 0; i < M; ++i) perm[(size_t)i * stride] = (T)i;
     for (int t = M - 1; t >= 1; --t) {
         const uint32_t j = below(st.word((uint32_t)(M - 1 - t)), (uint32_t)t + 1);
-        const uint16_t x = perm[t];
-        perm[t] = perm[j];
-        perm[j] = x;
+        const T x = perm[(size_t)t * stride];
+        perm[(size_t)t * stride] = perm[(size_t)j * stride];
+        perm[(size_t)j * stride] = x;
     }
 }
 
@@ -258,18 +260,25 @@ __device__ __forceinline__ bool key_less(const double *fit, int a, int b)
 
 // One child per thread (App. A): tournament selection of two parents, uniform
 // crossover of the ordering chromosome, repair, grouping and roles from one
-// parent, then at most one mutation.  Slots [0, Q) copy the elites.
+// parent, then at most one mutation.  Slots [0, Q) copy the elites.  The child
+// ordering and the repair bitmap live in shared memory, interleaved by thread
+// (element i of thread t at [i * blockDim + t]), and go to the population
+// buffer once at the end.
 __global__ void ga_kernel(Dims dm, DevPop src, DevPop dst, const double *fit, const int32_t *elite,
                           uint64_t seed, uint32_t gen, GaThr thr)
 {
+    extern __shared__ uint32_t ga_smem[];
     const int s = blockIdx.x * blockDim.x + threadIdx.x;
     if (s >= dm.P) return;
-    const int M = dm.M, K = dm.K, P = dm.P;
-    uint16_t *cp = dst.perm + (size_t)s * M;
+    const int M = dm.M, K = dm.K, P = dm.P, GT = blockDim.x, t = threadIdx.x;
+    const int words = (M + 31) >> 5;
+    uint32_t *cp = ga_smem + t;                                  // cp[i * GT]
+    uint32_t *seen = ga_smem + (size_t)M * GT + t;               // seen[w * GT]
+    uint16_t *out_perm = dst.perm + (size_t)s * M;
     uint16_t *cs = dst.sizes + (size_t)s * K;
     if (s < dm.Q) {
         const int e = elite[s];
-        for (int i = 0; i < M; ++i) cp[i] = src.perm[(size_t)e * M + i];
+        for (int i = 0; i < M; ++i) out_perm[i] = src.perm[(size_t)e * M + i];
         for (int i = 0; i < K; ++i) cs[i] = src.sizes[(size_t)e * K + i];
         dst.nclus[s] = src.nclus[e];
         dst.roles[s] = src.roles[e];
@@ -279,30 +288,35 @@ __global__ void ga_kernel(Dims dm, DevPop src, DevPop dst, const double *fit, co
     int par[2];
     for (int q = 0; q < 2; ++q) {
         int best = (int)below(sel.word((uint32_t)(q * dm.tournament)), (uint32_t)P);
-        for (int t = 1; t < dm.tournament; ++t) {
-            const int c = (int)below(sel.word((uint32_t)(q * dm.tournament + t)), (uint32_t)P);
+        for (int r = 1; r < dm.tournament; ++r) {
+            const int c = (int)below(sel.word((uint32_t)(q * dm.tournament + r)), (uint32_t)P);
             if (key_less(fit, c, best)) best = c;
         }
         par[q] = best;
     }
     const uint16_t *pa = src.perm + (size_t)par[0] * M, *pb = src.perm + (size_t)par[1] * M;
     Stream cx(seed, gen, (uint32_t)s, kCross);
-    for (int i = 0; i < M; ++i) cp[i] = (uint64_t)cx.word((uint32_t)i) < thr.cx ? pb[i] : pa[i];
-    // repair: a repeated device leaves a hole; holes take the missing devices in order
-    uint32_t seen[kBitmapWords];
-    const int words = (M + 31) >> 5;
-    for (int w = 0; w < words; ++w) seen[w] = 0;
+    for (int w = 0; w < words; ++w) seen[w * GT] = 0;
+    for (int i = 0; i < M; ++i) cp[i * GT] = (uint32_t)pa[i] | ((uint32_t)pb[i] << 16);   // both parents
+    // uniform crossover, then repair: a repeated device leaves a hole, holes
+    // take the missing devices in ascending order
     for (int i = 0; i < M; ++i) {
-        const int d = cp[i];
-        if ((seen[d >> 5] >> (d & 31)) & 1u) cp[i] = 0xFFFFu;
-        else seen[d >> 5] |= 1u << (d & 31);
+        const uint32_t pk = cp[i * GT];
+        const uint32_t d = (uint64_t)cx.word((uint32_t)i) < thr.cx ? (pk >> 16) : (pk & 0xFFFFu);
+        uint32_t &sw = seen[(d >> 5) * GT];
+        if ((sw >> (d & 31)) & 1u) {
+            cp[i * GT] = 0xFFFFu;
+        } else {
+            sw |= 1u << (d & 31);
+            cp[i * GT] = d;
+        }
     }
     int miss = 0;
     for (int i = 0; i < M; ++i) {
-        if (cp[i] != 0xFFFFu) continue;
-        while ((seen[miss >> 5] >> (miss & 31)) & 1u) ++miss;
-        cp[i] = (uint16_t)miss;
-        seen[miss >> 5] |= 1u << (miss & 31);
+        if (cp[i * GT] != 0xFFFFu) continue;
+        while ((seen[(miss >> 5) * GT] >> (miss & 31)) & 1u) ++miss;
+        cp[i * GT] = (uint32_t)miss;
+        seen[(miss >> 5) * GT] |= 1u << (miss & 31);
     }
     const int from = (uint64_t)cx.word((uint32_t)M) < thr.half ? par[1] : par[0];
     for (int i = 0; i < K; ++i) cs[i] = src.sizes[(size_t)from * K + i];
@@ -314,16 +328,16 @@ __global__ void ga_kernel(Dims dm, DevPop src, DevPop dst, const double *fit, co
         const uint64_t kind = mt.word(1);
         if (kind < thr.k1) {                                   // swap two positions
             const uint32_t x = below(mt.word(2), (uint32_t)M), y = below(mt.word(3), (uint32_t)M);
-            const uint16_t t = cp[x];
-            cp[x] = cp[y];
-            cp[y] = t;
+            const uint32_t tmp = cp[x * GT];
+            cp[x * GT] = cp[y * GT];
+            cp[y * GT] = tmp;
         } else {
             int r = 0;
             if (kind < thr.k2) {                               // regroup from a random replica
                 r = (int)below(mt.word(2), (uint32_t)R);
             } else if (kind >= thr.k3) {                       // regenerate both chromosomes
                 Stream sp(seed, gen, (uint32_t)s, kMutPerm);
-                random_perm(sp, M, cp);
+                random_perm(sp, M, cp, GT);
             }
             int kept = 0;
             for (int c = 0; c < r; ++c) kept += cs[c];
@@ -336,6 +350,7 @@ __global__ void ga_kernel(Dims dm, DevPop src, DevPop dst, const double *fit, co
             R = r + Rn;
         }
     }
+    for (int i = 0; i < M; ++i) out_perm[i] = (uint16_t)cp[i * GT];
     dst.nclus[s] = (uint8_t)R;
     dst.roles[s] = rl;
 }
@@ -396,7 +411,11 @@ cudaError_t launch_elites(const e2_ctx *c, const DevPop &p)
 cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen)
 {
     GaThr thr{c->thr_cx, c->thr_half, c->thr_mut, c->thr_k1, c->thr_k2, c->thr_k3};
-    ga_kernel<<<(c->dm.P + 31) / 32, 32, 0, c->stream>>>(c->dm, src, dst, c->fit, c->elite, seed, gen, thr);
+    const int per_thread = 4 * (c->dm.M + (c->dm.M + 31) / 32);
+    int gt = 32;
+    while (gt > 1 && (size_t)gt * per_thread > 40960) gt >>= 1;
+    ga_kernel<<<(c->dm.P + gt - 1) / gt, gt, (size_t)gt * per_thread, c->stream>>>(c->dm, src, dst, c->fit,
+                                                                               c->elite, seed, gen, thr);
     return cudaGetLastError();
 }
 
