@@ -228,31 +228,54 @@ __device__ __forceinline__ int item_bin(int level, int size)
     return (63 - lv) * kSizeBins + size;
 }
 
+// Outputs of a slot with nothing to run, or the bin and count of its work
+// items (returns 0 items for the former).
+__device__ __forceinline__ int slot_items(const Dims &dm, const DevPop &pop, const SlotInfo &si,
+                                          const EvalOut &out, int slot, int *bin)
+{
+    const int g = slot / dm.K, c = slot - g * dm.K;
+    si.best[slot] = -1;
+    if (c >= pop.nclus[g]) {
+        out.master[slot] = -1; out.bsel[slot] = -1;
+        out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
+        return 0;
+    }
+    const uint64_t mask = si.mask[slot];
+    const int m = pop.sizes[slot];
+    const int role = (int)((pop.roles[g] >> c) & 1ull);
+    if (!mask) {
+        write_unserved(out, slot, out.layers + (size_t)g * dm.M + si.off[slot], m);
+        atomicAdd(&out.stats[kStReplicas], 1ull);
+        if (m <= dm.N) atomicAdd(&out.stats[kStPaper], (role ? dm.b_max : 1) * paper_candidates(m, dm.N));
+        return 0;
+    }
+    const int W = dm.N - m + 1;
+    const int sz = (int)(1.0f * __log2f(1.0f + (float)m * (float)W));
+    const int size = sz < kSizeBins - 1 ? sz : kSizeBins - 1;
+    si.size[slot] = (uint8_t)size;
+    *bin = size;
+    return __popcll(mask);
+}
+
+// Item lv of a slot goes to bin item_bin(lv, size); emits (slot << 8) | bit.
+template <typename CursorFn>
+__device__ __forceinline__ void slot_emit(const SlotInfo &si, const WorkList &wl, int slot, CursorFn cursor)
+{
+    uint64_t mask = si.mask[slot];
+    const int size = si.size[slot];
+    for (int lv = 0; mask; ++lv) {
+        const int bit = 63 - __clzll((long long)mask);
+        mask &= ~(1ull << bit);
+        wl.items[cursor(item_bin(lv, size))] = ((uint64_t)slot << 8) | (uint64_t)bit;
+    }
+}
+
 __global__ void key_kernel(Dims dm, DevPop pop, SlotInfo si, EvalOut out, unsigned *bins)
 {
     const int total = dm.P * dm.K;
     for (int slot = blockIdx.x * blockDim.x + threadIdx.x; slot < total; slot += gridDim.x * blockDim.x) {
-        const int g = slot / dm.K, c = slot - g * dm.K;
-        si.best[slot] = -1;
-        if (c >= pop.nclus[g]) {
-            out.master[slot] = -1; out.bsel[slot] = -1;
-            out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
-            continue;
-        }
-        const uint64_t mask = si.mask[slot];
-        const int m = pop.sizes[slot];
-        if (!mask) {
-            const int role = (int)((pop.roles[g] >> c) & 1ull);
-            write_unserved(out, slot, out.layers + (size_t)g * dm.M + si.off[slot], m);
-            atomicAdd(&out.stats[kStReplicas], 1ull);
-            if (m <= dm.N) atomicAdd(&out.stats[kStPaper], (role ? dm.b_max : 1) * paper_candidates(m, dm.N));
-            continue;
-        }
-        const int W = dm.N - m + 1;
-        const int sz = (int)(1.0f * __log2f(1.0f + (float)m * (float)W));
-        const int size = sz < kSizeBins - 1 ? sz : kSizeBins - 1;
-        si.size[slot] = (uint8_t)size;
-        const int nv = __popcll(mask);
+        int size = 0;
+        const int nv = slot_items(dm, pop, si, out, slot, &size);
         for (int lv = 0; lv < nv; ++lv) atomicAdd(&bins[item_bin(lv, size)], 1u);
     }
 }
@@ -283,14 +306,8 @@ __global__ void order_scatter_kernel(Dims dm, DevPop pop, SlotInfo si, WorkList 
     const int total = dm.P * dm.K;
     for (int slot = blockIdx.x * blockDim.x + threadIdx.x; slot < total; slot += gridDim.x * blockDim.x) {
         const int g = slot / dm.K, c = slot - g * dm.K;
-        if (c >= pop.nclus[g]) continue;
-        uint64_t mask = si.mask[slot];
-        const int size = si.size[slot];
-        for (int lv = 0; mask; ++lv) {
-            const int bit = 63 - __clzll((long long)mask);
-            mask &= ~(1ull << bit);
-            wl.items[atomicAdd(&wl.ctrl[item_bin(lv, size)], 1u)] = ((uint64_t)slot << 8) | (uint64_t)bit;
-        }
+        if (c >= pop.nclus[g] || !si.mask[slot]) continue;
+        slot_emit(si, wl, slot, [&](int b) { return atomicAdd(&wl.ctrl[b], 1u); });
     }
 }
 
@@ -564,50 +581,58 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
   }
 }
 
-// Per slot with work: the largest accepted variant is the sweep's answer
-// (Alg. 2 keeps the highest feasible batch); its master, batch, times and
-// partition become the outputs.
-__global__ void finalize_kernel(Dims dm, DevPop pop, SlotInfo si, SplitOut so, EvalOut out)
-{
-    const int total = dm.P * dm.K;
-    for (int slot = blockIdx.x * blockDim.x + threadIdx.x; slot < total; slot += gridDim.x * blockDim.x) {
-        const int g = slot / dm.K, c = slot - g * dm.K;
-        if (c >= pop.nclus[g] || !si.mask[slot]) continue;
-        const int m = pop.sizes[slot], off = si.off[slot];
-        const int role = (int)((pop.roles[g] >> c) & 1ull);
-        const int best = si.best[slot];
-        int16_t *lay = out.layers + (size_t)g * dm.M + off;
-        unsigned long long nrun = role ? (unsigned long long)dm.b_max : 1ull;
-        if (best < 0) {
-            write_unserved(out, slot, lay, m);
-        } else {
-            const size_t sv = (size_t)slot * dm.b_max + best;
-            const int16_t *src = so.layers + ((size_t)g * dm.b_max + best) * dm.M + off;
-            for (int k = 0; k < m; ++k) lay[k] = src[k];
-            out.master[slot] = so.mu[sv];
-            out.bsel[slot] = (int16_t)(role ? best + 1 : 0);
-            out.T[slot] = so.T[sv];
-            out.L[slot] = so.L[sv];
-            if (role) nrun = (unsigned long long)(dm.b_max - best);   // variants b_max .. best+1
-            atomicAdd(&out.stats[kStServed], 1ull);
-        }
-        atomicAdd(&out.stats[kStReplicas], 1ull);
-        atomicAdd(&out.stats[kStPaper], nrun * paper_candidates(m, dm.N));
-    }
-}
-
-// Objective, one warp per genome (Sec. 3.3).  Each serving replica's rate
-// (NP / T for prefill, b / T for decode) is computed by its own lane; PS and
-// DS are then summed by lane 0 in ascending replica order, then Eq. 3
-// (bottleneck phase), Eq. 4 (backlog) and Eq. 5 (waiting time).  Also a
-// 64-bit fingerprint of the genome for the elites' duplicate test.
-__global__ void __launch_bounds__(128) score_kernel(Dims dm, DevPop pop, EvalOut out)
+// One warp per genome.  First each replica that had work gets its outputs:
+// the largest accepted variant is the sweep's answer (Alg. 2 keeps the highest
+// feasible batch), with its master, batch, times and partition.  Then the
+// objective (Sec. 3.3): each serving replica's rate (NP / T for prefill, b / T
+// for decode) by its own lane, PS and DS summed by lane 0 in ascending replica
+// order, Eq. 3 (bottleneck phase), Eq. 4 (backlog) and Eq. 5 (waiting time);
+// and a 64-bit fingerprint of the genome for the elites' duplicate test.
+__global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop, SlotInfo si, SplitOut so,
+                                                             EvalOut out)
 {
     const int g = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
     if (g >= dm.P) return;
     const int K = dm.K, M = dm.M;
     const int R = pop.nclus[g];
     const uint64_t roles = pop.roles[g];
+    unsigned long long n_rep = 0, n_served = 0, n_paper = 0;
+    for (int c = 0; c < R; ++c) {
+        const int slot = g * K + c;
+        if (!si.mask[slot]) continue;                      // done by the ordering pass
+        const int m = pop.sizes[slot], off = si.off[slot];
+        const int role = (int)((roles >> c) & 1ull);
+        const int best = si.best[slot];
+        int16_t *lay = out.layers + (size_t)g * M + off;
+        unsigned long long nrun = role ? (unsigned long long)dm.b_max : 1ull;
+        if (best < 0) {
+            for (int k = lane; k < m; k += 32) lay[k] = -1;
+            if (lane == 0) {
+                out.master[slot] = -1; out.bsel[slot] = -1;
+                out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
+            }
+        } else {
+            const size_t sv = (size_t)slot * dm.b_max + best;
+            const int16_t *src = so.layers + ((size_t)g * dm.b_max + best) * M + off;
+            for (int k = lane; k < m; k += 32) lay[k] = src[k];
+            if (lane == 0) {
+                out.master[slot] = so.mu[sv];
+                out.bsel[slot] = (int16_t)(role ? best + 1 : 0);
+                out.T[slot] = so.T[sv];
+                out.L[slot] = so.L[sv];
+            }
+            if (role) nrun = (unsigned long long)(dm.b_max - best);   // variants b_max .. best+1
+            ++n_served;
+        }
+        ++n_rep;
+        n_paper += nrun * paper_candidates(m, dm.N);
+    }
+    if (lane == 0 && n_rep) {
+        atomicAdd(&out.stats[kStReplicas], n_rep);
+        atomicAdd(&out.stats[kStPaper], n_paper);
+        if (n_served) atomicAdd(&out.stats[kStServed], n_served);
+    }
+    __syncwarp();
     double rate[2];
     int kind[2];                                   // -1 none, 0 prefill, 1 decode
 #pragma unroll
@@ -689,8 +714,8 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     order_scan_kernel<<<1, kOrderBins, 0, c->stream>>>(c->order_bins);
     order_scatter_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, wl);
     dp_eval_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so);
-    finalize_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, so, out);
-    score_kernel<<<(unsigned)(((size_t)c->dm.P * 32 + 127) / 128), 128, 0, c->stream>>>(c->dm, p, out);
+    finalize_score_kernel<<<(unsigned)(((size_t)c->dm.P * 32 + 127) / 128), 128, 0, c->stream>>>(c->dm, p, si, so,
+                                                                                               out);
     return cudaGetLastError();
 }
 

@@ -258,101 +258,169 @@ __device__ __forceinline__ bool key_less(const double *fit, int a, int b)
     return a < b;
 }
 
-// One child per thread (App. A): tournament selection of two parents, uniform
-// crossover of the ordering chromosome, repair, grouping and roles from one
-// parent, then at most one mutation.  Slots [0, Q) copy the elites.  The child
-// ordering and the repair bitmap live in shared memory, interleaved by thread
-// (element i of thread t at [i * blockDim + t]), and go to the population
-// buffer once at the end.
-__global__ void ga_kernel(Dims dm, DevPop src, DevPop dst, const double *fit, const int32_t *elite,
-                          uint64_t seed, uint32_t gen, GaThr thr)
+__device__ __forceinline__ bool key_before(uint64_t wa, uint64_t pa, int a, uint64_t wb, uint64_t pb, int b)
+{
+    if (wa != wb) return wa < wb;
+    if (pa != pb) return pa < pb;
+    return a < b;
+}
+
+__device__ __forceinline__ unsigned lanemask_lt()
+{
+    unsigned m;
+    asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+    return m;
+}
+
+// One child per warp (App. A).  Slots [0, Q) copy the elites.  Otherwise:
+//  * tournaments: lanes draw the candidates, a warp reduction keeps the
+//    fittest (the fitness order is strict, so this is the winner of the
+//    sequential tournament);
+//  * uniform crossover of the ordering chromosome, one position per lane;
+//  * repair: first occurrence of each device by shared-memory atomicMin; a
+//    later repeat is a hole; the h-th hole (by position) takes the h-th
+//    missing device (by id), ranks from warp ballots;
+//  * grouping and roles from one parent; then at most one mutation, its
+//    random words drawn by the lanes and the sequential steps (Fisher-Yates,
+//    selection sampling) taken by lane 0 in shared memory.
+// Per warp, shared memory holds the child ordering, the first-occurrence
+// table, the missing devices, the random words (M words each) and the sizes.
+__global__ void __launch_bounds__(256) ga_kernel(Dims dm, DevPop src, DevPop dst, const double *fit,
+                                                 const int32_t *elite, uint64_t seed, uint32_t gen, GaThr thr)
 {
     extern __shared__ uint32_t ga_smem[];
-    const int s = blockIdx.x * blockDim.x + threadIdx.x;
-    if (s >= dm.P) return;
-    const int M = dm.M, K = dm.K, P = dm.P, GT = blockDim.x, t = threadIdx.x;
-    const int words = (M + 31) >> 5;
-    uint32_t *cp = ga_smem + t;                                  // cp[i * GT]
-    uint32_t *seen = ga_smem + (size_t)M * GT + t;               // seen[w * GT]
-    uint16_t *out_perm = dst.perm + (size_t)s * M;
-    uint16_t *cs = dst.sizes + (size_t)s * K;
-    if (s < dm.Q) {
-        const int e = elite[s];
-        for (int i = 0; i < M; ++i) out_perm[i] = src.perm[(size_t)e * M + i];
-        for (int i = 0; i < K; ++i) cs[i] = src.sizes[(size_t)e * K + i];
-        dst.nclus[s] = src.nclus[e];
-        dst.roles[s] = src.roles[e];
-        return;
-    }
-    Stream sel(seed, gen, (uint32_t)s, kSelect);
-    int par[2];
-    for (int q = 0; q < 2; ++q) {
-        int best = (int)below(sel.word((uint32_t)(q * dm.tournament)), (uint32_t)P);
-        for (int r = 1; r < dm.tournament; ++r) {
-            const int c = (int)below(sel.word((uint32_t)(q * dm.tournament + r)), (uint32_t)P);
-            if (key_less(fit, c, best)) best = c;
+    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5, NWB = blockDim.x >> 5;
+    const int M = dm.M, K = dm.K, P = dm.P;
+    uint32_t *child = ga_smem + (size_t)wl * (4 * M + 64);
+    int32_t *first = reinterpret_cast<int32_t *>(child + M);
+    uint32_t *missing = reinterpret_cast<uint32_t *>(first + M);
+    uint32_t *words = missing + M;
+    uint32_t *ssz = words + M;                                    // [64] sizes
+    const uint64_t *fk = reinterpret_cast<const uint64_t *>(fit);
+    for (int s = blockIdx.x * NWB + wl; s < P; s += gridDim.x * NWB) {
+        uint16_t *out_perm = dst.perm + (size_t)s * M;
+        uint16_t *cs = dst.sizes + (size_t)s * K;
+        if (s < dm.Q) {
+            const int e = elite[s];
+            for (int i = lane; i < M; i += 32) out_perm[i] = src.perm[(size_t)e * M + i];
+            for (int i = lane; i < K; i += 32) cs[i] = src.sizes[(size_t)e * K + i];
+            if (lane == 0) { dst.nclus[s] = src.nclus[e]; dst.roles[s] = src.roles[e]; }
+            continue;
         }
-        par[q] = best;
-    }
-    const uint16_t *pa = src.perm + (size_t)par[0] * M, *pb = src.perm + (size_t)par[1] * M;
-    Stream cx(seed, gen, (uint32_t)s, kCross);
-    for (int w = 0; w < words; ++w) seen[w * GT] = 0;
-    for (int i = 0; i < M; ++i) cp[i * GT] = (uint32_t)pa[i] | ((uint32_t)pb[i] << 16);   // both parents
-    // uniform crossover, then repair: a repeated device leaves a hole, holes
-    // take the missing devices in ascending order
-    for (int i = 0; i < M; ++i) {
-        const uint32_t pk = cp[i * GT];
-        const uint32_t d = (uint64_t)cx.word((uint32_t)i) < thr.cx ? (pk >> 16) : (pk & 0xFFFFu);
-        uint32_t &sw = seen[(d >> 5) * GT];
-        if ((sw >> (d & 31)) & 1u) {
-            cp[i * GT] = 0xFFFFu;
-        } else {
-            sw |= 1u << (d & 31);
-            cp[i * GT] = d;
-        }
-    }
-    int miss = 0;
-    for (int i = 0; i < M; ++i) {
-        if (cp[i * GT] != 0xFFFFu) continue;
-        while ((seen[(miss >> 5) * GT] >> (miss & 31)) & 1u) ++miss;
-        cp[i * GT] = (uint32_t)miss;
-        seen[(miss >> 5) * GT] |= 1u << (miss & 31);
-    }
-    const int from = (uint64_t)cx.word((uint32_t)M) < thr.half ? par[1] : par[0];
-    for (int i = 0; i < K; ++i) cs[i] = src.sizes[(size_t)from * K + i];
-    int R = src.nclus[from];
-    uint64_t rl = src.roles[from];
-
-    Stream mt(seed, gen, (uint32_t)s, kMutate);
-    if ((uint64_t)mt.word(0) < thr.mut) {
-        const uint64_t kind = mt.word(1);
-        if (kind < thr.k1) {                                   // swap two positions
-            const uint32_t x = below(mt.word(2), (uint32_t)M), y = below(mt.word(3), (uint32_t)M);
-            const uint32_t tmp = cp[x * GT];
-            cp[x * GT] = cp[y * GT];
-            cp[y * GT] = tmp;
-        } else {
-            int r = 0;
-            if (kind < thr.k2) {                               // regroup from a random replica
-                r = (int)below(mt.word(2), (uint32_t)R);
-            } else if (kind >= thr.k3) {                       // regenerate both chromosomes
-                Stream sp(seed, gen, (uint32_t)s, kMutPerm);
-                random_perm(sp, M, cp, GT);
+        // ---- two tournaments
+        Stream sel(seed, gen, (uint32_t)s, kSelect);
+        int par[2];
+        for (int q = 0; q < 2; ++q) {
+            uint64_t bw = ~0ull, bp = ~0ull;
+            int bi = 0x7FFFFFFF;
+            for (int t = lane; t < dm.tournament; t += 32) {
+                const int cnd = (int)below(sel.word((uint32_t)(q * dm.tournament + t)), (uint32_t)P);
+                const uint64_t cw = fk[(size_t)cnd * 4], cp = fk[(size_t)cnd * 4 + 1];
+                if (key_before(cw, cp, cnd, bw, bp, bi)) { bw = cw; bp = cp; bi = cnd; }
             }
-            int kept = 0;
-            for (int c = 0; c < r; ++c) kept += cs[c];
-            for (int c = r; c < K; ++c) cs[c] = 0;
-            Stream sg(seed, gen, (uint32_t)s, kMutGroup), sr(seed, gen, (uint32_t)s, kMutRoles);
-            uint64_t nr;
-            const int Rn = random_grouping(sg, sr, M - kept, K - r, cs + r, &nr);
-            const uint64_t keep = r >= 64 ? ~0ull : ((1ull << r) - 1ull);
-            rl = (rl & keep) | (r >= 64 ? 0ull : (nr << r));
-            R = r + Rn;
+#pragma unroll
+            for (int o = 16; o; o >>= 1) {
+                const uint64_t w2 = __shfl_xor_sync(0xFFFFFFFFu, bw, o), p2 = __shfl_xor_sync(0xFFFFFFFFu, bp, o);
+                const int i2 = __shfl_xor_sync(0xFFFFFFFFu, bi, o);
+                if (key_before(w2, p2, i2, bw, bp, bi)) { bw = w2; bp = p2; bi = i2; }
+            }
+            par[q] = bi;
         }
+        // ---- uniform crossover and repair
+        const uint16_t *pa = src.perm + (size_t)par[0] * M, *pb = src.perm + (size_t)par[1] * M;
+        Stream cx(seed, gen, (uint32_t)s, kCross);
+        for (int i = lane; i < M; i += 32) {
+            child[i] = (uint64_t)cx.word((uint32_t)i) < thr.cx ? pb[i] : pa[i];
+            first[i] = 0x7FFFFFFF;
+        }
+        __syncwarp();
+        for (int i = lane; i < M; i += 32) atomicMin(&first[child[i]], i);
+        __syncwarp();
+        const unsigned lt = lanemask_lt();
+        int nmiss = 0;
+        for (int base = 0; base < M; base += 32) {
+            const int d = base + lane;
+            const bool pm = d < M && first[d] == 0x7FFFFFFF;
+            const unsigned bm = __ballot_sync(0xFFFFFFFFu, pm);
+            if (pm) missing[nmiss + __popc(bm & lt)] = (uint32_t)d;
+            nmiss += __popc(bm);
+        }
+        __syncwarp();
+        int nh = 0;
+        for (int base = 0; base < M; base += 32) {
+            const int i = base + lane;
+            const bool hole = i < M && first[child[i]] != i;
+            const unsigned bh = __ballot_sync(0xFFFFFFFFu, hole);
+            if (hole) child[i] = missing[nh + __popc(bh & lt)];
+            nh += __popc(bh);
+        }
+        // ---- grouping and roles from one parent
+        const int from = (uint64_t)cx.word((uint32_t)M) < thr.half ? par[1] : par[0];
+        for (int i = lane; i < K; i += 32) ssz[i] = src.sizes[(size_t)from * K + i];
+        int R = src.nclus[from];
+        uint64_t rl = src.roles[from];
+        __syncwarp();
+        // ---- mutation
+        Stream mt(seed, gen, (uint32_t)s, kMutate);
+        if ((uint64_t)mt.word(0) < thr.mut) {
+            const uint64_t kind = mt.word(1);
+            if (kind < thr.k1) {                                   // swap two positions
+                const uint32_t x = below(mt.word(2), (uint32_t)M), y = below(mt.word(3), (uint32_t)M);
+                if (lane == 0) { const uint32_t t = child[x]; child[x] = child[y]; child[y] = t; }
+            } else {
+                int r = 0;
+                if (kind < thr.k2) {                               // regroup from a random replica
+                    r = (int)below(mt.word(2), (uint32_t)R);
+                } else if (kind >= thr.k3) {                       // regenerate both chromosomes
+                    Stream sp(seed, gen, (uint32_t)s, kMutPerm);
+                    for (int t = lane; t < M - 1; t += 32) words[t] = sp.word((uint32_t)t);
+                    for (int i = lane; i < M; i += 32) child[i] = (uint32_t)i;
+                    __syncwarp();
+                    if (lane == 0)
+                        for (int t = M - 1; t >= 1; --t) {        // Fisher-Yates, word M-1-t for position t
+                            const uint32_t j = below(words[M - 1 - t], (uint32_t)t + 1);
+                            const uint32_t x = child[t];
+                            child[t] = child[j];
+                            child[j] = x;
+                        }
+                    __syncwarp();
+                }
+                int kept = 0;
+                for (int c = 0; c < r; ++c) kept += (int)ssz[c];
+                const int Mr = M - kept, Kr = K - r;
+                Stream sg(seed, gen, (uint32_t)s, kMutGroup), sr(seed, gen, (uint32_t)s, kMutRoles);
+                for (int t = lane; t < Mr; t += 32) words[t] = sg.word((uint32_t)t);
+                const uint64_t bits = (uint64_t)sr.word(0) | ((uint64_t)sr.word(1) << 32);
+                __syncwarp();
+                if (lane == 0) {
+                    // replica count from word 0, cut t taken with probability needed/remaining
+                    const int cap = Kr < Mr ? Kr : Mr;
+                    const int Rn = 1 + (int)below(words[0], (uint32_t)cap);
+                    int need = Rn - 1, prev = 0, cc = r;
+                    for (int t = 1; t <= Mr - 1 && need > 0; ++t) {
+                        if (below(words[t], (uint32_t)(Mr - t)) < (uint32_t)need) {
+                            ssz[cc++] = (uint32_t)(t - prev);
+                            prev = t;
+                            --need;
+                        }
+                    }
+                    ssz[cc++] = (uint32_t)(Mr - prev);
+                    for (; cc < K; ++cc) ssz[cc] = 0;
+                    const uint64_t nr = Rn >= 64 ? bits : (bits & ((1ull << Rn) - 1ull));
+                    const uint64_t keep = r >= 64 ? ~0ull : ((1ull << r) - 1ull);
+                    rl = (rl & keep) | (r >= 64 ? 0ull : (nr << r));
+                    R = r + Rn;
+                }
+                R = __shfl_sync(0xFFFFFFFFu, R, 0);
+                rl = __shfl_sync(0xFFFFFFFFu, rl, 0);
+            }
+        }
+        __syncwarp();
+        for (int i = lane; i < M; i += 32) out_perm[i] = (uint16_t)child[i];
+        for (int i = lane; i < K; i += 32) cs[i] = (uint16_t)ssz[i];
+        if (lane == 0) { dst.nclus[s] = (uint8_t)R; dst.roles[s] = rl; }
+        __syncwarp();
     }
-    for (int i = 0; i < M; ++i) out_perm[i] = (uint16_t)cp[i * GT];
-    dst.nclus[s] = (uint8_t)R;
-    dst.roles[s] = rl;
 }
 
 // 1D launch helpers
@@ -411,11 +479,17 @@ cudaError_t launch_elites(const e2_ctx *c, const DevPop &p)
 cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen)
 {
     GaThr thr{c->thr_cx, c->thr_half, c->thr_mut, c->thr_k1, c->thr_k2, c->thr_k3};
-    const int per_thread = 4 * (c->dm.M + (c->dm.M + 31) / 32);
-    int gt = 32;
-    while (gt > 1 && (size_t)gt * per_thread > 40960) gt >>= 1;
-    ga_kernel<<<(c->dm.P + gt - 1) / gt, gt, (size_t)gt * per_thread, c->stream>>>(c->dm, src, dst, c->fit,
-                                                                               c->elite, seed, gen, thr);
+    const size_t per_warp = 4 * (4 * (size_t)c->dm.M + 64);
+    int nw = 8;
+    while (nw > 1 && (size_t)nw * per_warp > 48 * 1024) nw >>= 1;
+    if ((size_t)nw * per_warp > 48 * 1024) {
+        const cudaError_t e = cudaFuncSetAttribute(ga_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                   (int)((size_t)nw * per_warp));
+        if (e != cudaSuccess) return e;
+    }
+    const long long blocks = ((long long)c->dm.P + nw - 1) / nw;
+    ga_kernel<<<(unsigned)(blocks < 152 * 64 ? blocks : 152 * 64), 32 * nw, (size_t)nw * per_warp, c->stream>>>(
+        c->dm, src, dst, c->fit, c->elite, seed, gen, thr);
     return cudaGetLastError();
 }
 
