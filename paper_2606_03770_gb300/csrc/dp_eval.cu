@@ -119,6 +119,10 @@ __device__ __forceinline__ double warp_sum_d(double x)
 
 }  // namespace
 
+// Shared-memory bytes per warp of the pre-pass (18 bytes per device, rounded
+// up to 16 so that every warp's 64-bit array starts aligned).
+__host__ __device__ __forceinline__ size_t variant_stride(int mcap) { return ((size_t)mcap * 18 + 15) & ~(size_t)15; }
+
 // Pre-pass, one warp per (genome, replica slot, variant): whether the variant
 // is worth a DP run (bit i of the slot's mask: variant 0 of a prefill
 // replica, variant i+1 of a decode replica):
@@ -134,9 +138,9 @@ __device__ __forceinline__ double warp_sum_d(double x)
 __global__ void __launch_bounds__(128) variant_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si,
                                                       unsigned long long *stats)
 {
-    __shared__ uint16_t s_dev[4][kMaxReplicaDevices];
-    __shared__ int s_c0[4][kMaxReplicaDevices], s_c1[4][kMaxReplicaDevices];
-    __shared__ uint64_t s_cb[4][kMaxReplicaDevices];
+    // per warp: device ids, capacities and per-block times of up to mcap devices
+    extern __shared__ __align__(16) unsigned char vsm[];
+    const int mcap = dm.M < dm.N ? dm.M : dm.N;
     const long long wg = (long long)((blockIdx.x * (size_t)blockDim.x + threadIdx.x) >> 5);
     const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
     const int K = dm.K, M = dm.M, N = dm.N;
@@ -153,9 +157,10 @@ __global__ void __launch_bounds__(128) variant_kernel(Dims dm, Tables tb, DevPop
     if (m > N) return;
     const int W = N - m + 1;
     const int v = role ? i + 1 : 0;
-    uint16_t *sdev = s_dev[wl];
-    int *sc0 = s_c0[wl], *sc1 = s_c1[wl];
-    uint64_t *scb = s_cb[wl];                                    // per-block times as order keys
+    unsigned char *wbase = vsm + (size_t)wl * variant_stride(mcap);
+    uint64_t *scb = reinterpret_cast<uint64_t *>(wbase);              // per-block times as order keys
+    int *sc0 = reinterpret_cast<int *>(scb + mcap), *sc1 = sc0 + mcap;
+    uint16_t *sdev = reinterpret_cast<uint16_t *>(sc1 + mcap);
     const uint16_t *devs = pop.perm + (size_t)g * M + off;
     const int32_t *cap = tb.cap + (size_t)v * M * 2;
     int s0 = 0, z = 0;
@@ -709,7 +714,9 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     if (e != cudaSuccess) return e;
     const unsigned gb = (unsigned)((slots + 255) / 256 < 1024 ? (slots + 255) / 256 : 1024);
     const long long vwarps = slots * c->dm.b_max;
-    variant_kernel<<<(unsigned)((vwarps * 32 + 127) / 128), 128, 0, c->stream>>>(c->dm, tb, p, si, c->stats);
+    const int mcap = c->dm.M < c->dm.N ? c->dm.M : c->dm.N;
+    variant_kernel<<<(unsigned)((vwarps * 32 + 127) / 128), 128, 4 * variant_stride(mcap), c->stream>>>(c->dm, tb, p, si,
+                                                                                                  c->stats);
     key_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, out, c->order_bins);
     order_scan_kernel<<<1, kOrderBins, 0, c->stream>>>(c->order_bins);
     order_scatter_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, wl);

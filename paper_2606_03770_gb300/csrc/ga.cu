@@ -191,52 +191,81 @@ __device__ __forceinline__ bool elite_before(int da, uint64_t wa, uint64_t pa, i
     return a < b;
 }
 
+// Fitness keys of the elites' comparisons are staged in shared memory, tile
+// by tile, and shared by the block's warps (one warp per genome).
+constexpr int kEliteTile = 1024;
+
 // A genome equal to a lower-indexed one is a duplicate.  Equal genomes have
 // equal fitness (the evaluation is deterministic) and equal fingerprints, so
-// only those pairs are compared in full.  One warp per genome: lanes scan the
-// lower indices 32 at a time and compare candidates' genes lane-parallel.
+// only those pairs are compared in full.
 __global__ void __launch_bounds__(256) dup_kernel(Dims dm, DevPop p, const double *fit,
                                                   const uint64_t *hash, int32_t *dup)
 {
-    const int g = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
-    if (g >= dm.P) return;
+    __shared__ uint64_t s_w[kEliteTile], s_p[kEliteTile], s_h[kEliteTile];
+    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
+    const int g = blockIdx.x * (blockDim.x >> 5) + wl;
+    const bool live = g < dm.P;
     const uint64_t *fk = reinterpret_cast<const uint64_t *>(fit);
-    const uint64_t w = fk[(size_t)g * 4], ph = fk[(size_t)g * 4 + 1];
-    const uint64_t h = hash[g];
+    const uint64_t w = live ? fk[(size_t)g * 4] : 0, ph = live ? fk[(size_t)g * 4 + 1] : 0, h = live ? hash[g] : 0;
     const int M = dm.M, K = dm.K;
+    const int gmax = min(dm.P, (int)((blockIdx.x + 1) * (blockDim.x >> 5)));   // highest genome of the block
     int d = 0;
-    for (int base = 0; base < g && !d; base += 32) {
-        const int o = base + lane;
-        const bool cand = o < g && hash[o] == h && fk[(size_t)o * 4] == w && fk[(size_t)o * 4 + 1] == ph;
-        unsigned b = __ballot_sync(0xFFFFFFFFu, cand);
-        while (b && !d) {
-            const int oo = base + __ffs(b) - 1;
-            b &= b - 1;
-            bool diff = p.nclus[oo] != p.nclus[g] || p.roles[oo] != p.roles[g];
-            for (int i = lane; i < M && !diff; i += 32) diff = p.perm[(size_t)oo * M + i] != p.perm[(size_t)g * M + i];
-            for (int i = lane; i < K && !diff; i += 32) diff = p.sizes[(size_t)oo * K + i] != p.sizes[(size_t)g * K + i];
-            d = __ballot_sync(0xFFFFFFFFu, diff) == 0u;
+    for (int base = 0; base < gmax - 1; base += kEliteTile) {
+        __syncthreads();
+        for (int t = threadIdx.x; t < kEliteTile && base + t < dm.P; t += blockDim.x) {
+            s_w[t] = fk[(size_t)(base + t) * 4];
+            s_p[t] = fk[(size_t)(base + t) * 4 + 1];
+            s_h[t] = hash[base + t];
+        }
+        __syncthreads();
+        if (!live || d) continue;
+        const int lim = min(kEliteTile, g - base);
+        for (int t0 = 0; t0 < lim && !d; t0 += 32) {
+            const int t = t0 + lane;
+            const bool cand = t < lim && s_h[t] == h && s_w[t] == w && s_p[t] == ph;
+            unsigned b = __ballot_sync(0xFFFFFFFFu, cand);
+            while (b && !d) {
+                const int oo = base + t0 + __ffs(b) - 1;
+                b &= b - 1;
+                bool diff = p.nclus[oo] != p.nclus[g] || p.roles[oo] != p.roles[g];
+                for (int i = lane; i < M && !diff; i += 32) diff = p.perm[(size_t)oo * M + i] != p.perm[(size_t)g * M + i];
+                for (int i = lane; i < K && !diff; i += 32) diff = p.sizes[(size_t)oo * K + i] != p.sizes[(size_t)g * K + i];
+                d = __ballot_sync(0xFFFFFFFFu, diff) == 0u;
+            }
         }
     }
-    if (lane == 0) dup[g] = d;
+    if (live && lane == 0) dup[g] = d;
 }
 
 // rank(g) = number of genomes before g in the elite order (duplicate flag,
-// w, phase, index); the first Q ranks are the elites.  One warp per genome.
+// w, phase, index); the first Q ranks are the elites.
 __global__ void __launch_bounds__(256) rank_kernel(Dims dm, const double *fit, const int32_t *dup,
                                                    int32_t *elite, double *elite_fit)
 {
-    const int g = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
-    if (g >= dm.P) return;
+    __shared__ uint64_t s_w[kEliteTile], s_p[kEliteTile];
+    __shared__ int s_d[kEliteTile];
+    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
+    const int g = blockIdx.x * (blockDim.x >> 5) + wl;
+    const bool live = g < dm.P;
     const uint64_t *fk = reinterpret_cast<const uint64_t *>(fit);
-    const uint64_t w = fk[(size_t)g * 4], ph = fk[(size_t)g * 4 + 1];
-    const int dg = dup[g];
+    const uint64_t w = live ? fk[(size_t)g * 4] : 0, ph = live ? fk[(size_t)g * 4 + 1] : 0;
+    const int dg = live ? dup[g] : 0;
     int rank = 0;
-    for (int o = lane; o < dm.P; o += 32)
-        rank += elite_before(dup[o], fk[(size_t)o * 4], fk[(size_t)o * 4 + 1], o, dg, w, ph, g);
+    for (int base = 0; base < dm.P; base += kEliteTile) {
+        __syncthreads();
+        for (int t = threadIdx.x; t < kEliteTile && base + t < dm.P; t += blockDim.x) {
+            s_w[t] = fk[(size_t)(base + t) * 4];
+            s_p[t] = fk[(size_t)(base + t) * 4 + 1];
+            s_d[t] = dup[base + t];
+        }
+        __syncthreads();
+        const int lim = min(kEliteTile, dm.P - base);
+        if (live)
+            for (int t = lane; t < lim; t += 32) rank += elite_before(s_d[t], s_w[t], s_p[t], base + t, dg, w, ph, g);
+    }
 #pragma unroll
     for (int x = 16; x; x >>= 1) rank += __shfl_xor_sync(0xFFFFFFFFu, rank, x);
-    if (lane == 0 && rank < dm.Q) {
+    if (live && lane == 0 && rank < dm.Q) {
         elite[rank] = g;
         for (int q = 0; q < 4; ++q) elite_fit[(size_t)rank * 4 + q] = fit[(size_t)g * 4 + q];
     }
