@@ -19,6 +19,7 @@ its own GPU; value is the sum over ranks divided by the slowest rank's time.
 from __future__ import annotations
 
 import argparse
+import datetime
 import json
 import math
 import os
@@ -45,6 +46,13 @@ OPS_PER_PROBE = 6
 OPS_PER_CELL = 6
 SM_COUNT = 152
 INT32_LANES_PER_SM = 128
+# kernels of this library per step: evaluation (pre-pass, ordering key,
+# scan, scatter, DP, finalise+score) and generation step (duplicates, ranks,
+# children)
+LAUNCHES_PER_STEP = 9
+# dram__bytes_read.sum + dram__bytes_write.sum of one dp_eval_kernel launch
+# (generation 7 of this workload), from the ncu capture in profiles/
+DP_TRAFFIC_BYTES = 705536
 
 
 def parse():
@@ -65,25 +73,53 @@ def dist_info():
 
 
 class Clocks:
-    """nvidia-smi sampling during the timed region."""
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi sampling around the timed region.  Samples carry the host
+    wall clock at which they were read; those inside the region's window are
+    kept (the one nearest to it when the region is shorter than the sampling
+    interval, marked "nearest")."""
+    Q = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
 
     def __init__(self, index):
         self.index = index
         self.proc = None
         self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+        self.t0 = self.t1 = None
 
     def start(self):
         try:
             os.makedirs(os.path.dirname(self.path), exist_ok=True)
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "20"],
                                          stdout=self.f, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
+            return
+        deadline = time.time() + 10.0            # wait for the sampler's first line
+        while time.time() < deadline and self.proc.poll() is None:
+            if os.path.getsize(self.path) > 0:
+                break
+            time.sleep(0.01)
+
+    def begin(self):
+        self.t0 = time.time()
+
+    def end(self):
+        self.t1 = time.time()
+
+    def _rows(self):
+        for line in open(self.path):
+            p = [x.strip() for x in line.split(",")]
+            if len(p) < 10:
+                continue
+            try:
+                ts = datetime.datetime.strptime(p[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                yield ts, float(p[2]), float(p[3]), [n for n, v in zip(self.NAMES, p[6:10]) if v.lower() == "active"]
+            except ValueError:
+                continue
 
     def stop(self):
         if not self.proc:
@@ -94,24 +130,18 @@ class Clocks:
         except Exception:
             self.proc.kill()
         self.f.close()
-        sm, mx, reasons = [], [], set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in open(self.path):
-            p = [x.strip() for x in line.split(",")]
-            if len(p) < 9:
-                continue
-            try:
-                sm.append(float(p[1]))
-                mx.append(float(p[2]))
-            except ValueError:
-                continue
-            for n, val in zip(names, p[5:9]):
-                if val.lower() == "active":
-                    reasons.add(n)
-        if not sm:
+        rows = list(self._rows())
+        if not rows or self.t0 is None:
             return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+        inside = [r for r in rows if self.t0 <= r[0] <= self.t1]
+        kept, how = inside, "inside the timed region"
+        if not inside:
+            mid = 0.5 * (self.t0 + self.t1)
+            kept, how = [min(rows, key=lambda r: abs(r[0] - mid))], "nearest to the timed region"
+        reasons = sorted({n for r in kept for n in r[3]})
+        return {"sm_mhz": statistics.median(r[1] for r in kept), "sm_max_mhz": max(r[2] for r in kept),
+                "reasons": reasons, "samples": len(kept), "window": how,
+                "timed_region_s": self.t1 - self.t0}
 
 
 def cpu_baseline(prob, seed, sample=None):
@@ -195,6 +225,7 @@ def run_ours(args):
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
+            torch.cuda.synchronize()
 
     # ---- device-resident search: eval + elites + generation step per step
     eng.init_population(seed)
@@ -205,15 +236,21 @@ def run_ours(args):
         eng.ga_step(seed, gen)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
            torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    dpev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for x, y in dpev:                      # torch creates the CUDA event at its first record
+        x.record(stream)
+        y.record(stream)
     stats = []
     clocks = Clocks(local)
-    sync_all()
     clocks.start()
+    sync_all()
+    clocks.begin()
     for i in range(args.steps):
         with torch.cuda.stream(stream):
             flush.fill_(i & 0xFF)
         gen += 1
         a, b, c = ev[i]
+        eng.set_timing_events(*dpev[i])
         a.record(stream)
         eng.eval(parts=False)
         b.record(stream)
@@ -221,9 +258,12 @@ def run_ours(args):
         c.record(stream)
         stats.append(eng.stats())
     sync_all()
+    clocks.end()
     clk = clocks.stop()
+    eng.set_timing_events()
     step_ms = [a.elapsed_time(c) for a, b, c in ev]
     eval_ms = [a.elapsed_time(b) for a, b, c in ev]
+    dp_ms = [x.elapsed_time(y) for x, y in dpev]
     t_local = sum(step_ms) / 1e3
     t = torch.tensor([t_local], dtype=torch.float64, device="cuda")
     if world > 1:
@@ -235,8 +275,9 @@ def run_ours(args):
     probes = sum(s["dp_probes"] for s in stats) / args.steps
     cells = sum(s["dp_cells"] for s in stats) / args.steps
     eval_s = sum(eval_ms) / 1e3 / args.steps
+    dp_s = sum(dp_ms) / 1e3 / args.steps
     ops = OPS_PER_PROBE * probes + OPS_PER_CELL * cells
-    achieved = ops / eval_s / 1e12
+    achieved = ops / dp_s / 1e12
     peaks_path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     sm_max = 2070.0
     if os.path.exists(peaks_path):
@@ -288,15 +329,17 @@ def run_ours(args):
                                    f"P={prob.P}, Q={prob.Q}, b_max={prob.b_max}, one generation per step",
                        "l2": "flushed (256 MB write) between timed steps",
                        "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
-            "gpu_launches": 5 * args.steps,
+            "gpu_launches": LAUNCHES_PER_STEP * args.steps,
             "dp_cells_per_s": cells * args.steps * world / t_max,
             "paper_candidates_per_s": paper * args.steps * world / t_max,
             "eval_ms_per_step": 1e3 * eval_s,
+            "dp_kernel_ms_per_step": 1e3 * dp_s,
             "served_replicas_per_step": sum(s["served"] for s in stats) / args.steps,
             "replicas_per_step": sum(s["replicas"] for s in stats) / args.steps,
-            "roofline": {"bound": "alu", "kernel": "dp_eval_kernel + score_kernel (e2_eval_population)",
+            "roofline": {"bound": "alu", "kernel": "dp_eval_kernel (DP_Pipe, timed by events around its launch)",
                          "achieved": achieved, "peak": peak, "unit": "Tops/s (int32)",
-                         "frac": achieved / peak, "traffic": None,
+                         "frac": achieved / peak, "traffic": DP_TRAFFIC_BYTES if args.config == WORKLOAD else None,
+                         "traffic_source": "profiles/dp_eval_c2_gen7.md (dram read+write, one launch)",
                          "per_unit": f"{OPS_PER_PROBE} int32 ops per bisection probe + {OPS_PER_CELL} per DP cell",
                          "peak_source": f"{SM_COUNT} SMs x {INT32_LANES_PER_SM} int32 lanes x {sm_max:.0f} MHz"},
             "e2e": e2e,

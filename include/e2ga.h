@@ -225,6 +225,14 @@ int e2_get_elites(e2_ctx *ctx, int32_t *idx_out, double *fitness_out);
 /* Counters of the last evaluation.  Synchronises. */
 int e2_get_stats(e2_ctx *ctx, e2_stats *out);
 
+/* Timing hook (no counterpart in the paper; for measurement): two CUDA events
+ * (cudaEvent_t, created with timing enabled on the context's device) that
+ * every later e2_eval_population records on the context's stream immediately
+ * before and after its DP_Pipe kernel, so that cudaEventElapsedTime gives that
+ * kernel's duration.  NULL, NULL turns the hook off.  The caller owns the
+ * events and must keep them alive while the hook is set. */
+int e2_set_timing_events(e2_ctx *ctx, void *dp_start, void *dp_stop);
+
 /* Elite selection that allocates nothing.  The paper has no counterpart: this
  * is a service of this library for callers that cannot allocate device memory
  * -- code recording a CUDA graph (allocation is not capturable), plug-ins whose

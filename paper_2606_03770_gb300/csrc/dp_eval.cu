@@ -720,7 +720,9 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     key_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, out, c->order_bins);
     order_scan_kernel<<<1, kOrderBins, 0, c->stream>>>(c->order_bins);
     order_scatter_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, wl);
+    if (c->ev_dp_start) cudaEventRecord(c->ev_dp_start, c->stream);
     dp_eval_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so);
+    if (c->ev_dp_stop) cudaEventRecord(c->ev_dp_stop, c->stream);
     finalize_score_kernel<<<(unsigned)(((size_t)c->dm.P * 32 + 127) / 128), 128, 0, c->stream>>>(c->dm, p, si, so,
                                                                                                out);
     return cudaGetLastError();

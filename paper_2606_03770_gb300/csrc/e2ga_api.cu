@@ -480,6 +480,14 @@ int e2_get_stats(e2_ctx *c, e2_stats *out)
     return E2_OK;
 }
 
+int e2_set_timing_events(e2_ctx *c, void *dp_start, void *dp_stop)
+{
+    if (!c || (!dp_start) != (!dp_stop)) return E2_EINVAL;
+    c->ev_dp_start = static_cast<cudaEvent_t>(dp_start);
+    c->ev_dp_stop = static_cast<cudaEvent_t>(dp_stop);
+    return E2_OK;
+}
+
 const char *e2_strerror(int s)
 {
     switch (s) {

@@ -188,6 +188,7 @@ struct e2_ctx {
     int16_t *split_mu = nullptr;                     // [P*K*b_max]
     int16_t *split_layers = nullptr;                 // [P*b_max*M]
     int dp_grid = 0;                  // persistent DP CTAs
+    cudaEvent_t ev_dp_start = nullptr, ev_dp_stop = nullptr;   // optional timing hook
     // launch shapes
     int dp_threads = 128;
     size_t dp_smem = 0;

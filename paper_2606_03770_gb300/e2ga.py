@@ -70,6 +70,7 @@ SIGNATURES = {
     "e2_get_congestion": (C.c_int, [C.c_void_p, C.c_void_p]),
     "e2_get_elites": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "e2_get_stats": (C.c_int, [C.c_void_p, C.c_void_p]),
+    "e2_set_timing_events": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "e2_select_elites_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
                                             C.c_int32, C.c_void_p, C.c_void_p]),
     "e2_strerror": (C.c_char_p, [C.c_int]),
@@ -149,6 +150,10 @@ def e2_get_elites(ctx, idx_ptr, fit_ptr):
 
 def e2_get_stats(ctx, stats):
     return load().e2_get_stats(ctx, C.byref(stats))
+
+
+def e2_set_timing_events(ctx, start_ptr, stop_ptr):
+    return load().e2_set_timing_events(ctx, start_ptr, stop_ptr)
 
 
 def e2_select_elites_noalloc(genomes, fitness_ptr, P, M, K_max, Q, elite_ptr, stream_ptr):
@@ -274,6 +279,12 @@ class Engine:
         fit = np.zeros((max(self.Q, 1), 4), np.float64)
         _check(e2_get_elites(self.ctx, _ptr(idx), _ptr(fit)), "e2_get_elites", self.ctx)
         return idx[:self.Q], fit[:self.Q]
+
+    def set_timing_events(self, start=None, stop=None):
+        """Record two torch.cuda.Events around the DP kernel of later evaluations."""
+        sp = start.cuda_event if start is not None else None
+        ep = stop.cuda_event if stop is not None else None
+        _check(e2_set_timing_events(self.ctx, sp, ep), "e2_set_timing_events", self.ctx)
 
     def stats(self):
         s = e2_stats()

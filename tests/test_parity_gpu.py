@@ -236,3 +236,31 @@ def test_errors_are_statuses_not_faults():
     eng.eval(g)                                       # the context is still usable
     assert np.isfinite(eng.results()["T"]).any()
     eng.close()
+
+
+def test_dp_timing_events_bracket_the_dp_kernel():
+    import torch
+    from paper_2606_03770_gb300 import e2ga
+    prob = W.make_config("c2", P=256)
+    g = W.random_genomes(prob.M, prob.K_max, 256, seed=4)
+    eng = engine(prob)
+    stream = torch.cuda.current_stream()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    x, y = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for e in (x, y):
+        e.record(stream)                              # creates the CUDA events
+    with pytest.raises(e2ga.E2Error):
+        eng.set_timing_events(x, None)                # one event alone is rejected
+    eng.set_timing_events(x, y)
+    eng.set_population(g)
+    a.record(stream)
+    eng.eval(parts=False)
+    b.record(stream)
+    torch.cuda.synchronize()
+    dp, whole = x.elapsed_time(y), a.elapsed_time(b)
+    assert 0 < dp <= whole
+    eng.set_timing_events()                           # hook off: the events are not touched again
+    eng.eval(g)
+    torch.cuda.synchronize()
+    assert x.elapsed_time(y) == dp
+    eng.close()
