@@ -72,6 +72,23 @@ def dist_info():
     return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
 
 
+def max_over_ranks(x, world, device="cpu"):
+    """Largest value of x over the ranks (the slowest replica's time)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(units_per_rank, world, t_max):
+    """Whole-job throughput of `world` independent replicas that each processed
+    `units_per_rank` units, the slowest in t_max seconds (weak scaling)."""
+    return units_per_rank * world / t_max
+
+
 class Clocks:
     """nvidia-smi sampling around the timed region.  Samples carry the host
     wall clock at which they were read; those inside the region's window are
@@ -182,15 +199,23 @@ def run_reference(args):
     pop = O.init_population(ga, args.seed)
     op = O.OracleProblem(prob)
     times = []
+    fit = np.zeros((prob.P, 4))
     for step in range(args.warmup + args.steps):
         sub = {k: np.ascontiguousarray(v[(step * sample) % prob.P:][:sample]) for k, v in pop.items()}
         t0 = time.perf_counter()
         out = op.eval_population(sub, prob.K_max, nthreads=nt)
-        dt = time.perf_counter() - t0
+        t_eval = time.perf_counter() - t0
+        fit[:] = 0.0
+        fit[:sample] = out["fitness"]
+        t0 = time.perf_counter()
+        e = O.elites(ga, pop, fit)
+        nxt = O.ga_step(ga, args.seed, step + 1, pop, fit, e)
+        t_ga = time.perf_counter() - t0
+        pop = nxt
         if step >= args.warmup:
-            times.append(dt)
+            times.append(t_eval * prob.P / sample + t_ga)     # one generation of P genomes
     t = sum(times)
-    value = sample * len(times) / t
+    value = prob.P * len(times) / t
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / len(times),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
@@ -198,7 +223,9 @@ def run_reference(args):
             "config": {"workload": f"{prob.name}: M={prob.M} devices, N={prob.N} blocks, K_max={prob.K_max}, "
                                    f"P={prob.P}", "sample_genomes_per_step": sample},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": nt, "kind": "oracle",
-                             "sample": f"{sample} genomes per step evaluated by the oracle on {nt} threads"},
+                             "sample": f"per step, {sample} of {prob.P} genomes evaluated by the oracle on "
+                                       f"{nt} threads and scaled to the population, plus the elites and "
+                                       f"generation step of the full population"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -232,6 +259,8 @@ def run_ours(args):
     gen = 0
     for _ in range(args.warmup):
         gen += 1
+        if prob.redraw:
+            eng.redraw_congestion(seed, gen)
         eng.eval(parts=False)
         eng.ga_step(seed, gen)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
@@ -252,6 +281,8 @@ def run_ours(args):
         a, b, c = ev[i]
         eng.set_timing_events(*dpev[i])
         a.record(stream)
+        if prob.redraw:                          # congestion redrawn every generation
+            eng.redraw_congestion(seed, gen)
         eng.eval(parts=False)
         b.record(stream)
         eng.ga_step(seed, gen)
@@ -265,11 +296,8 @@ def run_ours(args):
     eval_ms = [a.elapsed_time(b) for a, b, c in ev]
     dp_ms = [x.elapsed_time(y) for x, y in dpev]
     t_local = sum(step_ms) / 1e3
-    t = torch.tensor([t_local], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    t_max = float(t.item())
-    value = prob.P * args.steps * world / t_max
+    t_max = max_over_ranks(t_local, world, "cuda")
+    value = replica_throughput(prob.P * args.steps, world, t_max)
 
     # ---- roofline of the dominant kernel (DP_Pipe evaluation)
     probes = sum(s["dp_probes"] for s in stats) / args.steps
@@ -298,12 +326,14 @@ def run_ours(args):
         bytes_pop = P * (2 * M + 2 * K + 1 + 8)
 
         def e2e_step(g):
+            if prob.redraw:
+                eng.redraw_congestion(seed, g)
             eng.set_population(host)                 # host -> device, validated
             eng.eval(fitness=hfit, parts=False)      # fitness -> host
             eng.ga_step(seed, g)
             eng.get_population(host)                 # next population -> host
 
-        for _ in range(2):
+        for _ in range(args.warmup):
             gen += 1
             e2e_step(gen)
         sync_all()
@@ -311,11 +341,9 @@ def run_ours(args):
         for _ in range(args.steps):
             gen += 1
             e2e_step(gen)
-        torch.cuda.synchronize()
-        te = torch.tensor([time.perf_counter() - t0], dtype=torch.float64, device="cuda")
-        if world > 1:
-            dist.all_reduce(te, op=dist.ReduceOp.MAX)
-        e2e = {"value": P * args.steps * world / float(te.item()), "unit": UNIT,
+        sync_all()
+        te = max_over_ranks(time.perf_counter() - t0, world, "cuda")
+        e2e = {"value": replica_throughput(P * args.steps, world, te), "unit": UNIT,
                "h2d_bytes_per_step": bytes_pop, "d2h_bytes_per_step": bytes_pop + 32 * P}
 
     if rank == 0:

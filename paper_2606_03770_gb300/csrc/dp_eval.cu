@@ -1,12 +1,17 @@
 // dp_eval.cu -- population fitness: DP_Pipe per replica (Alg. 1, Eq. 1-2),
 // the decode batch sweep (Alg. 2), and the objective (Eq. 3-5).
 //
-// One CTA evaluates one (genome, replica slot).  With identical blocks
-// (Sec. 3.2: the premise that lets the paper fix the node order) a stage's time
-// depends only on its device, its block count n and whether it is the master,
-// so the replica's costs fit in two rows per device, l_k(n) and l_k^head(n),
-// staged in shared memory as 64-bit keys (non-negative doubles order like their
-// bit patterns).
+// Work is split over six kernels per evaluation: a pre-pass that decides,
+// per (genome, replica slot, variant), whether a DP run can matter (memory and
+// latency bounds); three small kernels that order the surviving runs into one
+// work list; persistent DP CTAs that drain the list; and a warp per genome that
+// picks each replica's answer and scores the genome.
+//
+// With identical blocks (Sec. 3.2: the premise that lets the paper fix the
+// node order) a stage's time depends only on its device, its block count n and
+// whether it is the master, so the replica's costs fit in two rows per device,
+// l_k(n) and l_k^head(n), staged in shared memory as 32-bit order keys (exact
+// ranks of the float64 times, built in ranks.cu).
 //
 // Band form of Eq. 1.  Device k can take at most W = N - m + 1 blocks.  Let
 // D_k[r] = DP(i = r + k - 1, k), r in [0, W).  Then
@@ -26,12 +31,12 @@
 // l_k(r-s+1) <= D.  So the traceback needs only the cell value D and the cost
 // row: n_k = largest n <= r + 1 with l_k(n) <= D.
 //
-// Masters.  Columns k < mu do not involve the master and are shared by every
-// mu (computed once by the CTA).  Warps take masters mu = w+1, w+1+NW, ... and
-// run columns mu..m in private ping-pong buffers; the last column needs only
-// its final cell.  mu* = the smallest mu with the least bottleneck (the
-// oracle's first-wins argmin).  The CTA then recomputes mu*'s columns into the
-// shared column store for the traceback.
+// Masters.  Alg. 1 reruns the whole table for every master mu.  Here the
+// master-free prefix columns F_k (devices 1..k) and suffix columns G_k
+// (devices k..m) are computed once per run, and each master's bottleneck
+// follows from F_{mu-1}, G_{mu+1} and the master's head row (dp_eval_kernel,
+// step 4).  mu* = the smallest mu with the least bottleneck (the oracle's
+// first-wins argmin); its columns are recomputed for the traceback.
 #include "e2ga_internal.cuh"
 
 namespace e2 {
@@ -203,7 +208,7 @@ __global__ void __launch_bounds__(128) variant_kernel(Dims dm, Tables tb, DevPop
             if (k >= 1) part += tau[(size_t)sdev[k - 1] * M + sdev[k]];
         }
         const double lb = warp_sum_d(part) * (1.0 - 1e-9);
-        if (lb > 0.0 && 1.0 / lb < dm.min_tps) {
+        if (lb > dm.lam_max) {                                  // 1.0 / lb < Min_TPS
             if (lane == 0) atomicAdd(&stats[kStTpsPruned], 1ull);
             return;
         }
@@ -375,7 +380,6 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
 
     unsigned long long st_runs = 0, st_cells = 0, st_probes = 0;
     bool served = false;
-    int served_v = -1;
 
     if (m <= N && vmask) {
         const int W = N - m + 1;
@@ -419,10 +423,11 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
                 cnt1[k] = c1 < W ? c1 : W;
                 tauk[k] = k ? tb.tau_rank[(vM + devs[k - 1]) * M + devs[k]] : 0u;
             }
-            for (int e = tid; e < m * W; e += blockDim.x) {
-                const int k = e / W, n = e - k * W;
-                leaf0[e] = tb.leaf_rank[(vM + devs[k]) * 2 * dm.LS + n];
+            for (int k = wid; k < m; k += NW) {                   // asynchronous: the loads overlap
+                const uint32_t *src = tb.leaf_rank + (vM + devs[k]) * 2 * dm.LS;
+                for (int n = lane; n < W; n += 32) cp_async4(leaf0 + (size_t)k * W + n, src + n);
             }
+            cp_async_wait_all();
             __syncthreads();
             // ---- 2. masters the memory allows (the pre-pass guarantees one)
             if (wid == 0) {
@@ -556,7 +561,7 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
                 if (lane == 0) {
                     s_L = lam;
                     s_T = keyd(tmax);
-                    s_done = (!role) || (1.0 / lam >= dm.min_tps);
+                    s_done = (!role) || lam <= dm.lam_max;       // 1.0 / lam >= Min_TPS
                 }
             }
             __syncthreads();
@@ -571,7 +576,6 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
                     atomicMax(&si.best[slot], code);
                 }
                 served = true;
-                served_v = v;
             }
             __syncthreads();
         }
@@ -582,7 +586,6 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
         atomicAdd(&out.stats[kStProbes], st_probes);
     }
     if (tid == 0 && st_runs) atomicAdd(&out.stats[kStDpRuns], st_runs);
-    (void)served_v;
   }
 }
 

@@ -244,6 +244,32 @@ size_t e2_workspace_bytes(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_
     return layout(M, N, b_max, P, Q, K_max).total;
 }
 
+// The decode test of Alg. 2 keeps batch b when 1.0 / Lambda_b >= Min_TPS,
+// the quotient rounded to nearest.  Correctly rounded division is monotone, so
+// for Lambda >= 0 the test holds exactly when Lambda <= Lambda_max, the largest
+// double that passes it; found here by bisection over the bit patterns of the
+// non-negative doubles (which order like the values), so that the kernels
+// compare instead of dividing (a float64 division costs hundreds of cycles).
+static double latency_ceiling(double min_tps)
+{
+    auto pass = [&](uint64_t bits) {
+        double x;
+        memcpy(&x, &bits, sizeof x);
+        return 1.0 / x >= min_tps;
+    };
+    const uint64_t inf_bits = 0x7FF0000000000000ull;
+    if (pass(inf_bits)) return HUGE_VAL;            // min_tps <= 0: every latency passes
+    uint64_t lo = 0, hi = inf_bits;                 // pass(lo) (1/0 = +inf), !pass(hi)
+    while (hi - lo > 1) {
+        const uint64_t mid = lo + (hi - lo) / 2;
+        if (pass(mid)) lo = mid;
+        else hi = mid;
+    }
+    double x;
+    memcpy(&x, &lo, sizeof x);
+    return x;
+}
+
 int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_profile *prof,
               const e2_params *prm, void *workspace, size_t workspace_bytes, void *stream, e2_ctx **out)
 {
@@ -267,7 +293,7 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     if (!c) return E2_ENOMEM;
     c->stream = static_cast<cudaStream_t>(stream);
     c->dm = Dims{M, N, b_max + 1, b_max, P, Q, K, l.LS, prm->tournament, prof->NP, prof->ND,
-                 prm->min_tps, prm->t_a};
+                 prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps)};
     c->cong_lo = links->cong_lo;
     c->cong_hi = links->cong_hi;
     c->thr_cx = threshold(prm->p_cx);

@@ -53,6 +53,7 @@ struct Dims {
     int tournament;
     uint64_t NP, ND;
     double min_tps, t_a;
+    double lam_max;      // largest latency Lambda with 1.0 / Lambda >= min_tps (see e2_create)
 };
 
 struct Tables {

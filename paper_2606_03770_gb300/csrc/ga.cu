@@ -275,18 +275,6 @@ struct GaThr {
     uint64_t cx, half, mut, k1, k2, k3;
 };
 
-// Fitness order (lower w, lower phase, lower index) on the bit patterns of
-// the non-negative w and phase.
-__device__ __forceinline__ bool key_less(const double *fit, int a, int b)
-{
-    const uint64_t *fk = reinterpret_cast<const uint64_t *>(fit);
-    const uint64_t wa = fk[(size_t)a * 4], wb = fk[(size_t)b * 4];
-    if (wa != wb) return wa < wb;
-    const uint64_t pa = fk[(size_t)a * 4 + 1], pb = fk[(size_t)b * 4 + 1];
-    if (pa != pb) return pa < pb;
-    return a < b;
-}
-
 __device__ __forceinline__ bool key_before(uint64_t wa, uint64_t pa, int a, uint64_t wb, uint64_t pb, int b)
 {
     if (wa != wb) return wa < wb;

@@ -264,3 +264,30 @@ def test_dp_timing_events_bracket_the_dp_kernel():
     torch.cuda.synchronize()
     assert x.elapsed_time(y) == dp
     eng.close()
+
+
+def test_min_tps_boundary_exact():
+    """Min_TPS set to exactly 1.0 / Lambda of a serving decode replica, then to
+    the next double above it: the decode test of Alg. 2 flips for that replica
+    exactly as the oracle's division-based test does."""
+    import dataclasses
+    import math
+    prob = W.make_config("c2", P=256)
+    g = W.random_genomes(prob.M, prob.K_max, 256, seed=21)
+    ora = O.OracleProblem(prob).eval_population(g, prob.K_max, nthreads=O.num_threads())
+    cand = [(p, c) for p in range(256) for c in range(int(g["nclus"][p]))
+            if (int(g["roles"][p]) >> c) & 1 and ora["bsel"][p, c] >= 1]
+    assert cand
+    p, c = cand[len(cand) // 2]
+    lam = float(ora["L"][p, c])
+    served = []
+    for tps in (1.0 / lam, math.nextafter(1.0 / lam, math.inf)):
+        pb = dataclasses.replace(prob, min_tps=tps)
+        eng = engine(pb)
+        eng.eval(g)
+        gpu = eng.results()
+        ref = O.OracleProblem(pb).eval_population(g, prob.K_max, nthreads=O.num_threads())
+        assert_eval_equal(gpu, ref)
+        served.append(int(ref["bsel"][p, c]))
+        eng.close()
+    assert served[0] == ora["bsel"][p, c] and served[1] != served[0]
