@@ -46,10 +46,10 @@ OPS_PER_PROBE = 6
 OPS_PER_CELL = 6
 SM_COUNT = 152
 INT32_LANES_PER_SM = 128
-# kernels of this library per step: evaluation (pre-pass, ordering key,
-# scan, scatter, DP, finalise+score) and generation step (duplicates, ranks,
+# kernels of this library per step: evaluation (pre-pass with the work count,
+# work-list scatter, DP, finalise+score) and generation step (duplicates, ranks,
 # children)
-LAUNCHES_PER_STEP = 9
+LAUNCHES_PER_STEP = 7
 # dram__bytes_read.sum + dram__bytes_write.sum of one dp_eval_kernel launch
 # (generation 7 of this workload), from the ncu capture in profiles/
 DP_TRAFFIC_BYTES = 704512

@@ -124,105 +124,9 @@ __device__ __forceinline__ double warp_sum_d(double x)
 
 }  // namespace
 
-// Shared-memory bytes per warp of the pre-pass (18 bytes per device, rounded
-// up to 16 so that every warp's 64-bit array starts aligned).
-__host__ __device__ __forceinline__ size_t variant_stride(int mcap) { return ((size_t)mcap * 18 + 15) & ~(size_t)15; }
-
-// Pre-pass, one warp per (genome, replica slot, variant): whether the variant
-// is worth a DP run (bit i of the slot's mask: variant 0 of a prefill
-// replica, variant i+1 of a decode replica):
-//  * memory: with identical blocks a partition with master mu exists iff every
-//    device holds >= 1 block and the capacities, capped at W = N - m + 1, add
-//    up to N (exact);
-//  * decode latency: Lambda >= sum of link times + sum_k n_k c_k (c_k the
-//    per-block time, the head only adds), whose least value puts one block on
-//    each device and the other N - m on the cheapest devices up to their
-//    capacity.  A variant whose bound misses Min_TPS fails whatever partition
-//    the DP returns; the 1e-9 margin exceeds the rounding of every sum here.
-// The variant-0 warp also records the replica's offset in the ordering.
-__global__ void __launch_bounds__(128) variant_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si,
-                                                      unsigned long long *stats)
-{
-    // per warp: device ids, capacities and per-block times of up to mcap devices
-    extern __shared__ __align__(16) unsigned char vsm[];
-    const int mcap = dm.M < dm.N ? dm.M : dm.N;
-    const long long wg = (long long)((blockIdx.x * (size_t)blockDim.x + threadIdx.x) >> 5);
-    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
-    const int K = dm.K, M = dm.M, N = dm.N;
-    if (wg >= (long long)dm.P * K * dm.b_max) return;
-    const int slot = (int)(wg / dm.b_max), i = (int)(wg - (long long)slot * dm.b_max);
-    const int g = slot / K, c = slot - g * K;
-    if (c >= pop.nclus[g]) return;
-    const uint16_t *sz = pop.sizes + (size_t)g * K;
-    const int m = sz[c];
-    const int role = (int)((pop.roles[g] >> c) & 1ull);
-    if (!role && i > 0) return;
-    const int off = warp_sum(lane < c ? sz[lane] : 0) + warp_sum(lane + 32 < c ? sz[lane + 32] : 0);
-    if (i == 0 && lane == 0) si.off[slot] = off;
-    if (m > N) return;
-    const int W = N - m + 1;
-    const int v = role ? i + 1 : 0;
-    unsigned char *wbase = vsm + (size_t)wl * variant_stride(mcap);
-    uint64_t *scb = reinterpret_cast<uint64_t *>(wbase);              // per-block times as order keys
-    int *sc0 = reinterpret_cast<int *>(scb + mcap), *sc1 = sc0 + mcap;
-    uint16_t *sdev = reinterpret_cast<uint16_t *>(sc1 + mcap);
-    const uint16_t *devs = pop.perm + (size_t)g * M + off;
-    const int32_t *cap = tb.cap + (size_t)v * M * 2;
-    int s0 = 0, z = 0;
-    for (int k = lane; k < m; k += 32) {
-        const int d = devs[k];
-        sdev[k] = (uint16_t)d;
-        const int c0 = min(cap[d * 2], W), c1 = min(cap[d * 2 + 1], W);
-        sc0[k] = c0;
-        sc1[k] = c1;
-        s0 += c0;
-        z += c0 == 0;
-    }
-    s0 = warp_sum(s0);
-    z = warp_sum(z);
-    __syncwarp();
-    bool ok = false;
-    for (int k = lane; k < m && !ok; k += 32)
-        ok = (z - (sc0[k] == 0)) == 0 && sc1[k] >= 1 && s0 - sc0[k] + sc1[k] >= N;
-    if (!__any_sync(0xFFFFFFFFu, ok)) {
-        if (lane == 0) atomicAdd(&stats[kStPrecheck], 1ull);
-        return;
-    }
-    if (role && dm.min_tps > 0.0) {
-        const double *cpb = tb.cpb + (size_t)v * M;
-        const double *tau = tb.tau + (size_t)v * M * M;
-        for (int k = lane; k < m; k += 32) scb[k] = dkey(cpb[sdev[k]]);
-        __syncwarp();
-        double part = 0.0;
-        for (int k = lane; k < m; k += 32) {
-            const uint64_t ck = scb[k];
-            long long before = 0;            // capacity of the cheaper devices
-            for (int j = 0; j < m; ++j) {
-                const uint64_t cj = scb[j];
-                if (cj < ck || (cj == ck && j < k)) before += sc0[j] - 1;
-            }
-            const long long ek = sc0[k] - 1;
-            const long long room = (long long)(N - m) - before;
-            const long long take = room <= 0 ? 0 : (room < ek ? room : ek);
-            part += keyd(ck) * (double)(1 + take);
-            if (k >= 1) part += tau[(size_t)sdev[k - 1] * M + sdev[k]];
-        }
-        const double lb = warp_sum_d(part) * (1.0 - 1e-9);
-        if (lb > dm.lam_max) {                                  // 1.0 / lb < Min_TPS
-            if (lane == 0) atomicAdd(&stats[kStTpsPruned], 1ull);
-            return;
-        }
-    }
-    if (lane == 0) atomicOr(reinterpret_cast<unsigned long long *>(&si.mask[slot]), 1ull << i);
-}
-
-// Writes the outputs of a replica that cannot serve.
-__device__ __forceinline__ void write_unserved(const EvalOut &out, size_t gk, int16_t *lay, int m)
-{
-    for (int k = 0; k < m; ++k) lay[k] = -1;
-    out.master[gk] = -1; out.bsel[gk] = -1;
-    out.T[gk] = keyd(kInfKey); out.L[gk] = keyd(kInfKey);
-}
+// Shared-memory bytes per warp of the pre-pass (26 bytes per device, rounded
+// up to 16 so that every warp's 64-bit arrays start aligned).
+__host__ __device__ __forceinline__ size_t variant_stride(int mcap) { return ((size_t)mcap * 26 + 15) & ~(size_t)15; }
 
 // Per slot: slots with nothing to run get their outputs here (empty slots,
 // more devices than blocks, no variant left by the pre-pass).  Every other
@@ -238,86 +142,206 @@ __device__ __forceinline__ int item_bin(int level, int size)
     return (63 - lv) * kSizeBins + size;
 }
 
-// Outputs of a slot with nothing to run, or the bin and count of its work
-// items (returns 0 items for the former).
-__device__ __forceinline__ int slot_items(const Dims &dm, const DevPop &pop, const SlotInfo &si,
-                                          const EvalOut &out, int slot, int *bin)
+// Pre-pass and work count, one warp per (genome, replica slot).  For each
+// variant of the replica (prefill: v = 0; decode: v = 1..b_max, bit v-1) the
+// warp decides whether a DP run can matter:
+//  * memory: with identical blocks a partition with master mu exists iff every
+//    device holds >= 1 block and the capacities, capped at W = N - m + 1, add
+//    up to N (exact);
+//  * decode latency: Lambda >= sum of link times + sum_k n_k c_k (c_k the
+//    per-block time, the head only adds), whose least value puts one block on
+//    each device and the other N - m on the cheapest devices up to their
+//    capacity.  A variant whose bound misses Min_TPS fails whatever partition
+//    the DP returns; the 1e-9 margin exceeds the rounding of every sum here.
+// Both tests are monotone in the batch: the capacities shrink as b grows (more
+// KV memory per block), and the bound is the least of a linear cost whose
+// coefficients (per-block and link times) grow with b over a feasible set that
+// shrinks with b.  So the variants are tested from the largest batch down and
+// the first that passes keeps every smaller batch as well (rounding could at
+// most keep a variant the bound would have dropped, which costs a DP run and
+// changes no result).  The surviving variants form the slot's mask.  A slot with nothing to run
+// (empty, more devices than blocks, no variant left) gets its outputs here;
+// the others count their work items into the ordering bins.  The last CTA to
+// finish (a ticket taken after a fence, no waiting) scans the bins into
+// starting offsets, heaviest first, and stores the item total.
+__global__ void __launch_bounds__(128, 12) slot_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si, EvalOut out,
+                                                   unsigned *ctrl)
 {
-    const int g = slot / dm.K, c = slot - g * dm.K;
-    si.best[slot] = -1;
-    if (c >= pop.nclus[g]) {
-        out.master[slot] = -1; out.bsel[slot] = -1;
-        out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
-        return 0;
+    // per warp: device ids, capacities and per-block times of up to mcap devices
+    extern __shared__ __align__(16) unsigned char vsm[];
+    __shared__ int s_last;
+    __shared__ unsigned s_part[4];
+    const int mcap = dm.M < dm.N ? dm.M : dm.N;
+    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
+    const int K = dm.K, M = dm.M, N = dm.N;
+    const long long slot = (long long)blockIdx.x * (blockDim.x >> 5) + wl;
+    if (slot < (long long)dm.P * K) {
+        const int g = (int)(slot / K), c = (int)(slot - (long long)g * K);
+        const int R = pop.nclus[g];
+        uint64_t mask = 0;
+        unsigned long long n_pre = 0, n_tps = 0;
+        int m = 0, off = 0, role = 0;
+        if (c < R) {
+            const uint16_t *sz = pop.sizes + (size_t)g * K;
+            m = sz[c];
+            role = (int)((pop.roles[g] >> c) & 1ull);
+            off = warp_sum(lane < c ? sz[lane] : 0) + warp_sum(lane + 32 < c ? sz[lane + 32] : 0);
+            if (lane == 0) si.off[slot] = off;
+        }
+        if (c < R && m <= N) {
+            const int W = N - m + 1;
+            unsigned char *wbase = vsm + (size_t)wl * variant_stride(mcap);
+            uint64_t *scb = reinterpret_cast<uint64_t *>(wbase);          // per-block times as order keys
+            double *stau = reinterpret_cast<double *>(scb + mcap);        // link (k-1) -> k
+            int *sc0 = reinterpret_cast<int *>(stau + mcap), *sc1 = sc0 + mcap;
+            uint16_t *sdev = reinterpret_cast<uint16_t *>(sc1 + mcap);
+            for (int k = lane; k < m; k += 32) sdev[k] = pop.perm[(size_t)g * M + off + k];
+            __syncwarp();
+            const int nvar = role ? dm.b_max : 1;
+            for (int i = nvar - 1; i >= 0; --i) {                 // largest batch first
+                const int v = role ? i + 1 : 0;
+                const int32_t *cap = tb.cap + (size_t)v * M * 2;
+                const bool bound = role && dm.min_tps > 0.0;
+                const double *cpb = tb.cpb + (size_t)v * M;
+                const double *tau = tb.tau + (size_t)v * M * M;
+                int s0 = 0, z = 0;
+                for (int k = lane; k < m; k += 32) {                   // every load of the variant at once
+                    const int d = sdev[k];
+                    const int c0 = min(cap[d * 2], W), c1 = min(cap[d * 2 + 1], W);
+                    if (bound) {
+                        scb[k] = dkey(cpb[d]);
+                        stau[k] = k ? tau[(size_t)sdev[k - 1] * M + d] : 0.0;
+                    }
+                    sc0[k] = c0;
+                    sc1[k] = c1;
+                    s0 += c0;
+                    z += c0 == 0;
+                }
+                s0 = warp_sum(s0);
+                z = warp_sum(z);
+                __syncwarp();
+                bool ok = false;
+                for (int k = lane; k < m && !ok; k += 32)
+                    ok = (z - (sc0[k] == 0)) == 0 && sc1[k] >= 1 && s0 - sc0[k] + sc1[k] >= N;
+                if (!__any_sync(0xFFFFFFFFu, ok)) {
+                    ++n_pre;
+                    continue;
+                }
+                if (bound) {
+                    double part = 0.0;
+                    for (int k = lane; k < m; k += 32) {
+                        const uint64_t ck = scb[k];
+                        long long before = 0;            // capacity of the cheaper devices
+                        for (int j = 0; j < m; ++j) {
+                            const uint64_t cj = scb[j];
+                            if (cj < ck || (cj == ck && j < k)) before += sc0[j] - 1;
+                        }
+                        const long long ek = sc0[k] - 1;
+                        const long long room = (long long)(N - m) - before;
+                        const long long take = room <= 0 ? 0 : (room < ek ? room : ek);
+                        part += keyd(ck) * (double)(1 + take);
+                        if (k >= 1) part += stau[k];
+                    }
+                    const double lb = warp_sum_d(part) * (1.0 - 1e-9);
+                    __syncwarp();
+                    if (lb > dm.lam_max) {                              // 1.0 / lb < Min_TPS
+                        ++n_tps;
+                        continue;
+                    }
+                }
+                mask = (2ull << i) - 1ull;         // this variant and every smaller batch
+                break;
+            }
+        }
+        // ---- the slot's outputs or its work count
+        if (c < R && !mask)                                          // a replica that cannot serve
+            for (int k = lane; k < m; k += 32) out.layers[(size_t)g * M + off + k] = -1;
+        if (lane == 0) {
+            si.mask[slot] = mask;
+            si.best[slot] = -1;
+            if (n_pre) atomicAdd(&out.stats[kStPrecheck], n_pre);
+            if (n_tps) atomicAdd(&out.stats[kStTpsPruned], n_tps);
+            if (!mask) {
+                out.master[slot] = -1; out.bsel[slot] = -1;
+                out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
+                if (c < R) {
+                    atomicAdd(&out.stats[kStReplicas], 1ull);
+                    if (m <= N) atomicAdd(&out.stats[kStPaper], (role ? dm.b_max : 1) * paper_candidates(m, N));
+                }
+            } else {
+                const int W = N - m + 1;
+                const int lg = (int)(1.0f * __log2f(1.0f + (float)m * (float)W));
+                const int size = lg < kSizeBins - 1 ? lg : kSizeBins - 1;
+                si.size[slot] = (uint8_t)size;
+                const int nv = __popcll(mask);
+                for (int lv = 0; lv < nv; ++lv) atomicAdd(&ctrl[item_bin(lv, size)], 1u);
+            }
+        }
     }
-    const uint64_t mask = si.mask[slot];
-    const int m = pop.sizes[slot];
-    const int role = (int)((pop.roles[g] >> c) & 1ull);
-    if (!mask) {
-        write_unserved(out, slot, out.layers + (size_t)g * dm.M + si.off[slot], m);
-        atomicAdd(&out.stats[kStReplicas], 1ull);
-        if (m <= dm.N) atomicAdd(&out.stats[kStPaper], (role ? dm.b_max : 1) * paper_candidates(m, dm.N));
-        return 0;
-    }
-    const int W = dm.N - m + 1;
-    const int sz = (int)(1.0f * __log2f(1.0f + (float)m * (float)W));
-    const int size = sz < kSizeBins - 1 ? sz : kSizeBins - 1;
-    si.size[slot] = (uint8_t)size;
-    *bin = size;
-    return __popcll(mask);
-}
-
-// Item lv of a slot goes to bin item_bin(lv, size); emits (slot << 8) | bit.
-template <typename CursorFn>
-__device__ __forceinline__ void slot_emit(const SlotInfo &si, const WorkList &wl, int slot, CursorFn cursor)
-{
-    uint64_t mask = si.mask[slot];
-    const int size = si.size[slot];
-    for (int lv = 0; mask; ++lv) {
-        const int bit = 63 - __clzll((long long)mask);
-        mask &= ~(1ull << bit);
-        wl.items[cursor(item_bin(lv, size))] = ((uint64_t)slot << 8) | (uint64_t)bit;
-    }
-}
-
-__global__ void key_kernel(Dims dm, DevPop pop, SlotInfo si, EvalOut out, unsigned *bins)
-{
-    const int total = dm.P * dm.K;
-    for (int slot = blockIdx.x * blockDim.x + threadIdx.x; slot < total; slot += gridDim.x * blockDim.x) {
-        int size = 0;
-        const int nv = slot_items(dm, pop, si, out, slot, &size);
-        for (int lv = 0; lv < nv; ++lv) atomicAdd(&bins[item_bin(lv, size)], 1u);
-    }
-}
-
-// Exclusive scan of the bins in descending key order (heaviest first); the
-// total number of work items goes to bins[kOrderBins].
-__global__ void order_scan_kernel(unsigned *bins)
-{
-    __shared__ unsigned s[kOrderBins];
-    const int t = threadIdx.x;
-    s[t] = bins[kOrderBins - 1 - t];
+    // ---- the last CTA scans the bins
     __syncthreads();
-    for (int o = 1; o < kOrderBins; o <<= 1) {
-        const unsigned v = t >= o ? s[t - o] : 0u;
-        __syncthreads();
-        s[t] += v;
-        __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        s_last = atomicAdd(&ctrl[kCtrlTicket], 1u) == gridDim.x - 1;
     }
-    const unsigned incl = s[t];
-    const unsigned cnt = bins[kOrderBins - 1 - t];
     __syncthreads();
-    bins[kOrderBins - 1 - t] = incl - cnt;
-    if (t == kOrderBins - 1) { bins[kOrderBins] = incl; bins[kOrderBins + 1] = 0u; }
+    if (!s_last) return;
+    __threadfence();
+    // thread t owns positions [8t, 8t + 8) of the descending bin order
+    constexpr int kPer = kOrderBins / 128;
+    unsigned *own = ctrl + kOrderBins - 1 - threadIdx.x * kPer;      // own[-j] = position 8t + j
+    unsigned sum = 0;
+    for (int j = 0; j < kPer; ++j) sum += __ldcg(own - j);
+    unsigned incl = sum;                                   // inclusive scan over the warp
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned x = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += x;
+    }
+    if (lane == 31) s_part[wl] = incl;
+    __syncthreads();
+    unsigned base = incl - sum;
+    for (int w = 0; w < wl; ++w) base += s_part[w];
+    for (int j = 0; j < kPer; ++j) {
+        const unsigned cnt = __ldcg(own - j);
+        own[-j] = base;
+        base += cnt;
+    }
+    if (threadIdx.x == 127) ctrl[kCtrlTotal] = base;
 }
 
+// Item lv of a slot (its variants from the largest batch down) goes to bin
+// item_bin(lv, size) as (slot << 8) | bit.  The lanes of a warp whose items
+// share a bin take their positions with one atomic.
 __global__ void order_scatter_kernel(Dims dm, DevPop pop, SlotInfo si, WorkList wl)
 {
-    const int total = dm.P * dm.K;
-    for (int slot = blockIdx.x * blockDim.x + threadIdx.x; slot < total; slot += gridDim.x * blockDim.x) {
-        const int g = slot / dm.K, c = slot - g * dm.K;
-        if (c >= pop.nclus[g] || !si.mask[slot]) continue;
-        slot_emit(si, wl, slot, [&](int b) { return atomicAdd(&wl.ctrl[b], 1u); });
+    const int total = dm.P * dm.K, lane = threadIdx.x & 31;
+    const unsigned below = (1u << lane) - 1u;
+    for (int base = blockIdx.x * blockDim.x + (threadIdx.x & ~31); base < total; base += gridDim.x * blockDim.x) {
+        const int slot = base + lane;
+        uint64_t mask = 0;
+        int size = 0;
+        if (slot < total) {
+            const int g = slot / dm.K, c = slot - g * dm.K;
+            if (c < pop.nclus[g]) mask = si.mask[slot];
+            if (mask) size = si.size[slot];
+        }
+        for (int lv = 0; __any_sync(0xFFFFFFFFu, mask != 0); ++lv) {
+            int bit = 0, bin = -1;
+            if (mask) {
+                bit = 63 - __clzll((long long)mask);
+                mask &= ~(1ull << bit);
+                bin = item_bin(lv, size);
+            }
+            const unsigned peers = __match_any_sync(0xFFFFFFFFu, bin);
+            if (bin >= 0) {
+                const int leader = __ffs(peers) - 1;
+                unsigned at = 0;
+                if (lane == leader) at = atomicAdd(&wl.ctrl[bin], (unsigned)__popc(peers));
+                at = __shfl_sync(peers, at, leader);
+                wl.items[at + __popc(peers & below)] = ((uint64_t)slot << 8) | (uint64_t)bit;
+            }
+        }
     }
 }
 
@@ -358,10 +382,10 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
 
     const int K = dm.K, M = dm.M, N = dm.N;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
-    const unsigned n_items = wl.ctrl[kOrderBins];
+    const unsigned n_items = wl.ctrl[kCtrlTotal];
   for (;;) {
     // ---- next work item (heaviest first)
-    if (tid == 0) s_item = atomicAdd(&wl.ctrl[kOrderBins + 1], 1u);
+    if (tid == 0) s_item = atomicAdd(&wl.ctrl[kCtrlNext], 1u);
     __syncthreads();
     const unsigned idx = s_item;
     __syncthreads();
@@ -589,58 +613,27 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
   }
 }
 
-// One warp per genome.  First each replica that had work gets its outputs:
-// the largest accepted variant is the sweep's answer (Alg. 2 keeps the highest
-// feasible batch), with its master, batch, times and partition.  Then the
-// objective (Sec. 3.3): each serving replica's rate (NP / T for prefill, b / T
-// for decode) by its own lane, PS and DS summed by lane 0 in ascending replica
-// order, Eq. 3 (bottleneck phase), Eq. 4 (backlog) and Eq. 5 (waiting time);
-// and a 64-bit fingerprint of the genome for the elites' duplicate test.
+// One warp per genome.  Each replica that had work gets its outputs from its
+// lane: the largest accepted variant is the sweep's answer (Alg. 2 keeps the
+// highest feasible batch), with its master, batch and times, and the serving
+// replica's rate (NP / T for prefill, b / T for decode).  The lanes then copy
+// the partition, position by position, from the accepted variant's split
+// results.  Lane 0 sums PS and DS in ascending replica order and applies
+// Eq. 3 (bottleneck phase), Eq. 4 (backlog) and Eq. 5 (waiting time).  A
+// 64-bit fingerprint of the genome, folded as a tree over the lanes, serves
+// the elites' duplicate test.
 __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop, SlotInfo si, SplitOut so,
                                                              EvalOut out)
 {
-    const int g = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    __shared__ int s_off[4][E2_MAX_CLUSTERS + 1];     // replica start in the ordering
+    __shared__ int s_best[4][E2_MAX_CLUSTERS];        // accepted variant bit, -1 none, -2 no work here
+    const int wl = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = blockIdx.x * 4 + wl;
     if (g >= dm.P) return;
     const int K = dm.K, M = dm.M;
     const int R = pop.nclus[g];
     const uint64_t roles = pop.roles[g];
     unsigned long long n_rep = 0, n_served = 0, n_paper = 0;
-    for (int c = 0; c < R; ++c) {
-        const int slot = g * K + c;
-        if (!si.mask[slot]) continue;                      // done by the ordering pass
-        const int m = pop.sizes[slot], off = si.off[slot];
-        const int role = (int)((roles >> c) & 1ull);
-        const int best = si.best[slot];
-        int16_t *lay = out.layers + (size_t)g * M + off;
-        unsigned long long nrun = role ? (unsigned long long)dm.b_max : 1ull;
-        if (best < 0) {
-            for (int k = lane; k < m; k += 32) lay[k] = -1;
-            if (lane == 0) {
-                out.master[slot] = -1; out.bsel[slot] = -1;
-                out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
-            }
-        } else {
-            const size_t sv = (size_t)slot * dm.b_max + best;
-            const int16_t *src = so.layers + ((size_t)g * dm.b_max + best) * M + off;
-            for (int k = lane; k < m; k += 32) lay[k] = src[k];
-            if (lane == 0) {
-                out.master[slot] = so.mu[sv];
-                out.bsel[slot] = (int16_t)(role ? best + 1 : 0);
-                out.T[slot] = so.T[sv];
-                out.L[slot] = so.L[sv];
-            }
-            if (role) nrun = (unsigned long long)(dm.b_max - best);   // variants b_max .. best+1
-            ++n_served;
-        }
-        ++n_rep;
-        n_paper += nrun * paper_candidates(m, dm.N);
-    }
-    if (lane == 0 && n_rep) {
-        atomicAdd(&out.stats[kStReplicas], n_rep);
-        atomicAdd(&out.stats[kStPaper], n_paper);
-        if (n_served) atomicAdd(&out.stats[kStServed], n_served);
-    }
-    __syncwarp();
     double rate[2];
     int kind[2];                                   // -1 none, 0 prefill, 1 decode
 #pragma unroll
@@ -649,13 +642,61 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
         kind[h] = -1;
         rate[h] = 0.0;
         if (c < R) {
-            const int b = out.bsel[(size_t)g * K + c];
-            if (b >= 0) {
-                const double T = out.T[(size_t)g * K + c];
-                kind[h] = (int)((roles >> c) & 1ull);
-                rate[h] = kind[h] ? (double)b / T : (double)dm.NP / T;
+            const int slot = g * K + c;
+            const uint64_t mask = si.mask[slot];
+            s_off[wl][c] = si.off[slot];
+            int best = -2;                         // no work: outputs written by the pre-pass
+            if (mask) {
+                const int m = pop.sizes[slot];
+                const int role = (int)((roles >> c) & 1ull);
+                best = si.best[slot];
+                unsigned long long nrun = role ? (unsigned long long)dm.b_max : 1ull;
+                if (best < 0) {
+                    out.master[slot] = -1; out.bsel[slot] = -1;
+                    out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
+                } else {
+                    const size_t sv = (size_t)slot * dm.b_max + best;
+                    const double T = so.T[sv];
+                    out.master[slot] = so.mu[sv];
+                    out.bsel[slot] = (int16_t)(role ? best + 1 : 0);
+                    out.T[slot] = T;
+                    out.L[slot] = so.L[sv];
+                    if (role) nrun = (unsigned long long)(dm.b_max - best);   // variants b_max .. best+1
+                    ++n_served;
+                    kind[h] = role;
+                    rate[h] = role ? (double)(best + 1) / T : (double)dm.NP / T;
+                }
+                ++n_rep;
+                n_paper += nrun * paper_candidates(m, dm.N);
             }
+            s_best[wl][c] = best;
         }
+    }
+    if (lane == 0) s_off[wl][R] = M;
+    __syncwarp();
+    // partition: position i belongs to the last replica c with off_c <= i
+    const int16_t *split = so.layers + (size_t)g * dm.b_max * M;
+    for (int i = lane; i < M; i += 32) {
+        int lo = 0, hi = R - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (s_off[wl][mid] <= i) lo = mid;
+            else hi = mid - 1;
+        }
+        const int best = s_best[wl][lo];
+        if (best >= 0) out.layers[(size_t)g * M + i] = split[(size_t)best * M + i];
+        else if (best == -1) out.layers[(size_t)g * M + i] = -1;
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        n_rep += __shfl_xor_sync(0xFFFFFFFFu, n_rep, o);
+        n_served += __shfl_xor_sync(0xFFFFFFFFu, n_served, o);
+        n_paper += __shfl_xor_sync(0xFFFFFFFFu, n_paper, o);
+    }
+    if (lane == 0 && n_rep) {
+        atomicAdd(&out.stats[kStReplicas], n_rep);
+        atomicAdd(&out.stats[kStPaper], n_paper);
+        if (n_served) atomicAdd(&out.stats[kStServed], n_served);
     }
     double PS = 0.0, DS = 0.0;
     for (int c = 0; c < R; ++c) {
@@ -665,14 +706,18 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
         if (k == 0) PS = PS + x;
         else if (k == 1) DS = DS + x;
     }
-    // fingerprint: lanes mix interleaved slices of the ordering, lane 0 folds
+    // fingerprint: lanes mix interleaved slices of the ordering, then a tree fold
     uint64_t hl = 0x9E3779B97F4A7C15ull ^ (uint64_t)lane;
     auto mix = [](uint64_t h, uint64_t x) { h = (h ^ x) * 0xBF58476D1CE4E5B9ull; return h ^ (h >> 31); };
     const uint16_t *pp = pop.perm + (size_t)g * M;
     for (int i = lane; i < M; i += 32) hl = mix(hl, pp[i]);
-    uint64_t h = 0;
-    for (int l = 0; l < 32; ++l) h = mix(h, __shfl_sync(0xFFFFFFFFu, hl, l));
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        const uint64_t other = __shfl_down_sync(0xFFFFFFFFu, hl, o);
+        if (lane < o) hl = mix(hl, other);
+    }
     if (lane != 0) return;
+    uint64_t h = hl;
     double w = keyd(kInfKey), phase = keyd(kInfKey);
     if (PS != 0.0 && DS != 0.0) {
         const double tp = (double)dm.NP / PS, td = (double)dm.ND / DS;
@@ -712,16 +757,12 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     WorkList wl{c->items, c->order_bins};
     SplitOut so{c->split_T, c->split_L, c->split_mu, c->split_layers};
     const long long slots = (long long)c->dm.P * c->dm.K;
-    cudaError_t e = cudaMemsetAsync(c->order_bins, 0, sizeof(unsigned) * (kOrderBins + 2), c->stream);
-    if (e == cudaSuccess) e = cudaMemsetAsync(c->slot_mask, 0, sizeof(uint64_t) * (size_t)slots, c->stream);
+    cudaError_t e = cudaMemsetAsync(c->order_bins, 0, sizeof(unsigned) * kCtrlWords, c->stream);
     if (e != cudaSuccess) return e;
     const unsigned gb = (unsigned)((slots + 255) / 256 < 1024 ? (slots + 255) / 256 : 1024);
-    const long long vwarps = slots * c->dm.b_max;
     const int mcap = c->dm.M < c->dm.N ? c->dm.M : c->dm.N;
-    variant_kernel<<<(unsigned)((vwarps * 32 + 127) / 128), 128, 4 * variant_stride(mcap), c->stream>>>(c->dm, tb, p, si,
-                                                                                                  c->stats);
-    key_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, out, c->order_bins);
-    order_scan_kernel<<<1, kOrderBins, 0, c->stream>>>(c->order_bins);
+    slot_kernel<<<(unsigned)((slots + 3) / 4), 128, 4 * variant_stride(mcap), c->stream>>>(c->dm, tb, p, si, out,
+                                                                                       c->order_bins);
     order_scatter_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, wl);
     if (c->ev_dp_start) cudaEventRecord(c->ev_dp_start, c->stream);
     dp_eval_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so);

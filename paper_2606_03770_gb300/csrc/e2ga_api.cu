@@ -75,7 +75,7 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K)
     l.elite_fit = take(32 * (size_t)(Q > 0 ? Q : 1));
     l.stats = take(8 * kNumStats);
     l.err = take(4);
-    l.order_bins = take(4 * (kOrderBins + 2));
+    l.order_bins = take(4 * (size_t)kCtrlWords);
     l.items = take(8 * (size_t)P * K * b_max);
     l.slot_off = take(4 * (size_t)P * K);
     l.slot_mask = take(8 * (size_t)P * K);

@@ -41,6 +41,9 @@ constexpr int kMaxReplicaDevices = 256;
 // variant among its replica's variants, largest batch first) x 16 work sizes.
 constexpr int kOrderBins = 1024;
 constexpr int kSizeBins = 16;
+// Control words after the ordering bins: item total, next item of the DP, the
+// pre-pass's CTA ticket.
+enum CtrlWord { kCtrlTotal = kOrderBins, kCtrlNext, kCtrlTicket, kCtrlWords };
 
 // Stats slots (unsigned long long, atomically accumulated).
 enum StatSlot { kStGenomes = 0, kStReplicas, kStDpRuns, kStCells, kStProbes, kStPaper, kStPrecheck,
@@ -79,7 +82,7 @@ struct SlotInfo {
 // Work items of the DP: (slot << 8) | variant bit.
 struct WorkList {
     uint64_t *items;           // [P*K*b_max]
-    unsigned *ctrl;            // [kOrderBins] bins/cursors, then [kOrderBins] = total, [+1] = next item
+    unsigned *ctrl;            // [kOrderBins] bins/cursors, then the CtrlWord words
 };
 
 // Results of the DP runs, per (slot, variant bit).
@@ -179,7 +182,7 @@ struct e2_ctx {
     double *elite_fit = nullptr;
     unsigned long long *stats = nullptr;
     int32_t *err = nullptr;
-    unsigned *order_bins = nullptr;   // [kOrderBins + 2]
+    unsigned *order_bins = nullptr;   // [kCtrlWords]
     uint64_t *items = nullptr;        // [P*K*b_max] DP work items, heaviest first
     int32_t *slot_off = nullptr;      // [P*K]
     uint64_t *slot_mask = nullptr;    // [P*K]
