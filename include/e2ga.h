@@ -222,6 +222,24 @@ int e2_get_congestion(e2_ctx *ctx, double *cong_out);
  * e2_ga_step) and their fitness [Q][4]; either may be NULL. */
 int e2_get_elites(e2_ctx *ctx, int32_t *idx_out, double *fitness_out);
 
+/* Copies the results of the most recent evaluation (by e2_eval_population or
+ * e2_run_generation): fitness P x 4 and, if parts is not NULL, the partitions;
+ * host or device pointers, NULL ones skipped.  Synchronises when a
+ * destination is host memory.  E2_ESTATE if nothing was evaluated yet. */
+int e2_get_results(e2_ctx *ctx, double *fitness_out, const e2_partitions *parts);
+
+/* One generation of Alg. 2 from the current population: its evaluation
+ * (as e2_eval_population(ctx, NULL, NULL, NULL)) followed by the elites and the
+ * next population (as e2_ga_step(ctx, seed, generation)), with the same
+ * results.  The context records this launch sequence as a CUDA graph on first
+ * use (one per population buffer, recorded on a private stream and again when
+ * the timing events of e2_set_timing_events change) and afterwards replays it
+ * on its stream, setting only the new seed and generation: one launch instead
+ * of nine (two memsets and seven kernels).  If recording fails the calls are
+ * issued one by one.
+ * E2_EINVAL for a NULL context; E2_ECUDA on a CUDA failure. */
+int e2_run_generation(e2_ctx *ctx, uint64_t seed, uint32_t generation);
+
 /* Counters of the last evaluation.  Synchronises. */
 int e2_get_stats(e2_ctx *ctx, e2_stats *out);
 

@@ -764,9 +764,15 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     slot_kernel<<<(unsigned)((slots + 3) / 4), 128, 4 * variant_stride(mcap), c->stream>>>(c->dm, tb, p, si, out,
                                                                                        c->order_bins);
     order_scatter_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, wl);
-    if (c->ev_dp_start) cudaEventRecord(c->ev_dp_start, c->stream);
+    // while a launch sequence is being recorded, the timing events become
+    // event-record nodes of the graph (an ordinary record would only mark a
+    // dependency)
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (c->ev_dp_start && (e = cudaStreamIsCapturing(c->stream, &cs)) != cudaSuccess) return e;
+    const unsigned rec = cs == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : cudaEventRecordDefault;
+    if (c->ev_dp_start && (e = cudaEventRecordWithFlags(c->ev_dp_start, c->stream, rec)) != cudaSuccess) return e;
     dp_eval_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so);
-    if (c->ev_dp_stop) cudaEventRecord(c->ev_dp_stop, c->stream);
+    if (c->ev_dp_stop && (e = cudaEventRecordWithFlags(c->ev_dp_stop, c->stream, rec)) != cudaSuccess) return e;
     finalize_score_kernel<<<(unsigned)(((size_t)c->dm.P * 32 + 127) / 128), 128, 0, c->stream>>>(c->dm, p, si, so,
                                                                                                out);
     return cudaGetLastError();

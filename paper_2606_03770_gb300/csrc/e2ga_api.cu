@@ -383,10 +383,63 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     return E2_OK;
 }
 
+namespace {
+
+void drop_generation_graph(e2_ctx *c, int b)
+{
+    if (c->gen_exec[b]) cudaGraphExecDestroy(c->gen_exec[b]);
+    if (c->gen_graph[b]) cudaGraphDestroy(c->gen_graph[b]);
+    c->gen_exec[b] = nullptr;
+    c->gen_graph[b] = nullptr;
+    c->gen_ga_node[b] = nullptr;
+}
+
+// Records the launches of one generation from population buffer b (the same
+// sequence e2_eval_population and e2_ga_step issue) on the private stream.
+cudaError_t record_generation(e2_ctx *c, int b)
+{
+    drop_generation_graph(c, b);
+    cudaError_t e = cudaSuccess;
+    if (!c->cap_stream) e = cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking);
+    if (e != cudaSuccess) return e;
+    const cudaStream_t user = c->stream;
+    c->stream = c->cap_stream;
+    e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
+    if (e == cudaSuccess) {
+        cudaError_t le = cudaMemsetAsync(c->stats, 0, 8 * kNumStats, c->stream);
+        if (le == cudaSuccess) le = launch_eval(c, c->pop[b]);
+        if (le == cudaSuccess) le = launch_elites(c, c->pop[b]);
+        if (le == cudaSuccess) le = launch_ga(c, c->pop[b], c->pop[b ^ 1], 0, 0);
+        cudaGraph_t g = nullptr;
+        e = cudaStreamEndCapture(c->cap_stream, &g);
+        if (le != cudaSuccess) e = le;
+        if (e == cudaSuccess) {
+            c->gen_graph[b] = g;
+            e = cudaGraphInstantiate(&c->gen_exec[b], g, 0);
+        } else if (g) {
+            cudaGraphDestroy(g);
+        }
+    }
+    c->stream = user;
+    if (e == cudaSuccess) e = find_ga_node(c->gen_graph[b], &c->gen_ga_node[b]);
+    if (e != cudaSuccess) {
+        drop_generation_graph(c, b);
+        cudaGetLastError();
+        return e;
+    }
+    c->gen_ev[b][0] = c->ev_dp_start;
+    c->gen_ev[b][1] = c->ev_dp_stop;
+    return cudaSuccess;
+}
+
+}  // namespace
+
 int e2_destroy(e2_ctx *c)
 {
     if (!c) return E2_OK;
     cudaError_t e = cudaStreamSynchronize(c->stream);
+    for (int b = 0; b < 2; ++b) drop_generation_graph(c, b);
+    if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
     delete c;
     return e == cudaSuccess ? E2_OK : E2_ECUDA;
 }
@@ -421,6 +474,14 @@ int e2_eval_population(e2_ctx *c, const e2_genomes *genomes, double *fitness_out
     E2_CUDA(c, cudaMemsetAsync(c->stats, 0, 8 * kNumStats, c->stream));
     E2_CUDA(c, launch_eval(c, c->pop[c->cur]));
     c->evaluated = true;
+    c->have_results = true;
+    return e2_get_results(c, fitness_out, parts);
+}
+
+int e2_get_results(e2_ctx *c, double *fitness_out, const e2_partitions *parts)
+{
+    if (!c) return E2_EINVAL;
+    if (!c->have_results) return fail(c, E2_ESTATE, "no population has been evaluated");
     const size_t P = c->dm.P, M = c->dm.M, K = c->dm.K;
     bool host = false;
     auto out = [&](void *dst, const void *src, size_t bytes) -> cudaError_t {
@@ -446,6 +507,25 @@ int e2_ga_step(e2_ctx *c, uint64_t seed, uint32_t generation)
     if (!c->evaluated) return fail(c, E2_ESTATE, "the current population has not been evaluated");
     E2_CUDA(c, launch_elites(c, c->pop[c->cur]));
     E2_CUDA(c, launch_ga(c, c->pop[c->cur], c->pop[c->cur ^ 1], seed, generation));
+    c->cur ^= 1;
+    c->evaluated = false;
+    c->have_elites = true;
+    return E2_OK;
+}
+
+int e2_run_generation(e2_ctx *c, uint64_t seed, uint32_t generation)
+{
+    if (!c) return E2_EINVAL;
+    const int b = c->cur;
+    if (!c->gen_eager && (!c->gen_exec[b] || c->gen_ev[b][0] != c->ev_dp_start || c->gen_ev[b][1] != c->ev_dp_stop))
+        c->gen_eager = record_generation(c, b) != cudaSuccess;
+    if (c->gen_eager) {                                         // the same work, launched one by one
+        int st = e2_eval_population(c, nullptr, nullptr, nullptr);
+        return st ? st : e2_ga_step(c, seed, generation);
+    }
+    E2_CUDA(c, set_ga_node(c, c->gen_exec[b], c->gen_ga_node[b], c->pop[b], c->pop[b ^ 1], seed, generation));
+    E2_CUDA(c, cudaGraphLaunch(c->gen_exec[b], c->stream));
+    c->have_results = true;
     c->cur ^= 1;
     c->evaluated = false;
     c->have_elites = true;

@@ -193,11 +193,19 @@ struct e2_ctx {
     int16_t *split_layers = nullptr;                 // [P*b_max*M]
     int dp_grid = 0;                  // persistent DP CTAs
     cudaEvent_t ev_dp_start = nullptr, ev_dp_stop = nullptr;   // optional timing hook
+    // recorded generation (e2_run_generation), one per population buffer
+    cudaStream_t cap_stream = nullptr;                          // private stream the graphs are recorded on
+    cudaGraph_t gen_graph[2] = {nullptr, nullptr};
+    cudaGraphExec_t gen_exec[2] = {nullptr, nullptr};
+    cudaGraphNode_t gen_ga_node[2] = {nullptr, nullptr};        // the generation kernel's node
+    cudaEvent_t gen_ev[2][2] = {{nullptr, nullptr}, {nullptr, nullptr}};   // timing events recorded in it
+    bool gen_eager = false;                                     // recording failed: eager launches
     // launch shapes
     int dp_threads = 128;
     size_t dp_smem = 0;
     bool evaluated = false;
     bool have_elites = false;
+    bool have_results = false;           // an evaluation has filled the result buffers
     std::string last_error;
 };
 
@@ -211,6 +219,10 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p);
 cudaError_t launch_init(const e2_ctx *c, const DevPop &p, uint64_t seed);
 cudaError_t launch_elites(const e2_ctx *c, const DevPop &p);
 cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen);
+// the generation kernel's node of a recorded graph, and new (seed, generation) for it
+cudaError_t find_ga_node(cudaGraph_t graph, cudaGraphNode_t *node);
+cudaError_t set_ga_node(const e2_ctx *c, cudaGraphExec_t exec, cudaGraphNode_t node, const DevPop &src,
+                        const DevPop &dst, uint64_t seed, uint32_t gen);
 size_t dp_smem_bytes(int M, int N, int threads);
 cudaError_t configure_eval(e2_ctx *c);   // shared memory limit and persistent grid size
 size_t rank_pow2(size_t n);

@@ -510,4 +510,45 @@ cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uin
     return cudaGetLastError();
 }
 
+cudaError_t find_ga_node(cudaGraph_t graph, cudaGraphNode_t *node)
+{
+    *node = nullptr;
+    size_t n = 0;
+    cudaError_t e = cudaGraphGetNodes(graph, nullptr, &n);
+    if (e != cudaSuccess) return e;
+    cudaGraphNode_t nodes[64];
+    if (n > 64) return cudaErrorInvalidValue;
+    e = cudaGraphGetNodes(graph, nodes, &n);
+    if (e != cudaSuccess) return e;
+    for (size_t i = 0; i < n; ++i) {
+        cudaGraphNodeType t;
+        if ((e = cudaGraphNodeGetType(nodes[i], &t)) != cudaSuccess) return e;
+        if (t != cudaGraphNodeTypeKernel) continue;
+        cudaKernelNodeParams p{};
+        if ((e = cudaGraphKernelNodeGetParams(nodes[i], &p)) != cudaSuccess) return e;
+        if (p.func == reinterpret_cast<void *>(ga_kernel)) {
+            *node = nodes[i];
+            return cudaSuccess;
+        }
+    }
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t set_ga_node(const e2_ctx *c, cudaGraphExec_t exec, cudaGraphNode_t node, const DevPop &src,
+                        const DevPop &dst, uint64_t seed, uint32_t gen)
+{
+    cudaKernelNodeParams p{};
+    cudaError_t e = cudaGraphKernelNodeGetParams(node, &p);     // launch shape as recorded
+    if (e != cudaSuccess) return e;
+    Dims dm = c->dm;
+    DevPop s = src, d = dst;
+    const double *fit = c->fit;
+    const int32_t *elite = c->elite;
+    GaThr thr{c->thr_cx, c->thr_half, c->thr_mut, c->thr_k1, c->thr_k2, c->thr_k3};
+    void *args[] = {&dm, &s, &d, &fit, &elite, &seed, &gen, &thr};
+    p.kernelParams = args;
+    p.extra = nullptr;
+    return cudaGraphExecKernelNodeSetParams(exec, node, &p);
+}
+
 }  // namespace e2

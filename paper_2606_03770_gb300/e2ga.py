@@ -71,6 +71,8 @@ SIGNATURES = {
     "e2_get_elites": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "e2_get_stats": (C.c_int, [C.c_void_p, C.c_void_p]),
     "e2_set_timing_events": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "e2_run_generation": (C.c_int, [C.c_void_p, C.c_uint64, C.c_uint32]),
+    "e2_get_results": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "e2_select_elites_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
                                             C.c_int32, C.c_void_p, C.c_void_p]),
     "e2_strerror": (C.c_char_p, [C.c_int]),
@@ -150,6 +152,14 @@ def e2_get_elites(ctx, idx_ptr, fit_ptr):
 
 def e2_get_stats(ctx, stats):
     return load().e2_get_stats(ctx, C.byref(stats))
+
+
+def e2_get_results(ctx, fitness_ptr, parts):
+    return load().e2_get_results(ctx, fitness_ptr, C.byref(parts) if parts is not None else None)
+
+
+def e2_run_generation(ctx, seed, generation):
+    return load().e2_run_generation(ctx, seed, generation)
 
 
 def e2_set_timing_events(ctx, start_ptr, stop_ptr):
@@ -257,7 +267,9 @@ class Engine:
         return fit
 
     def results(self):
-        """Copy the last evaluation's device results to numpy."""
+        """The most recent evaluation's results, as numpy arrays."""
+        ps = e2_partitions(_ptr(self.layers), _ptr(self.master), _ptr(self.bsel), _ptr(self.T), _ptr(self.L))
+        _check(e2_get_results(self.ctx, _ptr(self.fitness), ps), "e2_get_results", self.ctx)
         self.torch.cuda.synchronize()
         return dict(fitness=self.fitness.cpu().numpy(), layers=self.layers.cpu().numpy(),
                     master=self.master.cpu().numpy(), bsel=self.bsel.cpu().numpy(), T=self.T.cpu().numpy(),
@@ -265,6 +277,10 @@ class Engine:
 
     def ga_step(self, seed, generation):
         _check(e2_ga_step(self.ctx, seed, generation), "e2_ga_step", self.ctx)
+
+    def run_generation(self, seed, generation):
+        """Evaluation, elites and next population in one recorded launch."""
+        _check(e2_run_generation(self.ctx, seed, generation), "e2_run_generation", self.ctx)
 
     def redraw_congestion(self, seed, generation):
         _check(e2_redraw_congestion(self.ctx, seed, generation), "e2_redraw_congestion", self.ctx)

@@ -291,3 +291,38 @@ def test_min_tps_boundary_exact():
         served.append(int(ref["bsel"][p, c]))
         eng.close()
     assert served[0] == ora["bsel"][p, c] and served[1] != served[0]
+
+
+@pytest.mark.parametrize("name,P,gens", [("c1_tiny", 64, 5), ("c2", 1024, 5)])
+def test_recorded_generation_matches_separate_calls(name, P, gens):
+    """e2_run_generation (one recorded graph per population buffer) gives the
+    populations and fitness of e2_eval_population + e2_ga_step, also when
+    interleaved with the separate calls and after the timing events change."""
+    import torch
+    prob = W.make_config(name, P=P)
+    a, b = engine(prob), engine(prob)
+    a.init_population(5)
+    b.init_population(5)
+    x, y = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for e in (x, y):
+        e.record(torch.cuda.current_stream())
+    for gen in range(1, gens + 1):
+        a.eval(parts=False)
+        fa = a.results()["fitness"]
+        a.ga_step(5, gen)
+        if gen == 3:                                   # the separate calls on the recording engine
+            b.eval(parts=False)
+            fb = b.results()["fitness"]
+            b.ga_step(5, gen)
+        else:
+            if gen == 4:
+                b.set_timing_events(x, y)              # recorded again, with the events
+            b.run_generation(5, gen)
+            fb = b.results()["fitness"]
+        assert np.array_equal(fa, fb), gen
+        assert_genomes_equal(a.get_population(), b.get_population())
+    torch.cuda.synchronize()
+    assert x.elapsed_time(y) > 0
+    b.set_timing_events()
+    a.close()
+    b.close()
