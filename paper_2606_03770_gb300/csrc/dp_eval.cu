@@ -34,7 +34,7 @@
 // Masters.  Alg. 1 reruns the whole table for every master mu.  Here the
 // master-free prefix columns F_k (devices 1..k) and suffix columns G_k
 // (devices k..m) are computed once per run, and each master's bottleneck
-// follows from F_{mu-1}, G_{mu+1} and the master's head row (dp_eval_kernel,
+// follows from F_{mu-1}, G_{mu+1} and the master's head row (dp_eval_body,
 // step 4).  mu* = the smallest mu with the least bottleneck (the oracle's
 // first-wins argmin); its columns are recomputed for the traceback.
 #include "e2ga_internal.cuh"
@@ -43,9 +43,10 @@ namespace e2 {
 
 namespace {
 
-// D_k[r] for one cell (see the header comment), on 32-bit order keys.
-__device__ __forceinline__ uint32_t dp_cell(const uint32_t *__restrict__ prev,
-                                            const uint32_t *__restrict__ row, uint32_t tau, int r)
+// D_k[r] for one cell (see the header comment), on order keys (the largest
+// value is +inf).
+template <typename Key>
+__device__ __forceinline__ Key dp_cell(const Key *__restrict__ prev, const Key *__restrict__ row, Key tau, int r)
 {
     int lo = 0, hi = r + 1;
     while (lo < hi) {
@@ -53,7 +54,7 @@ __device__ __forceinline__ uint32_t dp_cell(const uint32_t *__restrict__ prev,
         if (prev[mid] >= row[r - mid]) hi = mid;
         else lo = mid + 1;
     }
-    uint32_t h = 0xFFFFFFFFu;
+    Key h = (Key)~(Key)0;
     if (lo <= r) h = prev[lo];
     if (lo >= 1) h = min(h, row[r - lo + 1]);
     return max(h, tau);
@@ -93,16 +94,17 @@ __device__ __forceinline__ unsigned long long column_probes(int W)
 
 }  // namespace
 
-// Shared-memory bytes for the largest replica the problem allows.
-size_t dp_smem_bytes(int M, int N, int threads)
+// Shared-memory bytes for the largest replica the problem allows, with keys of
+// key_bytes bytes.
+size_t dp_smem_bytes(int M, int N, int threads, int key_bytes)
 {
     const int NW = threads / 32;
     size_t best = 0;
     const int mmax = M < N ? M : N;
     for (int m = 1; m <= mmax; ++m) {
         const size_t W = (size_t)(N - m + 1);
-        const size_t u32s = 3 * (size_t)m * W + (size_t)(2 * NW + 2) * W + (size_t)m;
-        const size_t bytes = u32s * 4 + (size_t)m * (3 * sizeof(int)) + (size_t)m * sizeof(uint16_t) + 16;
+        const size_t keys = 3 * (size_t)m * W + (size_t)(2 * NW + 2) * W + (size_t)m;
+        const size_t bytes = (size_t)m * (3 * sizeof(int)) + keys * key_bytes + (size_t)m * sizeof(uint16_t) + 16;
         if (bytes > best) best = bytes;
     }
     return (best + 15) & ~(size_t)15;
@@ -345,6 +347,23 @@ __global__ void order_scatter_kernel(Dims dm, DevPop pop, SlotInfo si, WorkList 
     }
 }
 
+// A row of order keys from the rank table into shared memory, copied
+// asynchronously.
+__device__ __forceinline__ void stage_row(uint32_t *dst, const uint32_t *src, int W, int lane)
+{
+    for (int n = lane; n < W; n += 32) cp_async4(dst + n, src + n);
+}
+
+// The head row of a master, fetched asynchronously while the warp builds H.
+template <typename Key> struct HeadRow;
+template <> struct HeadRow<uint32_t> {
+    __device__ __forceinline__ void start(uint32_t *dst, const uint32_t *src, int W, int lane)
+    {
+        for (int r = lane; r < W; r += 32) cp_async4(dst + r, src + r);
+    }
+    __device__ __forceinline__ void finish(uint32_t *, const uint32_t *, int, int) { cp_async_wait_all(); }
+};
+
 // Persistent CTAs; each work item is one (genome, replica slot, variant) the
 // pre-pass kept, skipped if a larger batch of its replica was already
 // accepted.  Per item:
@@ -369,8 +388,9 @@ __global__ void order_scatter_kernel(Dims dm, DevPop pop, SlotInfo si, WorkList 
 // Every comparison is between ranks of the same stage and link times the
 // oracle compares, so V, mu*, the partition, T and Lambda are bit-identical to
 // Alg. 1.
-__global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out,
-                                                      WorkList wl, SlotInfo si, SplitOut so)
+template <typename Key>
+__device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, const DevPop &pop, const EvalOut &out,
+                                             const WorkList &wl, const SlotInfo &si, const SplitOut &so)
 {
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ int s_S0, s_Z, s_mu, s_done;
@@ -382,6 +402,7 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
 
     const int K = dm.K, M = dm.M, N = dm.N;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
+    constexpr Key kInf = (Key)~(Key)0;
     const unsigned n_items = wl.ctrl[kCtrlTotal];
   for (;;) {
     // ---- next work item (heaviest first)
@@ -407,28 +428,28 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
 
     if (m <= N && vmask) {
         const int W = N - m + 1;
-        uint32_t *leaf0 = reinterpret_cast<uint32_t *>(smem);   // [m][W] l_k(n)
-        uint32_t *Fst = leaf0 + (size_t)m * W;                  // [m][W] prefix / traceback columns
-        uint32_t *Gst = Fst + (size_t)m * W;                    // [m][W] suffix columns
-        uint32_t *Hb = Gst + (size_t)m * W;                     // [NW][W] per-warp convolution
-        uint32_t *Lb = Hb + (size_t)NW * W;                     // [NW][W] per-warp head row
-        uint32_t *row1s = Lb + (size_t)NW * W;                  // [W] head row of mu*
-        uint32_t *delta = row1s + W;                            // [W] the empty stage
-        uint32_t *tauk = delta + W;                             // [m] tauk[k] = link (k-1) -> k
-        int *cnt0 = reinterpret_cast<int *>(tauk + m);          // [m]
+        int *cnt0 = reinterpret_cast<int *>(smem);              // [m]
         int *cnt1 = cnt0 + m;                                   // [m]
         int *nk = cnt1 + m;                                     // [m]
-        uint16_t *devs = reinterpret_cast<uint16_t *>(nk + m);  // [m]
+        Key *leaf0 = reinterpret_cast<Key *>(nk + m);           // [m][W] l_k(n)
+        Key *Fst = leaf0 + (size_t)m * W;                       // [m][W] prefix / traceback columns
+        Key *Gst = Fst + (size_t)m * W;                         // [m][W] suffix columns
+        Key *Hb = Gst + (size_t)m * W;                          // [NW][W] per-warp convolution
+        Key *Lb = Hb + (size_t)NW * W;                          // [NW][W] per-warp head row
+        Key *row1s = Lb + (size_t)NW * W;                       // [W] head row of mu*
+        Key *delta = row1s + W;                                 // [W] the empty stage
+        Key *tauk = delta + W;                                  // [m] tauk[k] = link (k-1) -> k
+        uint16_t *devs = reinterpret_cast<uint16_t *>(tauk + m);  // [m]
 
         for (int k = tid; k < m; k += blockDim.x) devs[k] = pop.perm[(size_t)g * M + off + k];
-        for (int r = tid; r < W; r += blockDim.x) delta[r] = r ? 0xFFFFFFFFu : 0u;
+        for (int r = tid; r < W; r += blockDim.x) delta[r] = r ? kInf : (Key)0;
         __syncthreads();
 
         // column accessors (1-based device index k)
-        auto colF = [&](int k) -> const uint32_t * {
+        auto colF = [&](int k) -> const Key * {
             return k == 0 ? delta : k == 1 ? leaf0 : Fst + (size_t)(k - 1) * W;
         };
-        auto colG = [&](int k) -> const uint32_t * {
+        auto colG = [&](int k) -> const Key * {
             return k == m + 1 ? delta : k == m ? leaf0 + (size_t)(m - 1) * W : Gst + (size_t)(k - 1) * W;
         };
 
@@ -445,12 +466,10 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
                 const int c0 = tb.cap[vd * 2], c1 = tb.cap[vd * 2 + 1];
                 cnt0[k] = c0 < W ? c0 : W;
                 cnt1[k] = c1 < W ? c1 : W;
-                tauk[k] = k ? tb.tau_rank[(vM + devs[k - 1]) * M + devs[k]] : 0u;
+                tauk[k] = k ? (Key)tb.tau_rank[(vM + devs[k - 1]) * M + devs[k]] : (Key)0;
             }
-            for (int k = wid; k < m; k += NW) {                   // asynchronous: the loads overlap
-                const uint32_t *src = tb.leaf_rank + (vM + devs[k]) * 2 * dm.LS;
-                for (int n = lane; n < W; n += 32) cp_async4(leaf0 + (size_t)k * W + n, src + n);
-            }
+            for (int k = wid; k < m; k += NW)                       // the loads of a row overlap
+                stage_row(leaf0 + (size_t)k * W, tb.leaf_rank + (vM + devs[k]) * 2 * dm.LS, W, lane);
             cp_async_wait_all();
             __syncthreads();
             // ---- 2. masters the memory allows (the pre-pass guarantees one)
@@ -470,17 +489,17 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             // ---- 3. prefix columns (warps 0-1) and suffix columns (warps 2-3)
             if (wid < 2) {
                 for (int k = 2; k <= m - 1; ++k) {
-                    const uint32_t *prev = colF(k - 1), *row = leaf0 + (size_t)(k - 1) * W;
-                    const uint32_t t = tauk[k - 1];
-                    uint32_t *cur = Fst + (size_t)(k - 1) * W;
+                    const Key *prev = colF(k - 1), *row = leaf0 + (size_t)(k - 1) * W;
+                    const Key t = tauk[k - 1];
+                    Key *cur = Fst + (size_t)(k - 1) * W;
                     for (int r = tid; r < W; r += 64) cur[r] = dp_cell(prev, row, t, r);
                     bar_named(1, 64);
                 }
             } else {
                 for (int k = m - 1; k >= 2; --k) {
-                    const uint32_t *prev = colG(k + 1), *row = leaf0 + (size_t)(k - 1) * W;
-                    const uint32_t t = tauk[k];
-                    uint32_t *cur = Gst + (size_t)(k - 1) * W;
+                    const Key *prev = colG(k + 1), *row = leaf0 + (size_t)(k - 1) * W;
+                    const Key t = tauk[k];
+                    Key *cur = Gst + (size_t)(k - 1) * W;
                     for (int r = tid - 64; r < W; r += 64) cur[r] = dp_cell(prev, row, t, r);
                     bar_named(2, 64);
                 }
@@ -491,19 +510,20 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             }
             __syncthreads();
             // ---- 4. one master per warp at a time
-            uint32_t bestV = 0xFFFFFFFFu;
+            uint32_t bestV = kInf;
             int bestMu = 0x7FFFFFFF;
             unsigned long long w_cells = 0, w_probes = 0;
-            uint32_t *H = Hb + (size_t)wid * W, *L1 = Lb + (size_t)wid * W;
+            Key *H = Hb + (size_t)wid * W, *L1 = Lb + (size_t)wid * W;
             for (int mu = wid + 1; mu <= m; mu += NW) {
                 if (!mu_ok(mu)) continue;
                 const uint32_t *hrow = tb.leaf_rank + ((vM + devs[mu - 1]) * 2 + 1) * dm.LS;
-                for (int r = lane; r < W; r += 32) cp_async4(L1 + r, hrow + r);
-                const uint32_t *P = colF(mu - 1), *S = colG(mu + 1);
-                for (int r = lane; r < W; r += 32) H[r] = dp_cell(P, S, 0u, r);
-                cp_async_wait_all();
+                HeadRow<Key> hr;
+                hr.start(L1, hrow, W, lane);                          // in flight while H is built
+                const Key *P = colF(mu - 1), *S = colG(mu + 1);
+                for (int r = lane; r < W; r += 32) H[r] = dp_cell(P, S, (Key)0, r);
+                hr.finish(L1, hrow, W, lane);
                 __syncwarp();
-                uint32_t V = dp_cell(H, L1, 0u, W - 1);
+                uint32_t V = dp_cell(H, L1, (Key)0, W - 1);
                 if (mu >= 2) V = max(V, tauk[mu - 1]);
                 if (mu <= m - 1) V = max(V, tauk[mu]);
                 __syncwarp();
@@ -514,7 +534,7 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             if (lane == 0) { s_wV[wid] = bestV; s_wMu[wid] = bestMu; st_cells += w_cells; st_probes += w_probes; }
             __syncthreads();
             if (tid == 0) {
-                uint32_t V = 0xFFFFFFFFu;
+                uint32_t V = kInf;
                 int mu = 0x7FFFFFFF;
                 for (int w = 0; w < NW; ++w)
                     if (s_wV[w] < V || (s_wV[w] == V && s_wMu[w] < mu)) { V = s_wV[w]; mu = s_wMu[w]; }
@@ -523,20 +543,20 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
             __syncthreads();
             const uint32_t V = s_V;
             const int mus = s_mu;
-            if (V == 0xFFFFFFFFu) continue;   // cannot happen: the pre-pass checked memory
+            if (V == kInf) continue;   // cannot happen: the pre-pass checked memory
             for (int r = tid; r < W; r += blockDim.x)
-                row1s[r] = tb.leaf_rank[((vM + devs[mus - 1]) * 2 + 1) * dm.LS + r];
+                row1s[r] = (Key)tb.leaf_rank[((vM + devs[mus - 1]) * 2 + 1) * dm.LS + r];
             __syncthreads();
             // ---- 5. mu*'s prefix columns, for the traceback
-            auto rowk = [&](int k) -> const uint32_t * { return k == mus ? row1s : leaf0 + (size_t)(k - 1) * W; };
-            auto colD = [&](int k) -> const uint32_t * {
+            auto rowk = [&](int k) -> const Key * { return k == mus ? row1s : leaf0 + (size_t)(k - 1) * W; };
+            auto colD = [&](int k) -> const Key * {
                 if (k == 1) return mus == 1 ? row1s : leaf0;
                 return Fst + (size_t)(k - 1) * W;
             };
             for (int k = (mus > 2 ? mus : 2); k <= m - 1; ++k) {
-                const uint32_t *prev = colD(k - 1), *row = rowk(k);
-                const uint32_t t = tauk[k - 1];
-                uint32_t *cur = Fst + (size_t)(k - 1) * W;
+                const Key *prev = colD(k - 1), *row = rowk(k);
+                const Key t = tauk[k - 1];
+                Key *cur = Fst + (size_t)(k - 1) * W;
                 for (int r = tid; r < W; r += blockDim.x) cur[r] = dp_cell(prev, row, t, r);
                 __syncthreads();
                 if (tid == 0) { st_cells += W; st_probes += cprobe; }
@@ -546,7 +566,7 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
                 int r = W - 1;
                 uint32_t D = V;
                 for (int k = m; k >= 2; --k) {
-                    const uint32_t *row = rowk(k);
+                    const Key *row = rowk(k);
                     int n = 0;                                    // #{n <= r+1 : l_k(n) <= D}
                     for (int base = 0; base <= r; base += 32) {
                         const int p = base + lane;
@@ -611,6 +631,12 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
     }
     if (tid == 0 && st_runs) atomicAdd(&out.stats[kStDpRuns], st_runs);
   }
+}
+
+__global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out, WorkList wl,
+                                                      SlotInfo si, SplitOut so)
+{
+    dp_eval_body<uint32_t>(dm, tb, pop, out, wl, si, so);
 }
 
 // One warp per genome.  Each replica that had work gets its outputs from its
@@ -738,10 +764,11 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
 
 cudaError_t configure_eval(e2_ctx *c)
 {
-    cudaError_t e = cudaFuncSetAttribute(dp_eval_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c->dp_smem);
+    const void *kernel = reinterpret_cast<const void *>(dp_eval_kernel);
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c->dp_smem);
     if (e != cudaSuccess) return e;
     int per_sm = 0, sms = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, dp_eval_kernel, c->dp_threads, c->dp_smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, c->dp_threads, c->dp_smem);
     if (e != cudaSuccess) return e;
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
     if (e != cudaSuccess) return e;

@@ -310,7 +310,7 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, c->device) != cudaSuccess)
         return fail_free(E2_ECUDA, "cudaDeviceGetAttribute failed");
     c->dp_threads = 128;
-    c->dp_smem = dp_smem_bytes(M, N, c->dp_threads);
+    c->dp_smem = dp_smem_bytes(M, N, c->dp_threads, 4);
     if ((M < N ? M : N) > kMaxReplicaDevices)
         return fail_free(E2_EINVAL, "replicas could exceed 256 devices (min(M, N) > 256)");
     if (c->dp_smem + 1024 > (size_t)smem_optin)

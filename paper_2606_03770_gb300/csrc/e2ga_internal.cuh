@@ -223,7 +223,7 @@ cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uin
 cudaError_t find_ga_node(cudaGraph_t graph, cudaGraphNode_t *node);
 cudaError_t set_ga_node(const e2_ctx *c, cudaGraphExec_t exec, cudaGraphNode_t node, const DevPop &src,
                         const DevPop &dst, uint64_t seed, uint32_t gen);
-size_t dp_smem_bytes(int M, int N, int threads);
+size_t dp_smem_bytes(int M, int N, int threads, int key_bytes);
 cudaError_t configure_eval(e2_ctx *c);   // shared memory limit and persistent grid size
 size_t rank_pow2(size_t n);
 cudaError_t build_leaf_sorted(const e2_ctx *c);   // once per context
