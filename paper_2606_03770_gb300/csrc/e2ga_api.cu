@@ -304,7 +304,13 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->thr_k2 = threshold(s2);
     c->thr_k3 = threshold(s3);
 
-    auto fail_free = [&](int code, const char *why) { delete c; return reject(code, why); };
+    auto fail_free = [&](int code, const char *why) {
+        if (c->side) cudaStreamDestroy(c->side);
+        if (c->ev_fork) cudaEventDestroy(c->ev_fork);
+        if (c->ev_join) cudaEventDestroy(c->ev_join);
+        delete c;
+        return reject(code, why);
+    };
     if (cudaGetDevice(&c->device) != cudaSuccess) return fail_free(E2_ECUDA, "no CUDA device");
     int smem_optin = 0;
     if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, c->device) != cudaSuccess)
@@ -316,6 +322,10 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     if (c->dp_smem + 1024 > (size_t)smem_optin)
         return fail_free(E2_EINVAL, "the largest replica's DP does not fit in shared memory (N too large)");
     if (configure_eval(c) != cudaSuccess) return fail_free(E2_ECUDA, "configuring the DP kernel failed");
+    if (cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->ev_join, cudaEventDisableTiming) != cudaSuccess)
+        return fail_free(E2_ECUDA, "creating the side stream failed");
 
     unsigned char *ws = static_cast<unsigned char *>(workspace);
     c->rate = reinterpret_cast<double *>(ws + l.rate);
@@ -408,8 +418,7 @@ cudaError_t record_generation(e2_ctx *c, int b)
     if (e == cudaSuccess) {
         cudaError_t le = cudaMemsetAsync(c->stats, 0, 8 * kNumStats, c->stream);
         if (le == cudaSuccess) le = launch_eval(c, c->pop[b]);
-        if (le == cudaSuccess) le = launch_elites(c, c->pop[b]);
-        if (le == cudaSuccess) le = launch_ga(c, c->pop[b], c->pop[b ^ 1], 0, 0);
+        if (le == cudaSuccess) le = launch_step(c, c->pop[b], c->pop[b ^ 1], 0, 0);
         cudaGraph_t g = nullptr;
         e = cudaStreamEndCapture(c->cap_stream, &g);
         if (le != cudaSuccess) e = le;
@@ -440,6 +449,9 @@ int e2_destroy(e2_ctx *c)
     cudaError_t e = cudaStreamSynchronize(c->stream);
     for (int b = 0; b < 2; ++b) drop_generation_graph(c, b);
     if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
+    if (c->side) cudaStreamDestroy(c->side);
+    if (c->ev_fork) cudaEventDestroy(c->ev_fork);
+    if (c->ev_join) cudaEventDestroy(c->ev_join);
     delete c;
     return e == cudaSuccess ? E2_OK : E2_ECUDA;
 }
@@ -505,8 +517,7 @@ int e2_ga_step(e2_ctx *c, uint64_t seed, uint32_t generation)
 {
     if (!c) return E2_EINVAL;
     if (!c->evaluated) return fail(c, E2_ESTATE, "the current population has not been evaluated");
-    E2_CUDA(c, launch_elites(c, c->pop[c->cur]));
-    E2_CUDA(c, launch_ga(c, c->pop[c->cur], c->pop[c->cur ^ 1], seed, generation));
+    E2_CUDA(c, launch_step(c, c->pop[c->cur], c->pop[c->cur ^ 1], seed, generation));
     c->cur ^= 1;
     c->evaluated = false;
     c->have_elites = true;

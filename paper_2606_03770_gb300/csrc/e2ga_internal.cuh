@@ -156,6 +156,8 @@ __device__ __forceinline__ uint64_t umax64(uint64_t a, uint64_t b) { return a > 
 struct e2_ctx {
     int device = 0;
     cudaStream_t stream = nullptr;
+    cudaStream_t side = nullptr;                 // children of the generation step run here
+    cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
     e2::Dims dm{};
     double cong_lo = 0, cong_hi = 0;
     uint64_t thr_cx = 0, thr_half = 0, thr_mut = 0, thr_k1 = 0, thr_k2 = 0, thr_k3 = 0;
@@ -217,8 +219,11 @@ cudaError_t launch_redraw(const e2_ctx *c, uint64_t seed, uint32_t gen);
 cudaError_t launch_validate(const e2_ctx *c, const DevPop &p);
 cudaError_t launch_eval(const e2_ctx *c, const DevPop &p);
 cudaError_t launch_init(const e2_ctx *c, const DevPop &p, uint64_t seed);
-cudaError_t launch_elites(const e2_ctx *c, const DevPop &p);
-cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen);
+cudaError_t launch_elites(const e2_ctx *c, const DevPop &p, const DevPop &dst);
+cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen,
+                      cudaStream_t st);
+// elites and children of the next population (children on the side stream)
+cudaError_t launch_step(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen);
 // the generation kernel's node of a recorded graph, and new (seed, generation) for it
 cudaError_t find_ga_node(cudaGraph_t graph, cudaGraphNode_t *node);
 cudaError_t set_ga_node(const e2_ctx *c, cudaGraphExec_t exec, cudaGraphNode_t node, const DevPop &src,

@@ -238,9 +238,10 @@ __global__ void __launch_bounds__(256) dup_kernel(Dims dm, DevPop p, const doubl
 }
 
 // rank(g) = number of genomes before g in the elite order (duplicate flag,
-// w, phase, index); the first Q ranks are the elites.
+// w, phase, index); the first Q ranks are the elites, and the warp of an elite
+// copies it into slot rank(g) of the next population.
 __global__ void __launch_bounds__(256) rank_kernel(Dims dm, const double *fit, const int32_t *dup,
-                                                   int32_t *elite, double *elite_fit)
+                                                   int32_t *elite, double *elite_fit, DevPop src, DevPop dst)
 {
     __shared__ uint64_t s_w[kEliteTile], s_p[kEliteTile];
     __shared__ int s_d[kEliteTile];
@@ -265,9 +266,16 @@ __global__ void __launch_bounds__(256) rank_kernel(Dims dm, const double *fit, c
     }
 #pragma unroll
     for (int x = 16; x; x >>= 1) rank += __shfl_xor_sync(0xFFFFFFFFu, rank, x);
-    if (live && lane == 0 && rank < dm.Q) {
-        elite[rank] = g;
-        for (int q = 0; q < 4; ++q) elite_fit[(size_t)rank * 4 + q] = fit[(size_t)g * 4 + q];
+    if (live && rank < dm.Q) {
+        const int M = dm.M, K = dm.K;
+        for (int i = lane; i < M; i += 32) dst.perm[(size_t)rank * M + i] = src.perm[(size_t)g * M + i];
+        for (int i = lane; i < K; i += 32) dst.sizes[(size_t)rank * K + i] = src.sizes[(size_t)g * K + i];
+        if (lane == 0) {
+            dst.nclus[rank] = src.nclus[g];
+            dst.roles[rank] = src.roles[g];
+            elite[rank] = g;
+            for (int q = 0; q < 4; ++q) elite_fit[(size_t)rank * 4 + q] = fit[(size_t)g * 4 + q];
+        }
     }
 }
 
@@ -303,7 +311,7 @@ __device__ __forceinline__ unsigned lanemask_lt()
 // Per warp, shared memory holds the child ordering, the first-occurrence
 // table, the missing devices, the random words (M words each) and the sizes.
 __global__ void __launch_bounds__(256) ga_kernel(Dims dm, DevPop src, DevPop dst, const double *fit,
-                                                 const int32_t *elite, uint64_t seed, uint32_t gen, GaThr thr)
+                                                 uint64_t seed, uint32_t gen, GaThr thr)
 {
     extern __shared__ uint32_t ga_smem[];
     const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5, NWB = blockDim.x >> 5;
@@ -314,16 +322,9 @@ __global__ void __launch_bounds__(256) ga_kernel(Dims dm, DevPop src, DevPop dst
     uint32_t *words = missing + M;
     uint32_t *ssz = words + M;                                    // [64] sizes
     const uint64_t *fk = reinterpret_cast<const uint64_t *>(fit);
-    for (int s = blockIdx.x * NWB + wl; s < P; s += gridDim.x * NWB) {
+    for (int s = dm.Q + blockIdx.x * NWB + wl; s < P; s += gridDim.x * NWB) {   // the children
         uint16_t *out_perm = dst.perm + (size_t)s * M;
         uint16_t *cs = dst.sizes + (size_t)s * K;
-        if (s < dm.Q) {
-            const int e = elite[s];
-            for (int i = lane; i < M; i += 32) out_perm[i] = src.perm[(size_t)e * M + i];
-            for (int i = lane; i < K; i += 32) cs[i] = src.sizes[(size_t)e * K + i];
-            if (lane == 0) { dst.nclus[s] = src.nclus[e]; dst.roles[s] = src.roles[e]; }
-            continue;
-        }
         // ---- two tournaments
         Stream sel(seed, gen, (uint32_t)s, kSelect);
         int par[2];
@@ -485,16 +486,20 @@ cudaError_t launch_init(const e2_ctx *c, const DevPop &p, uint64_t seed)
     return cudaGetLastError();
 }
 
-cudaError_t launch_elites(const e2_ctx *c, const DevPop &p)
+// Duplicate flags, then ranks; the elites go to slots [0, Q) of dst.
+cudaError_t launch_elites(const e2_ctx *c, const DevPop &p, const DevPop &dst)
 {
     const unsigned blocks = (unsigned)(((size_t)c->dm.P * 32 + 255) / 256);
     dup_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, p, c->fit, c->hash, c->dup);
-    if (c->dm.Q > 0) rank_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, c->fit, c->dup, c->elite, c->elite_fit);
+    if (c->dm.Q > 0)
+        rank_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, c->fit, c->dup, c->elite, c->elite_fit, p, dst);
     return cudaGetLastError();
 }
 
-cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen)
+cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen,
+                      cudaStream_t st)
 {
+    if (c->dm.P <= c->dm.Q) return cudaSuccess;              // no children
     GaThr thr{c->thr_cx, c->thr_half, c->thr_mut, c->thr_k1, c->thr_k2, c->thr_k3};
     const size_t per_warp = 4 * (4 * (size_t)c->dm.M + 64);
     int nw = 8;
@@ -504,10 +509,25 @@ cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uin
                                                    (int)((size_t)nw * per_warp));
         if (e != cudaSuccess) return e;
     }
-    const long long blocks = ((long long)c->dm.P + nw - 1) / nw;
-    ga_kernel<<<(unsigned)(blocks < 152 * 64 ? blocks : 152 * 64), 32 * nw, (size_t)nw * per_warp, c->stream>>>(
-        c->dm, src, dst, c->fit, c->elite, seed, gen, thr);
+    const long long blocks = ((long long)(c->dm.P - c->dm.Q) + nw - 1) / nw;
+    ga_kernel<<<(unsigned)(blocks < 152 * 64 ? blocks : 152 * 64), 32 * nw, (size_t)nw * per_warp, st>>>(
+        c->dm, src, dst, c->fit, seed, gen, thr);
     return cudaGetLastError();
+}
+
+// The generation step: the children (which need only the fitness) on the side
+// stream, concurrently with the duplicate test and the ranks (which copy the
+// elites) on the context's stream; the context's stream then waits for the
+// children.
+cudaError_t launch_step(const e2_ctx *c, const DevPop &src, const DevPop &dst, uint64_t seed, uint32_t gen)
+{
+    cudaError_t e = cudaEventRecord(c->ev_fork, c->stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(c->side, c->ev_fork, 0);
+    if (e == cudaSuccess) e = launch_ga(c, src, dst, seed, gen, c->side);
+    if (e == cudaSuccess) e = cudaEventRecord(c->ev_join, c->side);
+    if (e == cudaSuccess) e = launch_elites(c, src, dst);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(c->stream, c->ev_join, 0);
+    return e;
 }
 
 cudaError_t find_ga_node(cudaGraph_t graph, cudaGraphNode_t *node)
@@ -543,9 +563,8 @@ cudaError_t set_ga_node(const e2_ctx *c, cudaGraphExec_t exec, cudaGraphNode_t n
     Dims dm = c->dm;
     DevPop s = src, d = dst;
     const double *fit = c->fit;
-    const int32_t *elite = c->elite;
     GaThr thr{c->thr_cx, c->thr_half, c->thr_mut, c->thr_k1, c->thr_k2, c->thr_k3};
-    void *args[] = {&dm, &s, &d, &fit, &elite, &seed, &gen, &thr};
+    void *args[] = {&dm, &s, &d, &fit, &seed, &gen, &thr};
     p.kernelParams = args;
     p.extra = nullptr;
     return cudaGraphExecKernelNodeSetParams(exec, node, &p);
