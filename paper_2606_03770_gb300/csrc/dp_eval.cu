@@ -103,7 +103,7 @@ size_t dp_smem_bytes(int M, int N, int threads, int key_bytes)
     const int mmax = M < N ? M : N;
     for (int m = 1; m <= mmax; ++m) {
         const size_t W = (size_t)(N - m + 1);
-        const size_t keys = 3 * (size_t)m * W + (size_t)(2 * NW + 2) * W + (size_t)m;
+        const size_t keys = 3 * (size_t)m * W + (size_t)(2 * NW + 2) * W + 2 * (size_t)m;
         const size_t bytes = (size_t)m * (3 * sizeof(int)) + keys * key_bytes + (size_t)m * sizeof(uint16_t) + 16;
         if (bytes > best) best = bytes;
     }
@@ -396,9 +396,9 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
     __shared__ int s_S0, s_Z, s_mu, s_done;
     __shared__ uint32_t s_V;
     __shared__ double s_L, s_T;
-    __shared__ uint32_t s_wV[4];
-    __shared__ int s_wMu[4];
     __shared__ unsigned s_item;
+    __shared__ unsigned long long s_bestkey;     // (V << 32) | mu of the best master so far
+    __shared__ uint32_t s_V0;
 
     const int K = dm.K, M = dm.M, N = dm.N;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
@@ -439,7 +439,8 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
         Key *row1s = Lb + (size_t)NW * W;                       // [W] head row of mu*
         Key *delta = row1s + W;                                 // [W] the empty stage
         Key *tauk = delta + W;                                  // [m] tauk[k] = link (k-1) -> k
-        uint16_t *devs = reinterpret_cast<uint16_t *>(tauk + m);  // [m]
+        Key *lbm = tauk + m;                                    // [m] l^head_k(1)
+        uint16_t *devs = reinterpret_cast<uint16_t *>(lbm + m);   // [m]
 
         for (int k = tid; k < m; k += blockDim.x) devs[k] = pop.perm[(size_t)g * M + off + k];
         for (int r = tid; r < W; r += blockDim.x) delta[r] = r ? kInf : (Key)0;
@@ -467,6 +468,7 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                 cnt0[k] = c0 < W ? c0 : W;
                 cnt1[k] = c1 < W ? c1 : W;
                 tauk[k] = k ? (Key)tb.tau_rank[(vM + devs[k - 1]) * M + devs[k]] : (Key)0;
+                lbm[k] = (Key)tb.leaf_rank[((vM + devs[k]) * 2 + 1) * dm.LS];   // l^head_k(1)
             }
             for (int k = wid; k < m; k += NW)                       // the loads of a row overlap
                 stage_row(leaf0 + (size_t)k * W, tb.leaf_rank + (vM + devs[k]) * 2 * dm.LS, W, lane);
@@ -495,6 +497,18 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                     for (int r = tid; r < W; r += 64) cur[r] = dp_cell(prev, row, t, r);
                     bar_named(1, 64);
                 }
+                if (wid == 0) {                                   // V0 = F_m[W-1], the master-free optimum:
+                    uint32_t v0 = 0;                              // the minimum over every split, by the lanes
+                    if (m >= 2) {
+                        const Key *prev = colF(m - 1), *row = leaf0 + (size_t)(m - 1) * W;
+                        v0 = kInf;
+                        for (int q = lane; q < W; q += 32) v0 = min(v0, (uint32_t)max(prev[q], row[W - 1 - q]));
+#pragma unroll
+                        for (int o = 16; o; o >>= 1) v0 = min(v0, __shfl_xor_sync(0xFFFFFFFFu, v0, o));
+                        v0 = max(v0, (uint32_t)tauk[m - 1]);
+                    }
+                    if (lane == 0) { s_V0 = v0; s_bestkey = ~0ull; }
+                }
             } else {
                 for (int k = m - 1; k >= 2; --k) {
                     const Key *prev = colG(k + 1), *row = leaf0 + (size_t)(k - 1) * W;
@@ -509,13 +523,21 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                 st_probes += 2ull * (m - 2) * cprobe;
             }
             __syncthreads();
-            // ---- 4. one master per warp at a time
-            uint32_t bestV = kInf;
-            int bestMu = 0x7FFFFFFF;
+            // ---- 4. one master per warp at a time, skipping a master whose lower
+            //      bound V_mu >= max(V0, l^head_mu(1)) (V0 the master-free
+            //      optimum F_m[W-1]: the head only adds) exceeds the best V found
+            //      so far, or ties it with a larger index
+            const uint32_t V0 = s_V0;
+            auto bound = [&](int k) -> uint32_t { return mu_ok(k + 1) ? max(V0, (uint32_t)lbm[k]) : (uint32_t)kInf; };
+
             unsigned long long w_cells = 0, w_probes = 0;
             Key *H = Hb + (size_t)wid * W, *L1 = Lb + (size_t)wid * W;
             for (int mu = wid + 1; mu <= m; mu += NW) {
                 if (!mu_ok(mu)) continue;
+                const uint32_t lb = bound(mu - 1);
+                const unsigned long long bk = *reinterpret_cast<volatile unsigned long long *>(&s_bestkey);
+                const uint32_t bv = (uint32_t)(bk >> 32);
+                if (lb > bv || (lb == bv && (unsigned)mu > (unsigned)(bk & 0xFFFFFFFFu))) continue;
                 const uint32_t *hrow = tb.leaf_rank + ((vM + devs[mu - 1]) * 2 + 1) * dm.LS;
                 HeadRow<Key> hr;
                 hr.start(L1, hrow, W, lane);                          // in flight while H is built
@@ -524,21 +546,19 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                 hr.finish(L1, hrow, W, lane);
                 __syncwarp();
                 uint32_t V = dp_cell(H, L1, (Key)0, W - 1);
-                if (mu >= 2) V = max(V, tauk[mu - 1]);
-                if (mu <= m - 1) V = max(V, tauk[mu]);
+                if (mu >= 2) V = max(V, (uint32_t)tauk[mu - 1]);
+                if (mu <= m - 1) V = max(V, (uint32_t)tauk[mu]);
                 __syncwarp();
                 w_cells += W + 1;
                 w_probes += cprobe + lprobe;
-                if (V < bestV) { bestV = V; bestMu = mu; }
+                if (lane == 0) atomicMin(&s_bestkey, ((unsigned long long)V << 32) | (unsigned)mu);
             }
-            if (lane == 0) { s_wV[wid] = bestV; s_wMu[wid] = bestMu; st_cells += w_cells; st_probes += w_probes; }
+            if (lane == 0) { st_cells += w_cells; st_probes += w_probes; }
+            if (tid == 0 && m >= 2) { st_cells += 1; st_probes += lprobe; }
             __syncthreads();
             if (tid == 0) {
-                uint32_t V = kInf;
-                int mu = 0x7FFFFFFF;
-                for (int w = 0; w < NW; ++w)
-                    if (s_wV[w] < V || (s_wV[w] == V && s_wMu[w] < mu)) { V = s_wV[w]; mu = s_wMu[w]; }
-                s_V = V; s_mu = mu;
+                s_V = (uint32_t)(s_bestkey >> 32);
+                s_mu = (int)(s_bestkey & 0xFFFFFFFFu);
             }
             __syncthreads();
             const uint32_t V = s_V;
