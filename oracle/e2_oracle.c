@@ -14,6 +14,7 @@
  *                                  Alg. 1
  *   per-request latency Lambda     Sec. 3.2 (text after Alg. 1)
  *   prefill / decode evaluation    Alg. 2 (replica loop, b sweep)
+ *   role assignment by brute force Alg. 2 (optional)
  *   objective Eq. 3, 4, 5 and the multi-replica aggregation
  *                                  Sec. 3.3
  *   GA: gene, crossover + repair, mutation mixture, elites
@@ -46,6 +47,8 @@ typedef struct {
     const uint64_t *act_bytes;   /* [V] activation bytes per microbatch       */
     uint64_t NP, ND;
     double min_tps, t_a;
+    int role_search;             /* 0: roles from the genome; 1: Alg. 2's     */
+                                 /* brute force over every role assignment    */
 } orc_problem;
 
 /* ------------------------------------------------------------------------ */
@@ -245,10 +248,63 @@ void orc_eval_genome(const orc_problem *p, int K, const uint16_t *perm, const ui
     orc_score(p, R, roles, T, bsel, fit);
 }
 
+/* Alg. 2 with its role search: every replica is evaluated in both roles
+ * (the prefill DP and the decode sweep), then every role assignment (bit c =
+ * 1: replica c decodes) is scored with Eq. 3-5, masks in increasing order; the
+ * first with the least (w, phase) wins.  The replicas' outputs are those of
+ * their chosen roles, and the chosen assignment goes to *roles_out. */
+void orc_eval_genome_roles(const orc_problem *p, int K, const uint16_t *perm, const uint16_t *sizes,
+                           int R, double fit[4], int16_t *layers, int16_t *master, int16_t *bsel,
+                           double *T, double *L, uint64_t *cand, uint64_t *roles_out)
+{
+    double Tr[2][64], Lr[2][64];
+    int mur[2][64], br[2][64];
+    int16_t *lay[2];
+    lay[0] = (int16_t *)malloc(sizeof(int16_t) * (size_t)p->M);
+    lay[1] = (int16_t *)malloc(sizeof(int16_t) * (size_t)p->M);
+    int off = 0;
+    for (int c = 0; c < K; ++c) {
+        master[c] = -1; bsel[c] = -1; T[c] = ORC_INF; L[c] = ORC_INF;
+    }
+    for (int c = 0; c < R; ++c) {
+        for (int role = 0; role < 2; ++role)
+            orc_eval_cluster(p, perm + off, sizes[c], role, &Tr[role][c], &Lr[role][c], &mur[role][c],
+                             &br[role][c], lay[role] + off, cand);
+        off += sizes[c];
+    }
+    uint64_t best = 0;
+    double bw = ORC_INF, bp = ORC_INF;
+    int have = 0;
+    for (uint64_t mask = 0; mask < ((uint64_t)1 << R); ++mask) {
+        double Tm[64], f[4];
+        int16_t bm[64];
+        for (int c = 0; c < R; ++c) {
+            const int role = (int)((mask >> c) & 1u);
+            Tm[c] = Tr[role][c];
+            bm[c] = (int16_t)br[role][c];
+        }
+        orc_score(p, R, mask, Tm, bm, f);
+        if (!have || f[0] < bw || (f[0] == bw && f[1] < bp)) {
+            have = 1; bw = f[0]; bp = f[1]; best = mask;
+        }
+    }
+    off = 0;
+    for (int c = 0; c < R; ++c) {
+        const int role = (int)((best >> c) & 1u);
+        T[c] = Tr[role][c]; L[c] = Lr[role][c]; master[c] = (int16_t)mur[role][c]; bsel[c] = (int16_t)br[role][c];
+        for (int k = 0; k < sizes[c]; ++k) layers[off + k] = lay[role][off + k];
+        off += sizes[c];
+    }
+    orc_score(p, R, best, T, bsel, fit);
+    *roles_out = best;
+    free(lay[0]);
+    free(lay[1]);
+}
+
 void orc_eval_population(const orc_problem *p, int P, int K, const uint16_t *perm,
                          const uint16_t *sizes, const uint8_t *nclus, const uint64_t *roles,
                          double *fitness, int16_t *layers, int16_t *master, int16_t *bsel,
-                         double *T, double *L, uint64_t *cand, int nthreads)
+                         double *T, double *L, uint64_t *cand, int nthreads, uint64_t *roles_out)
 {
     uint64_t total = 0;
     const int M = p->M;
@@ -257,9 +313,17 @@ void orc_eval_population(const orc_problem *p, int P, int K, const uint16_t *per
 #endif
     for (int g = 0; g < P; ++g) {
         uint64_t c = 0;
-        orc_eval_genome(p, K, perm + (size_t)g * M, sizes + (size_t)g * K, nclus[g], roles[g],
-                        fitness + (size_t)g * 4, layers + (size_t)g * M, master + (size_t)g * K,
-                        bsel + (size_t)g * K, T + (size_t)g * K, L + (size_t)g * K, &c);
+        if (p->role_search)
+            orc_eval_genome_roles(p, K, perm + (size_t)g * M, sizes + (size_t)g * K, nclus[g],
+                                  fitness + (size_t)g * 4, layers + (size_t)g * M, master + (size_t)g * K,
+                                  bsel + (size_t)g * K, T + (size_t)g * K, L + (size_t)g * K, &c,
+                                  roles_out + g);
+        else {
+            orc_eval_genome(p, K, perm + (size_t)g * M, sizes + (size_t)g * K, nclus[g], roles[g],
+                            fitness + (size_t)g * 4, layers + (size_t)g * M, master + (size_t)g * K,
+                            bsel + (size_t)g * K, T + (size_t)g * K, L + (size_t)g * K, &c);
+            roles_out[g] = roles[g];
+        }
         total += c;
     }
     (void)nthreads;

@@ -42,7 +42,7 @@ class _Problem(C.Structure):
                 ("blk_flops", C.c_void_p), ("blk_bytes", C.c_void_p), ("blk_mem", C.c_void_p),
                 ("head_flops", C.c_void_p), ("head_bytes", C.c_void_p), ("head_mem", C.c_void_p),
                 ("act_bytes", C.c_void_p), ("NP", C.c_uint64), ("ND", C.c_uint64),
-                ("min_tps", C.c_double), ("t_a", C.c_double)]
+                ("min_tps", C.c_double), ("t_a", C.c_double), ("role_search", C.c_int)]
 
 
 class _GA(C.Structure):
@@ -70,7 +70,8 @@ def lib():
         _lib.orc_score.restype = None
         _lib.orc_score.argtypes = [C.c_void_p, C.c_int, C.c_uint64, C.c_void_p, C.c_void_p, C.c_void_p]
         _lib.orc_eval_population.restype = None
-        _lib.orc_eval_population.argtypes = [C.c_void_p, C.c_int, C.c_int] + [C.c_void_p] * 11 + [C.c_int]
+        _lib.orc_eval_population.argtypes = [C.c_void_p, C.c_int, C.c_int] + [C.c_void_p] * 11 + [C.c_int,
+                                                                                                   C.c_void_p]
         _lib.orc_philox4x32_10.restype = None
         _lib.orc_philox4x32_10.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p]
         _lib.orc_word.restype = C.c_uint32
@@ -113,7 +114,7 @@ class OracleProblem:
         self.s = _Problem(prob.M, prob.N, prob.V, *[_p(a[k]) for k in
                           ("rate", "bw", "mem", "link_bw", "cong", "blk_flops", "blk_bytes",
                            "blk_mem", "head_flops", "head_bytes", "head_mem", "act_bytes")],
-                          prob.NP, prob.ND, prob.min_tps, prob.t_a)
+                          prob.NP, prob.ND, prob.min_tps, prob.t_a, int(getattr(prob, "role_search", 0)))
 
     def set_cong(self, cong):
         self.arrays["cong"] = np.ascontiguousarray(cong, dtype=np.float64)
@@ -169,12 +170,13 @@ class OracleProblem:
         P, M = perm.shape
         out = dict(fitness=np.zeros((P, 4), np.float64), layers=np.zeros((P, M), np.int16),
                    master=np.zeros((P, K), np.int16), bsel=np.zeros((P, K), np.int16),
-                   T=np.zeros((P, K), np.float64), L=np.zeros((P, K), np.float64))
+                   T=np.zeros((P, K), np.float64), L=np.zeros((P, K), np.float64),
+                   roles=np.zeros(P, np.uint64))
         cand = C.c_uint64(0)
         lib().orc_eval_population(self.ref, P, K, _p(perm), _p(sizes), _p(nclus), _p(roles),
                                   _p(out["fitness"]), _p(out["layers"]), _p(out["master"]),
                                   _p(out["bsel"]), _p(out["T"]), _p(out["L"]), C.byref(cand),
-                                  int(nthreads))
+                                  int(nthreads), _p(out["roles"]))
         out["cand"] = cand.value
         return out
 

@@ -53,6 +53,9 @@ class Problem:
     # objective
     min_tps: float = 7.0
     t_a: float = 1.0
+    # roles: 0 = one role bit per replica in the genome; 1 = Alg. 2's brute force
+    # over every role assignment of the genome's replicas
+    role_search: int = 0
     # genetic algorithm
     P: int = 64
     Q: int = 2

@@ -575,3 +575,35 @@ def test_latency_hand_value_and_tps_boundary():
     assert r["ok"] and r["b"] == 1 and r["T"] == 0.25 and r["L"] == 0.75
     r = O.OracleProblem(mk(np.nextafter(1.0 / 0.75, 2.0))).eval_cluster([0, 1], decode=True)
     assert not r["ok"] and r["b"] == -1
+
+
+def test_role_search_is_the_best_fixed_assignment():
+    """Alg. 2's role search: the fitness equals the least (w, phase) over every
+    role assignment evaluated with fixed role bits, the smallest such
+    assignment is chosen, the replicas' outputs are those of that assignment,
+    and the genome's own role bits do not matter."""
+    import dataclasses
+    prob = W.make_config("c1_tiny")
+    search = O.OracleProblem(dataclasses.replace(prob, role_search=1))
+    fixed = O.OracleProblem(prob)
+    K = 5
+    g = W.random_genomes(prob.M, K, 24, seed=31)
+    got = search.eval_population(g, K)
+    scrambled = dict(g, roles=np.ascontiguousarray(g["roles"] ^ np.uint64(0b10110)))
+    again = search.eval_population(scrambled, K)
+    for key in ("fitness", "layers", "master", "bsel", "T", "L", "roles"):
+        assert np.array_equal(got[key], again[key]), key
+    checked_feasible = 0
+    for p in range(24):
+        R = int(g["nclus"][p])
+        one = {k: np.repeat(v[p:p + 1], 1 << R, axis=0) for k, v in g.items()}
+        one["roles"] = np.arange(1 << R, dtype=np.uint64)
+        every = fixed.eval_population(one, K)
+        f = every["fitness"]
+        best = min(range(1 << R), key=lambda r: (f[r, 0], f[r, 1], r))
+        assert int(got["roles"][p]) == best
+        assert np.array_equal(got["fitness"][p], f[best])
+        for key in ("layers", "master", "bsel", "T", "L"):
+            assert np.array_equal(got[key][p], every[key][best]), key
+        checked_feasible += bool(np.isfinite(f[best, 0]))
+    assert checked_feasible >= 10
