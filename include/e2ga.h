@@ -106,6 +106,13 @@ typedef struct {
     double p_swap;          /* mutation kinds, App. A: swap two positions       */
     double p_regroup;       /*   regroup from a random replica onward           */
     double p_regroup_all;   /*   regroup everything; the rest: regenerate both  */
+    int32_t role_search;    /* 0: each replica's role is a bit of the genome;   */
+                            /* 1: Alg. 2's brute-force role assignment: every   */
+                            /* replica is evaluated in both roles, the best of  */
+                            /* the 2^R assignments (least w, then phase, then   */
+                            /* smallest mask) is taken and written back into    */
+                            /* the genome's role bits.  Needs K_max <=          */
+                            /* E2_MAX_ROLE_SEARCH and b_max <= 63.              */
 } e2_params;
 
 /* A population in the layout above; "host or device" pointers. */
@@ -155,6 +162,7 @@ typedef struct e2_ctx e2_ctx;
 #define E2_MAX_BATCH 64
 #define E2_MAX_CLUSTERS 64
 #define E2_MAX_POP (1 << 22)
+#define E2_MAX_ROLE_SEARCH 12
 
 /* Bytes of device workspace a context with these sizes needs.  Returns 0 on
  * invalid sizes.  Reads only M, N, b_max, P, Q, K_max. */

@@ -199,11 +199,16 @@ __global__ void __launch_bounds__(128, 12) slot_kernel(Dims dm, Tables tb, DevPo
             uint16_t *sdev = reinterpret_cast<uint16_t *>(sc1 + mcap);
             for (int k = lane; k < m; k += 32) sdev[k] = pop.perm[(size_t)g * M + off + k];
             __syncwarp();
-            const int nvar = role ? dm.b_max : 1;
+            // with the role search, the decode sweep and then the prefill variant
+            // (its result goes to bit b_max); otherwise the genome's role only
+            const int npass = dm.role_search ? 2 : 1;
+            for (int pass = 0; pass < npass; ++pass) {
+            const int prole = dm.role_search ? (pass == 0) : role;
+            const int nvar = prole ? dm.b_max : 1;
             for (int i = nvar - 1; i >= 0; --i) {                 // largest batch first
-                const int v = role ? i + 1 : 0;
+                const int v = prole ? i + 1 : 0;
                 const int32_t *cap = tb.cap + (size_t)v * M * 2;
-                const bool bound = role && dm.min_tps > 0.0;
+                const bool bound = prole && dm.min_tps > 0.0;
                 const double *cpb = tb.cpb + (size_t)v * M;
                 const double *tau = tb.tau + (size_t)v * M * M;
                 int s0 = 0, z = 0;
@@ -251,8 +256,10 @@ __global__ void __launch_bounds__(128, 12) slot_kernel(Dims dm, Tables tb, DevPo
                         continue;
                     }
                 }
-                mask = (2ull << i) - 1ull;         // this variant and every smaller batch
+                if (dm.role_search && !prole) mask |= 1ull << dm.b_max;
+                else mask |= (2ull << i) - 1ull;   // this variant and every smaller batch
                 break;
+            }
             }
         }
         // ---- the slot's outputs or its work count
@@ -268,7 +275,8 @@ __global__ void __launch_bounds__(128, 12) slot_kernel(Dims dm, Tables tb, DevPo
                 out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
                 if (c < R) {
                     atomicAdd(&out.stats[kStReplicas], 1ull);
-                    if (m <= N) atomicAdd(&out.stats[kStPaper], (role ? dm.b_max : 1) * paper_candidates(m, N));
+                    const int runs = dm.role_search ? dm.b_max + 1 : (role ? dm.b_max : 1);
+                    if (m <= N) atomicAdd(&out.stats[kStPaper], runs * paper_candidates(m, N));
                 }
             } else {
                 const int W = N - m + 1;
@@ -313,7 +321,9 @@ __global__ void __launch_bounds__(128, 12) slot_kernel(Dims dm, Tables tb, DevPo
 }
 
 // Item lv of a slot (its variants from the largest batch down) goes to bin
-// item_bin(lv, size) as (slot << 8) | bit.  The lanes of a warp whose items
+// item_bin(lv, size) as (slot << 8) | role << 7 | sweep << 6 | bit: role 1 =
+// decode; sweep 1 = an accepted result stops the smaller batches (every item
+// but the prefill run of a searched role).  The lanes of a warp whose items
 // share a bin take their positions with one atomic.
 __global__ void order_scatter_kernel(Dims dm, DevPop pop, SlotInfo si, WorkList wl)
 {
@@ -322,11 +332,14 @@ __global__ void order_scatter_kernel(Dims dm, DevPop pop, SlotInfo si, WorkList 
     for (int base = blockIdx.x * blockDim.x + (threadIdx.x & ~31); base < total; base += gridDim.x * blockDim.x) {
         const int slot = base + lane;
         uint64_t mask = 0;
-        int size = 0;
+        int size = 0, grole = 0;
         if (slot < total) {
             const int g = slot / dm.K, c = slot - g * dm.K;
             if (c < pop.nclus[g]) mask = si.mask[slot];
-            if (mask) size = si.size[slot];
+            if (mask) {
+                size = si.size[slot];
+                grole = (int)((pop.roles[g] >> c) & 1ull);
+            }
         }
         for (int lv = 0; __any_sync(0xFFFFFFFFu, mask != 0); ++lv) {
             int bit = 0, bin = -1;
@@ -341,7 +354,9 @@ __global__ void order_scatter_kernel(Dims dm, DevPop pop, SlotInfo si, WorkList 
                 unsigned at = 0;
                 if (lane == leader) at = atomicAdd(&wl.ctrl[bin], (unsigned)__popc(peers));
                 at = __shfl_sync(peers, at, leader);
-                wl.items[at + __popc(peers & below)] = ((uint64_t)slot << 8) | (uint64_t)bit;
+                const bool pre = dm.role_search ? bit == dm.b_max : !grole;
+                const uint64_t flags = (pre ? 0u : 0x80u) | (dm.role_search && pre ? 0u : 0x40u);
+                wl.items[at + __popc(peers & below)] = ((uint64_t)slot << 8) | flags | (uint64_t)bit;
             }
         }
     }
@@ -412,16 +427,17 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
     __syncthreads();
     if (idx >= n_items) break;
     const uint64_t item = wl.items[idx];
-    const int slot = (int)(item >> 8), code = (int)(item & 0xFFu);
+    const int slot = (int)(item >> 8), code = (int)(item & 0x3Fu);
     if (tid == 0) s_done = *(volatile const int32_t *)&si.best[slot] > code;   // a larger batch won
     __syncthreads();
     if (s_done) continue;
     const int g = slot / K, c = slot - g * K;
     const size_t gk = (size_t)g * K + c;
     const int off = si.off[slot], m = pop.sizes[gk];
-    const int role = (int)((pop.roles[g] >> c) & 1ull);
+    const int role = (int)((item >> 7) & 1u);                   // decode
+    const bool sweep = (item >> 6) & 1u;                        // the result advances the decode sweep
     uint64_t vmask = 1ull << code;
-    int16_t *lay_out = so.layers + ((size_t)g * dm.b_max + code) * M + off;
+    int16_t *lay_out = so.layers + ((size_t)g * dm.V + code) * M + off;
 
     unsigned long long st_runs = 0, st_cells = 0, st_probes = 0;
     bool served = false;
@@ -632,12 +648,12 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
             if (s_done) {
                 for (int k = tid; k < m; k += blockDim.x) lay_out[k] = (int16_t)nk[k];
                 if (tid == 0) {
-                    const size_t sv = gk * dm.b_max + code;
+                    const size_t sv = gk * dm.V + code;
                     so.mu[sv] = (int16_t)(mus - 1);
                     so.T[sv] = s_T;
                     so.L[sv] = s_L;
                     __threadfence();
-                    atomicMax(&si.best[slot], code);
+                    if (sweep) atomicMax(&si.best[slot], code);
                 }
                 served = true;
             }
@@ -701,7 +717,7 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
                     out.master[slot] = -1; out.bsel[slot] = -1;
                     out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
                 } else {
-                    const size_t sv = (size_t)slot * dm.b_max + best;
+                    const size_t sv = (size_t)slot * dm.V + best;
                     const double T = so.T[sv];
                     out.master[slot] = so.mu[sv];
                     out.bsel[slot] = (int16_t)(role ? best + 1 : 0);
@@ -721,7 +737,7 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
     if (lane == 0) s_off[wl][R] = M;
     __syncwarp();
     // partition: position i belongs to the last replica c with off_c <= i
-    const int16_t *split = so.layers + (size_t)g * dm.b_max * M;
+    const int16_t *split = so.layers + (size_t)g * dm.V * M;
     for (int i = lane; i < M; i += 32) {
         int lo = 0, hi = R - 1;
         while (lo < hi) {
@@ -782,6 +798,142 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
     atomicAdd(&out.stats[kStGenomes], 1ull);
 }
 
+// Alg. 2's role search, one warp per genome.  Each replica's lane reads its
+// two results: the prefill run (variant bit b_max, run when the memory allows)
+// and the decode sweep's answer (the largest accepted batch).  Every role
+// assignment r (bit c = 1: replica c decodes) is then scored as Eq. 3-5 score a
+// genome (PS and DS summed in ascending replica order over the replicas that
+// serve their role), the lanes taking r = lane, lane + 32, ...; the least
+// (w, phase, r) wins.  The replicas' outputs are those of their chosen roles,
+// the chosen roles are written into the genome, and the genome is scored.
+__global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop, SlotInfo si, SplitOut so,
+                                                             EvalOut out)
+{
+    __shared__ double s_ps[4][E2_MAX_ROLE_SEARCH], s_ds[4][E2_MAX_ROLE_SEARCH];
+    __shared__ int s_pv[4][E2_MAX_ROLE_SEARCH], s_dv[4][E2_MAX_ROLE_SEARCH];
+    __shared__ int s_off[4][E2_MAX_ROLE_SEARCH + 1], s_code[4][E2_MAX_ROLE_SEARCH];
+    const int wl = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = blockIdx.x * 4 + wl;
+    if (g >= dm.P) return;
+    const int K = dm.K, M = dm.M, V = dm.V, bp = dm.b_max;
+    const int R = pop.nclus[g];
+    auto score = [&](uint64_t r, double &PS, double &DS, double &w, double &phase) {
+        PS = 0.0; DS = 0.0;
+        for (int c = 0; c < R; ++c) {
+            if ((r >> c) & 1ull) { if (s_dv[wl][c]) DS = DS + s_ds[wl][c]; }
+            else if (s_pv[wl][c]) PS = PS + s_ps[wl][c];
+        }
+        w = keyd(kInfKey); phase = keyd(kInfKey);
+        if (PS != 0.0 && DS != 0.0) {
+            const double tp = (double)dm.NP / PS, td = (double)dm.ND / DS;
+            phase = tp >= td ? tp : td;                 // Eq. 3
+            const double x = phase - dm.t_a;
+            const double bn = x > 0.0 ? x : 0.0;        // Eq. 4
+            w = bn > 0.0 ? tp + bn : 0.0;               // Eq. 5
+        }
+    };
+    // ---- each replica's two results
+    int best = -1, pok = 0, m = 0;
+    if (lane < R) {
+        const int slot = g * K + lane;
+        const uint64_t mask = si.mask[slot];
+        m = pop.sizes[slot];
+        pok = (int)((mask >> bp) & 1ull);
+        best = mask ? si.best[slot] : -1;
+        s_off[wl][lane] = si.off[slot];
+        s_pv[wl][lane] = pok;
+        s_dv[wl][lane] = best >= 0;
+        s_ps[wl][lane] = pok ? (double)dm.NP / so.T[(size_t)slot * V + bp] : 0.0;
+        s_ds[wl][lane] = best >= 0 ? (double)(best + 1) / so.T[(size_t)slot * V + best] : 0.0;
+    }
+    if (lane == 0) s_off[wl][R] = M;
+    __syncwarp();
+    // ---- the best assignment
+    double bw = keyd(kInfKey), bph = keyd(kInfKey);
+    uint64_t br = ~0ull;
+    for (uint64_t r = lane; r < (1ull << R); r += 32) {
+        double PS, DS, w, ph;
+        score(r, PS, DS, w, ph);
+        if (w < bw || (w == bw && (ph < bph || (ph == bph && r < br)))) { bw = w; bph = ph; br = r; }
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        const double ow = __shfl_xor_sync(0xFFFFFFFFu, bw, o), op = __shfl_xor_sync(0xFFFFFFFFu, bph, o);
+        const uint64_t orr = __shfl_xor_sync(0xFFFFFFFFu, br, o);
+        if (ow < bw || (ow == bw && (op < bph || (op == bph && orr < br)))) { bw = ow; bph = op; br = orr; }
+    }
+    // ---- outputs of the chosen roles
+    unsigned long long n_rep = 0, n_served = 0, n_paper = 0;
+    if (lane < R) {
+        const int slot = g * K + lane;
+        const int role = (int)((br >> lane) & 1ull);
+        const int code = role ? best : (pok ? bp : -1);
+        s_code[wl][lane] = code;
+        if (code < 0) {
+            out.master[slot] = -1; out.bsel[slot] = -1;
+            out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
+        } else {
+            const size_t sv = (size_t)slot * V + code;
+            out.master[slot] = so.mu[sv];
+            out.bsel[slot] = (int16_t)(role ? code + 1 : 0);
+            out.T[slot] = so.T[sv];
+            out.L[slot] = so.L[sv];
+            ++n_served;
+        }
+        if (si.mask[slot]) {                         // replicas with no work were counted by the pre-pass
+            const unsigned long long ndec = best >= 0 ? (unsigned long long)(bp - best) : (unsigned long long)bp;
+            ++n_rep;
+            n_paper += (1 + ndec) * paper_candidates(m, dm.N);
+        }
+    }
+    __syncwarp();
+    const int16_t *split = so.layers + (size_t)g * V * M;
+    for (int i = lane; i < M; i += 32) {
+        int lo = 0, hi = R - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (s_off[wl][mid] <= i) lo = mid;
+            else hi = mid - 1;
+        }
+        const int code = s_code[wl][lo];
+        out.layers[(size_t)g * M + i] = code >= 0 ? split[(size_t)code * M + i] : (int16_t)-1;
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        n_rep += __shfl_xor_sync(0xFFFFFFFFu, n_rep, o);
+        n_served += __shfl_xor_sync(0xFFFFFFFFu, n_served, o);
+        n_paper += __shfl_xor_sync(0xFFFFFFFFu, n_paper, o);
+    }
+    // fingerprint of the genome with its chosen roles (a tree fold over the lanes)
+    uint64_t hl = 0x9E3779B97F4A7C15ull ^ (uint64_t)lane;
+    auto mix = [](uint64_t h, uint64_t x) { h = (h ^ x) * 0xBF58476D1CE4E5B9ull; return h ^ (h >> 31); };
+    const uint16_t *pp = pop.perm + (size_t)g * M;
+    for (int i = lane; i < M; i += 32) hl = mix(hl, pp[i]);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        const uint64_t other = __shfl_down_sync(0xFFFFFFFFu, hl, o);
+        if (lane < o) hl = mix(hl, other);
+    }
+    if (lane != 0) return;
+    if (n_rep) {
+        atomicAdd(&out.stats[kStReplicas], n_rep);
+        atomicAdd(&out.stats[kStPaper], n_paper);
+    }
+    if (n_served) atomicAdd(&out.stats[kStServed], n_served);
+    double PS, DS, w, phase;
+    score(br, PS, DS, w, phase);
+    double *f = out.fit + (size_t)g * 4;
+    f[0] = w; f[1] = phase; f[2] = PS; f[3] = DS;
+    pop.roles[g] = br;
+    uint64_t h = hl;
+    const uint16_t *ss = pop.sizes + (size_t)g * K;
+    for (int i = 0; i < R; ++i) h = mix(h, (uint64_t)ss[i] << 16);
+    h = mix(h, (uint64_t)R << 40);
+    h = mix(h, br);
+    out.hash[g] = h;
+    atomicAdd(&out.stats[kStGenomes], 1ull);
+}
+
 cudaError_t configure_eval(e2_ctx *c)
 {
     const void *kernel = reinterpret_cast<const void *>(dp_eval_kernel);
@@ -820,8 +972,9 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     if (c->ev_dp_start && (e = cudaEventRecordWithFlags(c->ev_dp_start, c->stream, rec)) != cudaSuccess) return e;
     dp_eval_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so);
     if (c->ev_dp_stop && (e = cudaEventRecordWithFlags(c->ev_dp_stop, c->stream, rec)) != cudaSuccess) return e;
-    finalize_score_kernel<<<(unsigned)(((size_t)c->dm.P * 32 + 127) / 128), 128, 0, c->stream>>>(c->dm, p, si, so,
-                                                                                               out);
+    const unsigned fb = (unsigned)(((size_t)c->dm.P * 32 + 127) / 128);
+    if (c->dm.role_search) finalize_roles_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
+    else finalize_score_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
     return cudaGetLastError();
 }
 

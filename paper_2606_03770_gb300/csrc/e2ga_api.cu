@@ -76,15 +76,15 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K)
     l.stats = take(8 * kNumStats);
     l.err = take(4);
     l.order_bins = take(4 * (size_t)kCtrlWords);
-    l.items = take(8 * (size_t)P * K * b_max);
+    l.items = take(8 * (size_t)P * K * V);
     l.slot_off = take(4 * (size_t)P * K);
     l.slot_mask = take(8 * (size_t)P * K);
     l.slot_size = take((size_t)P * K);
     l.slot_best = take(4 * (size_t)P * K);
-    l.split_T = take(8 * (size_t)P * K * b_max);
-    l.split_L = take(8 * (size_t)P * K * b_max);
-    l.split_mu = take(2 * (size_t)P * K * b_max);
-    l.split_layers = take(2 * (size_t)P * b_max * M);
+    l.split_T = take(8 * (size_t)P * K * V);                 // per (slot, variant bit): decode b = bit + 1,
+    l.split_L = take(8 * (size_t)P * K * V);                 // and bit b_max = prefill when roles are searched
+    l.split_mu = take(2 * (size_t)P * K * V);
+    l.split_layers = take(2 * (size_t)P * V * M);
     l.total = o;
     return l;
 }
@@ -185,6 +185,11 @@ int validate_inputs(const e2_devices *d, const e2_links *l, const e2_layer_profi
     for (double q : probs)
         if (!(q >= 0.0 && q <= 1.0)) { snprintf(msg, n, "probabilities must lie in [0, 1]"); return E2_EINVAL; }
     if (p->tournament < 1) { snprintf(msg, n, "tournament size must be >= 1"); return E2_EINVAL; }
+    if (p->role_search != 0 && p->role_search != 1) { snprintf(msg, n, "role_search must be 0 or 1"); return E2_EINVAL; }
+    if (p->role_search && (p->K_max > E2_MAX_ROLE_SEARCH || pf->b_max > 63)) {
+        snprintf(msg, n, "role_search needs K_max <= %d and b_max <= 63", E2_MAX_ROLE_SEARCH);
+        return E2_EINVAL;
+    }
     return E2_OK;
 }
 
@@ -293,7 +298,7 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     if (!c) return E2_ENOMEM;
     c->stream = static_cast<cudaStream_t>(stream);
     c->dm = Dims{M, N, b_max + 1, b_max, P, Q, K, l.LS, prm->tournament, prof->NP, prof->ND,
-                 prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps)};
+                 prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps), prm->role_search};
     c->cong_lo = links->cong_lo;
     c->cong_hi = links->cong_hi;
     c->thr_cx = threshold(prm->p_cx);

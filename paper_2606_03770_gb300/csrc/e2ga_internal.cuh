@@ -57,6 +57,7 @@ struct Dims {
     uint64_t NP, ND;
     double min_tps, t_a;
     double lam_max;      // largest latency Lambda with 1.0 / Lambda >= min_tps (see e2_create)
+    int role_search;     // 1: both roles per replica, best assignment per genome (Alg. 2)
 };
 
 struct Tables {
@@ -79,9 +80,9 @@ struct SlotInfo {
     int32_t *best;             // [P*K] largest variant bit accepted so far (-1: none)
 };
 
-// Work items of the DP: (slot << 8) | variant bit.
+// Work items of the DP: (slot << 8) | role << 7 | sweep << 6 | variant bit.
 struct WorkList {
-    uint64_t *items;           // [P*K*b_max]
+    uint64_t *items;           // [P*K*(b_max+1)] (slot << 8) | role << 7 | sweep << 6 | variant bit
     unsigned *ctrl;            // [kOrderBins] bins/cursors, then the CtrlWord words
 };
 

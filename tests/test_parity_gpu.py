@@ -326,3 +326,48 @@ def test_recorded_generation_matches_separate_calls(name, P, gens):
     b.set_timing_events()
     a.close()
     b.close()
+
+
+@pytest.mark.parametrize("name,P", [("c1_tiny", 64), ("c2", 1024)])
+def test_role_search_parity(name, P):
+    """Alg. 2's brute-force role assignment: every replica evaluated in both
+    roles, the best of the 2^R assignments chosen and written into the
+    genomes; compared with the oracle element by element."""
+    import dataclasses
+    prob = dataclasses.replace(W.make_config(name, P=P), role_search=1)
+    eng = engine(prob)
+    g = W.random_genomes(prob.M, prob.K_max, P, seed=13)
+    eng.eval(g)
+    gpu = eng.results()
+    ora = O.OracleProblem(prob).eval_population(g, prob.K_max, nthreads=O.num_threads())
+    assert_eval_equal(gpu, ora)
+    assert np.array_equal(eng.get_population()["roles"], ora["roles"])
+    st = eng.stats()
+    assert st["paper_candidates"] == ora["cand"]
+    assert st["served"] == int((ora["bsel"] >= 0).sum())
+    eng.close()
+
+
+def test_role_search_generations():
+    """Generations with the role search, recorded and separate calls alike,
+    against the oracle (whose population takes the roles it chose)."""
+    import dataclasses
+    prob = dataclasses.replace(W.make_config("c2", P=256), role_search=1)
+    ga = O.ga_of(prob)
+    op = O.OracleProblem(prob)
+    eng = engine(prob)
+    eng.init_population(9)
+    pop = O.init_population(ga, 9)
+    assert_genomes_equal(eng.get_population(), pop)
+    for gen in range(1, 5):
+        ora = op.eval_population(pop, prob.K_max, nthreads=O.num_threads())
+        if gen % 2:
+            eng.run_generation(9, gen)
+        else:
+            eng.eval(parts=False)
+            eng.ga_step(9, gen)
+        assert np.array_equal(eng.results()["fitness"], ora["fitness"]), gen
+        pop = dict(pop, roles=ora["roles"])
+        pop = O.ga_step(ga, 9, gen, pop, ora["fitness"], O.elites(ga, pop, ora["fitness"]))
+        assert_genomes_equal(eng.get_population(), pop)
+    eng.close()
