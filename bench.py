@@ -19,6 +19,7 @@ its own GPU; value is the sum over ranks divided by the slowest rank's time.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import datetime
 import json
 import math
@@ -65,7 +66,26 @@ def parse():
     ap.add_argument("--seed", type=int, default=2026)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--roles", default="bits", choices=["bits", "search"],
+                    help="replica roles: bits of the genome, or Alg. 2's brute-force search")
     return ap.parse_args()
+
+
+def problem(args):
+    prob = W.make_config(args.config)
+    if args.roles == "search":
+        prob = dataclasses.replace(prob, role_search=1)
+    return prob
+
+
+def workload_label(prob):
+    mdl = W.CONFIGS[prob.name]["model"]
+    kv = f"GQA {mdl['kv_heads']} KV heads" if mdl.get("kv_heads") else "MHA"
+    roles = "roles searched per genome (Alg. 2)" if prob.role_search else "one role bit per replica"
+    return (f"{prob.name}: M={prob.M} devices, N={prob.N} blocks (d={mdl['d']}, ffn={mdl['ffn']}, {kv}, "
+            f"{mdl['wbits']}-bit weights), K_max={prob.K_max} replicas, P={prob.P}, Q={prob.Q}, "
+            f"b_max={prob.b_max}, {roles}, one generation per step"
+            + (", congestion redrawn per generation" if prob.redraw else ""))
 
 
 def dist_info():
@@ -191,7 +211,7 @@ def run_reference(args):
     rank, world, _ = dist_info()
     if rank != 0:
         return
-    prob = W.make_config(args.config)
+    prob = problem(args)
     from oracle import oracle as O
     nt = O.num_threads()
     sample = min(prob.P, 16 * nt)
@@ -220,8 +240,7 @@ def run_reference(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / len(times),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded fleet, links and dense-decoder profile)",
-            "config": {"workload": f"{prob.name}: M={prob.M} devices, N={prob.N} blocks, K_max={prob.K_max}, "
-                                   f"P={prob.P}", "sample_genomes_per_step": sample},
+            "config": {"workload": workload_label(prob), "sample_genomes_per_step": sample},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": nt, "kind": "oracle",
                              "sample": f"per step, {sample} of {prob.P} genomes evaluated by the oracle on "
                                        f"{nt} threads and scaled to the population, plus the elites and "
@@ -242,7 +261,7 @@ def run_ours(args):
     ge.build()
     from paper_2606_03770_gb300.e2ga import Engine
 
-    prob = W.make_config(args.config)
+    prob = problem(args)
     seed = args.seed + 1000 * rank
     eng = Engine(prob)
     stream = eng.stream
@@ -348,9 +367,7 @@ def run_ours(args):
             "warmup": args.warmup, "ms_per_step": 1e3 * t_max / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded fleet, links and dense-decoder profile; no paper data)",
-            "config": {"workload": f"{prob.name}: M={prob.M} devices, N={prob.N} blocks (d=8192, ffn=28672, "
-                                   f"GQA 8 KV heads, 4-bit weights), K_max={prob.K_max} replicas, "
-                                   f"P={prob.P}, Q={prob.Q}, b_max={prob.b_max}, one generation per step",
+            "config": {"workload": workload_label(prob),
                        "l2": "flushed (256 MB write) between timed steps",
                        "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
             "gpu_launches": LAUNCHES_PER_STEP * args.steps,
