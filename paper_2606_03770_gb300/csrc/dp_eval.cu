@@ -117,18 +117,11 @@ __device__ __forceinline__ void bar_named(int id, int nthreads)
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-__device__ __forceinline__ double warp_sum_d(double x)
-{
-#pragma unroll
-    for (int o = 16; o; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
-    return x;
-}
-
 }  // namespace
 
-// Shared-memory bytes per warp of the pre-pass (26 bytes per device, rounded
-// up to 16 so that every warp's 64-bit arrays start aligned).
-__host__ __device__ __forceinline__ size_t variant_stride(int mcap) { return ((size_t)mcap * 26 + 15) & ~(size_t)15; }
+// Shared-memory bytes per warp of the pre-pass (18 bytes per device, rounded
+// up to 16 so that every warp's arrays start aligned).
+__host__ __device__ __forceinline__ size_t variant_stride(int mcap) { return ((size_t)mcap * 18 + 15) & ~(size_t)15; }
 
 // Per slot: slots with nothing to run get their outputs here (empty slots,
 // more devices than blocks, no variant left by the pre-pass).  Every other
@@ -153,26 +146,27 @@ __device__ __forceinline__ int item_bin(int level, int size)
 //  * decode latency: Lambda >= sum of link times + sum_k n_k c_k (c_k the
 //    per-block time, the head only adds), whose least value puts one block on
 //    each device and the other N - m on the cheapest devices up to their
-//    capacity.  A variant whose bound misses Min_TPS fails whatever partition
-//    the DP returns; the 1e-9 margin exceeds the rounding of every sum here.
+//    capacity.  It is summed in float from times rounded down, every operation
+//    rounded toward -inf, so it never exceeds the exact bound; a variant whose
+//    bound is above Lambda_max (rounded up to float) fails whatever partition
+//    the DP returns.
 // Both tests are monotone in the batch: the capacities shrink as b grows (more
 // KV memory per block), and the bound is the least of a linear cost whose
 // coefficients (per-block and link times) grow with b over a feasible set that
 // shrinks with b.  So the variants are tested from the largest batch down and
 // the first that passes keeps every smaller batch as well (rounding could at
 // most keep a variant the bound would have dropped, which costs a DP run and
-// changes no result).  The surviving variants form the slot's mask.  A slot with nothing to run
+// changes no result).
+// The surviving variants form the slot's mask.  A slot with nothing to run
 // (empty, more devices than blocks, no variant left) gets its outputs here;
-// the others count their work items into the ordering bins.  The last CTA to
+// the others count their work items into the ordering bins.  The last warp to
 // finish (a ticket taken after a fence, no waiting) scans the bins into
 // starting offsets, heaviest first, and stores the item total.
-__global__ void __launch_bounds__(128, 12) slot_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si, EvalOut out,
-                                                   unsigned *ctrl)
+__global__ void __launch_bounds__(64, 24) slot_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si, EvalOut out,
+                                                  unsigned *ctrl)
 {
     // per warp: device ids, capacities and per-block times of up to mcap devices
     extern __shared__ __align__(16) unsigned char vsm[];
-    __shared__ int s_last;
-    __shared__ unsigned s_part[4];
     const int mcap = dm.M < dm.N ? dm.M : dm.N;
     const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
     const int K = dm.K, M = dm.M, N = dm.N;
@@ -193,8 +187,8 @@ __global__ void __launch_bounds__(128, 12) slot_kernel(Dims dm, Tables tb, DevPo
         if (c < R && m <= N) {
             const int W = N - m + 1;
             unsigned char *wbase = vsm + (size_t)wl * variant_stride(mcap);
-            uint64_t *scb = reinterpret_cast<uint64_t *>(wbase);          // per-block times as order keys
-            double *stau = reinterpret_cast<double *>(scb + mcap);        // link (k-1) -> k
+            uint32_t *scb = reinterpret_cast<uint32_t *>(wbase);          // per-block times (float bits)
+            float *stau = reinterpret_cast<float *>(scb + mcap);          // link (k-1) -> k
             int *sc0 = reinterpret_cast<int *>(stau + mcap), *sc1 = sc0 + mcap;
             uint16_t *sdev = reinterpret_cast<uint16_t *>(sc1 + mcap);
             for (int k = lane; k < m; k += 32) sdev[k] = pop.perm[(size_t)g * M + off + k];
@@ -209,15 +203,15 @@ __global__ void __launch_bounds__(128, 12) slot_kernel(Dims dm, Tables tb, DevPo
                 const int v = prole ? i + 1 : 0;
                 const int32_t *cap = tb.cap + (size_t)v * M * 2;
                 const bool bound = prole && dm.min_tps > 0.0;
-                const double *cpb = tb.cpb + (size_t)v * M;
-                const double *tau = tb.tau + (size_t)v * M * M;
+                const float *cpb = tb.cpb + (size_t)v * M;
+                const float *tau = tb.tau_lb + (size_t)v * M * M;
                 int s0 = 0, z = 0;
                 for (int k = lane; k < m; k += 32) {                   // every load of the variant at once
                     const int d = sdev[k];
                     const int c0 = min(cap[d * 2], W), c1 = min(cap[d * 2 + 1], W);
                     if (bound) {
-                        scb[k] = dkey(cpb[d]);
-                        stau[k] = k ? tau[(size_t)sdev[k - 1] * M + d] : 0.0;
+                        scb[k] = __float_as_uint(cpb[d]);               // non-negative: bits order as values
+                        stau[k] = k ? tau[(size_t)sdev[k - 1] * M + d] : 0.0f;
                     }
                     sc0[k] = c0;
                     sc1[k] = c1;
@@ -235,23 +229,24 @@ __global__ void __launch_bounds__(128, 12) slot_kernel(Dims dm, Tables tb, DevPo
                     continue;
                 }
                 if (bound) {
-                    double part = 0.0;
+                    float part = 0.0f;
                     for (int k = lane; k < m; k += 32) {
-                        const uint64_t ck = scb[k];
-                        long long before = 0;            // capacity of the cheaper devices
+                        const uint32_t ck = scb[k];
+                        int before = 0;                  // capacity of the cheaper devices
                         for (int j = 0; j < m; ++j) {
-                            const uint64_t cj = scb[j];
+                            const uint32_t cj = scb[j];
                             if (cj < ck || (cj == ck && j < k)) before += sc0[j] - 1;
                         }
-                        const long long ek = sc0[k] - 1;
-                        const long long room = (long long)(N - m) - before;
-                        const long long take = room <= 0 ? 0 : (room < ek ? room : ek);
-                        part += keyd(ck) * (double)(1 + take);
-                        if (k >= 1) part += stau[k];
+                        const int ek = sc0[k] - 1;
+                        const int room = (N - m) - before;
+                        const int take = room <= 0 ? 0 : (room < ek ? room : ek);
+                        part = __fadd_rd(part, __fmul_rd(__uint_as_float(ck), (float)(1 + take)));
+                        if (k >= 1) part = __fadd_rd(part, stau[k]);
                     }
-                    const double lb = warp_sum_d(part) * (1.0 - 1e-9);
+#pragma unroll
+                    for (int o = 16; o; o >>= 1) part = __fadd_rd(part, __shfl_xor_sync(0xFFFFFFFFu, part, o));
                     __syncwarp();
-                    if (lb > dm.lam_max) {                              // 1.0 / lb < Min_TPS
+                    if (part > dm.lam_max_up) {                        // 1.0 / Lambda < Min_TPS
                         ++n_tps;
                         continue;
                     }
@@ -288,36 +283,33 @@ __global__ void __launch_bounds__(128, 12) slot_kernel(Dims dm, Tables tb, DevPo
             }
         }
     }
-    // ---- the last CTA scans the bins
-    __syncthreads();
-    if (threadIdx.x == 0) {
+    // ---- the last warp to finish scans the bins: lane t owns positions
+    //      [32t, 32t + 32) of the descending bin order
+    unsigned ticket = 0;
+    if (lane == 0) {
         __threadfence();
-        s_last = atomicAdd(&ctrl[kCtrlTicket], 1u) == gridDim.x - 1;
+        ticket = atomicAdd(&ctrl[kCtrlTicket], 1u);
     }
-    __syncthreads();
-    if (!s_last) return;
+    ticket = __shfl_sync(0xFFFFFFFFu, ticket, 0);
+    if (ticket != gridDim.x * (blockDim.x >> 5) - 1) return;
     __threadfence();
-    // thread t owns positions [8t, 8t + 8) of the descending bin order
-    constexpr int kPer = kOrderBins / 128;
-    unsigned *own = ctrl + kOrderBins - 1 - threadIdx.x * kPer;      // own[-j] = position 8t + j
+    constexpr int kPer = kOrderBins / 32;
+    unsigned *own = ctrl + kOrderBins - 1 - lane * kPer;           // own[-j] = position 32 lane + j
     unsigned sum = 0;
     for (int j = 0; j < kPer; ++j) sum += __ldcg(own - j);
-    unsigned incl = sum;                                   // inclusive scan over the warp
+    unsigned incl = sum;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
         const unsigned x = __shfl_up_sync(0xFFFFFFFFu, incl, o);
         if (lane >= o) incl += x;
     }
-    if (lane == 31) s_part[wl] = incl;
-    __syncthreads();
     unsigned base = incl - sum;
-    for (int w = 0; w < wl; ++w) base += s_part[w];
     for (int j = 0; j < kPer; ++j) {
         const unsigned cnt = __ldcg(own - j);
         own[-j] = base;
         base += cnt;
     }
-    if (threadIdx.x == 127) ctrl[kCtrlTotal] = base;
+    if (lane == 31) ctrl[kCtrlTotal] = base;
 }
 
 // Item lv of a slot (its variants from the largest batch down) goes to bin
@@ -950,7 +942,7 @@ cudaError_t configure_eval(e2_ctx *c)
 
 cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
 {
-    Tables tb{c->rate, c->bw, c->mem, c->prof, c->leaf, c->tau, c->cap, c->cpb, c->leaf_rank, c->tau_rank};
+    Tables tb{c->rate, c->bw, c->mem, c->prof, c->leaf, c->tau, c->cap, c->cpb, c->tau_lb, c->leaf_rank, c->tau_rank};
     EvalOut out{c->fit, c->layers, c->master, c->bsel, c->T, c->L, c->hash, c->stats};
     SlotInfo si{c->slot_off, c->slot_mask, c->slot_size, c->slot_best};
     WorkList wl{c->items, c->order_bins};
@@ -960,8 +952,8 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     if (e != cudaSuccess) return e;
     const unsigned gb = (unsigned)((slots + 255) / 256 < 1024 ? (slots + 255) / 256 : 1024);
     const int mcap = c->dm.M < c->dm.N ? c->dm.M : c->dm.N;
-    slot_kernel<<<(unsigned)((slots + 3) / 4), 128, 4 * variant_stride(mcap), c->stream>>>(c->dm, tb, p, si, out,
-                                                                                       c->order_bins);
+    slot_kernel<<<(unsigned)((slots + 1) / 2), 64, 2 * variant_stride(mcap), c->stream>>>(c->dm, tb, p, si, out,
+                                                                                      c->order_bins);
     order_scatter_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, wl);
     // while a launch sequence is being recorded, the timing events become
     // event-record nodes of the graph (an ordinary record would only mark a

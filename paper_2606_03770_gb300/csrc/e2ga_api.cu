@@ -20,7 +20,7 @@ thread_local char g_create_error[256] = "";
 size_t align_up(size_t x, size_t a = 256) { return (x + a - 1) / a * a; }
 
 struct Layout {
-    size_t rate, bw, mem, link_bw, cong, prof, leaf, tau, cap, cpb, leaf_sorted, beff_sorted, tau_sorted,
+    size_t rate, bw, mem, link_bw, cong, prof, leaf, tau, tau_lb, cap, cpb, leaf_sorted, beff_sorted, tau_sorted,
         leaf_rank, tau_rank;
     size_t perm[2], sizes[2], nclus[2], roles[2];
     size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, stats, err, order_bins, items, slot_off, slot_mask, slot_size, slot_best,
@@ -51,7 +51,8 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K)
     l.leaf = take(8 * V * M * 2 * (size_t)l.LS);
     l.tau = take(8 * V * MM);
     l.cap = take(4 * V * M * 2);
-    l.cpb = take(8 * V * M);
+    l.cpb = take(4 * V * M);
+    l.tau_lb = take(4 * V * MM);
     l.leaf_sorted = take(8 * V * rank_pow2((size_t)M * 2 * N));
     l.beff_sorted = take(8 * rank_pow2(MM));
     l.tau_sorted = take(8 * V * MM);
@@ -298,7 +299,13 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     if (!c) return E2_ENOMEM;
     c->stream = static_cast<cudaStream_t>(stream);
     c->dm = Dims{M, N, b_max + 1, b_max, P, Q, K, l.LS, prm->tournament, prof->NP, prof->ND,
-                 prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps), prm->role_search};
+                 prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps), prm->role_search, 0.0f};
+    {
+        const double lm = c->dm.lam_max;                       // rounded up to float
+        float f = (float)lm;
+        if ((double)f < lm) f = nextafterf(f, HUGE_VALF);
+        c->dm.lam_max_up = f;
+    }
     c->cong_lo = links->cong_lo;
     c->cong_hi = links->cong_hi;
     c->thr_cx = threshold(prm->p_cx);
@@ -342,7 +349,8 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->leaf = reinterpret_cast<double *>(ws + l.leaf);
     c->tau = reinterpret_cast<double *>(ws + l.tau);
     c->cap = reinterpret_cast<int32_t *>(ws + l.cap);
-    c->cpb = reinterpret_cast<double *>(ws + l.cpb);
+    c->cpb = reinterpret_cast<float *>(ws + l.cpb);
+    c->tau_lb = reinterpret_cast<float *>(ws + l.tau_lb);
     c->leaf_sorted = reinterpret_cast<uint64_t *>(ws + l.leaf_sorted);
     c->beff_sorted = reinterpret_cast<uint64_t *>(ws + l.beff_sorted);
     c->tau_sorted = reinterpret_cast<double *>(ws + l.tau_sorted);

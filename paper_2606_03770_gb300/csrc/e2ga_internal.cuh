@@ -58,6 +58,7 @@ struct Dims {
     double min_tps, t_a;
     double lam_max;      // largest latency Lambda with 1.0 / Lambda >= min_tps (see e2_create)
     int role_search;     // 1: both roles per replica, best assignment per genome (Alg. 2)
+    float lam_max_up;    // lam_max rounded up to float (the float latency bound is compared with it)
 };
 
 struct Tables {
@@ -67,7 +68,8 @@ struct Tables {
     const double *leaf;        // [V][M][2][LS]: leaf[((v*M+d)*2+mf)*LS + n-1] = l_d(n blocks, master mf)
     const double *tau;         // [V][M][M]
     const int32_t *cap;        // [V][M][2]: most blocks device d holds (memory), without / with the head
-    const double *cpb;         // [V][M]: per-block time max(blk_flops/rate, blk_bytes/bw)
+    const float *cpb;          // [V][M]: per-block time max(blk_flops/rate, blk_bytes/bw), rounded down
+    const float *tau_lb;       // [V][M][M]: tau rounded down
     const uint32_t *leaf_rank; // [V][M][2][LS]: order key of leaf within its variant's value set
     const uint32_t *tau_rank;  // [V][M][M]
 };
@@ -169,7 +171,8 @@ struct e2_ctx {
     uint64_t *prof = nullptr;
     double *leaf = nullptr, *tau = nullptr;
     int32_t *cap = nullptr;
-    double *cpb = nullptr;
+    float *cpb = nullptr;
+    float *tau_lb = nullptr;
     uint64_t *leaf_sorted = nullptr;  // [V][pow2(2 M N)] sorted stage-time keys
     uint64_t *beff_sorted = nullptr;  // [pow2(M M)] sorted effective link bandwidths
     double *tau_sorted = nullptr;     // [V][M M] sorted link times

@@ -45,9 +45,10 @@ __global__ void tables_kernel(Dims dm, const double *rate, const double *bw, con
 
 // Per (variant, device): the most blocks the device can hold, without and with
 // the LM head (the number of finite entries of its two cost rows), and the
-// per-block time max(blk_flops/rate, blk_bytes/bw) used by the latency bound.
+// per-block time max(blk_flops/rate, blk_bytes/bw) rounded down to float, used
+// by the latency bound.
 __global__ void captab_kernel(Dims dm, const double *rate, const double *bw, const uint64_t *mem,
-                              const uint64_t *prof, int32_t *cap, double *cpb)
+                              const uint64_t *prof, int32_t *cap, float *cpb)
 {
     const size_t total = (size_t)dm.V * dm.M;
     for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < total;
@@ -61,13 +62,14 @@ __global__ void captab_kernel(Dims dm, const double *rate, const double *bw, con
         cap[idx * 2 + 1] = (int32_t)(c1 < (uint64_t)dm.N ? c1 : (uint64_t)dm.N);
         const double tc = __ull2double_rn(prof[kBlkFlops * V + v]) / rate[d];
         const double tm = __ull2double_rn(prof[kBlkBytes * V + v]) / bw[d];
-        cpb[idx] = tc >= tm ? tc : tm;
+        cpb[idx] = __double2float_rd(tc >= tm ? tc : tm);
     }
 }
 
-// tau_v(a, b) = A_v / (B(a,b) * congestion(a,b)) (Sec. 3.2).
+// tau_v(a, b) = A_v / (B(a,b) * congestion(a,b)) (Sec. 3.2), and the same
+// rounded down to float for the latency bound.
 __global__ void tau_kernel(Dims dm, const double *link_bw, const double *cong, const uint64_t *prof,
-                           double *tau)
+                           double *tau, float *tau_lb)
 {
     const size_t MM = (size_t)dm.M * dm.M, total = (size_t)dm.V * MM;
     for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < total;
@@ -75,7 +77,9 @@ __global__ void tau_kernel(Dims dm, const double *link_bw, const double *cong, c
         const int v = (int)(idx / MM);
         const size_t ab = idx - (size_t)v * MM;
         const double beff = link_bw[ab] * cong[ab];
-        tau[idx] = __ull2double_rn(prof[kAct * dm.V + v]) / beff;
+        const double t = __ull2double_rn(prof[kAct * dm.V + v]) / beff;
+        tau[idx] = t;
+        tau_lb[idx] = __double2float_rd(t);
     }
 }
 
@@ -463,7 +467,7 @@ cudaError_t launch_tables(const e2_ctx *c)
 cudaError_t launch_tau(const e2_ctx *c)
 {
     const size_t total = (size_t)c->dm.V * c->dm.M * c->dm.M;
-    tau_kernel<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm, c->link_bw, c->cong, c->prof, c->tau);
+    tau_kernel<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm, c->link_bw, c->cong, c->prof, c->tau, c->tau_lb);
     return cudaGetLastError();
 }
 
