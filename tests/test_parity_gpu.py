@@ -371,3 +371,45 @@ def test_role_search_generations():
         pop = O.ga_step(ga, 9, gen, pop, ora["fitness"], O.elites(ga, pop, ora["fitness"]))
         assert_genomes_equal(eng.get_population(), pop)
     eng.close()
+
+
+def _genomes_from(M, K, groups, rng):
+    """Genomes with the given replica sizes (one list per genome) over random orderings."""
+    P = len(groups)
+    g = dict(perm=np.zeros((P, M), np.uint16), sizes=np.zeros((P, K), np.uint16),
+             nclus=np.zeros(P, np.uint8), roles=np.zeros(P, np.uint64))
+    for p, sz in enumerate(groups):
+        assert sum(sz) == M and len(sz) <= K
+        g["perm"][p] = rng.permutation(M)
+        g["sizes"][p, :len(sz)] = sz
+        g["nclus"][p] = len(sz)
+        g["roles"][p] = rng.integers(0, 1 << len(sz))
+    return g
+
+
+@pytest.mark.parametrize("case", ["wide rows", "largest replica"])
+def test_eval_parity_maximum_sizes(case):
+    """The largest shapes the ABI takes: cost rows of ~300 blocks (W > 256,
+    ~190 KB of DP shared memory), and a replica of 256 devices (the limit) next
+    to mixed ones; then a generation step on them."""
+    rng = np.random.default_rng(77)
+    if case == "wide rows":
+        M, N, K = 64, 300, 6
+        prob = _edge_problem(rng, M, N, 12, K, integer=False, Q=2, min_tps=0.02)
+        g = W.random_genomes(M, K, 12, seed=5)
+    else:
+        M, N, K = 256, 260, 2
+        prob = _edge_problem(rng, M, N, 3, K, integer=True, Q=1, min_tps=0.01)
+        g = _genomes_from(M, K, [[256], [250, 6], [200, 56]], rng)
+    eng = engine(prob)
+    eng.eval(g)
+    gpu = eng.results()
+    ora = O.OracleProblem(prob).eval_population(g, K, nthreads=O.num_threads())
+    assert_eval_equal(gpu, ora)
+    assert eng.stats()["paper_candidates"] == ora["cand"]
+    assert np.isfinite(ora["T"]).any()
+    ga = O.ga_of(prob)
+    eidx = O.elites(ga, g, ora["fitness"])
+    eng.ga_step(3, 1)
+    assert_genomes_equal(eng.get_population(), O.ga_step(ga, 3, 1, g, ora["fitness"], eidx))
+    eng.close()
