@@ -53,7 +53,7 @@ INT32_LANES_PER_SM = 128
 LAUNCHES_PER_STEP = 7
 # dram__bytes_read.sum + dram__bytes_write.sum of one dp_eval_kernel launch
 # (generation 7 of this workload), from the ncu capture in profiles/
-DP_TRAFFIC_BYTES = 708608
+DP_TRAFFIC_BYTES = 705536
 
 
 def parse():
