@@ -47,10 +47,6 @@ OPS_PER_PROBE = 6
 OPS_PER_CELL = 6
 SM_COUNT = 152
 INT32_LANES_PER_SM = 128
-# kernels of this library per step (one recorded graph launch): evaluation
-# (pre-pass with the work count, work-list scatter, DP, finalise+score) and
-# generation step (duplicates, ranks, children)
-LAUNCHES_PER_STEP = 7
 # dram__bytes_read.sum + dram__bytes_write.sum of one dp_eval_kernel launch
 # (generation 7 of this workload), from the ncu capture in profiles/
 DP_TRAFFIC_BYTES = 705536
@@ -290,6 +286,7 @@ def run_ours(args):
         eng.run_generation(seed, gen)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     stats, dp_ms = [], []
+    launched = eng.stats()["launches"]     # the library's own count of its kernel launches
     clocks = Clocks(local)
     clocks.start()
     sync_all()
@@ -370,11 +367,15 @@ def run_ours(args):
             "config": {"workload": workload_label(prob),
                        "l2": "flushed (256 MB write) between timed steps",
                        "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
-            "gpu_launches": LAUNCHES_PER_STEP * args.steps,
+            "gpu_launches": stats[-1]["launches"] - launched,
             "dp_cells_per_s": cells * args.steps * world / t_max,
             "paper_candidates_per_s": paper * args.steps * world / t_max,
             "dp_kernel_ms_per_step": 1e3 * dp_s,
             "served_replicas_per_step": sum(s["served"] for s in stats) / args.steps,
+            "dp_launches": {"ctas": [stats[-1]["dp_ctas"], stats[-1]["dp_ctas_small"]],
+                            "smem_bytes": [stats[-1]["dp_smem"], stats[-1]["dp_smem_small"]],
+                            "runs": [sum(s["dp_runs"] - s["dp_runs_small"] for s in stats) / args.steps,
+                                     sum(s["dp_runs_small"] for s in stats) / args.steps]},
             "replicas_per_step": sum(s["replicas"] for s in stats) / args.steps,
             "roofline": {"bound": "alu", "kernel": "dp_eval_kernel (DP_Pipe, timed by events around its launch)",
                          "achieved": achieved, "peak": peak, "unit": "Tops/s (int32)",

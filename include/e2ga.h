@@ -140,7 +140,9 @@ typedef struct {
     double *lambda;
 } e2_partitions;
 
-/* Counters of the last e2_eval_population (device-side tallies). */
+/* Counters of the last evaluation (device-side tallies), then host-side
+ * figures of the context: its DP launch shapes and its kernel launches so
+ * far. */
 typedef struct {
     uint64_t genomes;           /* genomes evaluated                           */
     uint64_t replicas;          /* replicas evaluated (sum of R)                */
@@ -153,6 +155,20 @@ typedef struct {
     uint64_t served;            /* replicas that can serve                      */
     uint64_t tps_pruned;        /* decode variants a latency lower bound proved
                                    to miss Min_TPS (their DP is skipped)        */
+    uint64_t dp_runs_small;     /* of dp_runs, those of the second DP launch:
+                                   replica sizes whose DP needs at most half the
+                                   largest one's shared memory, run with more
+                                   CTAs per SM (0 where that raises no
+                                   occupancy and one launch runs them all)      */
+    uint64_t dp_launches;       /* DP kernel launches per evaluation (1 or 2;
+                                   fixed at e2_create)                          */
+    uint64_t dp_ctas;           /* persistent CTAs of the first DP launch       */
+    uint64_t dp_smem;           /* and its dynamic shared memory per CTA (B)    */
+    uint64_t dp_ctas_small;     /* the same for the second launch (0: none)     */
+    uint64_t dp_smem_small;
+    uint64_t launches;          /* kernels this context has launched since
+                                   e2_create, cumulative (a recorded generation
+                                   counts its kernel nodes per replay)          */
 } e2_stats;
 
 typedef struct e2_ctx e2_ctx;

@@ -98,16 +98,13 @@ __device__ __forceinline__ unsigned long long column_probes(int W)
 // key_bytes bytes.
 size_t dp_smem_bytes(int M, int N, int threads, int key_bytes)
 {
-    const int NW = threads / 32;
     size_t best = 0;
     const int mmax = M < N ? M : N;
     for (int m = 1; m <= mmax; ++m) {
-        const size_t W = (size_t)(N - m + 1);
-        const size_t keys = 3 * (size_t)m * W + (size_t)(2 * NW + 2) * W + 2 * (size_t)m;
-        const size_t bytes = (size_t)m * (3 * sizeof(int)) + keys * key_bytes + (size_t)m * sizeof(uint16_t) + 16;
+        const size_t bytes = dp_item_bytes(m, N, threads / 32, key_bytes);
         if (bytes > best) best = bytes;
     }
-    return (best + 15) & ~(size_t)15;
+    return best;
 }
 
 namespace {
@@ -130,11 +127,13 @@ __host__ __device__ __forceinline__ size_t variant_stride(int mcap) { return ((s
 // first), then by work size (m * W, log scale), largest first.  A replica's
 // smaller batches thus come after every replica's larger ones, by which time
 // the larger batch has usually been decided: a variant below an accepted one
-// is skipped, as the sequential sweep of Alg. 2 would.
+// is skipped, as the sequential sweep of Alg. 2 would.  The items of DP class
+// 0 (size bit 4 clear) take the upper half of the bins, which the descending
+// scan places first; a replica's items all share its class.
 __device__ __forceinline__ int item_bin(int level, int size)
 {
     const int lv = level < 63 ? level : 63;
-    return (63 - lv) * kSizeBins + size;
+    return ((size >> 4) ? 0 : kOrderBins) + (63 - lv) * kSizeBins + (size & (kSizeBins - 1));
 }
 
 // Pre-pass and work count, one warp per (genome, replica slot).  For each
@@ -161,7 +160,8 @@ __device__ __forceinline__ int item_bin(int level, int size)
 // (empty, more devices than blocks, no variant left) gets its outputs here;
 // the others count their work items into the ordering bins.  The last warp to
 // finish (a ticket taken after a fence, no waiting) scans the bins into
-// starting offsets, heaviest first, and stores the item total.
+// starting offsets, class 0 first and heaviest first within a class, and
+// stores the item total and where class 1 starts.
 __global__ void __launch_bounds__(64, 24) slot_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si, EvalOut out,
                                                   unsigned *ctrl)
 {
@@ -276,15 +276,18 @@ __global__ void __launch_bounds__(64, 24) slot_kernel(Dims dm, Tables tb, DevPop
             } else {
                 const int W = N - m + 1;
                 const int lg = (int)(1.0f * __log2f(1.0f + (float)m * (float)W));
-                const int size = lg < kSizeBins - 1 ? lg : kSizeBins - 1;
+                const int cls = dp_item_bytes(m, N, dm.dp_warps, 4) <= dm.dp_small;
+                const int size = (lg < kSizeBins - 1 ? lg : kSizeBins - 1) | cls << 4;
                 si.size[slot] = (uint8_t)size;
                 const int nv = __popcll(mask);
                 for (int lv = 0; lv < nv; ++lv) atomicAdd(&ctrl[item_bin(lv, size)], 1u);
             }
         }
     }
-    // ---- the last warp to finish scans the bins: lane t owns positions
-    //      [32t, 32t + 32) of the descending bin order
+    // ---- the last warp to finish scans the bins: with nb bins in use (class
+    //      1's only where that class exists), lane t owns positions
+    //      [t nb/32, (t+1) nb/32) of the descending bin order (class 0's bins,
+    //      then class 1's), read eight at a time
     unsigned ticket = 0;
     if (lane == 0) {
         __threadfence();
@@ -293,10 +296,16 @@ __global__ void __launch_bounds__(64, 24) slot_kernel(Dims dm, Tables tb, DevPop
     ticket = __shfl_sync(0xFFFFFFFFu, ticket, 0);
     if (ticket != gridDim.x * (blockDim.x >> 5) - 1) return;
     __threadfence();
-    constexpr int kPer = kOrderBins / 32;
-    unsigned *own = ctrl + kOrderBins - 1 - lane * kPer;           // own[-j] = position 32 lane + j
+    const int per = (dm.dp_small ? kAllBins : kOrderBins) / 32;
+    unsigned *own = ctrl + kAllBins - 1 - lane * per;              // own[-j] = position per lane + j
     unsigned sum = 0;
-    for (int j = 0; j < kPer; ++j) sum += __ldcg(own - j);
+    for (int j = 0; j < per; j += 8) {
+        unsigned v[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) v[q] = __ldcg(own - j - q);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) sum += v[q];
+    }
     unsigned incl = sum;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -304,12 +313,24 @@ __global__ void __launch_bounds__(64, 24) slot_kernel(Dims dm, Tables tb, DevPop
         if (lane >= o) incl += x;
     }
     unsigned base = incl - sum;
-    for (int j = 0; j < kPer; ++j) {
-        const unsigned cnt = __ldcg(own - j);
-        own[-j] = base;
-        base += cnt;
+    if (dm.dp_small && lane == kOrderBins / per) {               // class 0 holds the first kOrderBins positions
+        ctrl[kCtrlEnd] = base;
+        ctrl[kCtrlNext + 1] = base;
     }
-    if (lane == 31) ctrl[kCtrlTotal] = base;
+    for (int j = 0; j < per; j += 8) {
+        unsigned v[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) v[q] = __ldcg(own - j - q);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            own[-j - q] = base;
+            base += v[q];
+        }
+    }
+    if (lane == 31) {
+        ctrl[kCtrlEnd + 1] = base;
+        if (!dm.dp_small) ctrl[kCtrlEnd] = ctrl[kCtrlNext + 1] = base;   // one class: class 1 is empty
+    }
 }
 
 // Item lv of a slot (its variants from the largest batch down) goes to bin
@@ -397,7 +418,7 @@ template <> struct HeadRow<uint32_t> {
 // Alg. 1.
 template <typename Key>
 __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, const DevPop &pop, const EvalOut &out,
-                                             const WorkList &wl, const SlotInfo &si, const SplitOut &so)
+                                             const WorkList &wl, const SlotInfo &si, const SplitOut &so, int cls)
 {
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ int s_S0, s_Z, s_mu, s_done;
@@ -410,10 +431,10 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
     const int K = dm.K, M = dm.M, N = dm.N;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
     constexpr Key kInf = (Key)~(Key)0;
-    const unsigned n_items = wl.ctrl[kCtrlTotal];
+    const unsigned n_items = wl.ctrl[kCtrlEnd + cls];         // this class's items end here
   for (;;) {
-    // ---- next work item (heaviest first)
-    if (tid == 0) s_item = atomicAdd(&wl.ctrl[kCtrlNext], 1u);
+    // ---- next work item of the class (heaviest first)
+    if (tid == 0) s_item = atomicAdd(&wl.ctrl[kCtrlNext + cls], 1u);
     __syncthreads();
     const unsigned idx = s_item;
     __syncthreads();
@@ -657,14 +678,16 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
         atomicAdd(&out.stats[kStCells], st_cells);
         atomicAdd(&out.stats[kStProbes], st_probes);
     }
-    if (tid == 0 && st_runs) atomicAdd(&out.stats[kStDpRuns], st_runs);
+    if (tid == 0 && st_runs) atomicAdd(&out.stats[cls ? kStDpRunsSmall : kStDpRuns], st_runs);
   }
 }
 
+// One launch per DP class (cls): the same code over the class's items, with
+// the class's shared-memory allocation.
 __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out, WorkList wl,
-                                                      SlotInfo si, SplitOut so)
+                                                      SlotInfo si, SplitOut so, int cls)
 {
-    dp_eval_body<uint32_t>(dm, tb, pop, out, wl, si, so);
+    dp_eval_body<uint32_t>(dm, tb, pop, out, wl, si, so, cls);
 }
 
 // One warp per genome.  Each replica that had work gets its outputs from its
@@ -926,17 +949,43 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     atomicAdd(&out.stats[kStGenomes], 1ull);
 }
 
+// Persistent grids of the DP.  Shared memory is what limits CTAs per SM when
+// the largest replica's DP is big (many blocks); the replica sizes whose DP
+// fits in half of it then form class 1, launched with that smaller allocation
+// and a grid of as many CTAs as fit, where this raises the CTAs per SM.
 cudaError_t configure_eval(e2_ctx *c)
 {
     const void *kernel = reinterpret_cast<const void *>(dp_eval_kernel);
     cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c->dp_smem);
     if (e != cudaSuccess) return e;
-    int per_sm = 0, sms = 0;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0, per_sm1 = 0, sms = 0;
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, c->dp_threads, c->dp_smem);
     if (e != cudaSuccess) return e;
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
     if (e != cudaSuccess) return e;
-    c->dp_grid = (per_sm > 0 ? per_sm : 1) * (sms > 0 ? sms : 1);
+    if (sms < 1) sms = 1;
+    c->dp_grid = (per_sm > 0 ? per_sm : 1) * sms;
+    const int warps = c->dp_threads / 32, mmax = c->dm.M < c->dm.N ? c->dm.M : c->dm.N;
+    size_t small = 0;
+    for (int m = 1; m <= mmax; ++m) {
+        const size_t b = dp_item_bytes(m, c->dm.N, warps, 4);
+        if (2 * b <= c->dp_smem && b > small) small = b;
+    }
+    c->dm.dp_warps = warps;
+    c->dm.dp_small = 0;
+    c->dp_grid1 = 0;
+    c->dp_smem1 = 0;
+    if (small > 0) {
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm1, kernel, c->dp_threads, small);
+        if (e != cudaSuccess) return e;
+        if (per_sm1 > per_sm) {
+            c->dm.dp_small = (unsigned)small;
+            c->dp_grid1 = per_sm1 * sms;
+            c->dp_smem1 = small;
+        }
+    }
     return cudaSuccess;
 }
 
@@ -962,11 +1011,23 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     if (c->ev_dp_start && (e = cudaStreamIsCapturing(c->stream, &cs)) != cudaSuccess) return e;
     const unsigned rec = cs == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : cudaEventRecordDefault;
     if (c->ev_dp_start && (e = cudaEventRecordWithFlags(c->ev_dp_start, c->stream, rec)) != cudaSuccess) return e;
-    dp_eval_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so);
+    if (c->dp_grid1 > 0) {                       // class 1 beside class 0, on the side stream
+        if ((e = cudaEventRecord(c->ev_dp_fork, c->stream)) != cudaSuccess) return e;
+        if ((e = cudaStreamWaitEvent(c->side, c->ev_dp_fork, 0)) != cudaSuccess) return e;
+    }
+    dp_eval_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so, 0);
+    if (c->dp_grid1 > 0) {
+        dp_eval_kernel<<<(unsigned)c->dp_grid1, c->dp_threads, c->dp_smem1, c->side>>>(c->dm, tb, p, out, wl, si, so,
+                                                                                      1);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        if ((e = cudaEventRecord(c->ev_dp_join, c->side)) != cudaSuccess) return e;
+        if ((e = cudaStreamWaitEvent(c->stream, c->ev_dp_join, 0)) != cudaSuccess) return e;
+    }
     if (c->ev_dp_stop && (e = cudaEventRecordWithFlags(c->ev_dp_stop, c->stream, rec)) != cudaSuccess) return e;
     const unsigned fb = (unsigned)(((size_t)c->dm.P * 32 + 127) / 128);
     if (c->dm.role_search) finalize_roles_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
     else finalize_score_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
+    c->launches += c->dp_grid1 > 0 ? 5 : 4;
     return cudaGetLastError();
 }
 

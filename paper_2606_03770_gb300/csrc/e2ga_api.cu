@@ -299,7 +299,7 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     if (!c) return E2_ENOMEM;
     c->stream = static_cast<cudaStream_t>(stream);
     c->dm = Dims{M, N, b_max + 1, b_max, P, Q, K, l.LS, prm->tournament, prof->NP, prof->ND,
-                 prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps), prm->role_search, 0.0f};
+                 prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps), prm->role_search, 0.0f, 0u, 4};
     {
         const double lm = c->dm.lam_max;                       // rounded up to float
         float f = (float)lm;
@@ -320,6 +320,8 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
         if (c->side) cudaStreamDestroy(c->side);
         if (c->ev_fork) cudaEventDestroy(c->ev_fork);
         if (c->ev_join) cudaEventDestroy(c->ev_join);
+        if (c->ev_dp_fork) cudaEventDestroy(c->ev_dp_fork);
+        if (c->ev_dp_join) cudaEventDestroy(c->ev_dp_join);
         delete c;
         return reject(code, why);
     };
@@ -336,7 +338,9 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     if (configure_eval(c) != cudaSuccess) return fail_free(E2_ECUDA, "configuring the DP kernel failed");
     if (cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking) != cudaSuccess ||
         cudaEventCreateWithFlags(&c->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
-        cudaEventCreateWithFlags(&c->ev_join, cudaEventDisableTiming) != cudaSuccess)
+        cudaEventCreateWithFlags(&c->ev_join, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->ev_dp_fork, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->ev_dp_join, cudaEventDisableTiming) != cudaSuccess)
         return fail_free(E2_ECUDA, "creating the side stream failed");
 
     unsigned char *ws = static_cast<unsigned char *>(workspace);
@@ -426,6 +430,7 @@ cudaError_t record_generation(e2_ctx *c, int b)
     if (!c->cap_stream) e = cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking);
     if (e != cudaSuccess) return e;
     const cudaStream_t user = c->stream;
+    const unsigned long long launched = c->launches;         // recording launches nothing
     c->stream = c->cap_stream;
     e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
     if (e == cudaSuccess) {
@@ -443,6 +448,8 @@ cudaError_t record_generation(e2_ctx *c, int b)
         }
     }
     c->stream = user;
+    c->gen_kernels[b] = c->launches - launched;
+    c->launches = launched;
     if (e == cudaSuccess) e = find_ga_node(c->gen_graph[b], &c->gen_ga_node[b]);
     if (e != cudaSuccess) {
         drop_generation_graph(c, b);
@@ -465,6 +472,8 @@ int e2_destroy(e2_ctx *c)
     if (c->side) cudaStreamDestroy(c->side);
     if (c->ev_fork) cudaEventDestroy(c->ev_fork);
     if (c->ev_join) cudaEventDestroy(c->ev_join);
+    if (c->ev_dp_fork) cudaEventDestroy(c->ev_dp_fork);
+    if (c->ev_dp_join) cudaEventDestroy(c->ev_dp_join);
     delete c;
     return e == cudaSuccess ? E2_OK : E2_ECUDA;
 }
@@ -549,6 +558,7 @@ int e2_run_generation(e2_ctx *c, uint64_t seed, uint32_t generation)
     }
     E2_CUDA(c, set_ga_node(c, c->gen_exec[b], c->gen_ga_node[b], c->pop[b], c->pop[b ^ 1], seed, generation));
     E2_CUDA(c, cudaGraphLaunch(c->gen_exec[b], c->stream));
+    c->launches += c->gen_kernels[b];
     c->have_results = true;
     c->cur ^= 1;
     c->evaluated = false;
@@ -600,13 +610,20 @@ int e2_get_stats(e2_ctx *c, e2_stats *out)
     E2_CUDA(c, cudaStreamSynchronize(c->stream));
     out->genomes = s[kStGenomes];
     out->replicas = s[kStReplicas];
-    out->dp_runs = s[kStDpRuns];
+    out->dp_runs = s[kStDpRuns] + s[kStDpRunsSmall];   // the kernel counts each launch's runs apart
     out->dp_cells = s[kStCells];
     out->dp_probes = s[kStProbes];
     out->paper_candidates = s[kStPaper];
     out->prechecked = s[kStPrecheck];
     out->served = s[kStServed];
     out->tps_pruned = s[kStTpsPruned];
+    out->dp_runs_small = s[kStDpRunsSmall];
+    out->dp_launches = c->dp_grid1 > 0 ? 2 : 1;
+    out->dp_ctas = (uint64_t)c->dp_grid;
+    out->dp_smem = c->dp_smem;
+    out->dp_ctas_small = (uint64_t)c->dp_grid1;
+    out->dp_smem_small = c->dp_smem1;
+    out->launches = c->launches;
     return E2_OK;
 }
 

@@ -38,16 +38,38 @@ struct DevPop {
 constexpr int kMaxReplicaDevices = 256;
 
 // Buckets of the work ordering of the evaluation: 64 levels (the rank of a
-// variant among its replica's variants, largest batch first) x 16 work sizes.
+// variant among its replica's variants, largest batch first) x 16 work sizes,
+// once per shared-memory class of the DP (class 0: every replica size; class
+// 1, where it exists: the sizes whose DP fits in the smaller allocation that
+// lets more CTAs share an SM).
 constexpr int kOrderBins = 1024;
 constexpr int kSizeBins = 16;
-// Control words after the ordering bins: item total, next item of the DP, the
-// pre-pass's CTA ticket.
-enum CtrlWord { kCtrlTotal = kOrderBins, kCtrlNext, kCtrlTicket, kCtrlWords };
+constexpr int kDpClasses = 2;
+constexpr int kAllBins = kDpClasses * kOrderBins;
+// Control words after the ordering bins: where each class's items end (class
+// 1's follow class 0's), each class's DP cursor (starting where its items
+// start), the pre-pass's warp ticket.
+enum CtrlWord { kCtrlEnd = kAllBins, kCtrlNext = kCtrlEnd + kDpClasses, kCtrlTicket = kCtrlNext + kDpClasses,
+                kCtrlWords };
+
+// Shared memory of one DP run on a replica of m devices over N blocks, with
+// `warps` warps per CTA and `key_bytes`-byte order keys: the per-device
+// counters, the cost rows and the prefix and suffix columns ([m][W] each),
+// the per-warp rows, the head row, the empty stage, the link and head keys and
+// the device ids (rounded up to 16 bytes).  No slack: a few bytes more per CTA
+// can cost a CTA per SM (the 80-block model's largest DP, 22,208 B, fits 10
+// per SM; 16 B more fit 9).
+__host__ __device__ __forceinline__ unsigned dp_item_bytes(int m, int N, int warps, int key_bytes)
+{
+    const unsigned W = (unsigned)(N - m + 1);
+    const unsigned keys = 3u * (unsigned)m * W + (unsigned)(2 * warps + 2) * W + 2u * (unsigned)m;
+    const unsigned bytes = (unsigned)m * 12u + keys * (unsigned)key_bytes + (unsigned)m * 2u;
+    return (bytes + 15u) & ~15u;
+}
 
 // Stats slots (unsigned long long, atomically accumulated).
 enum StatSlot { kStGenomes = 0, kStReplicas, kStDpRuns, kStCells, kStProbes, kStPaper, kStPrecheck,
-                kStServed, kStTpsPruned, kNumStats };
+                kStServed, kStTpsPruned, kStDpRunsSmall, kNumStats };
 
 // Everything a kernel needs, passed by value.
 struct Dims {
@@ -59,6 +81,9 @@ struct Dims {
     double lam_max;      // largest latency Lambda with 1.0 / Lambda >= min_tps (see e2_create)
     int role_search;     // 1: both roles per replica, best assignment per genome (Alg. 2)
     float lam_max_up;    // lam_max rounded up to float (the float latency bound is compared with it)
+    unsigned dp_small;   // shared-memory bytes of DP class 1 (0: one class); m is in class 1 iff
+                         // dp_item_bytes(m, N, dp_warps, 4) <= dp_small
+    int dp_warps;        // warps per DP CTA
 };
 
 struct Tables {
@@ -78,14 +103,14 @@ struct Tables {
 struct SlotInfo {
     int32_t *off;              // [P*K] offset of the replica in the ordering chromosome
     uint64_t *mask;            // [P*K] variants to run (bit i: prefill v=0 / decode v=i+1)
-    uint8_t *size;             // [P*K] log-scale work size of one DP run of the slot
+    uint8_t *size;             // [P*K] log-scale work size of one DP run of the slot | DP class << 4
     int32_t *best;             // [P*K] largest variant bit accepted so far (-1: none)
 };
 
 // Work items of the DP: (slot << 8) | role << 7 | sweep << 6 | variant bit.
 struct WorkList {
     uint64_t *items;           // [P*K*(b_max+1)] (slot << 8) | role << 7 | sweep << 6 | variant bit
-    unsigned *ctrl;            // [kOrderBins] bins/cursors, then the CtrlWord words
+    unsigned *ctrl;            // [kAllBins] bins/cursors, then the CtrlWord words
 };
 
 // Results of the DP runs, per (slot, variant bit).
@@ -197,7 +222,12 @@ struct e2_ctx {
     double *split_T = nullptr, *split_L = nullptr;   // [P*K*b_max]
     int16_t *split_mu = nullptr;                     // [P*K*b_max]
     int16_t *split_layers = nullptr;                 // [P*b_max*M]
-    int dp_grid = 0;                  // persistent DP CTAs
+    mutable unsigned long long launches = 0;   // kernels launched (a graph replay adds its kernel nodes)
+    unsigned long long gen_kernels[2] = {0, 0}; // kernel nodes of each recorded generation
+    int dp_grid = 0;                  // persistent DP CTAs of class 0
+    int dp_grid1 = 0;                 // persistent DP CTAs of class 1 (0: one class)
+    size_t dp_smem1 = 0;              // their shared memory
+    cudaEvent_t ev_dp_fork = nullptr, ev_dp_join = nullptr;   // class 1 runs on the side stream
     cudaEvent_t ev_dp_start = nullptr, ev_dp_stop = nullptr;   // optional timing hook
     // recorded generation (e2_run_generation), one per population buffer
     cudaStream_t cap_stream = nullptr;                          // private stream the graphs are recorded on

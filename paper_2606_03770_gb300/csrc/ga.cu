@@ -461,6 +461,7 @@ cudaError_t launch_tables(const e2_ctx *c)
     tables_kernel<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm, c->rate, c->bw, c->mem, c->prof, c->leaf);
     const size_t vm = (size_t)c->dm.V * c->dm.M;
     captab_kernel<<<grid_for(vm, 256), 256, 0, c->stream>>>(c->dm, c->rate, c->bw, c->mem, c->prof, c->cap, c->cpb);
+    c->launches += 2;
     return cudaGetLastError();
 }
 
@@ -468,6 +469,7 @@ cudaError_t launch_tau(const e2_ctx *c)
 {
     const size_t total = (size_t)c->dm.V * c->dm.M * c->dm.M;
     tau_kernel<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm, c->link_bw, c->cong, c->prof, c->tau, c->tau_lb);
+    ++c->launches;
     return cudaGetLastError();
 }
 
@@ -475,18 +477,21 @@ cudaError_t launch_redraw(const e2_ctx *c, uint64_t seed, uint32_t gen)
 {
     const size_t total = (size_t)c->dm.M * c->dm.M;
     redraw_kernel<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm.M, seed, gen, c->cong_lo, c->cong_hi, c->cong);
+    ++c->launches;
     return cudaGetLastError();
 }
 
 cudaError_t launch_validate(const e2_ctx *c, const DevPop &p)
 {
     validate_kernel<<<(c->dm.P + 127) / 128, 128, 0, c->stream>>>(c->dm, p, c->err);
+    ++c->launches;
     return cudaGetLastError();
 }
 
 cudaError_t launch_init(const e2_ctx *c, const DevPop &p, uint64_t seed)
 {
     init_kernel<<<(c->dm.P + 31) / 32, 32, 0, c->stream>>>(c->dm, p, seed);
+    ++c->launches;
     return cudaGetLastError();
 }
 
@@ -497,6 +502,7 @@ cudaError_t launch_elites(const e2_ctx *c, const DevPop &p, const DevPop &dst)
     dup_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, p, c->fit, c->hash, c->dup);
     if (c->dm.Q > 0)
         rank_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, c->fit, c->dup, c->elite, c->elite_fit, p, dst);
+    c->launches += c->dm.Q > 0 ? 2 : 1;
     return cudaGetLastError();
 }
 
@@ -516,6 +522,7 @@ cudaError_t launch_ga(const e2_ctx *c, const DevPop &src, const DevPop &dst, uin
     const long long blocks = ((long long)(c->dm.P - c->dm.Q) + nw - 1) / nw;
     ga_kernel<<<(unsigned)(blocks < 152 * 64 ? blocks : 152 * 64), 32 * nw, (size_t)nw * per_warp, st>>>(
         c->dm, src, dst, c->fit, seed, gen, thr);
+    ++c->launches;
     return cudaGetLastError();
 }
 

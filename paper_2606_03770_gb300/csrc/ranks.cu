@@ -158,14 +158,19 @@ inline unsigned grid_for(size_t n, int threads, size_t cap = 152 * 32)
     return (unsigned)(b ? b : 1);
 }
 
-cudaError_t bitonic_sort(uint64_t *data, size_t n_pow2, int arrays, cudaStream_t st)
+// Adds its launches to *launches.
+cudaError_t bitonic_sort(uint64_t *data, size_t n_pow2, int arrays, cudaStream_t st, unsigned long long *launches)
 {
     // n_pow2 >= kLocal, a power of two
     bitonic_local<<<dim3((unsigned)(n_pow2 / kLocal), arrays), 1024, 0, st>>>(data, n_pow2, 2, kLocal);
+    ++*launches;
     for (size_t k = 2 * kLocal; k <= n_pow2; k <<= 1) {
-        for (size_t j = k >> 1; j >= (size_t)kLocal; j >>= 1)
+        for (size_t j = k >> 1; j >= (size_t)kLocal; j >>= 1) {
             bitonic_global<<<dim3(grid_for(n_pow2 / 2, 256), arrays), 256, 0, st>>>(data, n_pow2, n_pow2, k, j);
+            ++*launches;
+        }
         bitonic_local<<<dim3((unsigned)(n_pow2 / kLocal), arrays), 1024, 0, st>>>(data, n_pow2, k, k);
+        ++*launches;
     }
     return cudaGetLastError();
 }
@@ -183,14 +188,16 @@ cudaError_t build_leaf_sorted(const e2_ctx *c)
 {
     const size_t cap = rank_pow2((size_t)c->dm.M * 2 * c->dm.N);
     leaf_keys<<<grid_for((size_t)c->dm.V * cap, 256), 256, 0, c->stream>>>(c->dm, c->leaf, c->leaf_sorted, cap);
-    return bitonic_sort(c->leaf_sorted, cap, c->dm.V, c->stream);
+    ++c->launches;
+    return bitonic_sort(c->leaf_sorted, cap, c->dm.V, c->stream, &c->launches);
 }
 
 cudaError_t build_ranks(const e2_ctx *c)
 {
     const size_t MM = (size_t)c->dm.M * c->dm.M, bcap = rank_pow2(MM);
     beff_keys<<<grid_for(bcap, 256), 256, 0, c->stream>>>(c->dm.M, c->link_bw, c->cong, c->beff_sorted, bcap);
-    cudaError_t e = bitonic_sort(c->beff_sorted, bcap, 1, c->stream);
+    ++c->launches;
+    cudaError_t e = bitonic_sort(c->beff_sorted, bcap, 1, c->stream, &c->launches);
     if (e != cudaSuccess) return e;
     tau_sorted_kernel<<<grid_for((size_t)c->dm.V * MM, 256), 256, 0, c->stream>>>(c->dm, c->beff_sorted, c->prof,
                                                                                 c->tau_sorted);
@@ -198,6 +205,7 @@ cudaError_t build_ranks(const e2_ctx *c)
     const size_t total = (size_t)c->dm.V * c->dm.M * 2 * c->dm.LS + (size_t)c->dm.V * MM;
     rank_kernel_tables<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm, c->leaf, c->tau, c->leaf_sorted, leaf_cap,
                                                                     c->tau_sorted, c->leaf_rank, c->tau_rank);
+    c->launches += 2;
     return cudaGetLastError();
 }
 

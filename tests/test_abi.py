@@ -36,6 +36,32 @@ def test_exports_every_declared_symbol(lib):
     assert set(e2ga.SIGNATURES) == set(names)
 
 
+def declared_struct_fields(name):
+    src = open(os.path.join(ROOT, "include", "e2ga.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    body = re.search(r"typedef struct \{([^}]*)\}\s*" + name + r"\s*;", src).group(1)
+    return [(t, n) for t, n in re.findall(r"(\w+)\s*\*?\s*(\w+)\s*;", body)]
+
+
+@pytest.mark.parametrize("name", ["e2_params", "e2_stats", "e2_genomes", "e2_partitions"])
+def test_binding_structs_follow_the_header(name):
+    """The ctypes mirrors of the header's structs: same fields in the same
+    order, with the same widths."""
+    from paper_2606_03770_gb300 import e2ga
+    widths = {"int32_t": 4, "uint32_t": 4, "int": 4, "uint64_t": 8, "int64_t": 8, "double": 8, "float": 4}
+    decl = declared_struct_fields(name)
+    mine = getattr(e2ga, name)._fields_
+    assert len(decl) == len(mine), (decl, mine)
+    src = open(os.path.join(ROOT, "include", "e2ga.h")).read()
+    for (t, n), (pn, pt) in zip(decl, mine):
+        assert pn.rstrip("_") == n, (n, pn)
+        pointer = re.search(r"\b" + t + r"\s*\*\s*" + n + r"\s*;", src) is not None
+        if pointer:
+            assert pt is C.c_void_p or issubclass(pt, C._Pointer), (n, pt)
+        else:
+            assert C.sizeof(pt) == widths[t], (n, t, pt)
+
+
 def test_workspace_bytes(lib):
     from paper_2606_03770_gb300 import e2ga
     for name in ("c1_tiny", "c2", "c4"):

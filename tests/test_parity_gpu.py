@@ -74,6 +74,15 @@ def test_eval_parity_full_size_sampled(name, P, sample):
     idx = np.sort(np.random.default_rng(5).choice(P, sample, replace=False))
     ora = O.OracleProblem(prob).eval_population(take(g, idx), prob.K_max, nthreads=O.num_threads())
     assert_eval_equal(gpu, ora, rows=idx)
+    # the 126-block model's largest DP leaves room for 4 CTAs per SM: the
+    # replica sizes that need half of it run in a second launch with more
+    st = eng.stats()
+    assert st["dp_launches"] == (2 if st["dp_ctas_small"] else 1)
+    assert st["dp_runs_small"] < st["dp_runs"]
+    assert (st["dp_runs_small"] > 0) == (st["dp_launches"] == 2), st
+    if name == "c4":
+        assert st["dp_launches"] == 2 and st["dp_ctas_small"] >= 2 * st["dp_ctas"], st
+        assert 2 * st["dp_smem_small"] <= st["dp_smem"], st
     eng.close()
 
 
@@ -293,7 +302,7 @@ def test_min_tps_boundary_exact():
     assert served[0] == ora["bsel"][p, c] and served[1] != served[0]
 
 
-@pytest.mark.parametrize("name,P,gens", [("c1_tiny", 64, 5), ("c2", 1024, 5)])
+@pytest.mark.parametrize("name,P,gens", [("c1_tiny", 64, 5), ("c2", 1024, 5), ("c4", 1024, 4)])
 def test_recorded_generation_matches_separate_calls(name, P, gens):
     """e2_run_generation (one recorded graph per population buffer) gives the
     populations and fitness of e2_eval_population + e2_ga_step, also when
@@ -307,6 +316,7 @@ def test_recorded_generation_matches_separate_calls(name, P, gens):
     for e in (x, y):
         e.record(torch.cuda.current_stream())
     for gen in range(1, gens + 1):
+        la, lb = a.stats()["launches"], b.stats()["launches"]
         a.eval(parts=False)
         fa = a.results()["fitness"]
         a.ga_step(5, gen)
@@ -321,6 +331,9 @@ def test_recorded_generation_matches_separate_calls(name, P, gens):
             fb = b.results()["fitness"]
         assert np.array_equal(fa, fb), gen
         assert_genomes_equal(a.get_population(), b.get_population())
+        # a replay counts the recorded kernel nodes: as many as the separate calls launch
+        sa, sb = a.stats(), b.stats()
+        assert sa["launches"] - la == sb["launches"] - lb == 6 + sa["dp_launches"], gen
     torch.cuda.synchronize()
     assert x.elapsed_time(y) > 0
     b.set_timing_events()
@@ -406,7 +419,13 @@ def test_eval_parity_maximum_sizes(case):
     gpu = eng.results()
     ora = O.OracleProblem(prob).eval_population(g, K, nthreads=O.num_threads())
     assert_eval_equal(gpu, ora)
-    assert eng.stats()["paper_candidates"] == ora["cand"]
+    st = eng.stats()
+    assert st["paper_candidates"] == ora["cand"]
+    if case != "wide rows":
+        # replicas of 6, 250 and 256 devices (W <= 255 with few devices, or a
+        # short row) need less than half the shared memory of the 56- and
+        # 200-device ones: they run in the second DP launch
+        assert st["dp_launches"] == 2 and 0 < st["dp_runs_small"] <= st["dp_runs"], st
     assert np.isfinite(ora["T"]).any()
     ga = O.ga_of(prob)
     eidx = O.elites(ga, g, ora["fitness"])
