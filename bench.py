@@ -372,6 +372,8 @@ def run_ours(args):
             "paper_candidates_per_s": paper * args.steps * world / t_max,
             "dp_kernel_ms_per_step": 1e3 * dp_s,
             "served_replicas_per_step": sum(s["served"] for s in stats) / args.steps,
+            "prepass_per_step": {"memory_rejected": sum(s["prechecked"] for s in stats) / args.steps,
+                                 "latency_rejected": sum(s["tps_pruned"] for s in stats) / args.steps},
             "dp_launches": {"ctas": [stats[-1]["dp_ctas"], stats[-1]["dp_ctas_small"]],
                             "smem_bytes": [stats[-1]["dp_smem"], stats[-1]["dp_smem_small"]],
                             "runs": [sum(s["dp_runs"] - s["dp_runs_small"] for s in stats) / args.steps,

@@ -152,17 +152,22 @@ __device__ __forceinline__ int item_bin(int level, int size)
 // Both tests are monotone in the batch: the capacities shrink as b grows (more
 // KV memory per block), and the bound is the least of a linear cost whose
 // coefficients (per-block and link times) grow with b over a feasible set that
-// shrinks with b.  So the variants are tested from the largest batch down and
-// the first that passes keeps every smaller batch as well (rounding could at
-// most keep a variant the bound would have dropped, which costs a DP run and
-// changes no result).
+// shrinks with b, when the profile's costs grow with the batch (physical
+// profiles do; checked at e2_create).  So the largest batch the memory allows
+// is found by a search (the largest batch first, then the smallest, then
+// bisection), and the largest the bound keeps by a second search below it;
+// every smaller batch is kept.  A failed test is exact (memory) or a proof
+// (the bound never exceeds the exact value), so every batch above it fails
+// too; rounding can only keep a variant the exact bound would drop, which
+// costs a DP run and changes no result.  Other profiles test every batch from
+// the largest down, and the first that passes keeps the smaller ones.
 // The surviving variants form the slot's mask.  A slot with nothing to run
 // (empty, more devices than blocks, no variant left) gets its outputs here;
 // the others count their work items into the ordering bins.  The last warp to
 // finish (a ticket taken after a fence, no waiting) scans the bins into
 // starting offsets, class 0 first and heaviest first within a class, and
 // stores the item total and where class 1 starts.
-__global__ void __launch_bounds__(64, 24) slot_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si, EvalOut out,
+__global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si, EvalOut out,
                                                   unsigned *ctrl)
 {
     // per warp: device ids, capacities and per-block times of up to mcap devices
@@ -196,16 +201,15 @@ __global__ void __launch_bounds__(64, 24) slot_kernel(Dims dm, Tables tb, DevPop
             // with the role search, the decode sweep and then the prefill variant
             // (its result goes to bit b_max); otherwise the genome's role only
             const int npass = dm.role_search ? 2 : 1;
-            for (int pass = 0; pass < npass; ++pass) {
-            const int prole = dm.role_search ? (pass == 0) : role;
-            const int nvar = prole ? dm.b_max : 1;
-            for (int i = nvar - 1; i >= 0; --i) {                 // largest batch first
+            // Stage variant i (capacities, and the per-block and link times
+            // when the latency bound applies) and return its memory verdict.
+            auto stage = [&](int prole, int i, bool bound) -> bool {
                 const int v = prole ? i + 1 : 0;
                 const int32_t *cap = tb.cap + (size_t)v * M * 2;
-                const bool bound = prole && dm.min_tps > 0.0;
                 const float *cpb = tb.cpb + (size_t)v * M;
                 const float *tau = tb.tau_lb + (size_t)v * M * M;
                 int s0 = 0, z = 0;
+                __syncwarp();
                 for (int k = lane; k < m; k += 32) {                   // every load of the variant at once
                     const int d = sdev[k];
                     const int c0 = min(cap[d * 2], W), c1 = min(cap[d * 2 + 1], W);
@@ -224,37 +228,69 @@ __global__ void __launch_bounds__(64, 24) slot_kernel(Dims dm, Tables tb, DevPop
                 bool ok = false;
                 for (int k = lane; k < m && !ok; k += 32)
                     ok = (z - (sc0[k] == 0)) == 0 && sc1[k] >= 1 && s0 - sc0[k] + sc1[k] >= N;
-                if (!__any_sync(0xFFFFFFFFu, ok)) {
-                    ++n_pre;
-                    continue;
-                }
-                if (bound) {
-                    float part = 0.0f;
-                    for (int k = lane; k < m; k += 32) {
-                        const uint32_t ck = scb[k];
-                        int before = 0;                  // capacity of the cheaper devices
-                        for (int j = 0; j < m; ++j) {
-                            const uint32_t cj = scb[j];
-                            if (cj < ck || (cj == ck && j < k)) before += sc0[j] - 1;
-                        }
-                        const int ek = sc0[k] - 1;
-                        const int room = (N - m) - before;
-                        const int take = room <= 0 ? 0 : (room < ek ? room : ek);
-                        part = __fadd_rd(part, __fmul_rd(__uint_as_float(ck), (float)(1 + take)));
-                        if (k >= 1) part = __fadd_rd(part, stau[k]);
+                return __any_sync(0xFFFFFFFFu, ok);
+            };
+            // The latency bound of the staged variant, against Lambda_max.
+            auto fast_enough = [&]() -> bool {
+                float part = 0.0f;
+                for (int k = lane; k < m; k += 32) {
+                    const uint32_t ck = scb[k];
+                    int before = 0;                  // capacity of the cheaper devices
+                    for (int j = 0; j < m; ++j) {
+                        const uint32_t cj = scb[j];
+                        if (cj < ck || (cj == ck && j < k)) before += sc0[j] - 1;
                     }
+                    const int ek = sc0[k] - 1;
+                    const int room = (N - m) - before;
+                    const int take = room <= 0 ? 0 : (room < ek ? room : ek);
+                    part = __fadd_rd(part, __fmul_rd(__uint_as_float(ck), (float)(1 + take)));
+                    if (k >= 1) part = __fadd_rd(part, stau[k]);
+                }
 #pragma unroll
-                    for (int o = 16; o; o >>= 1) part = __fadd_rd(part, __shfl_xor_sync(0xFFFFFFFFu, part, o));
-                    __syncwarp();
-                    if (part > dm.lam_max_up) {                        // 1.0 / Lambda < Min_TPS
-                        ++n_tps;
+                for (int o = 16; o; o >>= 1) part = __fadd_rd(part, __shfl_xor_sync(0xFFFFFFFFu, part, o));
+                return !(part > dm.lam_max_up);                         // 1.0 / Lambda >= Min_TPS possible
+            };
+            for (int pass = 0; pass < npass; ++pass) {
+                const int prole = dm.role_search ? (pass == 0) : role;
+                const int nvar = prole ? dm.b_max : 1;
+                const bool bound = prole && dm.min_tps > 0.0;
+                // When the costs grow with the batch both verdicts are monotone,
+                // so each is found by a search over the variants: the largest
+                // first (it usually decides), then the smallest, then bisection
+                // between the largest known pass (lo) and the smallest known
+                // failure (hi).  The memory search comes first; the bound then
+                // searches the variants the memory allows.  Otherwise each
+                // variant is tested from the largest down, and the first that
+                // passes both keeps the smaller ones.
+                int lo = -1, hi = nvar, next = nvar - 1, staged = -1, bm = -1;
+                bool tps = false;
+                while (hi - lo > 1) {
+                    bool pass = true;
+                    if (staged != next) {
+                        pass = stage(prole, next, bound);
+                        staged = next;
+                    }
+                    if (tps && pass) pass = fast_enough();
+                    if (pass) lo = next;
+                    else hi = next;
+                    if (!tps && hi - lo <= 1) {                 // the memory search is done
+                        bm = lo;
+                        if (!bound || bm < 0) break;
+                        tps = true;
+                        lo = -1;
+                        hi = bm + 1;
+                        next = bm;
                         continue;
                     }
+                    next = !dm.grows ? hi - 1 : lo < 0 ? 0 : (lo + hi) >> 1;
                 }
-                if (dm.role_search && !prole) mask |= 1ull << dm.b_max;
-                else mask |= (2ull << i) - 1ull;   // this variant and every smaller batch
-                break;
-            }
+                const int bs = tps ? lo : bm;               // largest variant both tests keep
+                n_pre += (unsigned long long)(nvar - 1 - bm);
+                n_tps += (unsigned long long)(bm - bs);
+                if (bs >= 0) {
+                    if (dm.role_search && !prole) mask |= 1ull << dm.b_max;
+                    else mask |= (2ull << bs) - 1ull;       // this variant and every smaller batch
+                }
             }
         }
         // ---- the slot's outputs or its work count

@@ -250,6 +250,20 @@ size_t e2_workspace_bytes(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_
     return layout(M, N, b_max, P, Q, K_max).total;
 }
 
+// Whether the decode variants' costs never shrink as the batch grows: block
+// and head memory (so capacities never grow), block flops and bytes (per-block
+// times) and activation bytes (link times), over v = 1..b_max.  Physical
+// profiles do; the evaluation pre-pass then searches its monotone tests
+// instead of testing every batch.
+static int costs_grow_with_batch(const e2_layer_profile *prof, int b_max)
+{
+    const uint64_t *rows[] = {prof->blk_mem, prof->head_mem, prof->blk_flops, prof->blk_bytes, prof->act_bytes};
+    for (const uint64_t *r : rows)
+        for (int v = 1; v < b_max; ++v)
+            if (r[v + 1] < r[v]) return 0;
+    return 1;
+}
+
 // The decode test of Alg. 2 keeps batch b when 1.0 / Lambda_b >= Min_TPS,
 // the quotient rounded to nearest.  Correctly rounded division is monotone, so
 // for Lambda >= 0 the test holds exactly when Lambda <= Lambda_max, the largest
@@ -299,7 +313,8 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     if (!c) return E2_ENOMEM;
     c->stream = static_cast<cudaStream_t>(stream);
     c->dm = Dims{M, N, b_max + 1, b_max, P, Q, K, l.LS, prm->tournament, prof->NP, prof->ND,
-                 prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps), prm->role_search, 0.0f, 0u, 4};
+                 prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps), prm->role_search, 0.0f, 0u, 4,
+                 costs_grow_with_batch(prof, b_max)};
     {
         const double lm = c->dm.lam_max;                       // rounded up to float
         float f = (float)lm;

@@ -84,6 +84,8 @@ struct Dims {
     unsigned dp_small;   // shared-memory bytes of DP class 1 (0: one class); m is in class 1 iff
                          // dp_item_bytes(m, N, dp_warps, 4) <= dp_small
     int dp_warps;        // warps per DP CTA
+    int grows;           // 1: block memory, head memory, block flops and bytes and activation bytes never
+                         // shrink from one decode batch to the next (the pre-pass tests are then monotone)
 };
 
 struct Tables {

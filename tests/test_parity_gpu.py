@@ -189,6 +189,34 @@ def test_eval_parity_edge_cases(case):
     eng.close()
 
 
+@pytest.mark.parametrize("case", range(6))
+def test_eval_parity_costs_growing_with_batch(case):
+    """The small-integer edge problems with each decode cost row sorted, so
+    that costs grow with the batch (ties between batches included): the
+    pre-pass then searches its monotone memory and latency tests instead of
+    testing every batch, with exact ties and memory walls at every step."""
+    rng = np.random.default_rng(2000 + case)
+    M, N, K, P = [(6, 5, 3, 40), (12, 12, 4, 129), (7, 30, 7, 255), (16, 9, 16, 300), (8, 8, 8, 513),
+                  (33, 64, 33, 70)][case]
+    prob = _edge_problem(rng, M, N, P, K, integer=case % 3 != 2, Q=3, min_tps=0.05 * (case % 4 + 1))
+    for f in ("blk_flops", "blk_bytes", "blk_mem", "head_flops", "head_bytes", "head_mem", "act_bytes"):
+        row = np.asarray(getattr(prob, f)).copy()       # prefill, then 8 decode batches drawn from the rows
+        row = np.concatenate([row[:1], rng.choice(row[1:], 8)])
+        row[1:] = np.sort(row[1:])
+        setattr(prob, f, row)
+    assert prob.b_max == 8
+    g = W.random_genomes(M, K, P, seed=case)
+    eng = engine(prob)
+    eng.eval(g)
+    gpu = eng.results()
+    ora = O.OracleProblem(prob).eval_population(g, K, nthreads=O.num_threads())
+    assert_eval_equal(gpu, ora)
+    st = eng.stats()
+    assert st["paper_candidates"] == ora["cand"]
+    assert st["served"] == int((ora["bsel"] >= 0).sum())
+    eng.close()
+
+
 def test_elites_with_duplicates_and_Q_extremes():
     prob = W.make_config("c1_tiny", P=96)
     g = W.random_genomes(prob.M, prob.K_max, 96, seed=4)
