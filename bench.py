@@ -10,9 +10,9 @@ workload is the 32-device fleet / 80-block model / 8-replica / population
 
 value: genome evaluations per second over the timed steps, device time with
 CUDA events on the engine's stream, L2 flushed (256 MB write) between steps.
-e2e: the same metric through the C ABI with pinned host buffers: each step
-uploads the population, evaluates, steps, and reads fitness and the next
-population back.  --impl reference times the CPU oracle on the host cores.
+e2e: the same metric through the C ABI with pinned host buffers: each step is
+one e2_run_generation_io call that uploads the population, evaluates, steps,
+and reads fitness and the next population back, synchronising once.  --impl reference times the CPU oracle on the host cores.
 Under torchrun each rank runs an independent replica search (its own seed) on
 its own GPU; value is the sum over ranks divided by the slowest rank's time.
 """
@@ -329,21 +329,24 @@ def run_ours(args):
     e2e = None
     if not args.no_e2e:
         P, M, K = prob.P, prob.M, prob.K_max
-        host = dict(perm=torch.empty((P, M), dtype=torch.int16).pin_memory(),
-                    sizes=torch.empty((P, K), dtype=torch.int16).pin_memory(),
-                    nclus=torch.empty(P, dtype=torch.uint8).pin_memory(),
-                    roles=torch.empty(P, dtype=torch.int64).pin_memory())
+        def pinned_population():
+            return dict(perm=torch.empty((P, M), dtype=torch.int16).pin_memory(),
+                        sizes=torch.empty((P, K), dtype=torch.int16).pin_memory(),
+                        nclus=torch.empty(P, dtype=torch.uint8).pin_memory(),
+                        roles=torch.empty(P, dtype=torch.int64).pin_memory())
+        host = [pinned_population(), pinned_population()]
         hfit = torch.empty((P, 4), dtype=torch.float64).pin_memory()
-        eng.get_population(host)
+        eng.get_population(host[0])
         bytes_pop = P * (2 * M + 2 * K + 1 + 8)
 
         def e2e_step(g):
+            # the population in from the host (validated on the device), one
+            # generation, its fitness and the next population back to the host:
+            # one call, one synchronisation
             if prob.redraw:
                 eng.redraw_congestion(seed, g)
-            eng.set_population(host)                 # host -> device, validated
-            eng.eval(fitness=hfit, parts=False)      # fitness -> host
-            eng.ga_step(seed, g)
-            eng.get_population(host)                 # next population -> host
+            eng.run_generation_io(seed, g, population=host[0], fitness=hfit, next_out=host[1])
+            host.reverse()
 
         for _ in range(args.warmup):
             gen += 1
@@ -356,7 +359,8 @@ def run_ours(args):
         sync_all()
         te = max_over_ranks(time.perf_counter() - t0, world, "cuda")
         e2e = {"value": replica_throughput(P * args.steps, world, te), "unit": UNIT,
-               "h2d_bytes_per_step": bytes_pop, "d2h_bytes_per_step": bytes_pop + 32 * P}
+               "h2d_bytes_per_step": bytes_pop, "d2h_bytes_per_step": bytes_pop + 32 * P + 4,
+               "call": "e2_run_generation_io (population in, fitness and next population out)"}
 
     if rank == 0:
         line = {

@@ -204,7 +204,9 @@ int e2_destroy(e2_ctx *ctx);
 /* Copy a population (host or device pointers) into the context's current
  * population and validate it (each ordering a permutation, 1 <= R <= K_max,
  * sizes >= 1 summing to M, zero sizes beyond R, no role bits at or above R).
- * Synchronises.  E2_EINVAL names the first bad genome via e2_last_error. */
+ * Synchronises.  E2_EINVAL names the first bad genome via e2_last_error; every
+ * invalid genome is then replaced by the identity ordering as one prefill
+ * replica, so that the context never holds an invalid population. */
 int e2_set_population(e2_ctx *ctx, const e2_genomes *g);
 
 /* Copy the context's current population out (host or device pointers). */
@@ -263,6 +265,22 @@ int e2_get_results(e2_ctx *ctx, double *fitness_out, const e2_partitions *parts)
  * issued one by one.
  * E2_EINVAL for a NULL context; E2_ECUDA on a CUDA failure. */
 int e2_run_generation(e2_ctx *ctx, uint64_t seed, uint32_t generation);
+
+/* One generation with the host in the loop, synchronising once (no
+ * counterpart in the paper; the host-driven form of Alg. 2's loop).  If
+ * `population` is not NULL it replaces the current population (host or device
+ * arrays, validated on the device like e2_set_population, without a separate
+ * synchronisation).  Then the work of e2_run_generation(ctx, seed,
+ * generation); then, where not NULL, the evaluated population's fitness
+ * [P][4] goes to fitness_out and the next population to next_out (host or
+ * device).  Synchronises when `population` is given or a destination is host
+ * memory.  E2_EINVAL when `population` holds an invalid genome (the smallest
+ * such index in e2_last_error): the generation ran with each invalid genome
+ * replaced by the identity ordering as one prefill replica, so the outputs
+ * are of that population and the context stays usable.  E2_EINVAL also for a
+ * NULL context or a NULL array in next_out; E2_ECUDA on a CUDA failure. */
+int e2_run_generation_io(e2_ctx *ctx, const e2_genomes *population, uint64_t seed, uint32_t generation,
+                         double *fitness_out, const e2_genomes *next_out);
 
 /* Counters of the last evaluation.  Synchronises. */
 int e2_get_stats(e2_ctx *ctx, e2_stats *out);

@@ -221,23 +221,38 @@ int copy_pop(e2_ctx *c, const DevPop &dst, const e2_genomes *g, bool out)
     return E2_OK;
 }
 
-int set_and_validate(e2_ctx *c, const e2_genomes *g)
+// Copy a population into the current buffer and validate it on the device
+// (invalid genomes are replaced there by a valid one); the smallest invalid
+// index lands in the error word, read back by check_validated.
+constexpr int32_t kNoBadGenome = 0x7F7F7F7F;   // the error word's bytes all 0x7F
+
+int upload_and_validate(e2_ctx *c, const e2_genomes *g)
 {
     int st = copy_pop(c, c->pop[c->cur], g, false);
     if (st) return st;
-    const int32_t big = 0x7FFFFFFF;
-    E2_CUDA(c, cudaMemcpyAsync(c->err, &big, 4, cudaMemcpyHostToDevice, c->stream));
+    E2_CUDA(c, cudaMemsetAsync(c->err, 0x7F, 4, c->stream));
     E2_CUDA(c, launch_validate(c, c->pop[c->cur]));
-    int32_t bad = big;
+    c->evaluated = false;
+    return E2_OK;
+}
+
+int check_validated(e2_ctx *c, int32_t bad)
+{
+    if (bad == kNoBadGenome) return E2_OK;
+    char buf[160];
+    snprintf(buf, sizeof buf, "genome %d is not a valid gene (ordering, grouping or roles); replaced by the identity "
+             "ordering as one replica", bad);
+    return fail(c, E2_EINVAL, buf);
+}
+
+int set_and_validate(e2_ctx *c, const e2_genomes *g)
+{
+    int st = upload_and_validate(c, g);
+    if (st) return st;
+    int32_t bad = kNoBadGenome;
     E2_CUDA(c, cudaMemcpyAsync(&bad, c->err, 4, cudaMemcpyDeviceToHost, c->stream));
     E2_CUDA(c, cudaStreamSynchronize(c->stream));
-    c->evaluated = false;
-    if (bad != big) {
-        char buf[128];
-        snprintf(buf, sizeof buf, "genome %d is not a valid gene (ordering, grouping or roles)", bad);
-        return fail(c, E2_EINVAL, buf);
-    }
-    return E2_OK;
+    return check_validated(c, bad);
 }
 
 }  // namespace
@@ -579,6 +594,37 @@ int e2_run_generation(e2_ctx *c, uint64_t seed, uint32_t generation)
     c->evaluated = false;
     c->have_elites = true;
     return E2_OK;
+}
+
+int e2_run_generation_io(e2_ctx *c, const e2_genomes *population, uint64_t seed, uint32_t generation,
+                         double *fitness_out, const e2_genomes *next_out)
+{
+    if (!c) return E2_EINVAL;
+    if (next_out && (!next_out->perm || !next_out->sizes || !next_out->nclus || !next_out->roles))
+        return fail(c, E2_EINVAL, "null genome array");
+    if (population) {
+        const int st = upload_and_validate(c, population);
+        if (st) return st;
+    }
+    const int st = e2_run_generation(c, seed, generation);
+    if (st) return st;
+    const size_t P = c->dm.P, M = c->dm.M, K = c->dm.K;
+    const DevPop &nx = c->pop[c->cur];
+    const cudaMemcpyKind k = cudaMemcpyDefault;
+    if (fitness_out) E2_CUDA(c, cudaMemcpyAsync(fitness_out, c->fit, 32 * P, k, c->stream));
+    if (next_out) {
+        E2_CUDA(c, cudaMemcpyAsync(next_out->perm, nx.perm, 2 * P * M, k, c->stream));
+        E2_CUDA(c, cudaMemcpyAsync(next_out->sizes, nx.sizes, 2 * P * K, k, c->stream));
+        E2_CUDA(c, cudaMemcpyAsync(next_out->nclus, nx.nclus, P, k, c->stream));
+        E2_CUDA(c, cudaMemcpyAsync(next_out->roles, nx.roles, 8 * P, k, c->stream));
+    }
+    int32_t bad = kNoBadGenome;
+    if (population) E2_CUDA(c, cudaMemcpyAsync(&bad, c->err, 4, cudaMemcpyDeviceToHost, c->stream));
+    const bool host = population || (fitness_out && is_host(fitness_out)) ||
+                      (next_out && (is_host(next_out->perm) || is_host(next_out->sizes) ||
+                                    is_host(next_out->nclus) || is_host(next_out->roles)));
+    if (host) E2_CUDA(c, cudaStreamSynchronize(c->stream));
+    return check_validated(c, bad);
 }
 
 int e2_redraw_congestion(e2_ctx *c, uint64_t seed, uint32_t generation)

@@ -128,7 +128,15 @@ __global__ void validate_kernel(Dims dm, DevPop p, int32_t *err)
         if (d >= M || ((seen[d >> 5] >> (d & 31)) & 1u)) ok = false;
         else seen[d >> 5] |= 1u << (d & 31);
     }
-    if (!ok) atomicMin(err, g);
+    if (!ok) {
+        atomicMin(err, g);
+        // replaced by a valid genome (the identity ordering as one prefill
+        // replica), so that no later kernel reads an invalid one
+        for (int i = 0; i < M; ++i) p.perm[(size_t)g * M + i] = (uint16_t)i;
+        for (int c = 0; c < K; ++c) p.sizes[(size_t)g * K + c] = (uint16_t)(c ? 0 : M);
+        p.nclus[g] = 1;
+        p.roles[g] = 0;
+    }
 }
 
 // Fisher-Yates shuffle of the identity ordering (word M-1-t draws position t);

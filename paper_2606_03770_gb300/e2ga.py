@@ -75,6 +75,8 @@ SIGNATURES = {
     "e2_get_stats": (C.c_int, [C.c_void_p, C.c_void_p]),
     "e2_set_timing_events": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "e2_run_generation": (C.c_int, [C.c_void_p, C.c_uint64, C.c_uint32]),
+    "e2_run_generation_io": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint64, C.c_uint32, C.c_void_p,
+                                       C.c_void_p]),
     "e2_get_results": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "e2_select_elites_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
                                             C.c_int32, C.c_void_p, C.c_void_p]),
@@ -163,6 +165,11 @@ def e2_get_results(ctx, fitness_ptr, parts):
 
 def e2_run_generation(ctx, seed, generation):
     return load().e2_run_generation(ctx, seed, generation)
+
+
+def e2_run_generation_io(ctx, population, seed, generation, fitness_ptr, next_out):
+    return load().e2_run_generation_io(ctx, C.byref(population) if population is not None else None, seed,
+                                       generation, fitness_ptr, C.byref(next_out) if next_out is not None else None)
 
 
 def e2_set_timing_events(ctx, start_ptr, stop_ptr):
@@ -284,6 +291,16 @@ class Engine:
     def run_generation(self, seed, generation):
         """Evaluation, elites and next population in one recorded launch."""
         _check(e2_run_generation(self.ctx, seed, generation), "e2_run_generation", self.ctx)
+
+    def run_generation_io(self, seed, generation, population=None, fitness=None, next_out=None):
+        """One generation with the host in the loop: optionally upload a
+        population, run the generation, copy the fitness and the next
+        population out (any of them host or device arrays); one
+        synchronisation."""
+        pin = self.genome_struct(population) if population is not None else None
+        pout = self.genome_struct(next_out) if next_out is not None else None
+        _check(e2_run_generation_io(self.ctx, pin, seed, generation, _ptr(fitness), pout),
+               "e2_run_generation_io", self.ctx)
 
     def redraw_congestion(self, seed, generation):
         _check(e2_redraw_congestion(self.ctx, seed, generation), "e2_redraw_congestion", self.ctx)

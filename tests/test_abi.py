@@ -146,6 +146,7 @@ def test_null_context_calls_are_rejected(lib):
     assert lib.e2_set_timing_events(None, None, None) == e2ga.E2_EINVAL
     assert lib.e2_run_generation(None, 1, 1) == e2ga.E2_EINVAL
     assert lib.e2_get_results(None, None, None) == e2ga.E2_EINVAL
+    assert lib.e2_run_generation_io(None, None, 1, 1, None, None) == e2ga.E2_EINVAL
     assert e2ga.e2_strerror(e2ga.E2_ESTATE) == "call out of order"
 
 

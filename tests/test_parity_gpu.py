@@ -369,6 +369,78 @@ def test_recorded_generation_matches_separate_calls(name, P, gens):
     b.close()
 
 
+def test_generation_io_matches_separate_calls():
+    """e2_run_generation_io (population in, one generation, fitness and next
+    population out, one synchronisation) gives what e2_set_population +
+    e2_run_generation + e2_get_results + e2_get_population give, with host
+    arrays and with device arrays, and chains over generations."""
+    import torch
+    prob = W.make_config("c2", P=512)
+    a, b = engine(prob), engine(prob)
+    g = W.random_genomes(prob.M, prob.K_max, prob.P, seed=21)
+    cur = {k: v.copy() for k, v in g.items()}
+    for gen in range(1, 5):
+        a.set_population(cur)
+        a.run_generation(9, gen)
+        fa = a.results()["fitness"]
+        na = a.get_population()
+        if gen % 2:                                    # host arrays
+            fb = np.zeros((prob.P, 4), np.float64)
+            nb = {k: np.zeros_like(v) for k, v in cur.items()}
+            b.run_generation_io(9, gen, population=cur, fitness=fb, next_out=nb)
+        else:                                          # device arrays
+            dev = {k: torch.from_numpy(v.view(np.int16) if v.dtype == np.uint16 else
+                                       v.view(np.int64) if v.dtype == np.uint64 else v).cuda()
+                   for k, v in cur.items()}
+            fd = torch.zeros((prob.P, 4), dtype=torch.float64, device="cuda")
+            nd = {k: torch.empty_like(t) for k, t in dev.items()}
+            b.run_generation_io(9, gen, population=dev, fitness=fd, next_out=nd)
+            torch.cuda.synchronize()
+            fb = fd.cpu().numpy()
+            nb = {k: nd[k].cpu().numpy().view(cur[k].dtype) for k in cur}
+        assert np.array_equal(fa, fb), gen
+        assert_genomes_equal(na, nb)
+        cur = nb
+    # chained without an upload: the context's own next population
+    a.run_generation(9, 5)
+    fb = np.zeros((prob.P, 4), np.float64)
+    b.run_generation_io(9, 5, fitness=fb)
+    assert np.array_equal(a.results()["fitness"], fb)
+    a.close()
+    b.close()
+
+
+def test_generation_io_invalid_genome_is_replaced():
+    """An invalid genome in the uploaded population: E2_EINVAL naming it, the
+    generation ran with it replaced by the identity ordering as one prefill
+    replica, and the context stays usable."""
+    from paper_2606_03770_gb300 import e2ga
+    prob = W.make_config("c1_tiny", P=16)
+    eng = engine(prob)
+    g = W.random_genomes(prob.M, prob.K_max, prob.P, seed=4)
+    bad = {k: v.copy() for k, v in g.items()}
+    bad["perm"][7, 2] = bad["perm"][7, 3]
+    fit = np.zeros((prob.P, 4), np.float64)
+    with pytest.raises(e2ga.E2Error) as ei:
+        eng.run_generation_io(3, 1, population=bad, fitness=fit)
+    assert ei.value.status == e2ga.E2_EINVAL and "genome 7" in str(ei.value)
+    fixed = {k: v.copy() for k, v in g.items()}
+    fixed["perm"][7] = np.arange(prob.M)
+    fixed["sizes"][7] = 0
+    fixed["sizes"][7, 0] = prob.M
+    fixed["nclus"][7] = 1
+    fixed["roles"][7] = 0
+    ora = O.OracleProblem(prob).eval_population(fixed, prob.K_max, nthreads=O.num_threads())
+    assert np.array_equal(fit, ora["fitness"])
+    # the same replacement by e2_set_population; then evaluation is safe
+    with pytest.raises(e2ga.E2Error):
+        eng.set_population(bad)
+    assert_genomes_equal(eng.get_population(), fixed)
+    eng.eval()
+    assert np.array_equal(eng.results()["fitness"], ora["fitness"])
+    eng.close()
+
+
 @pytest.mark.parametrize("name,P", [("c1_tiny", 64), ("c2", 1024)])
 def test_role_search_parity(name, P):
     """Alg. 2's brute-force role assignment: every replica evaluated in both
