@@ -178,7 +178,7 @@ typedef struct e2_ctx e2_ctx;
 #define E2_MAX_BATCH 64
 #define E2_MAX_CLUSTERS 64
 #define E2_MAX_POP (1 << 22)
-#define E2_MAX_ROLE_SEARCH 12
+#define E2_MAX_ROLE_SEARCH 20
 
 /* Bytes of device workspace a context with these sizes needs.  Returns 0 on
  * invalid sizes.  Reads only M, N, b_max, P, Q, K_max. */

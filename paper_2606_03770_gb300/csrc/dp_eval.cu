@@ -854,8 +854,7 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
 // and the decode sweep's answer (the largest accepted batch).  Every role
 // assignment r (bit c = 1: replica c decodes) is then scored as Eq. 3-5 score a
 // genome (PS and DS summed in ascending replica order over the replicas that
-// serve their role), the lanes taking r = lane, lane + 32, ...; the least
-// (w, phase, r) wins.  The replicas' outputs are those of their chosen roles,
+// serve their role); the least (w, phase, r) wins.  The replicas' outputs are those of their chosen roles,
 // the chosen roles are written into the genome, and the genome is scored.
 __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop, SlotInfo si, SplitOut so,
                                                              EvalOut out)
@@ -863,6 +862,7 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     __shared__ double s_ps[4][E2_MAX_ROLE_SEARCH], s_ds[4][E2_MAX_ROLE_SEARCH];
     __shared__ int s_pv[4][E2_MAX_ROLE_SEARCH], s_dv[4][E2_MAX_ROLE_SEARCH];
     __shared__ int s_off[4][E2_MAX_ROLE_SEARCH + 1], s_code[4][E2_MAX_ROLE_SEARCH];
+    __shared__ long long s_qp[4][E2_MAX_ROLE_SEARCH], s_qd[4][E2_MAX_ROLE_SEARCH];
     const int wl = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int g = blockIdx.x * 4 + wl;
     if (g >= dm.P) return;
@@ -899,13 +899,153 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     }
     if (lane == 0) s_off[wl][R] = M;
     __syncwarp();
-    // ---- the best assignment
+    // ---- the best assignment.  Lane l owns the assignments whose first
+    //      low = min(R, 5) replicas' roles are the bits of l, and walks the
+    //      other H = R - low replicas' roles in Gray-code order (one role flips
+    //      per step).  Along the walk PS and DS are kept as exact fixed-point
+    //      sums (each rate rounded to an integer multiple of 2^-s, s per warp
+    //      so that the total stays below 2^62), with the counts of replicas
+    //      serving each role.  Two screens skip assignments that can only
+    //      lose.  (1) Integer compares: a w no larger than the best w needs
+    //      NP/PS <= max(w, T_a) and ND/DS <= T_a + w (the phase exceeds T_a
+    //      by at most w, and w >= NP/PS once it does), i.e. PS and DS above
+    //      thresholds derived from the best, with margins for the fixed-point
+    //      rounding; with a best w of 0, both must stay within the best phase.
+    //      (2) A lower bound on w and the phase from the float values of the
+    //      sums, without a division (relative error below 1e-6, against a 1e-5
+    //      margin), against the best.  The others are scored exactly: PS and DS
+    //      summed in float64 in ascending replica order, then Eq. 3-5, as the
+    //      oracle does.  The best key is shared over the warp whenever a lane
+    //      improves it, so that few steps of the warp take the exact path.
+    //      With at most 8 replicas every assignment is scored exactly.
     double bw = keyd(kInfKey), bph = keyd(kInfKey);
     uint64_t br = ~0ull;
-    for (uint64_t r = lane; r < (1ull << R); r += 32) {
-        double PS, DS, w, ph;
-        score(r, PS, DS, w, ph);
-        if (w < bw || (w == bw && (ph < bph || (ph == bph && r < br)))) { bw = w; bph = ph; br = r; }
+    const int low = R < 5 ? R : 5, H = R - low;
+    // fixed-point scales: totals below 2^62; the screen needs every serving
+    // rate to be at least 2^24 units (else every assignment is scored exactly)
+    double totp = 0.0, totd = 0.0;
+    for (int c = 0; c < R; ++c) { totp = totp + s_ps[wl][c]; totd = totd + s_ds[wl][c]; }
+    const int sp_ = totp > 0.0 ? 61 - ilogb(totp) : 0, sd_ = totd > 0.0 ? 61 - ilogb(totd) : 0;
+    bool in_range = isfinite(totp) && isfinite(totd) && sp_ > -126 + 64 && sp_ < 126 && sd_ > -126 + 64 &&
+                    sd_ < 126;
+    if (lane < R) {
+        const long long qp = in_range && s_pv[wl][lane] ? __double2ll_rn(ldexp(s_ps[wl][lane], sp_)) : 0ll;
+        const long long qd = in_range && s_dv[wl][lane] ? __double2ll_rn(ldexp(s_ds[wl][lane], sd_)) : 0ll;
+        s_qp[wl][lane] = qp;
+        s_qd[wl][lane] = qd;
+        if ((s_pv[wl][lane] && qp < (1ll << 24)) || (s_dv[wl][lane] && qd < (1ll << 24))) in_range = false;
+    }
+    in_range = __all_sync(0xFFFFFFFFu, in_range);
+    __syncwarp();
+    if (H <= 3) {                                               // at most 256 assignments: score them all
+        for (uint64_t r = lane; r < (1ull << R); r += 32) {
+            double PS, DS, w, ph;
+            score(r, PS, DS, w, ph);
+            if (w < bw || (w == bw && (ph < bph || (ph == bph && r < br)))) { bw = w; bph = ph; br = r; }
+        }
+    } else {
+        long long P = 0, D = 0;                                 // fixed-point PS and DS
+        int np = 0, nd = 0;                                     // replicas serving prefill / decode
+        for (int c = 0; c < R; ++c) {                           // replicas above low start as prefill
+            const bool dec = c < low && ((lane >> c) & 1);
+            if (dec) { if (s_dv[wl][c]) { D += s_qd[wl][c]; ++nd; } }
+            else if (s_pv[wl][c]) { P += s_qp[wl][c]; ++np; }
+        }
+        // float value of a fixed-point sum (truncated to 24 bits, then scaled)
+        auto to_float = [](long long x, int s) -> float {
+            const int lz = __clzll(x), sh = lz < 40 ? 40 - lz : 0;
+            return __uint2float_rn((unsigned)(x >> sh)) * __int_as_float((127 + sh - s) << 23);
+        };
+        const float npf = (float)dm.NP, ndf = (float)dm.ND;
+        const float ta_up = (float)dm.t_a * (1.0f + 1e-6f);
+        bool finite = false, zero = false;                      // the best w: finite / 0
+        bool improved = false;                                  // this lane found a better one
+        float bw_up = 0.0f, bph_up = 0.0f;                      // its w and phase, rounded up to float
+        long long pthr = 0, dthr = 0;                           // screen (1): P, D below these lose
+        // one assignment: the screens, then the exact score where they cannot decide
+        auto consider = [&](long long P, long long D, int np, int nd, uint64_t r) {
+            if (np == 0 || nd == 0) {                              // PS or DS is 0: w = phase = +inf
+                if (!finite && r < br) br = r;
+                return;
+            }
+            if (finite && in_range) {
+                if (P < pthr || D < dthr) return;
+                const float tp = npf * __frcp_rn(to_float(P, sp_)), td = ndf * __frcp_rn(to_float(D, sd_));
+                const float ph_lo = fmaxf(tp, td) * (1.0f - 1e-5f);
+                const float w_lo = ph_lo > ta_up ? (tp * (1.0f - 1e-5f) + ph_lo) - ta_up : 0.0f;
+                if (w_lo > bw_up || (zero && ph_lo > bph_up)) return;
+            }
+            double PS, DS, w, ph;
+            score(r, PS, DS, w, ph);
+            if (w < bw || (w == bw && (ph < bph || (ph == bph && r < br)))) {
+                bw = w; bph = ph; br = r;
+                improved = true;
+            }
+        };
+        // the first U = min(H, 2) walked replicas are taken in all 2^U
+        // combinations at every step (independent work for the lane); the
+        // Gray code walks the other H - U
+        const int U = H < 2 ? H : 2;
+        long long dP[2] = {0, 0}, dD[2] = {0, 0};
+        int dn[2] = {0, 0}, dm_[2] = {0, 0};
+        for (int j = 0; j < U; ++j) {                           // replica low + j: prefill -> decode
+            const int c = low + j;
+            dP[j] = -s_qp[wl][c]; dD[j] = s_qd[wl][c];
+            dn[j] = -s_pv[wl][c]; dm_[j] = s_dv[wl][c];
+        }
+        uint64_t gq = 0;                                        // Gray code of the outer step
+        const uint64_t nq = 1ull << (H - U);
+        for (uint64_t q = 0;; ) {
+            const uint64_t rb = (uint64_t)lane | (gq << (low + U));
+            consider(P, D, np, nd, rb);
+            if (U >= 1) consider(P + dP[0], D + dD[0], np + dn[0], nd + dm_[0], rb | (1ull << low));
+            if (U >= 2) {
+                consider(P + dP[1], D + dD[1], np + dn[1], nd + dm_[1], rb | (2ull << low));
+                consider(P + dP[0] + dP[1], D + dD[0] + dD[1], np + dn[0] + dn[1], nd + dm_[0] + dm_[1],
+                         rb | (3ull << low));
+            }
+            // every lane screens against the warp's best: when a lane improved
+            // on its own, the best key (w, phase, r) is shared (all 32 lanes
+            // run the same number of steps once R >= 5)
+            if (H > 0 && __any_sync(0xFFFFFFFFu, improved)) {
+#pragma unroll
+                for (int o = 16; o; o >>= 1) {
+                    const double ow = __shfl_xor_sync(0xFFFFFFFFu, bw, o), op = __shfl_xor_sync(0xFFFFFFFFu, bph, o);
+                    const uint64_t orr = __shfl_xor_sync(0xFFFFFFFFu, br, o);
+                    if (ow < bw || (ow == bw && (op < bph || (op == bph && orr < br)))) { bw = ow; bph = op; br = orr; }
+                }
+                improved = true;                                    // every lane's best may have changed
+            }
+            if (improved) {                                         // the float copies of the best
+                improved = false;
+                if (bw < keyd(kInfKey)) {
+                    finite = true;
+                    zero = bw == 0.0;
+                    bw_up = (float)bw;
+                    if ((double)bw_up < bw) bw_up = nextafterf(bw_up, HUGE_VALF);
+                    bph_up = (float)bph;
+                    if ((double)bph_up < bph) bph_up = nextafterf(bph_up, HUGE_VALF);
+                    if (in_range) {
+                        // PS >= NP / max(w, T_a) and DS >= ND / (T_a + w) (with w = 0: both
+                        // phases within the best), less 1e-9 relative and R units
+                        const double ptp = zero ? bph : (bw > dm.t_a ? bw : dm.t_a);
+                        const double ptd = zero ? bph : dm.t_a + bw;
+                        const double pmin = ldexp((double)dm.NP / ptp, sp_) * (1.0 - 1e-9);
+                        const double dmin = ldexp((double)dm.ND / ptd, sd_) * (1.0 - 1e-9);
+                        pthr = pmin < 4e18 ? (long long)pmin - R : (long long)4e18;
+                        dthr = dmin < 4e18 ? (long long)dmin - R : (long long)4e18;
+                    }
+                }
+            }
+            if (++q == nq) break;
+            // the next Gray code flips bit t: replica low + U + t changes role
+            const int t = __ffsll((long long)q) - 1, c = low + U + t;
+            gq ^= 1ull << t;
+            const long long qp = s_qp[wl][c], qd = s_qd[wl][c];     // 0 where the role is not served
+            const int pv = s_pv[wl][c], dv = s_dv[wl][c];
+            if ((gq >> t) & 1ull) { P -= qp; D += qd; np -= pv; nd += dv; }   // prefill -> decode
+            else { P += qp; D -= qd; np += pv; nd -= dv; }                     // decode -> prefill
+        }
     }
 #pragma unroll
     for (int o = 16; o; o >>= 1) {

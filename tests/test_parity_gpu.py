@@ -441,7 +441,7 @@ def test_generation_io_invalid_genome_is_replaced():
     eng.close()
 
 
-@pytest.mark.parametrize("name,P", [("c1_tiny", 64), ("c2", 1024)])
+@pytest.mark.parametrize("name,P", [("c1_tiny", 64), ("c2", 1024), ("c3", 256)])
 def test_role_search_parity(name, P):
     """Alg. 2's brute-force role assignment: every replica evaluated in both
     roles, the best of the 2^R assignments chosen and written into the
@@ -458,6 +458,33 @@ def test_role_search_parity(name, P):
     st = eng.stats()
     assert st["paper_candidates"] == ora["cand"]
     assert st["served"] == int((ora["bsel"] >= 0).sum())
+    eng.close()
+
+
+@pytest.mark.parametrize("integer,kw", [(True, dict(min_tps=0.05)), (True, dict(min_tps=0.05, t_a=100.0)),
+                                        (False, dict(min_tps=1e-5)), (False, dict(min_tps=1e-6, t_a=1e4))])
+def test_role_search_twenty_replicas(integer, kw):
+    """The largest role search the ABI takes: genomes of 9 to 20 replicas (up
+    to 2^20 assignments, walked in Gray-code order with screens), small-integer
+    or fractional costs, with w > 0 or on the w = 0 plateau (a large T_a),
+    where the phase decides; against the oracle's plain enumeration."""
+    rng = np.random.default_rng(31 + integer)
+    M, N, K, P = 40, 24, 20, 24
+    prob = _edge_problem(rng, M, N, P, K, integer=integer, Q=2, role_search=1, **kw)
+    groups = []
+    for p in range(P):
+        R = int(rng.integers(9, 21)) if p % 3 == 0 else int(rng.integers(17, 21))
+        cuts = np.sort(rng.choice(np.arange(1, M), R - 1, replace=False))
+        groups.append(list(np.diff(np.concatenate([[0], cuts, [M]])).astype(int)))
+    g = _genomes_from(M, K, groups, rng)
+    eng = engine(prob)
+    eng.eval(g)
+    gpu = eng.results()
+    ora = O.OracleProblem(prob).eval_population(g, K, nthreads=O.num_threads())
+    assert_eval_equal(gpu, ora)
+    assert np.array_equal(eng.get_population()["roles"], ora["roles"])
+    assert np.isfinite(ora["fitness"][:, 0]).all()
+    assert (ora["fitness"][:, 0] == 0).any() == ("t_a" in kw)
     eng.close()
 
 
