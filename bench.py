@@ -40,16 +40,18 @@ METRIC = "genome evaluations/sec (GA generations on device)"
 UNIT = "genomes/s"
 WORKLOAD = "c2"
 L2_FLUSH_BYTES = 256 << 20
-# algorithmic int32 ALU operations: per bisection probe (two key loads, a 64-bit
-# compare = 2 ops, midpoint = 2 ops, index = 1 op, interval update = 1 op) and
-# per DP cell to finish it (two 64-bit min/max = 4 ops, two guards = 2 ops)
+# algorithmic int32 ALU operations: per crossover probe, of a bisection or of
+# the one-step advance to the next cell (two key loads, a compare, midpoint or
+# step = 2 ops, index = 1 op, interval update = 1 op), and per DP cell to
+# finish it (min/max = 2 ops, two guards = 2 ops, store and index = 2 ops);
+# the probes are the kernel's own tally of those it makes
 OPS_PER_PROBE = 6
 OPS_PER_CELL = 6
 SM_COUNT = 152
 INT32_LANES_PER_SM = 128
 # dram__bytes_read.sum + dram__bytes_write.sum of one dp_eval_kernel launch
 # (generation 7 of this workload), from the ncu capture in profiles/
-DP_TRAFFIC_BYTES = 704000
+DP_TRAFFIC_BYTES = 701184
 
 
 def parse():
@@ -387,7 +389,7 @@ def run_ours(args):
                          "achieved": achieved, "peak": peak, "unit": "Tops/s (int32)",
                          "frac": achieved / peak, "traffic": DP_TRAFFIC_BYTES if args.config == WORKLOAD else None,
                          "traffic_source": "profiles/dp_eval_c2_gen7.md (dram read+write, one launch)",
-                         "per_unit": f"{OPS_PER_PROBE} int32 ops per bisection probe + {OPS_PER_CELL} per DP cell",
+                         "per_unit": f"{OPS_PER_PROBE} int32 ops per crossover probe + {OPS_PER_CELL} per DP cell",
                          "peak_source": f"{SM_COUNT} SMs x {INT32_LANES_PER_SM} int32 lanes x {sm_max:.0f} MHz"},
             "e2e": e2e,
             "clocks": clk,

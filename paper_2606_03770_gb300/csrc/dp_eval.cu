@@ -60,6 +60,32 @@ __device__ __forceinline__ Key dp_cell(const Key *__restrict__ prev, const Key *
     return max(h, tau);
 }
 
+// D_k[r] for the cells r0 <= r < r1 of one column: the first crossover by
+// bisection, then each next one from the last.  With both operands
+// non-decreasing, the crossover of r + 1 is that of r or one more (if
+// prev[s] >= row[r-s] then prev[s+1] >= row[(r+1)-(s+1)]), so every cell after
+// the first costs one probe.
+template <typename Key>
+__device__ __forceinline__ void dp_span(const Key *__restrict__ prev, const Key *__restrict__ row, Key tau,
+                                        Key *__restrict__ cur, int r0, int r1)
+{
+    if (r0 >= r1) return;
+    int r = r0, lo = 0, hi = r0 + 1;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (prev[mid] >= row[r - mid]) hi = mid;
+        else lo = mid + 1;
+    }
+    for (;;) {
+        Key h = (Key)~(Key)0;
+        if (lo <= r) h = prev[lo];
+        if (lo >= 1) h = min(h, row[r - lo + 1]);
+        cur[r] = max(h, tau);
+        if (++r >= r1) break;
+        if (!(prev[lo] >= row[r - lo])) ++lo;                // lo <= r: the crossover moves by at most one
+    }
+}
+
 __device__ __forceinline__ void cp_async4(void *smem_dst, const void *gmem_src)
 {
     const unsigned sa = (unsigned)__cvta_generic_to_shared(smem_dst);
@@ -85,12 +111,10 @@ __device__ __forceinline__ unsigned long long paper_candidates(int m, int N)
     return (unsigned long long)m * ((unsigned long long)N + s);
 }
 
-// Bisection probes of one full column of W cells: sum_{n=1..W} (floor(log2 n) + 1).
-__device__ __forceinline__ unsigned long long column_probes(int W)
-{
-    const int L = 31 - __clz(W);
-    return (unsigned long long)W + (unsigned long long)(W + 1) * L - (2ull << L) + 2ull;
-}
+// Probes of one column of W cells split into contiguous spans over T = 32,
+// 64 or 128 threads (index 0, 1, 2): per span the bisection of its first cell
+// (floor(log2(r + 1)) + 1 probes for cell r), then one per further cell.
+__constant__ uint16_t c_span_probes[3][E2_MAX_BLOCKS + 1];
 
 }  // namespace
 
@@ -463,6 +487,7 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
     __shared__ unsigned s_item;
     __shared__ unsigned long long s_bestkey;     // (V << 32) | mu of the best master so far
     __shared__ uint32_t s_V0;
+    __shared__ unsigned s_prb[3];                // probes of a column over 32, 64, 128 threads
 
     const int K = dm.K, M = dm.M, N = dm.N;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
@@ -508,6 +533,7 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
         uint16_t *devs = reinterpret_cast<uint16_t *>(lbm + m);   // [m]
 
         for (int k = tid; k < m; k += blockDim.x) devs[k] = pop.perm[(size_t)g * M + off + k];
+        if (tid < 3) s_prb[tid] = c_span_probes[tid][W];
         for (int r = tid; r < W; r += blockDim.x) delta[r] = r ? kInf : (Key)0;
         __syncthreads();
 
@@ -519,7 +545,6 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
             return k == m + 1 ? delta : k == m ? leaf0 + (size_t)(m - 1) * W : Gst + (size_t)(k - 1) * W;
         };
 
-        const unsigned long long cprobe = column_probes(W);
         const unsigned long long lprobe = 32 - __clz(W);
         while (vmask && !served) {
             const int bit = 63 - __clzll((long long)vmask);          // highest batch first
@@ -559,7 +584,8 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                     const Key *prev = colF(k - 1), *row = leaf0 + (size_t)(k - 1) * W;
                     const Key t = tauk[k - 1];
                     Key *cur = Fst + (size_t)(k - 1) * W;
-                    for (int r = tid; r < W; r += 64) cur[r] = dp_cell(prev, row, t, r);
+                    const int per = (W + 63) >> 6;                 // cells per thread
+                    dp_span(prev, row, t, cur, tid * per, min(W, (tid + 1) * per));
                     bar_named(1, 64);
                 }
                 if (wid == 0) {                                   // V0 = F_m[W-1], the master-free optimum:
@@ -579,13 +605,14 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                     const Key *prev = colG(k + 1), *row = leaf0 + (size_t)(k - 1) * W;
                     const Key t = tauk[k];
                     Key *cur = Gst + (size_t)(k - 1) * W;
-                    for (int r = tid - 64; r < W; r += 64) cur[r] = dp_cell(prev, row, t, r);
+                    const int per = (W + 63) >> 6;
+                    dp_span(prev, row, t, cur, (tid - 64) * per, min(W, (tid - 63) * per));
                     bar_named(2, 64);
                 }
             }
             if (tid == 0 && m >= 3) {
                 st_cells += 2ull * (m - 2) * W;
-                st_probes += 2ull * (m - 2) * cprobe;
+                st_probes += 2ull * (m - 2) * s_prb[1];
             }
             __syncthreads();
             // ---- 4. one master per warp at a time, skipping a master whose lower
@@ -607,7 +634,8 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                 HeadRow<Key> hr;
                 hr.start(L1, hrow, W, lane);                          // in flight while H is built
                 const Key *P = colF(mu - 1), *S = colG(mu + 1);
-                for (int r = lane; r < W; r += 32) H[r] = dp_cell(P, S, (Key)0, r);
+                const int per = (W + 31) >> 5;
+                dp_span(P, S, (Key)0, H, lane * per, min(W, (lane + 1) * per));
                 hr.finish(L1, hrow, W, lane);
                 __syncwarp();
                 uint32_t V = dp_cell(H, L1, (Key)0, W - 1);
@@ -615,7 +643,7 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                 if (mu <= m - 1) V = max(V, (uint32_t)tauk[mu]);
                 __syncwarp();
                 w_cells += W + 1;
-                w_probes += cprobe + lprobe;
+                w_probes += s_prb[0] + lprobe;
                 if (lane == 0) atomicMin(&s_bestkey, ((unsigned long long)V << 32) | (unsigned)mu);
             }
             if (lane == 0) { st_cells += w_cells; st_probes += w_probes; }
@@ -642,9 +670,10 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                 const Key *prev = colD(k - 1), *row = rowk(k);
                 const Key t = tauk[k - 1];
                 Key *cur = Fst + (size_t)(k - 1) * W;
-                for (int r = tid; r < W; r += blockDim.x) cur[r] = dp_cell(prev, row, t, r);
+                const int per = (W + 127) >> 7;
+                dp_span(prev, row, t, cur, tid * per, min(W, (tid + 1) * per));
                 __syncthreads();
-                if (tid == 0) { st_cells += W; st_probes += cprobe; }
+                if (tid == 0) { st_cells += W; st_probes += s_prb[2]; }
             }
             // ---- 6. traceback (smallest split on ties), T and Lambda
             if (wid == 0) {
@@ -1129,10 +1158,33 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
 // the largest replica's DP is big (many blocks); the replica sizes whose DP
 // fits in half of it then form class 1, launched with that smaller allocation
 // and a grid of as many CTAs as fit, where this raises the CTAs per SM.
+// The probe counts of c_span_probes (a function of W alone).
+static cudaError_t load_span_probes()
+{
+    static uint16_t t[3][E2_MAX_BLOCKS + 1];
+    for (int i = 0; i < 3; ++i) {
+        const int T = 32 << i;
+        t[i][0] = 0;
+        for (int W = 1; W <= E2_MAX_BLOCKS; ++W) {
+            const int per = (W + T - 1) / T, spans = (W + per - 1) / per;
+            unsigned n = (unsigned)(W - spans);
+            for (int j = 0; j < spans; ++j) {
+                unsigned bits = 0;
+                for (unsigned x = (unsigned)(j * per + 1); x; x >>= 1) ++bits;   // floor(log2(r + 1)) + 1
+                n += bits;
+            }
+            t[i][W] = (uint16_t)n;
+        }
+    }
+    return cudaMemcpyToSymbol(c_span_probes, t, sizeof t);
+}
+
 cudaError_t configure_eval(e2_ctx *c)
 {
     const void *kernel = reinterpret_cast<const void *>(dp_eval_kernel);
-    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c->dp_smem);
+    cudaError_t e = load_span_probes();
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c->dp_smem);
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
