@@ -26,6 +26,7 @@ import math
 import os
 import statistics
 import subprocess
+import tempfile
 import sys
 import time
 
@@ -64,6 +65,8 @@ def parse():
     ap.add_argument("--seed", type=int, default=2026)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--clocks-dir", default=tempfile.gettempdir(),
+                    help="folder for the raw nvidia-smi samples of the timed region (clocks_rank<i>.csv)")
     ap.add_argument("--roles", default="bits", choices=["bits", "search"],
                     help="replica roles: bits of the genome, or Alg. 2's brute-force search")
     return ap.parse_args()
@@ -117,10 +120,10 @@ class Clocks:
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
     NAMES = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
 
-    def __init__(self, index):
+    def __init__(self, index, folder):
         self.index = index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+        self.path = os.path.join(folder, f"clocks_rank{index}.csv")
         self.t0 = self.t1 = None
 
     def start(self):
@@ -289,7 +292,7 @@ def run_ours(args):
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     stats, dp_ms = [], []
     launched = eng.stats()["launches"]     # the library's own count of its kernel launches
-    clocks = Clocks(local)
+    clocks = Clocks(local, args.clocks_dir)
     clocks.start()
     sync_all()
     clocks.begin()
