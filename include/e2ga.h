@@ -95,7 +95,8 @@ typedef struct {
 
 /* Search parameters (Alg. 2 inputs P, G, Q, Min_TPS; App. A mutation mix). */
 typedef struct {
-    int32_t P;              /* population, 1..E2_MAX_POP                        */
+    int32_t P;              /* population, 1..E2_MAX_POP, with                  */
+                            /* P * K_max * (b_max + 1) < 2^31                   */
     int32_t Q;              /* elites, 0..P                                     */
     int32_t K_max;          /* replicas per genome, 1..E2_MAX_CLUSTERS          */
     int32_t tournament;     /* tournament size, >= 1                            */
@@ -181,7 +182,8 @@ typedef struct e2_ctx e2_ctx;
 #define E2_MAX_ROLE_SEARCH 20
 
 /* Bytes of device workspace a context with these sizes needs.  Returns 0 on
- * invalid sizes.  Reads only M, N, b_max, P, Q, K_max. */
+ * invalid sizes (each within its E2_MAX_* bound, Q <= P, and
+ * P * K_max * (b_max + 1) < 2^31).  Reads only M, N, b_max, P, Q, K_max. */
 size_t e2_workspace_bytes(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_t Q,
                           int32_t K_max);
 

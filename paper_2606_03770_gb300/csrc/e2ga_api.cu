@@ -30,9 +30,11 @@ struct Layout {
 
 bool dims_ok(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_t Q, int32_t K)
 {
+    // the evaluation's work items, P * K_max * (b_max + 1), are counted and
+    // indexed in 32 bits
     return M >= 1 && M <= E2_MAX_DEVICES && N >= 1 && N <= E2_MAX_BLOCKS && b_max >= 1 &&
            b_max <= E2_MAX_BATCH && P >= 1 && P <= E2_MAX_POP && Q >= 0 && Q <= P && K >= 1 &&
-           K <= E2_MAX_CLUSTERS;
+           K <= E2_MAX_CLUSTERS && (uint64_t)P * (uint64_t)K * (uint64_t)(b_max + 1) < (1ull << 31);
 }
 
 Layout layout(int M, int N, int b_max, int P, int Q, int K)

@@ -73,6 +73,9 @@ def test_workspace_bytes(lib):
     assert e2ga.e2_workspace_bytes(0, 10, 8, 10, 1, 2) == 0
     assert e2ga.e2_workspace_bytes(8, 10, 8, 10, 11, 2) == 0      # Q > P
     assert e2ga.e2_workspace_bytes(8, 10, 8, 10, 1, 65) == 0      # K_max > 64
+    # work items P * K_max * (b_max + 1) must stay below 2^31
+    assert e2ga.e2_workspace_bytes(8, 10, 63, (1 << 22) - 1, 1, 8) > 0
+    assert e2ga.e2_workspace_bytes(8, 10, 63, (1 << 22), 1, 8) == 0
 
 
 def _structs(prob):
