@@ -484,7 +484,7 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
     __shared__ int s_S0, s_Z, s_mu, s_done;
     __shared__ uint32_t s_V;
     __shared__ double s_L, s_T;
-    __shared__ unsigned s_item;
+    __shared__ unsigned s_item, s_next;           // s_next: an item claimed during the last traceback
     __shared__ unsigned long long s_bestkey;     // (V << 32) | mu of the best master so far
     __shared__ uint32_t s_V0;
     __shared__ unsigned s_prb[3];                // probes of a column over 32, 64, 128 threads
@@ -493,9 +493,15 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
     constexpr Key kInf = (Key)~(Key)0;
     const unsigned n_items = wl.ctrl[kCtrlEnd + cls];         // this class's items end here
+    if (tid == 0) s_next = ~0u;
   for (;;) {
-    // ---- next work item of the class (heaviest first)
-    if (tid == 0) s_item = atomicAdd(&wl.ctrl[kCtrlNext + cls], 1u);
+    // ---- next work item of the class (heaviest first); warp 1 claims it
+    //      while warp 0 traces the last one back
+    if (tid == 0) {
+        const unsigned nx = s_next;
+        s_next = ~0u;
+        s_item = nx != ~0u ? nx : atomicAdd(&wl.ctrl[kCtrlNext + cls], 1u);
+    }
     __syncthreads();
     const unsigned idx = s_item;
     __syncthreads();
@@ -721,6 +727,8 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                     s_T = keyd(tmax);
                     s_done = (!role) || lam <= dm.lam_max;       // 1.0 / lam >= Min_TPS
                 }
+            } else if (wid == 1 && lane == 0) {
+                s_next = atomicAdd(&wl.ctrl[kCtrlNext + cls], 1u);
             }
             __syncthreads();
             if (s_done) {
