@@ -202,15 +202,19 @@ __global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop
     const long long slot = (long long)blockIdx.x * (blockDim.x >> 5) + wl;
     if (slot < (long long)dm.P * K) {
         const int g = (int)(slot / K), c = (int)(slot - (long long)g * K);
+        // the genome's replica count, sizes and roles, loaded together (all in bounds)
+        const uint16_t *sz = pop.sizes + (size_t)g * K;
         const int R = pop.nclus[g];
+        const int m_c = sz[c];
+        const uint64_t roles = pop.roles[g];
+        const int s_lo = lane < c ? sz[lane] : 0, s_hi = lane + 32 < c ? sz[lane + 32] : 0;
         uint64_t mask = 0;
         unsigned long long n_pre = 0, n_tps = 0;
         int m = 0, off = 0, role = 0;
         if (c < R) {
-            const uint16_t *sz = pop.sizes + (size_t)g * K;
-            m = sz[c];
-            role = (int)((pop.roles[g] >> c) & 1ull);
-            off = warp_sum(lane < c ? sz[lane] : 0) + warp_sum(lane + 32 < c ? sz[lane + 32] : 0);
+            m = m_c;
+            role = (int)((roles >> c) & 1ull);
+            off = warp_sum(s_lo) + warp_sum(s_hi);
             if (lane == 0) si.off[slot] = off;
         }
         if (c < R && m <= N) {
@@ -783,6 +787,16 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
     const int K = dm.K, M = dm.M;
     const int R = pop.nclus[g];
     const uint64_t roles = pop.roles[g];
+    // the fingerprint's inputs, loaded up front: replica sizes (lane c holds
+    // sizes[c] and sizes[c + 32]) and the ordering folded by the lanes
+    auto mix = [](uint64_t h, uint64_t x) { h = (h ^ x) * 0xBF58476D1CE4E5B9ull; return h ^ (h >> 31); };
+    const int sz_lo = lane < K ? pop.sizes[(size_t)g * K + lane] : 0;
+    const int sz_hi = lane + 32 < K ? pop.sizes[(size_t)g * K + lane + 32] : 0;
+    uint64_t hl = 0x9E3779B97F4A7C15ull ^ (uint64_t)lane;
+    {
+        const uint16_t *pp = pop.perm + (size_t)g * M;
+        for (int i = lane; i < M; i += 32) hl = mix(hl, pp[i]);
+    }
     unsigned long long n_rep = 0, n_served = 0, n_paper = 0;
     double rate[2];
     int kind[2];                                   // -1 none, 0 prefill, 1 decode
@@ -797,7 +811,7 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
             s_off[wl][c] = si.off[slot];
             int best = -2;                         // no work: outputs written by the pre-pass
             if (mask) {
-                const int m = pop.sizes[slot];
+                const int m = h ? sz_hi : sz_lo;
                 const int role = (int)((roles >> c) & 1ull);
                 best = si.best[slot];
                 unsigned long long nrun = role ? (unsigned long long)dm.b_max : 1ull;
@@ -856,18 +870,19 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
         if (k == 0) PS = PS + x;
         else if (k == 1) DS = DS + x;
     }
-    // fingerprint: lanes mix interleaved slices of the ordering, then a tree fold
-    uint64_t hl = 0x9E3779B97F4A7C15ull ^ (uint64_t)lane;
-    auto mix = [](uint64_t h, uint64_t x) { h = (h ^ x) * 0xBF58476D1CE4E5B9ull; return h ^ (h >> 31); };
-    const uint16_t *pp = pop.perm + (size_t)g * M;
-    for (int i = lane; i < M; i += 32) hl = mix(hl, pp[i]);
+    // fingerprint: lanes mixed interleaved slices of the ordering; a tree fold,
+    // then the sizes in replica order (from the lanes that hold them)
 #pragma unroll
     for (int o = 16; o; o >>= 1) {
         const uint64_t other = __shfl_down_sync(0xFFFFFFFFu, hl, o);
         if (lane < o) hl = mix(hl, other);
     }
-    if (lane != 0) return;
     uint64_t h = hl;
+    for (int i = 0; i < R; ++i) {
+        const int si_ = __shfl_sync(0xFFFFFFFFu, i < 32 ? sz_lo : sz_hi, i & 31);
+        h = mix(h, (uint64_t)si_ << 16);
+    }
+    if (lane != 0) return;
     double w = keyd(kInfKey), phase = keyd(kInfKey);
     if (PS != 0.0 && DS != 0.0) {
         const double tp = (double)dm.NP / PS, td = (double)dm.ND / DS;
@@ -878,8 +893,6 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
     }
     double *f = out.fit + (size_t)g * 4;
     f[0] = w; f[1] = phase; f[2] = PS; f[3] = DS;
-    const uint16_t *ss = pop.sizes + (size_t)g * K;
-    for (int i = 0; i < R; ++i) h = mix(h, (uint64_t)ss[i] << 16);
     h = mix(h, (uint64_t)R << 40);
     h = mix(h, roles);
     out.hash[g] = h;
