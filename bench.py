@@ -52,7 +52,7 @@ SM_COUNT = 152
 INT32_LANES_PER_SM = 128
 # dram__bytes_read.sum + dram__bytes_write.sum of one dp_eval_kernel launch
 # (generation 7 of this workload), from the ncu capture in profiles/
-DP_TRAFFIC_BYTES = 701184
+DP_TRAFFIC_BYTES = 703232
 
 
 def parse():
