@@ -149,7 +149,9 @@ typedef struct {
     uint64_t replicas;          /* replicas evaluated (sum of R)                */
     uint64_t dp_runs;           /* DP_Pipe runs that reached the recurrence     */
     uint64_t dp_cells;          /* DP cells D_mu(i,k) computed                  */
-    uint64_t dp_probes;         /* split-point probes over all cells            */
+    uint64_t dp_probes;         /* split-point probes made: a bisection for the
+                                   first cell of each thread's span of a column,
+                                   one probe for each further cell              */
     uint64_t paper_candidates;  /* (mu,k,i,j) candidates Alg. 1 would examine   */
     uint64_t prechecked;        /* variants rejected by the memory count check
                                    (over each replica's whole sweep)            */
