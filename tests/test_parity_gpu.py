@@ -238,6 +238,34 @@ def test_elites_with_duplicates_and_Q_extremes():
         eng.close()
 
 
+@pytest.mark.parametrize("P,Q", [(5000, 157), (8200, 8200)])
+def test_elites_large_population_with_duplicates(P, Q):
+    """Populations of several thousand genomes (many tiles of the duplicate
+    test and the ranks): a ragged size, many planted duplicates (copies of a
+    few genomes spread over the population, ties in every key), Q = ceil(P/32)
+    and Q = P; elites and next population against the oracle."""
+    prob = W.make_config("c1_tiny", P=P)
+    prob.Q = Q
+    rng = np.random.default_rng(17)
+    g = W.random_genomes(prob.M, prob.K_max, P, seed=5)
+    src = rng.integers(0, 50, 600)
+    dst = rng.choice(np.arange(50, P), 600, replace=False)
+    for a, b in zip(dst, src):
+        for k in g:
+            g[k][a] = g[k][b]
+    eng = engine(prob)
+    eng.eval(g)
+    fit = eng.results()["fitness"]
+    ga = O.ga_of(prob)
+    eidx = O.elites(ga, g, fit)
+    eng.ga_step(8, 3)
+    gi, gf = eng.elites()
+    assert np.array_equal(gi, eidx)
+    assert np.array_equal(gf, fit[eidx])
+    assert_genomes_equal(eng.get_population(), O.ga_step(ga, 8, 3, g, fit, eidx))
+    eng.close()
+
+
 def test_host_and_device_buffers_agree():
     import torch
     prob = W.make_config("c1_tiny", P=64)
