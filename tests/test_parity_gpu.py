@@ -516,6 +516,24 @@ def test_role_search_twenty_replicas(integer, kw):
     eng.close()
 
 
+def test_role_search_with_two_dp_launches():
+    """The role search on a fleet whose DP runs in two shared-memory classes
+    (220-block rows): both roles of every replica through both launches."""
+    rng = np.random.default_rng(41)
+    M, N, K, P = 48, 220, 8, 24
+    prob = _edge_problem(rng, M, N, P, K, integer=True, Q=2, min_tps=0.01, role_search=1)
+    g = W.random_genomes(M, K, P, seed=9)
+    eng = engine(prob)
+    eng.eval(g)
+    gpu = eng.results()
+    ora = O.OracleProblem(prob).eval_population(g, K, nthreads=O.num_threads())
+    assert_eval_equal(gpu, ora)
+    assert np.array_equal(eng.get_population()["roles"], ora["roles"])
+    st = eng.stats()
+    assert st["dp_launches"] == 2 and 0 < st["dp_runs_small"] < st["dp_runs"], st
+    eng.close()
+
+
 def test_role_search_generations():
     """Generations with the role search, recorded and separate calls alike,
     against the oracle (whose population takes the roles it chose)."""
