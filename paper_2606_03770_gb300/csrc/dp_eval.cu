@@ -906,6 +906,7 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
 // genome (PS and DS summed in ascending replica order over the replicas that
 // serve their role); the least (w, phase, r) wins.  The replicas' outputs are those of their chosen roles,
 // the chosen roles are written into the genome, and the genome is scored.
+template <int WPG>
 __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop, SlotInfo si, SplitOut so,
                                                              EvalOut out)
 {
@@ -913,16 +914,25 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     __shared__ int s_pv[4][E2_MAX_ROLE_SEARCH], s_dv[4][E2_MAX_ROLE_SEARCH];
     __shared__ int s_off[4][E2_MAX_ROLE_SEARCH + 1], s_code[4][E2_MAX_ROLE_SEARCH];
     __shared__ long long s_qp[4][E2_MAX_ROLE_SEARCH], s_qd[4][E2_MAX_ROLE_SEARCH];
+    __shared__ double s_bw[4], s_bph[4];
+    __shared__ unsigned long long s_wmin[4];           // the least w a warp of the genome has scored (bits)
+    __shared__ uint64_t s_br[4];
     const int wl = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int g = blockIdx.x * 4 + wl;
+    // WPG warps per genome: 1 (four genomes per block), or 4 (one genome per
+    // block, its assignments split over the block's 128 threads)
+    const int g = WPG == 1 ? (int)blockIdx.x * 4 + wl : (int)blockIdx.x;
+    const int gw = WPG == 1 ? wl : 0;                  // the genome's shared-memory row
+    const int id = WPG == 1 ? lane : (int)threadIdx.x; // the thread's place in its genome's search
+    const bool lead = WPG == 1 || wl == 0;              // the warp that reads and writes the genome
     if (g >= dm.P) return;
     const int K = dm.K, M = dm.M, V = dm.V, bp = dm.b_max;
     const int R = pop.nclus[g];
+    const uint64_t roles0 = pop.roles[g];
     auto score = [&](uint64_t r, double &PS, double &DS, double &w, double &phase) {
         PS = 0.0; DS = 0.0;
         for (int c = 0; c < R; ++c) {
-            if ((r >> c) & 1ull) { if (s_dv[wl][c]) DS = DS + s_ds[wl][c]; }
-            else if (s_pv[wl][c]) PS = PS + s_ps[wl][c];
+            if ((r >> c) & 1ull) { if (s_dv[gw][c]) DS = DS + s_ds[gw][c]; }
+            else if (s_pv[gw][c]) PS = PS + s_ps[gw][c];
         }
         w = keyd(kInfKey); phase = keyd(kInfKey);
         if (PS != 0.0 && DS != 0.0) {
@@ -935,20 +945,21 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     };
     // ---- each replica's two results
     int best = -1, pok = 0, m = 0;
-    if (lane < R) {
+    if (lead && lane < R) {
         const int slot = g * K + lane;
         const uint64_t mask = si.mask[slot];
         m = pop.sizes[slot];
         pok = (int)((mask >> bp) & 1ull);
         best = mask ? si.best[slot] : -1;
-        s_off[wl][lane] = si.off[slot];
-        s_pv[wl][lane] = pok;
-        s_dv[wl][lane] = best >= 0;
-        s_ps[wl][lane] = pok ? (double)dm.NP / so.T[(size_t)slot * V + bp] : 0.0;
-        s_ds[wl][lane] = best >= 0 ? (double)(best + 1) / so.T[(size_t)slot * V + best] : 0.0;
+        s_off[gw][lane] = si.off[slot];
+        s_pv[gw][lane] = pok;
+        s_dv[gw][lane] = best >= 0;
+        s_ps[gw][lane] = pok ? (double)dm.NP / so.T[(size_t)slot * V + bp] : 0.0;
+        s_ds[gw][lane] = best >= 0 ? (double)(best + 1) / so.T[(size_t)slot * V + best] : 0.0;
     }
-    if (lane == 0) s_off[wl][R] = M;
-    __syncwarp();
+    if (lead && lane == 0) s_off[gw][R] = M;
+    if (WPG == 1) __syncwarp();
+    else __syncthreads();
     // ---- the best assignment.  Lane l owns the assignments whose first
     //      low = min(R, 5) replicas' roles are the bits of l, and walks the
     //      other H = R - low replicas' roles in Gray-code order (one role flips
@@ -970,25 +981,30 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     //      With at most 8 replicas every assignment is scored exactly.
     double bw = keyd(kInfKey), bph = keyd(kInfKey);
     uint64_t br = ~0ull;
-    const int low = R < 5 ? R : 5, H = R - low;
+    constexpr int kFixed = WPG == 1 ? 5 : 7;            // replicas whose roles are the bits of id
+    const int low = R < kFixed ? R : kFixed, H = R - low;
     // fixed-point scales: totals below 2^62; the screen needs every serving
     // rate to be at least 2^24 units (else every assignment is scored exactly)
     double totp = 0.0, totd = 0.0;
-    for (int c = 0; c < R; ++c) { totp = totp + s_ps[wl][c]; totd = totd + s_ds[wl][c]; }
+    for (int c = 0; c < R; ++c) { totp = totp + s_ps[gw][c]; totd = totd + s_ds[gw][c]; }
     const int sp_ = totp > 0.0 ? 61 - ilogb(totp) : 0, sd_ = totd > 0.0 ? 61 - ilogb(totd) : 0;
     bool in_range = isfinite(totp) && isfinite(totd) && sp_ > -126 + 64 && sp_ < 126 && sd_ > -126 + 64 &&
                     sd_ < 126;
     if (lane < R) {
-        const long long qp = in_range && s_pv[wl][lane] ? __double2ll_rn(ldexp(s_ps[wl][lane], sp_)) : 0ll;
-        const long long qd = in_range && s_dv[wl][lane] ? __double2ll_rn(ldexp(s_ds[wl][lane], sd_)) : 0ll;
-        s_qp[wl][lane] = qp;
-        s_qd[wl][lane] = qd;
-        if ((s_pv[wl][lane] && qp < (1ll << 24)) || (s_dv[wl][lane] && qd < (1ll << 24))) in_range = false;
+        const long long qp = in_range && s_pv[gw][lane] ? __double2ll_rn(ldexp(s_ps[gw][lane], sp_)) : 0ll;
+        const long long qd = in_range && s_dv[gw][lane] ? __double2ll_rn(ldexp(s_ds[gw][lane], sd_)) : 0ll;
+        if (lead) {
+            s_qp[gw][lane] = qp;
+            s_qd[gw][lane] = qd;
+        }
+        if ((s_pv[gw][lane] && qp < (1ll << 24)) || (s_dv[gw][lane] && qd < (1ll << 24))) in_range = false;
     }
     in_range = __all_sync(0xFFFFFFFFu, in_range);
-    __syncwarp();
-    if (H <= 3) {                                               // at most 256 assignments: score them all
-        for (uint64_t r = lane; r < (1ull << R); r += 32) {
+    if (lead && lane == 0) s_wmin[gw] = dkey(keyd(kInfKey));
+    if (WPG == 1) __syncwarp();
+    else __syncthreads();
+    if (R <= 8) {                                               // at most 256 assignments: score them all
+        for (uint64_t r = id; r < (1ull << R); r += 32 * WPG) {
             double PS, DS, w, ph;
             score(r, PS, DS, w, ph);
             if (w < bw || (w == bw && (ph < bph || (ph == bph && r < br)))) { bw = w; bph = ph; br = r; }
@@ -997,9 +1013,9 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
         long long P = 0, D = 0;                                 // fixed-point PS and DS
         int np = 0, nd = 0;                                     // replicas serving prefill / decode
         for (int c = 0; c < R; ++c) {                           // replicas above low start as prefill
-            const bool dec = c < low && ((lane >> c) & 1);
-            if (dec) { if (s_dv[wl][c]) { D += s_qd[wl][c]; ++nd; } }
-            else if (s_pv[wl][c]) { P += s_qp[wl][c]; ++np; }
+            const bool dec = c < low && ((id >> c) & 1);
+            if (dec) { if (s_dv[gw][c]) { D += s_qd[gw][c]; ++nd; } }
+            else if (s_pv[gw][c]) { P += s_qp[gw][c]; ++np; }
         }
         // float value of a fixed-point sum (truncated to 24 bits, then scaled)
         auto to_float = [](long long x, int s) -> float {
@@ -1008,14 +1024,27 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
         };
         const float npf = (float)dm.NP, ndf = (float)dm.ND;
         const float ta_up = (float)dm.t_a * (1.0f + 1e-6f);
-        bool finite = false, zero = false;                      // the best w: finite / 0
+        bool finite = false, zero = false;                      // the screen's w: finite / own best w of 0
         bool improved = false;                                  // this lane found a better one
-        float bw_up = 0.0f, bph_up = 0.0f;                      // its w and phase, rounded up to float
+        float bw_up = 0.0f, bph_up = 0.0f;                      // the screen's w and phase, rounded up to float
         long long pthr = 0, dthr = 0;                           // screen (1): P, D below these lose
+        // the screens compare with we = min(own best w, the least w any warp of
+        // the genome has scored); the phase screen only with the own best
+        double wsh = keyd(kInfKey);                             // the shared least w last taken
+        // start from the genome's own roles: a real assignment, scored exactly
+        bool own_fin;                                           // the lane's own best w is finite
+        {
+            const uint64_t r0 = roles0 & ((2ull << (R - 1)) - 1ull);
+            double PS, DS, w, ph;
+            score(r0, PS, DS, w, ph);
+            bw = w; bph = ph; br = r0;
+            own_fin = w < keyd(kInfKey);
+            improved = true;
+        }
         // one assignment: the screens, then the exact score where they cannot decide
         auto consider = [&](long long P, long long D, int np, int nd, uint64_t r) {
             if (np == 0 || nd == 0) {                              // PS or DS is 0: w = phase = +inf
-                if (!finite && r < br) br = r;
+                if (!own_fin && r < br) br = r;                    // ties the own best only while it is +inf
                 return;
             }
             if (finite && in_range) {
@@ -1029,6 +1058,7 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
             score(r, PS, DS, w, ph);
             if (w < bw || (w == bw && (ph < bph || (ph == bph && r < br)))) {
                 bw = w; bph = ph; br = r;
+                own_fin = true;                                    // PS, DS > 0: w is finite
                 improved = true;
             }
         };
@@ -1040,13 +1070,13 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
         int dn[2] = {0, 0}, dm_[2] = {0, 0};
         for (int j = 0; j < U; ++j) {                           // replica low + j: prefill -> decode
             const int c = low + j;
-            dP[j] = -s_qp[wl][c]; dD[j] = s_qd[wl][c];
-            dn[j] = -s_pv[wl][c]; dm_[j] = s_dv[wl][c];
+            dP[j] = -s_qp[gw][c]; dD[j] = s_qd[gw][c];
+            dn[j] = -s_pv[gw][c]; dm_[j] = s_dv[gw][c];
         }
         uint64_t gq = 0;                                        // Gray code of the outer step
         const uint64_t nq = 1ull << (H - U);
         for (uint64_t q = 0;; ) {
-            const uint64_t rb = (uint64_t)lane | (gq << (low + U));
+            const uint64_t rb = (uint64_t)id | (gq << (low + U));
             consider(P, D, np, nd, rb);
             if (U >= 1) consider(P + dP[0], D + dD[0], np + dn[0], nd + dm_[0], rb | (1ull << low));
             if (U >= 2) {
@@ -1065,21 +1095,29 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
                     if (ow < bw || (ow == bw && (op < bph || (op == bph && orr < br)))) { bw = ow; bph = op; br = orr; }
                 }
                 improved = true;                                    // every lane's best may have changed
+                own_fin = bw < keyd(kInfKey);
+                if (lane == 0 && own_fin) atomicMin(&s_wmin[gw], (unsigned long long)dkey(bw));
             }
-            if (improved) {                                         // the float copies of the best
+            {                                                       // another warp's better w
+                const double ws = keyd(*reinterpret_cast<volatile unsigned long long *>(&s_wmin[gw]));
+                if (ws < wsh) { wsh = ws; improved = true; }
+            }
+            if (improved) {                                         // the float copies of the screen's state
                 improved = false;
-                if (bw < keyd(kInfKey)) {
+                const double we = bw < wsh ? bw : wsh;
+                if (we < keyd(kInfKey)) {
                     finite = true;
                     zero = bw == 0.0;
-                    bw_up = (float)bw;
-                    if ((double)bw_up < bw) bw_up = nextafterf(bw_up, HUGE_VALF);
+                    bw_up = (float)we;
+                    if ((double)bw_up < we) bw_up = nextafterf(bw_up, HUGE_VALF);
                     bph_up = (float)bph;
                     if ((double)bph_up < bph) bph_up = nextafterf(bph_up, HUGE_VALF);
                     if (in_range) {
-                        // PS >= NP / max(w, T_a) and DS >= ND / (T_a + w) (with w = 0: both
-                        // phases within the best), less 1e-9 relative and R units
-                        const double ptp = zero ? bph : (bw > dm.t_a ? bw : dm.t_a);
-                        const double ptd = zero ? bph : dm.t_a + bw;
+                        // PS >= NP / max(w, T_a) and DS >= ND / (T_a + w) for a w no larger than
+                        // we (with an own best w of 0: both phases within its phase), less
+                        // 1e-9 relative and R units
+                        const double ptp = zero ? bph : (we > dm.t_a ? we : dm.t_a);
+                        const double ptd = zero ? bph : dm.t_a + we;
                         const double pmin = ldexp((double)dm.NP / ptp, sp_) * (1.0 - 1e-9);
                         const double dmin = ldexp((double)dm.ND / ptd, sd_) * (1.0 - 1e-9);
                         pthr = pmin < 4e18 ? (long long)pmin - R : (long long)4e18;
@@ -1091,8 +1129,8 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
             // the next Gray code flips bit t: replica low + U + t changes role
             const int t = __ffsll((long long)q) - 1, c = low + U + t;
             gq ^= 1ull << t;
-            const long long qp = s_qp[wl][c], qd = s_qd[wl][c];     // 0 where the role is not served
-            const int pv = s_pv[wl][c], dv = s_dv[wl][c];
+            const long long qp = s_qp[gw][c], qd = s_qd[gw][c];     // 0 where the role is not served
+            const int pv = s_pv[gw][c], dv = s_dv[gw][c];
             if ((gq >> t) & 1ull) { P -= qp; D += qd; np -= pv; nd += dv; }   // prefill -> decode
             else { P += qp; D -= qd; np += pv; nd -= dv; }                     // decode -> prefill
         }
@@ -1103,13 +1141,23 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
         const uint64_t orr = __shfl_xor_sync(0xFFFFFFFFu, br, o);
         if (ow < bw || (ow == bw && (op < bph || (op == bph && orr < br)))) { bw = ow; bph = op; br = orr; }
     }
-    // ---- outputs of the chosen roles
+    if (WPG > 1) {                                      // the best of the genome's warps
+        if (lane == 0) { s_bw[wl] = bw; s_bph[wl] = bph; s_br[wl] = br; }
+        __syncthreads();
+        if (wl != 0) return;
+        for (int o = 1; o < WPG; ++o) {
+            const double ow = s_bw[o], op = s_bph[o];
+            const uint64_t orr = s_br[o];
+            if (ow < bw || (ow == bw && (op < bph || (op == bph && orr < br)))) { bw = ow; bph = op; br = orr; }
+        }
+    }
+    // ---- outputs of the chosen roles (the genome's first warp)
     unsigned long long n_rep = 0, n_served = 0, n_paper = 0;
     if (lane < R) {
         const int slot = g * K + lane;
         const int role = (int)((br >> lane) & 1ull);
         const int code = role ? best : (pok ? bp : -1);
-        s_code[wl][lane] = code;
+        s_code[gw][lane] = code;
         if (code < 0) {
             out.master[slot] = -1; out.bsel[slot] = -1;
             out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
@@ -1133,10 +1181,10 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
         int lo = 0, hi = R - 1;
         while (lo < hi) {
             const int mid = (lo + hi + 1) >> 1;
-            if (s_off[wl][mid] <= i) lo = mid;
+            if (s_off[gw][mid] <= i) lo = mid;
             else hi = mid - 1;
         }
-        const int code = s_code[wl][lo];
+        const int code = s_code[gw][lo];
         out.layers[(size_t)g * M + i] = code >= 0 ? split[(size_t)code * M + i] : (int16_t)-1;
     }
 #pragma unroll
@@ -1274,7 +1322,9 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     }
     if (c->ev_dp_stop && (e = cudaEventRecordWithFlags(c->ev_dp_stop, c->stream, rec)) != cudaSuccess) return e;
     const unsigned fb = (unsigned)(((size_t)c->dm.P * 32 + 127) / 128);
-    if (c->dm.role_search) finalize_roles_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
+    if (c->dm.role_search && c->dm.K >= 12)           // up to 2^K_max assignments: a block per genome
+        finalize_roles_kernel<4><<<(unsigned)c->dm.P, 128, 0, c->stream>>>(c->dm, p, si, so, out);
+    else if (c->dm.role_search) finalize_roles_kernel<1><<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
     else finalize_score_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
     c->launches += c->dp_grid1 > 0 ? 5 : 4;
     return cudaGetLastError();
