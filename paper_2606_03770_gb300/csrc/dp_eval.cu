@@ -928,9 +928,12 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     const int K = dm.K, M = dm.M, V = dm.V, bp = dm.b_max;
     const int R = pop.nclus[g];
     const uint64_t roles0 = pop.roles[g];
-    auto score = [&](uint64_t r, double &PS, double &DS, double &w, double &phase) {
-        PS = 0.0; DS = 0.0;
-        for (int c = 0; c < R; ++c) {
+    // Eq. 3-5 for assignment r, PS and DS summed in ascending replica order
+    // from replica c0 on, the sums over replicas 0..c0-1 given
+    auto score_from = [&](uint64_t r, int c0, double PS0, double DS0, double &PS, double &DS, double &w,
+                          double &phase) {
+        PS = PS0; DS = DS0;
+        for (int c = c0; c < R; ++c) {
             if ((r >> c) & 1ull) { if (s_dv[gw][c]) DS = DS + s_ds[gw][c]; }
             else if (s_pv[gw][c]) PS = PS + s_ps[gw][c];
         }
@@ -942,6 +945,9 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
             const double bn = x > 0.0 ? x : 0.0;        // Eq. 4
             w = bn > 0.0 ? tp + bn : 0.0;               // Eq. 5
         }
+    };
+    auto score = [&](uint64_t r, double &PS, double &DS, double &w, double &phase) {
+        score_from(r, 0, 0.0, 0.0, PS, DS, w, phase);
     };
     // ---- each replica's two results
     int best = -1, pok = 0, m = 0;
@@ -1042,7 +1048,10 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
             improved = true;
         }
         // one assignment: the screens, then the exact score where they cannot decide
-        auto consider = [&](long long P, long long D, int np, int nd, uint64_t r) {
+        // with a block per genome the roles of replicas 0..low+U-1 are fixed per
+        // thread and combination: their exact sums are taken once (prefix)
+        double preP[4] = {0.0, 0.0, 0.0, 0.0}, preD[4] = {0.0, 0.0, 0.0, 0.0};
+        auto consider = [&](long long P, long long D, int np, int nd, uint64_t r, int j) {
             if (np == 0 || nd == 0) {                              // PS or DS is 0: w = phase = +inf
                 if (!own_fin && r < br) br = r;                    // ties the own best only while it is +inf
                 return;
@@ -1055,7 +1064,8 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
                 if (w_lo > bw_up || (zero && ph_lo > bph_up)) return;
             }
             double PS, DS, w, ph;
-            score(r, PS, DS, w, ph);
+            if (WPG > 1) score_from(r, low + 2, preP[j], preD[j], PS, DS, w, ph);
+            else score(r, PS, DS, w, ph);
             if (w < bw || (w == bw && (ph < bph || (ph == bph && r < br)))) {
                 bw = w; bph = ph; br = r;
                 own_fin = true;                                    // PS, DS > 0: w is finite
@@ -1065,7 +1075,14 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
         // the first U = min(H, 2) walked replicas are taken in all 2^U
         // combinations at every step (independent work for the lane); the
         // Gray code walks the other H - U
-        const int U = H < 2 ? H : 2;
+        const int U = H < 2 ? H : 2;                            // 2 with a block per genome (R >= 9)
+        if (WPG > 1)
+            for (int j = 0; j < 4; ++j)
+                for (int c = 0; c < low + 2; ++c) {
+                    const bool dec = c < low ? ((id >> c) & 1) : ((j >> (c - low)) & 1);
+                    if (dec) { if (s_dv[gw][c]) preD[j] = preD[j] + s_ds[gw][c]; }
+                    else if (s_pv[gw][c]) preP[j] = preP[j] + s_ps[gw][c];
+                }
         long long dP[2] = {0, 0}, dD[2] = {0, 0};
         int dn[2] = {0, 0}, dm_[2] = {0, 0};
         for (int j = 0; j < U; ++j) {                           // replica low + j: prefill -> decode
@@ -1077,12 +1094,12 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
         const uint64_t nq = 1ull << (H - U);
         for (uint64_t q = 0;; ) {
             const uint64_t rb = (uint64_t)id | (gq << (low + U));
-            consider(P, D, np, nd, rb);
-            if (U >= 1) consider(P + dP[0], D + dD[0], np + dn[0], nd + dm_[0], rb | (1ull << low));
+            consider(P, D, np, nd, rb, 0);
+            if (U >= 1) consider(P + dP[0], D + dD[0], np + dn[0], nd + dm_[0], rb | (1ull << low), 1);
             if (U >= 2) {
-                consider(P + dP[1], D + dD[1], np + dn[1], nd + dm_[1], rb | (2ull << low));
+                consider(P + dP[1], D + dD[1], np + dn[1], nd + dm_[1], rb | (2ull << low), 2);
                 consider(P + dP[0] + dP[1], D + dD[0] + dD[1], np + dn[0] + dn[1], nd + dm_[0] + dm_[1],
-                         rb | (3ull << low));
+                         rb | (3ull << low), 3);
             }
             // every lane screens against the warp's best: when a lane improved
             // on its own, the best key (w, phase, r) is shared (all 32 lanes
