@@ -1,11 +1,13 @@
 // dp_eval.cu -- population fitness: DP_Pipe per replica (Alg. 1, Eq. 1-2),
 // the decode batch sweep (Alg. 2), and the objective (Eq. 3-5).
 //
-// Work is split over six kernels per evaluation: a pre-pass that decides,
-// per (genome, replica slot, variant), whether a DP run can matter (memory and
-// latency bounds); three small kernels that order the surviving runs into one
-// work list; persistent DP CTAs that drain the list; and a warp per genome that
-// picks each replica's answer and scores the genome.
+// Work is split over four or five kernels per evaluation: a pre-pass that
+// decides, per (genome, replica slot, variant), whether a DP run can matter
+// (memory and latency bounds) and counts and orders the surviving runs; a
+// scatter that writes them into one work list; persistent DP CTAs that drain
+// the list (two launches where the replica sizes fall into two shared-memory
+// classes); and a warp per genome (a block per genome for a wide role search)
+// that picks each replica's answer and scores the genome.
 //
 // With identical blocks (Sec. 3.2: the premise that lets the paper fix the
 // node order) a stage's time depends only on its device, its block count n and
@@ -23,7 +25,9 @@
 // then rises: its minimum sits at the crossover s0 = first s with
 // D_{k-1}[s] >= l_k(r - s + 1) and equals min(l_k(r - s0 + 2), D_{k-1}[s0]).
 // A bisection over s finds s0, so a cell costs O(log W) probes instead of the
-// O(W) scan, with bit-identical values (min and max are exact).
+// O(W) scan, with bit-identical values (min and max are exact); and the
+// crossover of cell r + 1 is that of cell r or one more, so a thread that owns
+// a span of cells bisects only for the first (dp_span).
 //
 // Tie rule.  The oracle keeps the smallest split j attaining the minimum.  The
 // set of minimisers is {s : D_{k-1}[s] <= D and l_k(r-s+1) <= D} (tau <= D
@@ -463,7 +467,8 @@ template <> struct HeadRow<uint32_t> {
 //     order keys (exact ranks, see ranks.cu);
 //  2. masters the memory allows;
 //  3. prefix columns F_k (no master, devices 1..k) on warps 0-1 and suffix
-//     columns G_k (no master, devices k..m) on warps 2-3, concurrently:
+//     columns G_k (no master, devices k..m) on warps 2-3, concurrently, each
+//     thread a span of a column:
 //        F_k[r] = min_s max(F_{k-1}[s], l_k(r-s+1), tau_k)
 //        G_k[r] = min_s max(G_{k+1}[s], l_k(r-s+1), tau_{k+1})
 //  4. master mu: the prefix holds a extra blocks, the suffix b, the master
@@ -476,7 +481,8 @@ template <> struct HeadRow<uint32_t> {
 //  6. traceback with the smallest-split rule (n_k = number of n <= r+1 with
 //     l_k(n) <= D, counted with warp ballots); the bottleneck T (the largest
 //     stage or link time of the partition, equal to V) and Lambda (summed in
-//     pipeline order) in float64 from the stage and link tables.
+//     pipeline order) in float64 from the stage and link tables; meanwhile
+//     warp 1 claims the next item.
 // Every comparison is between ranks of the same stage and link times the
 // oracle compares, so V, mu*, the partition, T and Lambda are bit-identical to
 // Alg. 1.
