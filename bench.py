@@ -53,6 +53,9 @@ INT32_LANES_PER_SM = 128
 # dram__bytes_read.sum + dram__bytes_write.sum of one dp_eval_kernel launch
 # (generation 7 of this workload), from the ncu capture in profiles/
 DP_TRAFFIC_BYTES = 703232
+# smsp__issue_active (fraction of peak, active cycles) of the same launch: the
+# kernel is bound by issue and dependent latency, not by one pipe
+DP_ISSUE_ACTIVE = 0.663
 
 
 def parse():
@@ -392,6 +395,7 @@ def run_ours(args):
                          "achieved": achieved, "peak": peak, "unit": "Tops/s (int32)",
                          "frac": achieved / peak, "traffic": DP_TRAFFIC_BYTES if args.config == WORKLOAD else None,
                          "traffic_source": "profiles/dp_eval_c2_gen7.md (dram read+write, one launch)",
+                         "issue_active": DP_ISSUE_ACTIVE if args.config == WORKLOAD else None,
                          "per_unit": f"{OPS_PER_PROBE} int32 ops per crossover probe + {OPS_PER_CELL} per DP cell",
                          "peak_source": f"{SM_COUNT} SMs x {INT32_LANES_PER_SM} int32 lanes x {sm_max:.0f} MHz"},
             "e2e": e2e,
