@@ -192,9 +192,9 @@ __device__ __forceinline__ int item_bin(int level, int size)
 // The surviving variants form the slot's mask.  A slot with nothing to run
 // (empty, more devices than blocks, no variant left) gets its outputs here;
 // the others count their work items into the ordering bins.  The last warp to
-// finish (a ticket taken after a fence, no waiting) scans the bins into
-// starting offsets, class 0 first and heaviest first within a class, and
-// stores the item total and where class 1 starts.
+// finish (a ticket taken after a fence where the warp counted, no waiting)
+// scans the bins into starting offsets, class 0 first and heaviest first
+// within a class, and stores the item total and where class 1 starts.
 __global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si, EvalOut out,
                                                   unsigned *ctrl)
 {
@@ -204,6 +204,7 @@ __global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop
     const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
     const int K = dm.K, M = dm.M, N = dm.N;
     const long long slot = (long long)blockIdx.x * (blockDim.x >> 5) + wl;
+    bool counted = false;                                     // this warp added to the bins
     if (slot < (long long)dm.P * K) {
         const int g = (int)(slot / K), c = (int)(slot - (long long)g * K);
         // the genome's replica count, sizes and roles, loaded together (all in bounds)
@@ -349,6 +350,7 @@ __global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop
                 si.size[slot] = (uint8_t)size;
                 const int nv = __popcll(mask);
                 for (int lv = 0; lv < nv; ++lv) atomicAdd(&ctrl[item_bin(lv, size)], 1u);
+                counted = true;
             }
         }
     }
@@ -358,7 +360,7 @@ __global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop
     //      then class 1's), read eight at a time
     unsigned ticket = 0;
     if (lane == 0) {
-        __threadfence();
+        if (counted) __threadfence();                         // publish the bin counts (only they are read)
         ticket = atomicAdd(&ctrl[kCtrlTicket], 1u);
     }
     ticket = __shfl_sync(0xFFFFFFFFu, ticket, 0);
