@@ -381,7 +381,11 @@ def test_decode_picks_highest_feasible_batch():
             d = op.dp_pipe(b, devs)
             assert d["V"] == r["T"] and 1.0 / r["L"] >= prob.min_tps
             seen_mid += 0 < b < prob.b_max
-    assert seen_mid >= 0
+    # the sweep must stop inside the range, not only at its ends: on these 80
+    # random clusters 52 serve and 9 of them stop at a batch strictly between
+    # 1 and b_max (a sweep that only tried b_max, or that stopped at the first
+    # feasible batch from below, would not)
+    assert seen_mid >= 5
 
 
 # ---------------------------------------------------------------------------
@@ -475,6 +479,159 @@ def test_ga_mutation_kinds_act_as_described():
     _valid(bo, base.M, base.K)
     changed = sum(not np.array_equal(bo["perm"][s], plain["perm"][s]) for s in range(Q, base.P))
     assert changed > (base.P - Q) * 0.9
+
+
+def _distinct_population(P, M, K, seed):
+    """P genomes with pairwise distinct orderings (so that an ordering names
+    its genome) and at least two replicas each; drawn by numpy."""
+    rng = np.random.default_rng(seed)
+    perms = set()
+    g = O.empty_genomes(P, M, K)
+    s = 0
+    while s < P:
+        perm = tuple(int(x) for x in rng.permutation(M))
+        R = int(rng.integers(2, K + 1))
+        cuts = tuple(sorted(int(x) for x in rng.choice(np.arange(1, M), R - 1, replace=False)))
+        if perm in perms:
+            continue
+        perms.add(perm)
+        edges = (0,) + cuts + (M,)
+        g["perm"][s] = perm
+        g["sizes"][s, :R] = np.diff(edges)
+        g["nclus"][s] = R
+        g["roles"][s] = int(rng.integers(0, 1 << R))
+        s += 1
+    return g
+
+
+def _same_genome(a, i, b, j):
+    return all(np.array_equal(a[k][i], b[k][j]) for k in ("perm", "sizes", "nclus", "roles"))
+
+
+def test_tournament_keeps_the_fittest():
+    # App. A selects parents "based on fitness": a tournament returns its best
+    # entrant.  One genome is strictly best; with 256 entrants per tournament
+    # over 16 genomes it is drawn with probability 1 - (15/16)^256 > 1 - 1e-7,
+    # so with no mutation both parents of every child are that genome and the
+    # child equals it (crossover of two copies, repair a no-op).  Keeping the
+    # worst entrant instead would clone the worst genome.
+    P, M, K = 16, 9, 4
+    g = _distinct_population(P, M, K, 31)
+    f = np.zeros((P, 4))
+    f[:, 0] = np.arange(P, 0, -1, dtype=float)      # genome P-1 is the best (w = 1)
+    best = P - 1
+    ga = O._ga_struct(P, M, K, 0, 256, 0.5, 0.0, (0.2, 0.5, 0.15, 0.15))
+    nxt = O.ga_step(ga, 4, 1, g, f, np.zeros(0, np.int32))
+    for s in range(P):
+        assert _same_genome(nxt, s, g, best)
+    # ties on w are broken by the bottleneck phase, then by the lower index
+    f[:, 0] = 1.0
+    f[:, 1] = 2.0
+    f[5, 1] = 1.5
+    nxt = O.ga_step(ga, 4, 1, g, f, np.zeros(0, np.int32))
+    assert all(_same_genome(nxt, s, g, 5) for s in range(P))
+    f[:, 1] = 2.0
+    nxt = O.ga_step(ga, 4, 1, g, f, np.zeros(0, np.int32))
+    assert all(_same_genome(nxt, s, g, 0) for s in range(P))
+
+
+def test_grouping_comes_whole_from_either_parent():
+    # Sec. 3.4: crossover recombines the ordering and inherits the grouping
+    # chromosome from one parent.  With p_cx = 0 the child's ordering is parent
+    # A's, with p_cx = 1 parent B's (the parent draws do not depend on p_cx), so
+    # the two runs name both parents of every child; the grouping and roles
+    # must then be A's or B's whole, and over many children each parent gives
+    # it about half the time (a fair coin).
+    P, M, K = 600, 12, 5
+    g = _distinct_population(P, M, K, 32)
+    rng = np.random.default_rng(33)
+    f = np.zeros((P, 4))
+    f[:, 0] = rng.permutation(P).astype(float)
+    order_of = {tuple(g["perm"][i]): i for i in range(P)}
+    ga0 = O._ga_struct(P, M, K, 0, 2, 0.0, 0.0, (0.2, 0.5, 0.15, 0.15))
+    ga1 = O._ga_struct(P, M, K, 0, 2, 1.0, 0.0, (0.2, 0.5, 0.15, 0.15))
+    none = np.zeros(0, np.int32)
+    a_run = O.ga_step(ga0, 8, 3, g, f, none)
+    b_run = O.ga_step(ga1, 8, 3, g, f, none)
+    from_b = both = 0
+    for s in range(P):
+        A = order_of[tuple(a_run["perm"][s])]
+        B = order_of[tuple(b_run["perm"][s])]
+        for run in (a_run, b_run):
+            src = [x for x in (A, B) if np.array_equal(run["sizes"][s], g["sizes"][x])
+                   and run["nclus"][s] == g["nclus"][x] and run["roles"][s] == g["roles"][x]]
+            assert src, "grouping and roles must come whole from a parent"
+        # the same coin in both runs: the grouping source does not depend on p_cx
+        assert np.array_equal(a_run["sizes"][s], b_run["sizes"][s])
+        if not np.array_equal(g["sizes"][A], g["sizes"][B]):
+            both += 1
+            from_b += np.array_equal(a_run["sizes"][s], g["sizes"][B])
+    assert both > 450
+    assert 0.42 < from_b / both < 0.58
+
+
+def test_regroup_from_a_position_keeps_the_prefix():
+    # App. A: "regenerates the grouping from a random position".  The replica r
+    # is uniform over the source's R replicas (word 2 of the mutation stream);
+    # replicas [0, r) keep their sizes and roles, the ordering is untouched, and
+    # the devices from replica r on are regrouped.  Most children (all with
+    # r >= 1) therefore keep a non-empty prefix.
+    P, M, K = 400, 40, 8
+    g = _distinct_population(P, M, K, 34)
+    rng = np.random.default_rng(35)
+    f = np.zeros((P, 4))
+    f[:, 0] = rng.permutation(P).astype(float)
+    none = np.zeros(0, np.int32)
+    plain = O.ga_step(O._ga_struct(P, M, K, 0, 4, 0.5, 0.0, (0.2, 0.5, 0.15, 0.15)), 6, 2, g, f, none)
+    rg = O.ga_step(O._ga_struct(P, M, K, 0, 4, 0.5, 1.0, (0.0, 1.0, 0.0, 0.0)), 6, 2, g, f, none)
+    _valid(rg, M, K)
+    kept_some = 0
+    for s in range(P):
+        assert np.array_equal(rg["perm"][s], plain["perm"][s])
+        R = int(plain["nclus"][s])
+        r = (O.word(6, 2, s, O.PURPOSE["MUTATE"], 2) * R) >> 32
+        assert np.array_equal(rg["sizes"][s][:r], plain["sizes"][s][:r])
+        mask = (1 << r) - 1
+        assert int(rg["roles"][s]) & mask == int(plain["roles"][s]) & mask
+        assert int(rg["nclus"][s]) >= r + 1
+        kept_some += r >= 1
+    # R >= 2 for every source, so r >= 1 for at least half of the children
+    assert kept_some > 0.5 * P
+
+
+def test_regroup_all_keeps_the_ordering():
+    # App. A's third mutation kind regenerates the grouping entirely and leaves
+    # the ordering as crossover made it; the fourth regenerates both.  With
+    # every mutation of the third kind, no ordering changes and (almost) every
+    # grouping does.
+    P, M, K = 300, 20, 6
+    g = _distinct_population(P, M, K, 36)
+    rng = np.random.default_rng(37)
+    f = np.zeros((P, 4))
+    f[:, 0] = rng.permutation(P).astype(float)
+    none = np.zeros(0, np.int32)
+    plain = O.ga_step(O._ga_struct(P, M, K, 0, 4, 0.5, 0.0, (0.2, 0.5, 0.15, 0.15)), 7, 5, g, f, none)
+    ra = O.ga_step(O._ga_struct(P, M, K, 0, 4, 0.5, 1.0, (0.0, 0.0, 1.0, 0.0)), 7, 5, g, f, none)
+    _valid(ra, M, K)
+    changed = 0
+    for s in range(P):
+        assert np.array_equal(ra["perm"][s], plain["perm"][s])
+        changed += not (np.array_equal(ra["sizes"][s], plain["sizes"][s]) and ra["roles"][s] == plain["roles"][s])
+    assert changed > 0.9 * P
+    # and the kind boundaries sit at the cumulative 0.2 / 0.7 / 0.85: with the
+    # paper's mix, a child mutated with a kind word in [0.7, 0.85) keeps its
+    # ordering, one with a word at or above 0.85 gets a new one
+    mix = O.ga_step(O._ga_struct(P, M, K, 0, 4, 0.5, 1.0, (0.2, 0.5, 0.15, 0.15)), 7, 5, g, f, none)
+    t2, t3 = O.threshold(0.7), O.threshold(0.85)
+    n3 = n4 = 0
+    for s in range(P):
+        kw = O.word(7, 5, s, O.PURPOSE["MUTATE"], 1)
+        if t2 <= kw < t3:
+            n3 += 1
+            assert np.array_equal(mix["perm"][s], plain["perm"][s])
+        elif kw >= t3:
+            n4 += not np.array_equal(mix["perm"][s], plain["perm"][s])
+    assert n3 > 20 and n4 > 20
 
 
 def test_crossover_mixes_both_parents_evenly():
