@@ -310,16 +310,34 @@ int e2_set_timing_events(e2_ctx *ctx, void *dp_start, void *dp_stop);
  *   fitness   [P][4] {w, phase, PS, DS} from e2_eval_population, DEVICE
  *   elite_idx [Q] output, DEVICE; may be NULL when Q == 0
  *   stream    cudaStream_t the work is enqueued on (asynchronous)
+ * The order is e2_ga_step's: w and phase compared as their bit patterns.
  * Returns E2_EINVAL for P > E2_NOALLOC_MAX_POP, other out-of-range sizes, null or
- * host pointers; E2_ECUDA if the scratch address cannot be obtained or a launch
- * fails.  The first call on each device looks up the scratch array's device
- * address with that device current; make that first call before any stream
- * capture.  All calls share the one scratch array and overwrite it; calls that
- * overlap on the GPU (other streams, other host threads) race and must be
- * serialised by the caller. */
+ * host pointers, or device memory of another GPU than the current one; E2_ECUDA
+ * if the scratch address cannot be obtained or a launch fails.  The first call
+ * on each device (and again the first after a reset of that device, which gives
+ * it a new context) looks up the scratch array's device address with that
+ * device current; make that first call before any stream capture.  All calls
+ * share the one scratch array and overwrite it; calls that overlap on the GPU
+ * (other streams, other host threads) race and must be serialised by the
+ * caller.  Cost: two O(P^2) passes over shared-memory tiles of the fitness
+ * keys, one warp per genome (the same shape as e2_ga_step's elites). */
 #define E2_NOALLOC_MAX_POP 65536
 int e2_select_elites_noalloc(const e2_genomes *pop, const double *fitness, int32_t P, int32_t M,
                              int32_t K_max, int32_t Q, int32_t *elite_idx, void *stream);
+
+/* Measurement hook (no counterpart in the paper): the integer issue rate of
+ * the instruction mix the DP_Pipe kernel is bound by, on the current device.
+ * One launch of a full-occupancy grid in which every thread runs 8
+ * independent chains of `iters` steps:
+ *   kind 0: unsigned 32-bit min and max (2 operations per chain and step);
+ *   kind 1: 32-bit adds (2 per step);
+ *   kind 2: the DP's mix -- min, max, compare, select, add (5 per step).
+ * *ops_per_launch receives the operations the launch executes and *ms_out its
+ * duration from CUDA events recorded on `stream` (a cudaStream_t; NULL = the
+ * legacy default stream) around it; the call synchronises on the second
+ * event.  Allocates no device memory.  E2_EINVAL for a kind outside 0..2,
+ * iters outside 1..2^24 or null outputs; E2_ECUDA on a CUDA failure. */
+int e2_probe_int_rate(int32_t kind, int32_t iters, void *stream, double *ops_per_launch, float *ms_out);
 
 /* Text of a status code, and the context's last detailed error message.  With
  * ctx == NULL: the message of the calling thread's last failed e2_create ("" if

@@ -17,20 +17,64 @@
 // it has to start at zero (each call writes every entry it reads), but two
 // calls that overlap on the GPU -- on different streams, or from different
 // host threads -- race on it and must be serialised by the caller.
+//
+// The duplicate test and the ranks follow the same order as e2_ga_step's
+// elites: fitness keys compared as the bit patterns of w and phase (the order
+// of the values for the non-negative and +inf results an evaluation produces,
+// and a total order for any other input), staged tile by tile in shared
+// memory with one warp per genome.
+#include <mutex>
+
 #include "e2ga_internal.cuh"
 
 namespace {
 
 constexpr int kNoallocMaxPop = E2_NOALLOC_MAX_POP;
 constexpr int kMaxDeviceIds = 64;
+constexpr int kTile = 1024;
+constexpr int kWarps = 8;
 
 // Scratch: [0, P) fingerprints (u64), then [P, 2P) duplicate flags (stored in
 // the low word of a u64 slot so that the array stays one type).
 static __device__ __align__(256) unsigned long long g_noalloc_scratch[2 * kNoallocMaxPop];
 
-// Device address of g_noalloc_scratch per device id, set up on the first call
-// made with that device current.
-unsigned long long *g_scratch_addr[kMaxDeviceIds] = {};
+// Device address of g_noalloc_scratch per device id, with the CUDA context
+// that was current when it was looked up (a reset device gets a new context,
+// and the address is looked up again).
+struct ScratchSlot {
+    void *ctx = nullptr;
+    unsigned long long *addr = nullptr;
+};
+ScratchSlot g_scratch[kMaxDeviceIds];
+std::mutex g_scratch_mutex;
+
+// cuCtxGetCurrent, reached through the runtime's entry-point table (no link
+// against the driver library).
+typedef int (*CtxGetCurrentFn)(void **);
+
+void *current_context()
+{
+    static CtxGetCurrentFn fn = nullptr;
+    static bool looked = false;
+    if (!looked) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<CtxGetCurrentFn>(p);
+        else
+            cudaGetLastError();
+        looked = true;
+    }
+    void *ctx = nullptr;
+    if (!fn || fn(&ctx) != 0) return nullptr;
+    return ctx;
+}
+
+__device__ __forceinline__ uint64_t key_bits(const double *fit, size_t i, int q)
+{
+    return (uint64_t)__double_as_longlong(fit[i * 4 + q]);
+}
 
 __global__ void fingerprint_noalloc(e2::DevPop p, int P, int M, int K, unsigned long long *hash)
 {
@@ -46,56 +90,94 @@ __global__ void fingerprint_noalloc(e2::DevPop p, int P, int M, int K, unsigned 
     hash[g] = h;
 }
 
-// Duplicate flag: equal to a lower-indexed genome (compared in full when the
-// fitness and fingerprint agree).
-__global__ void __launch_bounds__(256) dup_noalloc(e2::DevPop p, int P, int M, int K, const double *fit,
-                                                   const unsigned long long *hash, unsigned long long *dup)
+// Duplicate flag, one warp per genome: equal to a lower-indexed genome
+// (compared in full only where the fitness keys and the fingerprint agree).
+__global__ void __launch_bounds__(32 * kWarps) dup_noalloc(e2::DevPop p, int P, int M, int K, const double *fit,
+                                                           const unsigned long long *hash, unsigned long long *dup)
 {
-    const int g = blockIdx.x * blockDim.x + threadIdx.x;
-    if (g >= P) return;
-    const double w = fit[(size_t)g * 4], ph = fit[(size_t)g * 4 + 1];
-    const unsigned long long h = hash[g];
-    unsigned long long d = 0;
-    for (int o = 0; o < g && !d; ++o) {
-        if (hash[o] != h || fit[(size_t)o * 4] != w || fit[(size_t)o * 4 + 1] != ph) continue;
-        bool eq = p.nclus[o] == p.nclus[g] && p.roles[o] == p.roles[g];
-        for (int i = 0; i < M && eq; ++i) eq = p.perm[(size_t)o * M + i] == p.perm[(size_t)g * M + i];
-        for (int i = 0; i < K && eq; ++i) eq = p.sizes[(size_t)o * K + i] == p.sizes[(size_t)g * K + i];
-        d = eq;
+    __shared__ uint64_t s_w[kTile], s_p[kTile], s_h[kTile];
+    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
+    const int g = blockIdx.x * kWarps + wl;
+    const bool live = g < P;
+    const uint64_t w = live ? key_bits(fit, g, 0) : 0, ph = live ? key_bits(fit, g, 1) : 0;
+    const uint64_t h = live ? hash[g] : 0;
+    const int gmax = min(P, (int)(blockIdx.x + 1) * kWarps);
+    int d = 0;
+    for (int base = 0; base < gmax - 1; base += kTile) {
+        __syncthreads();
+        for (int t = threadIdx.x; t < kTile && base + t < P; t += blockDim.x) {
+            s_w[t] = key_bits(fit, base + t, 0);
+            s_p[t] = key_bits(fit, base + t, 1);
+            s_h[t] = hash[base + t];
+        }
+        __syncthreads();
+        if (!live || d) continue;
+        const int lim = min(kTile, g - base);
+        for (int t0 = 0; t0 < lim && !d; t0 += 32) {
+            const int t = t0 + lane;
+            const bool cand = t < lim && s_h[t] == h && s_w[t] == w && s_p[t] == ph;
+            unsigned b = __ballot_sync(0xFFFFFFFFu, cand);
+            while (b && !d) {
+                const int o = base + t0 + __ffs(b) - 1;
+                b &= b - 1;
+                bool diff = p.nclus[o] != p.nclus[g] || p.roles[o] != p.roles[g];
+                for (int i = lane; i < M && !diff; i += 32) diff = p.perm[(size_t)o * M + i] != p.perm[(size_t)g * M + i];
+                for (int i = lane; i < K && !diff; i += 32) diff = p.sizes[(size_t)o * K + i] != p.sizes[(size_t)g * K + i];
+                d = __ballot_sync(0xFFFFFFFFu, diff) == 0u;
+            }
+        }
     }
-    dup[g] = d;
+    if (live && lane == 0) dup[g] = (unsigned long long)d;
 }
 
-// rank(g) in the order (duplicate, w, phase, index); ranks below Q are elites.
-__global__ void __launch_bounds__(256) rank_noalloc(int P, int Q, const double *fit,
-                                                    const unsigned long long *dup, int32_t *elite)
+// rank(g) in the order (duplicate, w bits, phase bits, index), one warp per
+// genome over shared-memory tiles of the keys; ranks below Q are the elites.
+__global__ void __launch_bounds__(32 * kWarps) rank_noalloc(int P, int Q, const double *fit,
+                                                            const unsigned long long *dup, int32_t *elite)
 {
-    const int g = blockIdx.x * blockDim.x + threadIdx.x;
-    if (g >= P) return;
-    const unsigned long long dg = dup[g];
-    const double w = fit[(size_t)g * 4], ph = fit[(size_t)g * 4 + 1];
+    __shared__ uint64_t s_w[kTile], s_p[kTile];
+    __shared__ int s_d[kTile];
+    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
+    const int g = blockIdx.x * kWarps + wl;
+    const bool live = g < P;
+    const uint64_t w = live ? key_bits(fit, g, 0) : 0, ph = live ? key_bits(fit, g, 1) : 0;
+    const int dg = live ? (int)dup[g] : 0;
     int rank = 0;
-    for (int o = 0; o < P; ++o) {
-        const unsigned long long d = dup[o];
-        const double wo = fit[(size_t)o * 4], po = fit[(size_t)o * 4 + 1];
-        bool before;
-        if (d != dg) before = d < dg;
-        else if (wo != w) before = wo < w;
-        else if (po != ph) before = po < ph;
-        else before = o < g;
-        rank += before;
+    for (int base = 0; base < P; base += kTile) {
+        __syncthreads();
+        for (int t = threadIdx.x; t < kTile && base + t < P; t += blockDim.x) {
+            s_w[t] = key_bits(fit, base + t, 0);
+            s_p[t] = key_bits(fit, base + t, 1);
+            s_d[t] = (int)dup[base + t];
+        }
+        __syncthreads();
+        const int lim = min(kTile, P - base);
+        if (live)
+            for (int t = lane; t < lim; t += 32) {
+                const int o = base + t;
+                bool before;
+                if (s_d[t] != dg) before = s_d[t] < dg;
+                else if (s_w[t] != w) before = s_w[t] < w;
+                else if (s_p[t] != ph) before = s_p[t] < ph;
+                else before = o < g;
+                rank += before;
+            }
     }
-    if (rank < Q) elite[rank] = g;
+#pragma unroll
+    for (int x = 16; x; x >>= 1) rank += __shfl_xor_sync(0xFFFFFFFFu, rank, x);
+    if (live && lane == 0 && rank < Q) elite[rank] = g;
 }
 
-bool on_device(const void *p)
+// Device memory of device `dev` (or managed memory).
+bool on_device(const void *p, int dev)
 {
     cudaPointerAttributes a;
     if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
         cudaGetLastError();
         return false;
     }
-    return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+    if (a.type == cudaMemoryTypeManaged) return true;
+    return a.type == cudaMemoryTypeDevice && a.device == dev;
 }
 
 // Statuses only: this entry point keeps no error text.
@@ -112,26 +194,39 @@ extern "C" int e2_select_elites_noalloc(const e2_genomes *pop, const double *fit
     if (M < 1 || M > E2_MAX_DEVICES || K_max < 1 || K_max > E2_MAX_CLUSTERS || Q < 0 || Q > P)
         return reject(E2_EINVAL, "M, K_max or Q out of range");
     if (Q > 0 && !elite_idx) return reject(E2_EINVAL, "null output");
-    if (!on_device(pop->perm) || !on_device(pop->sizes) || !on_device(pop->nclus) || !on_device(pop->roles) ||
-        !on_device(fitness) || (Q > 0 && !on_device(elite_idx)))
-        return reject(E2_EINVAL, "inputs and output must be device memory of the current device");
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return reject(E2_ECUDA, "cudaGetDevice failed");
     if (dev < 0 || dev >= kMaxDeviceIds) return reject(E2_EINVAL, "device id beyond the supported range");
-    if (!g_scratch_addr[dev]) {
-        void *addr = nullptr;
-        const cudaError_t e = cudaGetSymbolAddress(&addr, g_noalloc_scratch);
-        if (e != cudaSuccess || !addr) return reject(E2_ECUDA, "cudaGetSymbolAddress of the scratch array failed");
-        g_scratch_addr[dev] = static_cast<unsigned long long *>(addr);
+    if (!on_device(pop->perm, dev) || !on_device(pop->sizes, dev) || !on_device(pop->nclus, dev) ||
+        !on_device(pop->roles, dev) || !on_device(fitness, dev) || (Q > 0 && !on_device(elite_idx, dev)))
+        return reject(E2_EINVAL, "inputs and output must be device memory of the current device");
+    unsigned long long *hash = nullptr;
+    {
+        // set-up, once per device and context: the scratch array's device
+        // address, looked up with that device current
+        std::lock_guard<std::mutex> lock(g_scratch_mutex);
+        void *ctx = current_context();
+        ScratchSlot &sl = g_scratch[dev];
+        if (!sl.addr || sl.ctx != ctx) {
+            void *addr = nullptr;
+            const cudaError_t e = cudaGetSymbolAddress(&addr, g_noalloc_scratch);
+            if (e != cudaSuccess || !addr) {
+                cudaGetLastError();
+                return reject(E2_ECUDA, "cudaGetSymbolAddress of the scratch array failed");
+            }
+            sl.addr = static_cast<unsigned long long *>(addr);
+            sl.ctx = ctx;
+        }
+        hash = sl.addr;
     }
-    unsigned long long *hash = g_scratch_addr[dev];
     unsigned long long *dup = hash + P;
     const e2::DevPop p{pop->perm, pop->sizes, pop->nclus, pop->roles};
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const unsigned blocks = (unsigned)((P + 255) / 256);
+    const unsigned wblocks = (unsigned)((P + kWarps - 1) / kWarps);
     fingerprint_noalloc<<<blocks, 256, 0, s>>>(p, P, M, K_max, hash);
-    dup_noalloc<<<blocks, 256, 0, s>>>(p, P, M, K_max, fitness, hash, dup);
-    if (Q > 0) rank_noalloc<<<blocks, 256, 0, s>>>(P, Q, fitness, dup, elite_idx);
+    dup_noalloc<<<wblocks, 32 * kWarps, 0, s>>>(p, P, M, K_max, fitness, hash, dup);
+    if (Q > 0) rank_noalloc<<<wblocks, 32 * kWarps, 0, s>>>(P, Q, fitness, dup, elite_idx);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return reject(E2_ECUDA, cudaGetErrorString(e));
     return E2_OK;

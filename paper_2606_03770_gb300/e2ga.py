@@ -80,6 +80,7 @@ SIGNATURES = {
     "e2_get_results": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "e2_select_elites_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
                                             C.c_int32, C.c_void_p, C.c_void_p]),
+    "e2_probe_int_rate": (C.c_int, [C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p]),
     "e2_strerror": (C.c_char_p, [C.c_int]),
     "e2_last_error": (C.c_char_p, [C.c_void_p]),
 }
@@ -178,6 +179,13 @@ def e2_set_timing_events(ctx, start_ptr, stop_ptr):
 
 def e2_select_elites_noalloc(genomes, fitness_ptr, P, M, K_max, Q, elite_ptr, stream_ptr):
     return load().e2_select_elites_noalloc(C.byref(genomes), fitness_ptr, P, M, K_max, Q, elite_ptr, stream_ptr)
+
+
+def e2_probe_int_rate(kind, iters, stream_ptr):
+    """(status, operations executed, milliseconds) of one probe launch."""
+    ops, ms = C.c_double(), C.c_float()
+    st = load().e2_probe_int_rate(kind, iters, stream_ptr, C.byref(ops), C.byref(ms))
+    return st, ops.value, ms.value
 
 
 def e2_strerror(status):
