@@ -110,10 +110,28 @@ typedef struct {
     int32_t role_search;    /* 0: each replica's role is a bit of the genome;   */
                             /* 1: Alg. 2's brute-force role assignment: every   */
                             /* replica is evaluated in both roles, the best of  */
-                            /* the 2^R assignments (least w, then phase, then   */
-                            /* smallest mask) is taken and written back into    */
-                            /* the genome's role bits.  Needs K_max <=          */
-                            /* E2_MAX_ROLE_SEARCH and b_max <= 63.              */
+                            /* the 2^R assignments (least objective, then       */
+                            /* phase, then smallest mask) is taken and written  */
+                            /* back into the genome's role bits.  Needs K_max   */
+                            /* <= E2_MAX_ROLE_SEARCH and b_max <= 63.           */
+                            /* 2: the adapted-SplitWise rule of the paper's     */
+                            /* comparison (Sec. 4.2 "Baseline chosen"): both    */
+                            /* roles evaluated; the n_P strongest replicas      */
+                            /* (prefill throughput NP/T, ties to the lower      */
+                            /* index; a replica that cannot prefill is the      */
+                            /* weakest) prefill, the rest decode, with          */
+                            /* n_P = R*NP/(NP+ND) rounded half up, clamped to   */
+                            /* [1, R-1] (R = 1: 1); the roles are written back  */
+                            /* into the genome.  Needs b_max <= 63.             */
+    int32_t objective;      /* fitness[0] of a genome: 0 the waiting time w of  */
+                            /* Eq. 3-5; 1 the per-request finishing time of the */
+                            /* FT comparison (Sec. 2, Sec. 4.2: HexGen-2's      */
+                            /* objective), FT = (sum_P PS_c Lambda_c) / PS +    */
+                            /* ND (sum_D DS_c Lambda_c) / DS, the sums in       */
+                            /* ascending replica order (+inf when PS or DS is   */
+                            /* 0).  Either way fitness[1] is Eq. 3's phase and  */
+                            /* the fitness order is (fitness[0], fitness[1],    */
+                            /* index).                                          */
 } e2_params;
 
 /* A population in the layout above; "host or device" pointers. */
@@ -225,8 +243,9 @@ int e2_init_population(e2_ctx *ctx, uint64_t seed);
  * sweep, and the objective of Eq. 3-5.  `genomes` (host or device) replaces
  * the current population when not NULL (validated like e2_set_population);
  * NULL evaluates the current one.  fitness_out [P][4] = {w, phase, PS, DS}
- * (host or device, may be NULL); `parts` may be NULL.  The results also stay
- * in the context for e2_ga_step. */
+ * (host or device, may be NULL; fitness[0] is the objective e2_params.objective
+ * selects); `parts` may be NULL.  The results also stay in the context for
+ * e2_ga_step. */
 int e2_eval_population(e2_ctx *ctx, const e2_genomes *genomes, double *fitness_out,
                        const e2_partitions *parts);
 

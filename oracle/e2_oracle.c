@@ -15,8 +15,12 @@
  *   per-request latency Lambda     Sec. 3.2 (text after Alg. 1)
  *   prefill / decode evaluation    Alg. 2 (replica loop, b sweep)
  *   role assignment by brute force Alg. 2 (optional)
+ *   role assignment by the adapted-SplitWise rule
+ *                                  Sec. 4.2 "Baseline chosen" (optional)
  *   objective Eq. 3, 4, 5 and the multi-replica aggregation
  *                                  Sec. 3.3
+ *   finishing-time objective (HexGen-2's, the FT baseline)
+ *                                  Sec. 2, Sec. 4.2 (optional)
  *   GA: gene, crossover + repair, mutation mixture, elites
  *                                  Sec. 3.4, App. A
  *   Philox-4x32-10 counter-based generator
@@ -48,7 +52,10 @@ typedef struct {
     uint64_t NP, ND;
     double min_tps, t_a;
     int role_search;             /* 0: roles from the genome; 1: Alg. 2's     */
-                                 /* brute force over every role assignment    */
+                                 /* brute force over every role assignment;   */
+                                 /* 2: adapted SplitWise (strongest prefill)  */
+    int objective;               /* 0: waiting time w (Eq. 3-5); 1: per-      */
+                                 /* request finishing time FT                 */
 } orc_problem;
 
 /* ------------------------------------------------------------------------ */
@@ -203,24 +210,47 @@ int orc_eval_cluster(const orc_problem *p, const uint16_t *devs, int m, int deco
 
 /* Objective (Sec. 3.3): PS and DS are summed over the replicas of each role
  * in ascending replica order; Eq. 3 bottleneck phase, Eq. 4 backlog, Eq. 5
- * per-request waiting time.  No prefill or no decode capacity: +inf. */
-void orc_score(const orc_problem *p, int R, const uint64_t roles, const double *T,
+ * per-request waiting time.  No prefill or no decode capacity: +inf.
+ *
+ * With objective 1 the first fitness entry is instead the per-request
+ * finishing time that HexGen-2 minimises (Sec. 2: a sum of computation and
+ * communication time; Sec. 4.2: the FT baseline keeps the planner and swaps
+ * the objective).  A request spends Lambda_c, the end-to-end pass latency of
+ * its prefill replica c (every stage and link time added), in prefill, and ND
+ * passes of Lambda_c' on its decode replica c'.  Requests are routed in
+ * proportion to the replicas' rates (PS_c = NP/T_c, DS_c = b_c/T_c), so the
+ * expected finishing time is
+ *     FT = (sum_P PS_c * Lambda_c) / PS + ND * ((sum_D DS_c * Lambda_c) / DS),
+ * the sums in ascending replica order.  The phase of Eq. 3 stays the second
+ * key. */
+void orc_score(const orc_problem *p, int R, const uint64_t roles, const double *T, const double *L,
                const int16_t *bsel, double fit[4])
 {
-    double PS = 0.0, DS = 0.0;
+    double PS = 0.0, DS = 0.0, PL = 0.0, DL = 0.0;
     for (int c = 0; c < R; ++c) {
         if (bsel[c] < 0) continue;
-        if (((roles >> c) & 1u) == 0) PS = PS + (double)p->NP / T[c];
-        else DS = DS + (double)bsel[c] / T[c];
+        if (((roles >> c) & 1u) == 0) {
+            double r = (double)p->NP / T[c];
+            PS = PS + r;
+            PL = PL + r * L[c];
+        } else {
+            double r = (double)bsel[c] / T[c];
+            DS = DS + r;
+            DL = DL + r * L[c];
+        }
     }
     double w = ORC_INF, phase = ORC_INF;
     if (PS != 0.0 && DS != 0.0) {
         double tp = (double)p->NP / PS;
         double td = (double)p->ND / DS;
         phase = dmax(tp, td);                              /* Eq. 3 */
-        double x = phase - p->t_a;
-        double bn = x > 0.0 ? x : 0.0;                     /* Eq. 4 */
-        w = bn > 0.0 ? tp + bn : 0.0;                      /* Eq. 5 */
+        if (p->objective == 1) {
+            w = PL / PS + (double)p->ND * (DL / DS);       /* finishing time */
+        } else {
+            double x = phase - p->t_a;
+            double bn = x > 0.0 ? x : 0.0;                 /* Eq. 4 */
+            w = bn > 0.0 ? tp + bn : 0.0;                  /* Eq. 5 */
+        }
     }
     fit[0] = w; fit[1] = phase; fit[2] = PS; fit[3] = DS;
 }
@@ -245,7 +275,7 @@ void orc_eval_genome(const orc_problem *p, int K, const uint16_t *perm, const ui
         T[c] = Tc; L[c] = Lc; master[c] = (int16_t)mu; bsel[c] = (int16_t)b;
         off += m;
     }
-    orc_score(p, R, roles, T, bsel, fit);
+    orc_score(p, R, roles, T, L, bsel, fit);
 }
 
 /* Alg. 2 with its role search: every replica is evaluated in both roles
@@ -276,14 +306,15 @@ void orc_eval_genome_roles(const orc_problem *p, int K, const uint16_t *perm, co
     double bw = ORC_INF, bp = ORC_INF;
     int have = 0;
     for (uint64_t mask = 0; mask < ((uint64_t)1 << R); ++mask) {
-        double Tm[64], f[4];
+        double Tm[64], Lm[64], f[4];
         int16_t bm[64];
         for (int c = 0; c < R; ++c) {
             const int role = (int)((mask >> c) & 1u);
             Tm[c] = Tr[role][c];
+            Lm[c] = Lr[role][c];
             bm[c] = (int16_t)br[role][c];
         }
-        orc_score(p, R, mask, Tm, bm, f);
+        orc_score(p, R, mask, Tm, Lm, bm, f);
         if (!have || f[0] < bw || (f[0] == bw && f[1] < bp)) {
             have = 1; bw = f[0]; bp = f[1]; best = mask;
         }
@@ -295,8 +326,74 @@ void orc_eval_genome_roles(const orc_problem *p, int K, const uint16_t *perm, co
         for (int k = 0; k < sizes[c]; ++k) layers[off + k] = lay[role][off + k];
         off += sizes[c];
     }
-    orc_score(p, R, best, T, bsel, fit);
+    orc_score(p, R, best, T, L, bsel, fit);
     *roles_out = best;
+    free(lay[0]);
+    free(lay[1]);
+}
+
+/* Number of prefill replicas of the adapted-SplitWise rule: SplitWise sizes
+ * each phase's pool by the input-to-generated token ratio, so R replicas split
+ * as NP : ND, rounded half up, with at least one replica in each role (one
+ * replica: prefill). */
+int orc_splitwise_prefill_count(uint64_t NP, uint64_t ND, int R)
+{
+    if (R <= 1) return R;
+    uint64_t den = NP + ND;
+    int n = (int)((2 * (uint64_t)R * NP + den) / (2 * den));
+    if (n < 1) n = 1;
+    if (n > R - 1) n = R - 1;
+    return n;
+}
+
+/* Adapted SplitWise (Sec. 4.2, "Baseline chosen"): every replica is
+ * evaluated in both roles; within the genome the strongest replicas take the
+ * prefill role and the rest decode.  A replica's strength is its prefill
+ * throughput NP/T from its prefill partition (the quantity that exists only
+ * after partitioning, Sec. 2); a replica that cannot serve prefill is the
+ * weakest.  Ties go to the lower replica index.  The prefill count is
+ * orc_splitwise_prefill_count.  The chosen roles are written to *roles_out. */
+void orc_eval_genome_splitwise(const orc_problem *p, int K, const uint16_t *perm, const uint16_t *sizes,
+                               int R, double fit[4], int16_t *layers, int16_t *master, int16_t *bsel,
+                               double *T, double *L, uint64_t *cand, uint64_t *roles_out)
+{
+    double Tr[2][64], Lr[2][64];
+    int mur[2][64], br[2][64];
+    int ok[2][64];
+    int16_t *lay[2];
+    lay[0] = (int16_t *)malloc(sizeof(int16_t) * (size_t)p->M);
+    lay[1] = (int16_t *)malloc(sizeof(int16_t) * (size_t)p->M);
+    int off = 0;
+    for (int c = 0; c < K; ++c) {
+        master[c] = -1; bsel[c] = -1; T[c] = ORC_INF; L[c] = ORC_INF;
+    }
+    for (int c = 0; c < R; ++c) {
+        for (int role = 0; role < 2; ++role)
+            ok[role][c] = orc_eval_cluster(p, perm + off, sizes[c], role, &Tr[role][c], &Lr[role][c],
+                                           &mur[role][c], &br[role][c], lay[role] + off, cand);
+        off += sizes[c];
+    }
+    const int nP = orc_splitwise_prefill_count(p->NP, p->ND, R);
+    uint64_t roles = 0;
+    for (int c = 0; c < R; ++c) {
+        double sc = ok[0][c] ? (double)p->NP / Tr[0][c] : -1.0;
+        int rank = 0;                          /* replicas stronger than c, ties to the lower index */
+        for (int o = 0; o < R; ++o) {
+            if (o == c) continue;
+            double so = ok[0][o] ? (double)p->NP / Tr[0][o] : -1.0;
+            if (so > sc || (so == sc && o < c)) ++rank;
+        }
+        if (rank >= nP) roles |= (uint64_t)1 << c;
+    }
+    off = 0;
+    for (int c = 0; c < R; ++c) {
+        const int role = (int)((roles >> c) & 1u);
+        T[c] = Tr[role][c]; L[c] = Lr[role][c]; master[c] = (int16_t)mur[role][c]; bsel[c] = (int16_t)br[role][c];
+        for (int k = 0; k < sizes[c]; ++k) layers[off + k] = lay[role][off + k];
+        off += sizes[c];
+    }
+    orc_score(p, R, roles, T, L, bsel, fit);
+    *roles_out = roles;
     free(lay[0]);
     free(lay[1]);
 }
@@ -313,7 +410,12 @@ void orc_eval_population(const orc_problem *p, int P, int K, const uint16_t *per
 #endif
     for (int g = 0; g < P; ++g) {
         uint64_t c = 0;
-        if (p->role_search)
+        if (p->role_search == 2)
+            orc_eval_genome_splitwise(p, K, perm + (size_t)g * M, sizes + (size_t)g * K, nclus[g],
+                                      fitness + (size_t)g * 4, layers + (size_t)g * M, master + (size_t)g * K,
+                                      bsel + (size_t)g * K, T + (size_t)g * K, L + (size_t)g * K, &c,
+                                      roles_out + g);
+        else if (p->role_search)
             orc_eval_genome_roles(p, K, perm + (size_t)g * M, sizes + (size_t)g * K, nclus[g],
                                   fitness + (size_t)g * 4, layers + (size_t)g * M, master + (size_t)g * K,
                                   bsel + (size_t)g * K, T + (size_t)g * K, L + (size_t)g * K, &c,

@@ -42,7 +42,8 @@ class _Problem(C.Structure):
                 ("blk_flops", C.c_void_p), ("blk_bytes", C.c_void_p), ("blk_mem", C.c_void_p),
                 ("head_flops", C.c_void_p), ("head_bytes", C.c_void_p), ("head_mem", C.c_void_p),
                 ("act_bytes", C.c_void_p), ("NP", C.c_uint64), ("ND", C.c_uint64),
-                ("min_tps", C.c_double), ("t_a", C.c_double), ("role_search", C.c_int)]
+                ("min_tps", C.c_double), ("t_a", C.c_double), ("role_search", C.c_int),
+                ("objective", C.c_int)]
 
 
 class _GA(C.Structure):
@@ -68,7 +69,10 @@ def lib():
         _lib.orc_eval_cluster.argtypes = [C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_void_p,
                                           C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]
         _lib.orc_score.restype = None
-        _lib.orc_score.argtypes = [C.c_void_p, C.c_int, C.c_uint64, C.c_void_p, C.c_void_p, C.c_void_p]
+        _lib.orc_score.argtypes = [C.c_void_p, C.c_int, C.c_uint64, C.c_void_p, C.c_void_p, C.c_void_p,
+                                   C.c_void_p]
+        _lib.orc_splitwise_prefill_count.restype = C.c_int
+        _lib.orc_splitwise_prefill_count.argtypes = [C.c_uint64, C.c_uint64, C.c_int]
         _lib.orc_eval_population.restype = None
         _lib.orc_eval_population.argtypes = [C.c_void_p, C.c_int, C.c_int] + [C.c_void_p] * 11 + [C.c_int,
                                                                                                    C.c_void_p]
@@ -114,7 +118,8 @@ class OracleProblem:
         self.s = _Problem(prob.M, prob.N, prob.V, *[_p(a[k]) for k in
                           ("rate", "bw", "mem", "link_bw", "cong", "blk_flops", "blk_bytes",
                            "blk_mem", "head_flops", "head_bytes", "head_mem", "act_bytes")],
-                          prob.NP, prob.ND, prob.min_tps, prob.t_a, int(getattr(prob, "role_search", 0)))
+                          prob.NP, prob.ND, prob.min_tps, prob.t_a, int(getattr(prob, "role_search", 0)),
+                          int(getattr(prob, "objective", 0)))
 
     def set_cong(self, cong):
         self.arrays["cong"] = np.ascontiguousarray(cong, dtype=np.float64)
@@ -155,11 +160,12 @@ class OracleProblem:
                                     C.byref(mu), C.byref(b), _p(layers), None)
         return dict(ok=bool(ok), T=T.value, L=L.value, mu=mu.value, b=b.value, layers=layers[:m].copy())
 
-    def score(self, roles, T, bsel):
+    def score(self, roles, T, bsel, L=None):
         T = np.ascontiguousarray(T, dtype=np.float64)
+        L = np.ascontiguousarray(np.zeros(len(T)) if L is None else L, dtype=np.float64)
         bsel = np.ascontiguousarray(bsel, dtype=np.int16)
         fit = np.zeros(4, np.float64)
-        lib().orc_score(self.ref, len(T), int(roles), _p(T), _p(bsel), _p(fit))
+        lib().orc_score(self.ref, len(T), int(roles), _p(T), _p(L), _p(bsel), _p(fit))
         return fit
 
     def eval_population(self, genomes, K, nthreads=1):
@@ -247,6 +253,10 @@ def repair(perm):
     seen = np.zeros(len(cp), np.uint8)
     lib().orc_repair(_p(cp), len(cp), _p(seen))
     return cp
+
+
+def splitwise_prefill_count(NP, ND, R):
+    return lib().orc_splitwise_prefill_count(NP, ND, R)
 
 
 def num_threads():

@@ -775,6 +775,31 @@ __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop
     dp_eval_body<uint32_t>(dm, tb, pop, out, wl, si, so, cls);
 }
 
+// The genome's objective from the role sums (PS, DS; PL, DL the rate-weighted
+// latencies sum_P PS_c Lambda_c and sum_D DS_c Lambda_c, all summed in
+// ascending replica order).  Objective 0: Eq. 3 bottleneck phase, Eq. 4
+// backlog, Eq. 5 waiting time.  Objective 1: the per-request finishing time of
+// the FT comparison, a request's prefill pass plus ND decode passes, each
+// averaged over its role's replicas in proportion to their rates.  Either way
+// the second key is Eq. 3's phase; no prefill or no decode capacity: +inf.
+__device__ __forceinline__ void objective(const Dims &dm, double PS, double DS, double PL, double DL, double &w,
+                                          double &phase)
+{
+    w = keyd(kInfKey);
+    phase = keyd(kInfKey);
+    if (PS != 0.0 && DS != 0.0) {
+        const double tp = (double)dm.NP / PS, td = (double)dm.ND / DS;
+        phase = tp >= td ? tp : td;                 // Eq. 3
+        if (dm.objective == 1) {
+            w = PL / PS + (double)dm.ND * (DL / DS);
+        } else {
+            const double x = phase - dm.t_a;
+            const double bn = x > 0.0 ? x : 0.0;    // Eq. 4
+            w = bn > 0.0 ? tp + bn : 0.0;           // Eq. 5
+        }
+    }
+}
+
 // One warp per genome.  Each replica that had work gets its outputs from its
 // lane: the largest accepted variant is the sweep's answer (Alg. 2 keeps the
 // highest feasible batch), with its master, batch and times, and the serving
@@ -806,13 +831,14 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
         for (int i = lane; i < M; i += 32) hl = mix(hl, pp[i]);
     }
     unsigned long long n_rep = 0, n_served = 0, n_paper = 0;
-    double rate[2];
+    double rate[2], lat[2];
     int kind[2];                                   // -1 none, 0 prefill, 1 decode
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
         const int c = lane + 32 * h;
         kind[h] = -1;
         rate[h] = 0.0;
+        lat[h] = 0.0;
         if (c < R) {
             const int slot = g * K + c;
             const uint64_t mask = si.mask[slot];
@@ -832,7 +858,8 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
                     out.master[slot] = so.mu[sv];
                     out.bsel[slot] = (int16_t)(role ? best + 1 : 0);
                     out.T[slot] = T;
-                    out.L[slot] = so.L[sv];
+                    lat[h] = so.L[sv];
+                    out.L[slot] = lat[h];
                     if (role) nrun = (unsigned long long)(dm.b_max - best);   // variants b_max .. best+1
                     ++n_served;
                     kind[h] = role;
@@ -870,13 +897,14 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
         atomicAdd(&out.stats[kStPaper], n_paper);
         if (n_served) atomicAdd(&out.stats[kStServed], n_served);
     }
-    double PS = 0.0, DS = 0.0;
+    double PS = 0.0, DS = 0.0, PL = 0.0, DL = 0.0;   // PL, DL: rate-weighted latencies (finishing time)
     for (int c = 0; c < R; ++c) {
         const int h = c >> 5;
         const double x = __shfl_sync(0xFFFFFFFFu, h ? rate[1] : rate[0], c & 31);
+        const double l = __shfl_sync(0xFFFFFFFFu, h ? lat[1] : lat[0], c & 31);
         const int k = __shfl_sync(0xFFFFFFFFu, h ? kind[1] : kind[0], c & 31);
-        if (k == 0) PS = PS + x;
-        else if (k == 1) DS = DS + x;
+        if (k == 0) { PS = PS + x; PL = PL + x * l; }
+        else if (k == 1) { DS = DS + x; DL = DL + x * l; }
     }
     // fingerprint: lanes mixed interleaved slices of the ordering; a tree fold,
     // then the sizes in replica order (from the lanes that hold them)
@@ -891,14 +919,8 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
         h = mix(h, (uint64_t)si_ << 16);
     }
     if (lane != 0) return;
-    double w = keyd(kInfKey), phase = keyd(kInfKey);
-    if (PS != 0.0 && DS != 0.0) {
-        const double tp = (double)dm.NP / PS, td = (double)dm.ND / DS;
-        phase = tp >= td ? tp : td;                 // Eq. 3
-        const double x = phase - dm.t_a;
-        const double bn = x > 0.0 ? x : 0.0;        // Eq. 4
-        w = bn > 0.0 ? tp + bn : 0.0;               // Eq. 5
-    }
+    double w, phase;
+    objective(dm, PS, DS, PL, DL, w, phase);
     double *f = out.fit + (size_t)g * 4;
     f[0] = w; f[1] = phase; f[2] = PS; f[3] = DS;
     h = mix(h, (uint64_t)R << 40);
@@ -914,11 +936,12 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
 // genome (PS and DS summed in ascending replica order over the replicas that
 // serve their role); the least (w, phase, r) wins.  The replicas' outputs are those of their chosen roles,
 // the chosen roles are written into the genome, and the genome is scored.
-template <int WPG>
+template <int WPG, bool FT>
 __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop, SlotInfo si, SplitOut so,
                                                              EvalOut out)
 {
     __shared__ double s_ps[4][E2_MAX_ROLE_SEARCH], s_ds[4][E2_MAX_ROLE_SEARCH];
+    __shared__ double s_pl[4][E2_MAX_ROLE_SEARCH], s_dl[4][E2_MAX_ROLE_SEARCH];   // rate x Lambda (FT)
     __shared__ int s_pv[4][E2_MAX_ROLE_SEARCH], s_dv[4][E2_MAX_ROLE_SEARCH];
     __shared__ int s_off[4][E2_MAX_ROLE_SEARCH + 1], s_code[4][E2_MAX_ROLE_SEARCH];
     __shared__ long long s_qp[4][E2_MAX_ROLE_SEARCH], s_qd[4][E2_MAX_ROLE_SEARCH];
@@ -936,26 +959,27 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     const int K = dm.K, M = dm.M, V = dm.V, bp = dm.b_max;
     const int R = pop.nclus[g];
     const uint64_t roles0 = pop.roles[g];
-    // Eq. 3-5 for assignment r, PS and DS summed in ascending replica order
-    // from replica c0 on, the sums over replicas 0..c0-1 given
-    auto score_from = [&](uint64_t r, int c0, double PS0, double DS0, double &PS, double &DS, double &w,
+    // the objective of assignment r, PS and DS (and, for the finishing time,
+    // the rate-weighted latencies) summed in ascending replica order from
+    // replica c0 on, the sums over replicas 0..c0-1 given
+    constexpr bool ft = FT;                            // objective 1: the finishing time
+    auto score_from = [&](uint64_t r, int c0, const double *pre, double &PS, double &DS, double &w,
                           double &phase) {
-        PS = PS0; DS = DS0;
+        PS = pre[0]; DS = pre[1];
+        double PL = pre[2], DL = pre[3];
         for (int c = c0; c < R; ++c) {
-            if ((r >> c) & 1ull) { if (s_dv[gw][c]) DS = DS + s_ds[gw][c]; }
-            else if (s_pv[gw][c]) PS = PS + s_ps[gw][c];
+            if ((r >> c) & 1ull) {
+                if (s_dv[gw][c]) { DS = DS + s_ds[gw][c]; if (ft) DL = DL + s_dl[gw][c]; }
+            } else if (s_pv[gw][c]) {
+                PS = PS + s_ps[gw][c];
+                if (ft) PL = PL + s_pl[gw][c];
+            }
         }
-        w = keyd(kInfKey); phase = keyd(kInfKey);
-        if (PS != 0.0 && DS != 0.0) {
-            const double tp = (double)dm.NP / PS, td = (double)dm.ND / DS;
-            phase = tp >= td ? tp : td;                 // Eq. 3
-            const double x = phase - dm.t_a;
-            const double bn = x > 0.0 ? x : 0.0;        // Eq. 4
-            w = bn > 0.0 ? tp + bn : 0.0;               // Eq. 5
-        }
+        objective(dm, PS, DS, PL, DL, w, phase);
     };
+    const double zero4[4] = {0.0, 0.0, 0.0, 0.0};
     auto score = [&](uint64_t r, double &PS, double &DS, double &w, double &phase) {
-        score_from(r, 0, 0.0, 0.0, PS, DS, w, phase);
+        score_from(r, 0, zero4, PS, DS, w, phase);
     };
     // ---- each replica's two results
     int best = -1, pok = 0, m = 0;
@@ -970,6 +994,8 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
         s_dv[gw][lane] = best >= 0;
         s_ps[gw][lane] = pok ? (double)dm.NP / so.T[(size_t)slot * V + bp] : 0.0;
         s_ds[gw][lane] = best >= 0 ? (double)(best + 1) / so.T[(size_t)slot * V + best] : 0.0;
+        s_pl[gw][lane] = pok ? s_ps[gw][lane] * so.L[(size_t)slot * V + bp] : 0.0;
+        s_dl[gw][lane] = best >= 0 ? s_ds[gw][lane] * so.L[(size_t)slot * V + best] : 0.0;
     }
     if (lead && lane == 0) s_off[gw][R] = M;
     if (WPG == 1) __syncwarp();
@@ -1002,7 +1028,8 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     double totp = 0.0, totd = 0.0;
     for (int c = 0; c < R; ++c) { totp = totp + s_ps[gw][c]; totd = totd + s_ds[gw][c]; }
     const int sp_ = totp > 0.0 ? 61 - ilogb(totp) : 0, sd_ = totd > 0.0 ? 61 - ilogb(totd) : 0;
-    bool in_range = isfinite(totp) && isfinite(totd) && sp_ > -126 + 64 && sp_ < 126 && sd_ > -126 + 64 &&
+    // the screens bound the waiting time; the finishing time is scored exactly
+    bool in_range = !ft && isfinite(totp) && isfinite(totd) && sp_ > -126 + 64 && sp_ < 126 && sd_ > -126 + 64 &&
                     sd_ < 126;
     if (lane < R) {
         const long long qp = in_range && s_pv[gw][lane] ? __double2ll_rn(ldexp(s_ps[gw][lane], sp_)) : 0ll;
@@ -1058,7 +1085,8 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
         // one assignment: the screens, then the exact score where they cannot decide
         // with a block per genome the roles of replicas 0..low+U-1 are fixed per
         // thread and combination: their exact sums are taken once (prefix)
-        double preP[4] = {0.0, 0.0, 0.0, 0.0}, preD[4] = {0.0, 0.0, 0.0, 0.0};
+        double pre[4][4] = {{0.0, 0.0, 0.0, 0.0}, {0.0, 0.0, 0.0, 0.0}, {0.0, 0.0, 0.0, 0.0},
+                            {0.0, 0.0, 0.0, 0.0}};     // [combination][PS, DS, PL, DL]
         auto consider = [&](long long P, long long D, int np, int nd, uint64_t r, int j) {
             if (np == 0 || nd == 0) {                              // PS or DS is 0: w = phase = +inf
                 if (!own_fin && r < br) br = r;                    // ties the own best only while it is +inf
@@ -1072,7 +1100,7 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
                 if (w_lo > bw_up || (zero && ph_lo > bph_up)) return;
             }
             double PS, DS, w, ph;
-            if (WPG > 1) score_from(r, low + 2, preP[j], preD[j], PS, DS, w, ph);
+            if (WPG > 1) score_from(r, low + 2, pre[j], PS, DS, w, ph);
             else score(r, PS, DS, w, ph);
             if (w < bw || (w == bw && (ph < bph || (ph == bph && r < br)))) {
                 bw = w; bph = ph; br = r;
@@ -1088,8 +1116,15 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
             for (int j = 0; j < 4; ++j)
                 for (int c = 0; c < low + 2; ++c) {
                     const bool dec = c < low ? ((id >> c) & 1) : ((j >> (c - low)) & 1);
-                    if (dec) { if (s_dv[gw][c]) preD[j] = preD[j] + s_ds[gw][c]; }
-                    else if (s_pv[gw][c]) preP[j] = preP[j] + s_ps[gw][c];
+                    if (dec) {
+                        if (s_dv[gw][c]) {
+                            pre[j][1] = pre[j][1] + s_ds[gw][c];
+                            if (ft) pre[j][3] = pre[j][3] + s_dl[gw][c];
+                        }
+                    } else if (s_pv[gw][c]) {
+                        pre[j][0] = pre[j][0] + s_ps[gw][c];
+                        if (ft) pre[j][2] = pre[j][2] + s_pl[gw][c];
+                    }
                 }
         long long dP[2] = {0, 0}, dD[2] = {0, 0};
         int dn[2] = {0, 0}, dm_[2] = {0, 0};
@@ -1248,6 +1283,156 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     atomicAdd(&out.stats[kStGenomes], 1ull);
 }
 
+// The adapted-SplitWise rule of the paper's comparison (Sec. 4.2, "Baseline
+// chosen"), one warp per genome; lane l holds replicas l and l + 32.  Every
+// replica was evaluated in both roles (as for the role search): its prefill
+// run (variant bit b_max, present when the memory allows) and its decode
+// sweep's answer (the largest accepted batch).  A replica's strength is its
+// prefill throughput NP/T (-1 when it cannot prefill); the n_P strongest
+// replicas prefill (ties to the lower index), the rest decode, with
+// n_P = R NP / (NP + ND) rounded half up and clamped to [1, R-1] (R = 1: 1).
+// The replicas' outputs are those of their roles, the roles are written into
+// the genome, and the genome is scored.
+__global__ void __launch_bounds__(128) finalize_splitwise_kernel(Dims dm, DevPop pop, SlotInfo si, SplitOut so,
+                                                                 EvalOut out)
+{
+    __shared__ int s_off[4][E2_MAX_CLUSTERS + 1];     // replica start in the ordering
+    __shared__ int s_code[4][E2_MAX_CLUSTERS];        // variant bit of the chosen role's result, -1 none
+    const int wl = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = blockIdx.x * 4 + wl;
+    if (g >= dm.P) return;
+    const int K = dm.K, M = dm.M, V = dm.V, bp = dm.b_max;
+    const int R = pop.nclus[g];
+    double strength[2];
+    int pok[2], best[2], m[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int c = lane + 32 * h;
+        strength[h] = -1.0;
+        pok[h] = 0;
+        best[h] = -1;
+        m[h] = 0;
+        if (c < R) {
+            const int slot = g * K + c;
+            const uint64_t mask = si.mask[slot];
+            m[h] = pop.sizes[slot];
+            pok[h] = (int)((mask >> bp) & 1ull);
+            best[h] = mask ? si.best[slot] : -1;
+            s_off[wl][c] = si.off[slot];
+            if (pok[h]) strength[h] = (double)dm.NP / so.T[(size_t)slot * V + bp];
+        }
+    }
+    if (lane == 0) s_off[wl][R] = M;
+    // prefill count from the token ratio, in integers
+    int nP = R;
+    if (R > 1) {
+        const uint64_t den = dm.NP + dm.ND;
+        nP = (int)((2ull * (uint64_t)R * dm.NP + den) / (2ull * den));
+        nP = nP < 1 ? 1 : (nP > R - 1 ? R - 1 : nP);
+    }
+    // rank of each replica by strength (stronger first, ties to the lower index)
+    int rank[2] = {0, 0};
+    for (int o = 0; o < R; ++o) {
+        const double so_ = __shfl_sync(0xFFFFFFFFu, o < 32 ? strength[0] : strength[1], o & 31);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int c = lane + 32 * h;
+            if (c < R && o != c && (so_ > strength[h] || (so_ == strength[h] && o < c))) ++rank[h];
+        }
+    }
+    const unsigned dec_lo = __ballot_sync(0xFFFFFFFFu, lane < R && rank[0] >= nP);
+    const unsigned dec_hi = __ballot_sync(0xFFFFFFFFu, lane + 32 < R && rank[1] >= nP);
+    const uint64_t roles = (uint64_t)dec_lo | ((uint64_t)dec_hi << 32);
+    // outputs of the chosen roles
+    unsigned long long n_rep = 0, n_served = 0, n_paper = 0;
+    double rate[2] = {0.0, 0.0}, lat[2] = {0.0, 0.0};
+    int kind[2] = {-1, -1};
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int c = lane + 32 * h;
+        if (c >= R) continue;
+        const int slot = g * K + c;
+        const int role = (int)((roles >> c) & 1ull);
+        const int code = role ? best[h] : (pok[h] ? bp : -1);
+        s_code[wl][c] = code;
+        if (code < 0) {
+            out.master[slot] = -1; out.bsel[slot] = -1;
+            out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
+        } else {
+            const size_t sv = (size_t)slot * V + code;
+            const double T = so.T[sv];
+            out.master[slot] = so.mu[sv];
+            out.bsel[slot] = (int16_t)(role ? code + 1 : 0);
+            out.T[slot] = T;
+            lat[h] = so.L[sv];
+            out.L[slot] = lat[h];
+            kind[h] = role;
+            rate[h] = role ? (double)(code + 1) / T : (double)dm.NP / T;
+            ++n_served;
+        }
+        if (si.mask[slot]) {                         // replicas with no work were counted by the pre-pass
+            const unsigned long long ndec = best[h] >= 0 ? (unsigned long long)(bp - best[h]) : (unsigned long long)bp;
+            ++n_rep;
+            n_paper += (1 + ndec) * paper_candidates(m[h], dm.N);
+        }
+    }
+    __syncwarp();
+    const int16_t *split = so.layers + (size_t)g * V * M;
+    for (int i = lane; i < M; i += 32) {
+        int lo = 0, hi = R - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (s_off[wl][mid] <= i) lo = mid;
+            else hi = mid - 1;
+        }
+        const int code = s_code[wl][lo];
+        out.layers[(size_t)g * M + i] = code >= 0 ? split[(size_t)code * M + i] : (int16_t)-1;
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        n_rep += __shfl_xor_sync(0xFFFFFFFFu, n_rep, o);
+        n_served += __shfl_xor_sync(0xFFFFFFFFu, n_served, o);
+        n_paper += __shfl_xor_sync(0xFFFFFFFFu, n_paper, o);
+    }
+    double PS = 0.0, DS = 0.0, PL = 0.0, DL = 0.0;
+    for (int c = 0; c < R; ++c) {
+        const int h = c >> 5;
+        const double x = __shfl_sync(0xFFFFFFFFu, h ? rate[1] : rate[0], c & 31);
+        const double l = __shfl_sync(0xFFFFFFFFu, h ? lat[1] : lat[0], c & 31);
+        const int k = __shfl_sync(0xFFFFFFFFu, h ? kind[1] : kind[0], c & 31);
+        if (k == 0) { PS = PS + x; PL = PL + x * l; }
+        else if (k == 1) { DS = DS + x; DL = DL + x * l; }
+    }
+    // fingerprint of the genome with its roles (a tree fold over the lanes)
+    auto mix = [](uint64_t h, uint64_t x) { h = (h ^ x) * 0xBF58476D1CE4E5B9ull; return h ^ (h >> 31); };
+    uint64_t hl = 0x9E3779B97F4A7C15ull ^ (uint64_t)lane;
+    const uint16_t *pp = pop.perm + (size_t)g * M;
+    for (int i = lane; i < M; i += 32) hl = mix(hl, pp[i]);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        const uint64_t other = __shfl_down_sync(0xFFFFFFFFu, hl, o);
+        if (lane < o) hl = mix(hl, other);
+    }
+    if (lane != 0) return;
+    if (n_rep) {
+        atomicAdd(&out.stats[kStReplicas], n_rep);
+        atomicAdd(&out.stats[kStPaper], n_paper);
+    }
+    if (n_served) atomicAdd(&out.stats[kStServed], n_served);
+    double w, phase;
+    objective(dm, PS, DS, PL, DL, w, phase);
+    double *f = out.fit + (size_t)g * 4;
+    f[0] = w; f[1] = phase; f[2] = PS; f[3] = DS;
+    pop.roles[g] = roles;
+    uint64_t h = hl;
+    const uint16_t *ss = pop.sizes + (size_t)g * K;
+    for (int i = 0; i < R; ++i) h = mix(h, (uint64_t)ss[i] << 16);
+    h = mix(h, (uint64_t)R << 40);
+    h = mix(h, roles);
+    out.hash[g] = h;
+    atomicAdd(&out.stats[kStGenomes], 1ull);
+}
+
 // Persistent grids of the DP.  Shared memory is what limits CTAs per SM when
 // the largest replica's DP is big (many blocks); the replica sizes whose DP
 // fits in half of it then form class 1, launched with that smaller allocation
@@ -1347,9 +1532,15 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     }
     if (c->ev_dp_stop && (e = cudaEventRecordWithFlags(c->ev_dp_stop, c->stream, rec)) != cudaSuccess) return e;
     const unsigned fb = (unsigned)(((size_t)c->dm.P * 32 + 127) / 128);
-    if (c->dm.role_search && c->dm.K >= 12)           // up to 2^K_max assignments: a block per genome
-        finalize_roles_kernel<4><<<(unsigned)c->dm.P, 128, 0, c->stream>>>(c->dm, p, si, so, out);
-    else if (c->dm.role_search) finalize_roles_kernel<1><<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
+    if (c->dm.role_search == 2)
+        finalize_splitwise_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
+    else if (c->dm.role_search && c->dm.K >= 12) {    // up to 2^K_max assignments: a block per genome
+        if (c->dm.objective == 1) finalize_roles_kernel<4, true><<<(unsigned)c->dm.P, 128, 0, c->stream>>>(c->dm, p, si, so, out);
+        else finalize_roles_kernel<4, false><<<(unsigned)c->dm.P, 128, 0, c->stream>>>(c->dm, p, si, so, out);
+    } else if (c->dm.role_search) {
+        if (c->dm.objective == 1) finalize_roles_kernel<1, true><<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
+        else finalize_roles_kernel<1, false><<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
+    }
     else finalize_score_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
     c->launches += c->dp_grid1 > 0 ? 5 : 4;
     return cudaGetLastError();

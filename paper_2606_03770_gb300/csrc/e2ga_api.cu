@@ -188,11 +188,13 @@ int validate_inputs(const e2_devices *d, const e2_links *l, const e2_layer_profi
     for (double q : probs)
         if (!(q >= 0.0 && q <= 1.0)) { snprintf(msg, n, "probabilities must lie in [0, 1]"); return E2_EINVAL; }
     if (p->tournament < 1) { snprintf(msg, n, "tournament size must be >= 1"); return E2_EINVAL; }
-    if (p->role_search != 0 && p->role_search != 1) { snprintf(msg, n, "role_search must be 0 or 1"); return E2_EINVAL; }
-    if (p->role_search && (p->K_max > E2_MAX_ROLE_SEARCH || pf->b_max > 63)) {
-        snprintf(msg, n, "role_search needs K_max <= %d and b_max <= 63", E2_MAX_ROLE_SEARCH);
+    if (p->role_search < 0 || p->role_search > 2) { snprintf(msg, n, "role_search must be 0, 1 or 2"); return E2_EINVAL; }
+    if (p->role_search == 1 && (p->K_max > E2_MAX_ROLE_SEARCH || pf->b_max > 63)) {
+        snprintf(msg, n, "role_search 1 needs K_max <= %d and b_max <= 63", E2_MAX_ROLE_SEARCH);
         return E2_EINVAL;
     }
+    if (p->role_search == 2 && pf->b_max > 63) { snprintf(msg, n, "role_search 2 needs b_max <= 63"); return E2_EINVAL; }
+    if (p->objective != 0 && p->objective != 1) { snprintf(msg, n, "objective must be 0 or 1"); return E2_EINVAL; }
     return E2_OK;
 }
 
@@ -331,7 +333,7 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->stream = static_cast<cudaStream_t>(stream);
     c->dm = Dims{M, N, b_max + 1, b_max, P, Q, K, l.LS, prm->tournament, prof->NP, prof->ND,
                  prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps), prm->role_search, 0.0f, 0u, 4,
-                 costs_grow_with_batch(prof, b_max)};
+                 costs_grow_with_batch(prof, b_max), prm->objective};
     {
         const double lm = c->dm.lam_max;                       // rounded up to float
         float f = (float)lm;

@@ -79,13 +79,15 @@ struct Dims {
     uint64_t NP, ND;
     double min_tps, t_a;
     double lam_max;      // largest latency Lambda with 1.0 / Lambda >= min_tps (see e2_create)
-    int role_search;     // 1: both roles per replica, best assignment per genome (Alg. 2)
+    int role_search;     // 1: both roles per replica, best assignment per genome (Alg. 2);
+                         // 2: both roles per replica, the adapted-SplitWise rule picks the roles
     float lam_max_up;    // lam_max rounded up to float (the float latency bound is compared with it)
     unsigned dp_small;   // shared-memory bytes of DP class 1 (0: one class); m is in class 1 iff
                          // dp_item_bytes(m, N, dp_warps, 4) <= dp_small
     int dp_warps;        // warps per DP CTA
     int grows;           // 1: block memory, head memory, block flops and bytes and activation bytes never
                          // shrink from one decode batch to the next (the pre-pass tests are then monotone)
+    int objective;       // 0: waiting time w (Eq. 3-5); 1: per-request finishing time FT
 };
 
 struct Tables {

@@ -40,7 +40,7 @@ class e2_params(C.Structure):
     _fields_ = [("P", C.c_int32), ("Q", C.c_int32), ("K_max", C.c_int32), ("tournament", C.c_int32),
                 ("min_tps", C.c_double), ("t_a", C.c_double), ("p_cx", C.c_double), ("p_mut", C.c_double),
                 ("p_swap", C.c_double), ("p_regroup", C.c_double), ("p_regroup_all", C.c_double),
-                ("role_search", C.c_int32)]
+                ("role_search", C.c_int32), ("objective", C.c_int32)]
 
 
 class e2_genomes(C.Structure):
@@ -235,7 +235,8 @@ class Engine:
             prob.NP, prob.ND)
         pk = prob.p_kind
         self.params = e2_params(self.P, self.Q, self.K, prob.tournament, prob.min_tps, prob.t_a, prob.p_cx,
-                                prob.p_mut, pk[0], pk[1], pk[2], int(getattr(prob, "role_search", 0)))
+                                prob.p_mut, pk[0], pk[1], pk[2], int(getattr(prob, "role_search", 0)),
+                                int(getattr(prob, "objective", 0)))
         self.ws_bytes = e2_workspace_bytes(self.M, self.N, self.b_max, self.P, self.Q, self.K)
         if self.ws_bytes == 0:
             raise E2Error(E2_EINVAL, "e2_workspace_bytes")

@@ -54,8 +54,11 @@ class Problem:
     min_tps: float = 7.0
     t_a: float = 1.0
     # roles: 0 = one role bit per replica in the genome; 1 = Alg. 2's brute force
-    # over every role assignment of the genome's replicas
+    # over every role assignment of the genome's replicas; 2 = the adapted-SplitWise
+    # rule (the strongest replicas prefill)
     role_search: int = 0
+    # objective: 0 = the waiting time of Eq. 3-5; 1 = the per-request finishing time
+    objective: int = 0
     # genetic algorithm
     P: int = 64
     Q: int = 2

@@ -93,12 +93,13 @@ def _structs(prob):
     pf = e2ga.e2_layer_profile(prob.N, prob.b_max, *[p(u64(getattr(prob, k))) for k in (
         "blk_flops", "blk_bytes", "blk_mem", "head_flops", "head_bytes", "head_mem", "act_bytes")], prob.NP, prob.ND)
     pr = e2ga.e2_params(prob.P, prob.Q, prob.K_max, prob.tournament, prob.min_tps, prob.t_a, prob.p_cx,
-                        prob.p_mut, *prob.p_kind[:3], prob.role_search)
+                        prob.p_mut, *prob.p_kind[:3], prob.role_search, prob.objective)
     return d, l, pf, pr, keep
 
 
 BAD = {
-    "role search mode": lambda p: setattr(p, "role_search", 2),
+    "role search mode": lambda p: setattr(p, "role_search", 3),
+    "objective": lambda p: setattr(p, "objective", 2),
     "role search with many replicas": lambda p: (setattr(p, "role_search", 1), setattr(p, "K_max", 21)),
     "negative rate": lambda p: p.rate.__setitem__(0, -1.0),
     "nan bandwidth": lambda p: p.bw.__setitem__(1, np.nan),

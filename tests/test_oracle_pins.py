@@ -764,3 +764,131 @@ def test_role_search_is_the_best_fixed_assignment():
             assert np.array_equal(got[key][p], every[key][best]), key
         checked_feasible += bool(np.isfinite(f[best, 0]))
     assert checked_feasible >= 10
+
+
+# ---------------------------------------------------------------------------
+# comparison objectives (Sec. 4.2 "Baseline chosen")
+# ---------------------------------------------------------------------------
+def _ft_problem(NP, ND):
+    import dataclasses
+    return dataclasses.replace(_objective_problem(NP, ND, 1.0), objective=1)
+
+
+def test_finishing_time_hand_cases():
+    """HexGen-2's per-request finishing time: a request's prefill pass plus ND
+    decode passes, each the end-to-end latency Lambda of its replica (stages
+    and links added), averaged over the replicas of a role in proportion to
+    their rates."""
+    op = O.OracleProblem(_ft_problem(100, 50))
+    # one replica per role: FT = Lambda_P + ND * Lambda_D = 5 + 50 * 3
+    f = op.score(0b10, [2.0, 0.5], [0, 4], L=[5.0, 3.0])
+    assert f[0] == 155.0
+    assert f[2] == 50.0 and f[3] == 8.0 and f[1] == max(100 / 50, 50 / 8)   # PS, DS and Eq. 3 unchanged
+    # two equally fast prefill replicas with latencies 2 and 6: their mean, 4
+    f = op.score(0b100, [1.0, 1.0, 1.0], [0, 0, 1], L=[2.0, 6.0, 1.0])
+    assert f[0] == 4.0 + 50 * 1.0
+    # rate-weighted: prefill rates 3 and 1 tok/s (NP = 3, T = 1 and 3), latencies
+    # 1 and 3 -> (3*1 + 1*3) / 4 = 1.5
+    op3 = O.OracleProblem(_ft_problem(3, 1))
+    f = op3.score(0b100, [1.0, 3.0, 1.0], [0, 0, 1], L=[1.0, 3.0, 2.0])
+    assert f[0] == 1.5 + 1 * 2.0
+    # the waiting-time objective on the same replicas ignores Lambda
+    assert O.OracleProblem(_objective_problem(3, 1, 1.0)).score(0b100, [1.0, 3.0, 1.0], [0, 0, 1],
+                                                                L=[1.0, 3.0, 2.0])[0] == 0.0
+    # no decode capacity, or an infeasible replica alone in its role: +inf
+    assert op.score(0b00, [1.0, 1.0], [0, 0], L=[1.0, 1.0])[0] == INF
+    assert op.score(0b10, [1.0, INF], [0, -1], L=[1.0, INF])[0] == INF
+
+
+def test_finishing_time_scales_with_time():
+    """Every rate, bandwidth and link speed doubled: every stage and link time
+    halves exactly, and so does FT (a sum of latencies; ND is a count)."""
+    import dataclasses
+    prob = dataclasses.replace(W.make_config("c1_tiny"), objective=1)
+    fast = dataclasses.replace(prob, rate=prob.rate * 2, bw=prob.bw * 2, link_bw=prob.link_bw * 2,
+                               min_tps=prob.min_tps * 2)
+    g = W.random_genomes(prob.M, prob.K_max, 240, seed=41)
+    a = O.OracleProblem(prob).eval_population(g, prob.K_max)
+    b = O.OracleProblem(fast).eval_population(g, prob.K_max)
+    fin = np.isfinite(a["fitness"][:, 0])
+    assert fin.sum() >= 20
+    assert np.array_equal(a["fitness"][:, 0] / 2, b["fitness"][:, 0])
+    assert np.array_equal(a["layers"], b["layers"]) and np.array_equal(a["bsel"], b["bsel"])
+
+
+def test_finishing_time_role_search_is_the_best_fixed_assignment():
+    import dataclasses
+    prob = dataclasses.replace(W.make_config("c1_tiny"), objective=1)
+    search = O.OracleProblem(dataclasses.replace(prob, role_search=1))
+    fixed = O.OracleProblem(prob)
+    K = 4
+    g = W.random_genomes(prob.M, K, 16, seed=43)
+    got = search.eval_population(g, K)
+    finite = 0
+    for p in range(16):
+        R = int(g["nclus"][p])
+        one = {k: np.repeat(v[p:p + 1], 1 << R, axis=0) for k, v in g.items()}
+        one["roles"] = np.arange(1 << R, dtype=np.uint64)
+        f = fixed.eval_population(one, K)["fitness"]
+        best = min(range(1 << R), key=lambda r: (f[r, 0], f[r, 1], r))
+        assert int(got["roles"][p]) == best and np.array_equal(got["fitness"][p], f[best])
+        finite += bool(np.isfinite(f[best, 0]))
+    assert finite >= 6
+
+
+def test_splitwise_prefill_count():
+    """SplitWise sizes its pools by the input-to-generated token ratio: R
+    replicas split NP : ND, rounded half up, at least one per role."""
+    cases = {(1, 1, 4): 2, (1, 1, 1): 1, (1, 1, 2): 1, (3, 1, 4): 3, (1, 3, 4): 1, (1, 1, 3): 2,
+             (1, 100, 3): 1, (100, 1, 3): 2, (2291, 1385, 10): 6, (576, 746, 10): 4, (5, 5, 64): 32}
+    for (NP, ND, R), n in cases.items():
+        assert O.splitwise_prefill_count(NP, ND, R) == n, (NP, ND, R)
+
+
+def _single_device_replicas(rates, NP=64, ND=64):
+    """Replicas of one device each, identical but for the compute rate, with
+    ample memory and free links: the prefill throughput orders as the rate."""
+    M = len(rates)
+    V = 3
+    return W.make_problem(rates, [1e12] * M, [10 ** 12] * M, np.full((M, M), np.inf), np.ones((M, M)), 4,
+                          [1000] * V, [10] * V, [1] * V, [0] * V, [0] * V, [0] * V, [16] * V, NP=NP, ND=ND,
+                          min_tps=0.0, role_search=2)
+
+
+def test_splitwise_strongest_replicas_prefill():
+    prob = _single_device_replicas([1e6, 4e6, 2e6, 3e6])
+    op = O.OracleProblem(prob)
+    g = dict(perm=np.array([[0, 1, 2, 3]], np.uint16), sizes=np.array([[1, 1, 1, 1]], np.uint16),
+             nclus=np.array([4], np.uint8), roles=np.array([0b1111], np.uint64))
+    out = op.eval_population(g, 4)
+    # the two strongest (rates 4e6 and 3e6, replicas 1 and 3) prefill; 0 and 2 decode
+    assert int(out["roles"][0]) == 0b0101
+    assert list(out["bsel"][0]) == [2, 0, 2, 0]
+    # equal strengths: the lower index prefills first
+    op2 = O.OracleProblem(_single_device_replicas([2e6, 2e6, 2e6, 2e6]))
+    assert int(op2.eval_population(g, 4)["roles"][0]) == 0b1100
+    # NP : ND = 3 : 1 -> three prefill replicas
+    op3 = O.OracleProblem(_single_device_replicas([1e6, 4e6, 2e6, 3e6], NP=96, ND=32))
+    assert int(op3.eval_population(g, 4)["roles"][0]) == 0b0001
+
+
+def test_splitwise_never_beats_the_role_search():
+    """The adapted-SplitWise rule picks one of the 2^R assignments, so its
+    (w, phase) is never below Alg. 2's brute force; its fitness is the
+    objective of the assignment it picked, and its prefill replicas are at
+    least as strong as its decode replicas."""
+    import dataclasses
+    for objective in (0, 1):
+        prob = dataclasses.replace(W.make_config("c1_tiny"), objective=objective)
+        K = 5
+        g = W.random_genomes(prob.M, K, 40, seed=47 + objective)
+        spw = O.OracleProblem(dataclasses.replace(prob, role_search=2)).eval_population(g, K)
+        bf = O.OracleProblem(dataclasses.replace(prob, role_search=1)).eval_population(g, K)
+        fixed = O.OracleProblem(prob).eval_population(dict(g, roles=spw["roles"]), K)
+        assert np.array_equal(fixed["fitness"], spw["fitness"])
+        worse = 0
+        for p in range(40):
+            a, b = spw["fitness"][p], bf["fitness"][p]
+            assert (a[0], a[1]) >= (b[0], b[1])
+            worse += (a[0], a[1]) > (b[0], b[1])
+        assert worse >= 1
