@@ -56,12 +56,27 @@ typedef enum {
     E2_ESTATE = 6     /* call order: e.g. e2_ga_step before any evaluation    */
 } e2_status;
 
-/* Fleet (Sec. 3.1: profiled devices).  M >= 1, M <= E2_MAX_DEVICES. */
+/* Fleet (Sec. 3.1: profiled devices).  M >= 1, M <= E2_MAX_DEVICES.
+ *
+ * GPU-CPU offload (Sec. 1: offloading is part of the cost model; the plans'
+ * G--C column, Sec. 4.3): a device with host memory mem_cpu[d] > 0 keeps as
+ * many of a stage's blocks in its own memory as fit there (beside the LM head
+ * and output layer on the master, which never leave it) and the rest in host
+ * memory, if they fit, where they run at rate_cpu[d] and bw_cpu[d]; the two
+ * parts run one after the other, so the stage time is
+ *   max(g*F (+F_head)/rate, g*B (+B_head)/bw) + max(c*F/rate_cpu, c*B/bw_cpu)
+ * for g blocks in device memory and c = n - g offloaded.  mem_cpu NULL (or 0
+ * for a device, e.g. unified memory) means no offload there. */
 typedef struct {
     int32_t M;
     const double *rate;     /* [M] compute rate, FLOP/s, finite > 0   (host)  */
     const double *bw;       /* [M] memory bandwidth, bytes/s, finite > 0      */
     const uint64_t *mem;    /* [M] memory available to the model, bytes       */
+    const double *rate_cpu; /* [M] host FLOP/s for offloaded blocks, finite   */
+                            /*     > 0 where mem_cpu > 0; NULL if mem_cpu is  */
+    const double *bw_cpu;   /* [M] host bytes/s, likewise                     */
+    const uint64_t *mem_cpu;/* [M] host memory for offloaded blocks, bytes,   */
+                            /*     or NULL (no device offloads)               */
 } e2_devices;
 
 /* Links (Sec. 3.2: tau(k-1,k) = A / B(k-1,k)).  Row = sender.  The effective
@@ -150,13 +165,17 @@ typedef struct {
  *   bsel   [P][K_max]  0 prefill, b >= 1 chosen decode batch, -1 no service
  *                      (or replica index >= R);
  *   T      [P][K_max]  bottleneck stage time of the chosen variant (+inf if none);
- *   lambda [P][K_max]  per-request latency Lambda of the chosen variant (+inf). */
+ *   lambda [P][K_max]  per-request latency Lambda of the chosen variant (+inf);
+ *   gpu_layers [P][M]  of layers[p], the blocks in the device's own memory
+ *                      (the rest offloaded to host memory: the plans' G--C
+ *                      split), -1 when the replica cannot serve. */
 typedef struct {
     int16_t *layers;
     int16_t *master;
     int16_t *bsel;
     double *T;
     double *lambda;
+    int16_t *gpu_layers;
 } e2_partitions;
 
 /* Counters of the last evaluation (device-side tallies), then host-side

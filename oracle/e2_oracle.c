@@ -56,26 +56,61 @@ typedef struct {
                                  /* 2: adapted SplitWise (strongest prefill)  */
     int objective;               /* 0: waiting time w (Eq. 3-5); 1: per-      */
                                  /* request finishing time FT                 */
+    const double *rate_cpu;      /* [M] host FLOP/s of offloaded blocks, or   */
+    const double *bw_cpu;        /* [M] host bytes/s; mem_cpu [M] host bytes  */
+    const uint64_t *mem_cpu;     /* for blocks; NULL: no offload anywhere     */
 } orc_problem;
 
 /* ------------------------------------------------------------------------ */
 /* Cost model.                                                               */
 /* ------------------------------------------------------------------------ */
 
+/* Blocks of a stage of n blocks on device d that sit in the device's own
+ * (GPU or unified) memory, the rest being offloaded to host memory: as many
+ * as fit next to the LM head and output layer when d is the master (the head
+ * itself never leaves device memory), the "G" of the plans' G--C column
+ * (Sec. 4.3).  -1 when the head does not fit at all. */
+int orc_gpu_blocks(const orc_problem *p, int v, int d, int n, int master)
+{
+    uint64_t hm = master ? p->head_mem[v] : 0;
+    if (hm > p->mem[d]) return -1;
+    uint64_t bm = p->blk_mem[v];
+    uint64_t cap = bm ? (p->mem[d] - hm) / bm : (uint64_t)n;
+    return (uint64_t)n < cap ? n : (int)cap;
+}
+
 /* l_k(j,i,m): time of n = i-j+1 identical blocks on device d, plus the LM head
  * and output layer when the device is the master (Sec. 3.1: both live on the
  * master).  A block's time is the larger of its compute time and its memory
- * streaming time; a stage that does not fit in the device's memory costs +inf
- * (Sec. 3.2: memory-infeasible candidates take +inf). */
+ * streaming time; a stage that does not fit in memory costs +inf (Sec. 3.2:
+ * memory-infeasible candidates take +inf).
+ *
+ * GPU--CPU offload (Sec. 1: offloading is a first-class part of the cost
+ * model; the plans' G--C column, Sec. 4.3): the g = orc_gpu_blocks blocks in
+ * device memory run at the device's rate and bandwidth, the other n - g in
+ * host memory (mem_cpu) at the host's, one after the other, so their times
+ * add.  Without host memory (mem_cpu NULL or 0: unified-memory devices) every
+ * block must fit in device memory, as before. */
 double orc_stage_cost(const orc_problem *p, int v, int d, int n, int master)
 {
-    uint64_t need = (uint64_t)n * p->blk_mem[v] + (master ? p->head_mem[v] : 0);
-    if (need > p->mem[d]) return ORC_INF;
-    uint64_t fl = (uint64_t)n * p->blk_flops[v] + (master ? p->head_flops[v] : 0);
-    uint64_t by = (uint64_t)n * p->blk_bytes[v] + (master ? p->head_bytes[v] : 0);
+    int g = orc_gpu_blocks(p, v, d, n, master);
+    if (g < 0) return ORC_INF;
+    uint64_t c = (uint64_t)(n - g);                     /* offloaded blocks */
+    if (c > 0) {
+        uint64_t host = p->mem_cpu ? p->mem_cpu[d] : 0;
+        if (c * p->blk_mem[v] > host) return ORC_INF;
+    }
+    uint64_t fl = (uint64_t)g * p->blk_flops[v] + (master ? p->head_flops[v] : 0);
+    uint64_t by = (uint64_t)g * p->blk_bytes[v] + (master ? p->head_bytes[v] : 0);
     double tc = (double)fl / p->rate[d];
     double tm = (double)by / p->bw[d];
-    return tc >= tm ? tc : tm;
+    double t = tc >= tm ? tc : tm;
+    if (c > 0) {
+        double hc = (double)(c * p->blk_flops[v]) / p->rate_cpu[d];
+        double hmm = (double)(c * p->blk_bytes[v]) / p->bw_cpu[d];
+        t = t + (hc >= hmm ? hc : hmm);
+    }
+    return t;
 }
 
 /* tau(k-1,k) = A / B(k-1,k): time to move one microbatch of activations over

@@ -43,7 +43,8 @@ class _Problem(C.Structure):
                 ("head_flops", C.c_void_p), ("head_bytes", C.c_void_p), ("head_mem", C.c_void_p),
                 ("act_bytes", C.c_void_p), ("NP", C.c_uint64), ("ND", C.c_uint64),
                 ("min_tps", C.c_double), ("t_a", C.c_double), ("role_search", C.c_int),
-                ("objective", C.c_int)]
+                ("objective", C.c_int), ("rate_cpu", C.c_void_p), ("bw_cpu", C.c_void_p),
+                ("mem_cpu", C.c_void_p)]
 
 
 class _GA(C.Structure):
@@ -58,6 +59,8 @@ def lib():
         _lib = C.CDLL(build())
         _lib.orc_stage_cost.restype = C.c_double
         _lib.orc_stage_cost.argtypes = [C.c_void_p, C.c_int, C.c_int, C.c_int, C.c_int]
+        _lib.orc_gpu_blocks.restype = C.c_int
+        _lib.orc_gpu_blocks.argtypes = [C.c_void_p, C.c_int, C.c_int, C.c_int, C.c_int]
         _lib.orc_link_cost.restype = C.c_double
         _lib.orc_link_cost.argtypes = [C.c_void_p, C.c_int, C.c_int, C.c_int]
         _lib.orc_dp_pipe.restype = C.c_int
@@ -114,12 +117,16 @@ class OracleProblem:
                            blk_mem=u64(prob.blk_mem), head_flops=u64(prob.head_flops),
                            head_bytes=u64(prob.head_bytes), head_mem=u64(prob.head_mem),
                            act_bytes=u64(prob.act_bytes))
+        off = getattr(prob, "mem_cpu", None) is not None
+        if off:
+            self.arrays.update(rate_cpu=f64(prob.rate_cpu), bw_cpu=f64(prob.bw_cpu), mem_cpu=u64(prob.mem_cpu))
         a = self.arrays
         self.s = _Problem(prob.M, prob.N, prob.V, *[_p(a[k]) for k in
                           ("rate", "bw", "mem", "link_bw", "cong", "blk_flops", "blk_bytes",
                            "blk_mem", "head_flops", "head_bytes", "head_mem", "act_bytes")],
                           prob.NP, prob.ND, prob.min_tps, prob.t_a, int(getattr(prob, "role_search", 0)),
-                          int(getattr(prob, "objective", 0)))
+                          int(getattr(prob, "objective", 0)),
+                          *([_p(a[k]) for k in ("rate_cpu", "bw_cpu", "mem_cpu")] if off else [None] * 3))
 
     def set_cong(self, cong):
         self.arrays["cong"] = np.ascontiguousarray(cong, dtype=np.float64)
@@ -131,6 +138,9 @@ class OracleProblem:
 
     def stage_cost(self, v, d, n, master):
         return lib().orc_stage_cost(self.ref, v, d, n, int(master))
+
+    def gpu_blocks(self, v, d, n, master):
+        return lib().orc_gpu_blocks(self.ref, v, d, n, int(master))
 
     def link_cost(self, v, a, b):
         return lib().orc_link_cost(self.ref, v, a, b)

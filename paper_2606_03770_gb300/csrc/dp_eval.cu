@@ -1433,6 +1433,54 @@ __global__ void __launch_bounds__(128) finalize_splitwise_kernel(Dims dm, DevPop
     atomicAdd(&out.stats[kStGenomes], 1ull);
 }
 
+// The G--C split of the plans (Sec. 4.3) under GPU-CPU offload, one warp per
+// genome: of the n blocks at ordering position i, the ones in the device's own
+// memory, min(n, capg), for the variant its replica serves (bsel: 0 prefill,
+// b decode) and whether the device is the replica's master; -1 where the
+// replica cannot serve.  Runs after the replicas' outputs are final.
+__global__ void __launch_bounds__(128) gc_split_kernel(Dims dm, DevPop pop, const int32_t *capg, EvalOut out)
+{
+    __shared__ int s_off[4][E2_MAX_CLUSTERS + 1];
+    const int wl = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = blockIdx.x * 4 + wl;
+    if (g >= dm.P) return;
+    const int K = dm.K, M = dm.M;
+    const int R = pop.nclus[g];
+    // replica offsets: an exclusive scan of the sizes (lane l: replicas l and l + 32)
+    const int s_lo = lane < R ? pop.sizes[(size_t)g * K + lane] : 0;
+    const int s_hi = lane + 32 < R ? pop.sizes[(size_t)g * K + lane + 32] : 0;
+    int in_lo = s_lo, in_hi = s_hi;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int a = __shfl_up_sync(0xFFFFFFFFu, in_lo, o), b = __shfl_up_sync(0xFFFFFFFFu, in_hi, o);
+        if (lane >= o) { in_lo += a; in_hi += b; }
+    }
+    const int total_lo = __shfl_sync(0xFFFFFFFFu, in_lo, 31);
+    if (lane < R) s_off[wl][lane] = in_lo - s_lo;
+    if (lane + 32 < R) s_off[wl][lane + 32] = total_lo + in_hi - s_hi;
+    if (lane == 0) s_off[wl][R] = M;
+    __syncwarp();
+    for (int i = lane; i < M; i += 32) {
+        int lo = 0, hi = R - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (s_off[wl][mid] <= i) lo = mid;
+            else hi = mid - 1;
+        }
+        const size_t slot = (size_t)g * K + lo;
+        const int n = out.layers[(size_t)g * M + i];
+        int16_t gb = -1;
+        if (n >= 0) {
+            const int v = out.bsel[slot];
+            const int mf = (i - s_off[wl][lo]) == out.master[slot];
+            const int d = pop.perm[(size_t)g * M + i];
+            const int c = capg[((size_t)v * M + d) * 2 + mf];
+            gb = (int16_t)(n < c ? n : c);
+        }
+        out.gpu_layers[(size_t)g * M + i] = gb;
+    }
+}
+
 // Persistent grids of the DP.  Shared memory is what limits CTAs per SM when
 // the largest replica's DP is big (many blocks); the replica sizes whose DP
 // fits in half of it then form class 1, launched with that smaller allocation
@@ -1498,8 +1546,9 @@ cudaError_t configure_eval(e2_ctx *c)
 
 cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
 {
-    Tables tb{c->rate, c->bw, c->mem, c->prof, c->leaf, c->tau, c->cap, c->cpb, c->tau_lb, c->leaf_rank, c->tau_rank};
-    EvalOut out{c->fit, c->layers, c->master, c->bsel, c->T, c->L, c->hash, c->stats};
+    Tables tb{c->rate, c->bw, c->mem, c->rate_cpu, c->bw_cpu, c->mem_cpu, c->prof, c->leaf, c->tau, c->cap,
+              c->capg, c->cpb, c->tau_lb, c->leaf_rank, c->tau_rank};
+    EvalOut out{c->fit, c->layers, c->master, c->bsel, c->T, c->L, c->hash, c->stats, c->gpu_layers};
     SlotInfo si{c->slot_off, c->slot_mask, c->slot_size, c->slot_best};
     WorkList wl{c->items, c->order_bins};
     SplitOut so{c->split_T, c->split_L, c->split_mu, c->split_layers};
@@ -1543,6 +1592,10 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     }
     else finalize_score_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
     c->launches += c->dp_grid1 > 0 ? 5 : 4;
+    if (c->dm.offload) {
+        gc_split_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, c->capg, out);
+        ++c->launches;
+    }
     return cudaGetLastError();
 }
 

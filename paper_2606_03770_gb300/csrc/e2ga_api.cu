@@ -20,8 +20,8 @@ thread_local char g_create_error[256] = "";
 size_t align_up(size_t x, size_t a = 256) { return (x + a - 1) / a * a; }
 
 struct Layout {
-    size_t rate, bw, mem, link_bw, cong, prof, leaf, tau, tau_lb, cap, cpb, leaf_sorted, beff_sorted, tau_sorted,
-        leaf_rank, tau_rank;
+    size_t rate, bw, mem, rate_cpu, bw_cpu, mem_cpu, link_bw, cong, prof, leaf, tau, tau_lb, cap, capg, cpb,
+        leaf_sorted, beff_sorted, tau_sorted, leaf_rank, tau_rank, gpu_layers;
     size_t perm[2], sizes[2], nclus[2], roles[2];
     size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, stats, err, order_bins, items, slot_off, slot_mask, slot_size, slot_best,
         split_T, split_L, split_mu, split_layers, total;
@@ -47,12 +47,16 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K)
     l.rate = take(8 * (size_t)M);
     l.bw = take(8 * (size_t)M);
     l.mem = take(8 * (size_t)M);
+    l.rate_cpu = take(8 * (size_t)M);
+    l.bw_cpu = take(8 * (size_t)M);
+    l.mem_cpu = take(8 * (size_t)M);
     l.link_bw = take(8 * MM);
     l.cong = take(8 * MM);
     l.prof = take(8 * kNumProf * V);
     l.leaf = take(8 * V * M * 2 * (size_t)l.LS);
     l.tau = take(8 * V * MM);
     l.cap = take(4 * V * M * 2);
+    l.capg = take(4 * V * M * 2);
     l.cpb = take(4 * V * M);
     l.tau_lb = take(4 * V * MM);
     l.leaf_sorted = take(8 * V * rank_pow2((size_t)M * 2 * N));
@@ -68,6 +72,7 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K)
     }
     l.fit = take(32 * (size_t)P);
     l.layers = take(2 * (size_t)P * M);
+    l.gpu_layers = take(2 * (size_t)P * M);
     l.master = take(2 * (size_t)P * K);
     l.bsel = take(2 * (size_t)P * K);
     l.T = take(8 * (size_t)P * K);
@@ -152,6 +157,14 @@ int validate_inputs(const e2_devices *d, const e2_links *l, const e2_layer_profi
             snprintf(msg, n, "device %d: rate and bandwidth must be finite and > 0", i);
             return E2_EINVAL;
         }
+    }
+    if (d->mem_cpu) {
+        if (!d->rate_cpu || !d->bw_cpu) { snprintf(msg, n, "mem_cpu given without rate_cpu and bw_cpu"); return E2_EINVAL; }
+        for (int i = 0; i < M; ++i)
+            if (d->mem_cpu[i] && (!finite_pos(d->rate_cpu[i]) || !finite_pos(d->bw_cpu[i]))) {
+                snprintf(msg, n, "device %d: host rate and bandwidth must be finite and > 0 where mem_cpu > 0", i);
+                return E2_EINVAL;
+            }
     }
     for (int a = 0; a < M; ++a)
         for (int b = 0; b < M; ++b) {
@@ -334,6 +347,9 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->dm = Dims{M, N, b_max + 1, b_max, P, Q, K, l.LS, prm->tournament, prof->NP, prof->ND,
                  prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps), prm->role_search, 0.0f, 0u, 4,
                  costs_grow_with_batch(prof, b_max), prm->objective};
+    c->dm.offload = 0;
+    if (devs->mem_cpu)
+        for (int i = 0; i < M; ++i) c->dm.offload |= devs->mem_cpu[i] != 0;
     {
         const double lm = c->dm.lam_max;                       // rounded up to float
         float f = (float)lm;
@@ -381,6 +397,11 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->rate = reinterpret_cast<double *>(ws + l.rate);
     c->bw = reinterpret_cast<double *>(ws + l.bw);
     c->mem = reinterpret_cast<uint64_t *>(ws + l.mem);
+    c->rate_cpu = reinterpret_cast<double *>(ws + l.rate_cpu);
+    c->bw_cpu = reinterpret_cast<double *>(ws + l.bw_cpu);
+    c->mem_cpu = reinterpret_cast<uint64_t *>(ws + l.mem_cpu);
+    c->capg = reinterpret_cast<int32_t *>(ws + l.capg);
+    c->gpu_layers = reinterpret_cast<int16_t *>(ws + l.gpu_layers);
     c->link_bw = reinterpret_cast<double *>(ws + l.link_bw);
     c->cong = reinterpret_cast<double *>(ws + l.cong);
     c->prof = reinterpret_cast<uint64_t *>(ws + l.prof);
@@ -430,6 +451,11 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     chk(cudaMemcpyAsync(c->rate, devs->rate, 8 * (size_t)M, cudaMemcpyHostToDevice, c->stream));
     chk(cudaMemcpyAsync(c->bw, devs->bw, 8 * (size_t)M, cudaMemcpyHostToDevice, c->stream));
     chk(cudaMemcpyAsync(c->mem, devs->mem, 8 * (size_t)M, cudaMemcpyHostToDevice, c->stream));
+    if (c->dm.offload) {                       // otherwise the host side stays zero (no offload)
+        chk(cudaMemcpyAsync(c->rate_cpu, devs->rate_cpu, 8 * (size_t)M, cudaMemcpyHostToDevice, c->stream));
+        chk(cudaMemcpyAsync(c->bw_cpu, devs->bw_cpu, 8 * (size_t)M, cudaMemcpyHostToDevice, c->stream));
+        chk(cudaMemcpyAsync(c->mem_cpu, devs->mem_cpu, 8 * (size_t)M, cudaMemcpyHostToDevice, c->stream));
+    }
     chk(cudaMemcpyAsync(c->link_bw, links->bw, 8 * MM, cudaMemcpyHostToDevice, c->stream));
     chk(cudaMemcpyAsync(c->cong, links->cong, 8 * MM, cudaMemcpyHostToDevice, c->stream));
     chk(cudaMemcpyAsync(c->prof, prof_h, 8 * kNumProf * V, cudaMemcpyHostToDevice, c->stream));
@@ -564,6 +590,8 @@ int e2_get_results(e2_ctx *c, double *fitness_out, const e2_partitions *parts)
         E2_CUDA(c, out(parts->bsel, c->bsel, 2 * P * K));
         E2_CUDA(c, out(parts->T, c->T, 8 * P * K));
         E2_CUDA(c, out(parts->lambda, c->L, 8 * P * K));
+        // without offload every block sits in device memory: the split is the partition
+        E2_CUDA(c, out(parts->gpu_layers, c->dm.offload ? c->gpu_layers : c->layers, 2 * P * M));
     }
     if (host) E2_CUDA(c, cudaStreamSynchronize(c->stream));
     return E2_OK;

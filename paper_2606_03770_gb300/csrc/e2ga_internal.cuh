@@ -88,15 +88,20 @@ struct Dims {
     int grows;           // 1: block memory, head memory, block flops and bytes and activation bytes never
                          // shrink from one decode batch to the next (the pre-pass tests are then monotone)
     int objective;       // 0: waiting time w (Eq. 3-5); 1: per-request finishing time FT
+    int offload;         // 1: some device has host memory for offloaded blocks
 };
 
 struct Tables {
     const double *rate, *bw;
     const uint64_t *mem;
+    const double *rate_cpu, *bw_cpu;   // [M] host side of offloaded blocks (offload only)
+    const uint64_t *mem_cpu;           // [M] host memory for blocks, bytes (offload only)
     const uint64_t *prof;      // [kNumProf][V]
     const double *leaf;        // [V][M][2][LS]: leaf[((v*M+d)*2+mf)*LS + n-1] = l_d(n blocks, master mf)
     const double *tau;         // [V][M][M]
-    const int32_t *cap;        // [V][M][2]: most blocks device d holds (memory), without / with the head
+    const int32_t *cap;        // [V][M][2]: most blocks device d holds (device + host memory), without / with
+                               // the head
+    const int32_t *capg;       // [V][M][2]: of those, the most in device memory (-1: the head does not fit)
     const float *cpb;          // [V][M]: per-block time max(blk_flops/rate, blk_bytes/bw), rounded down
     const float *tau_lb;       // [V][M][M]: tau rounded down
     const uint32_t *leaf_rank; // [V][M][2][LS]: order key of leaf within its variant's value set
@@ -131,6 +136,7 @@ struct EvalOut {
     double *T, *L;             // [P][K]
     uint64_t *hash;            // [P]
     unsigned long long *stats; // [kNumStats]
+    int16_t *gpu_layers;       // [P][M] blocks in device memory (offload only)
 };
 
 // ---------------------------------------------------------------------------
@@ -196,6 +202,10 @@ struct e2_ctx {
     // device pointers (all inside the caller's workspace)
     double *rate = nullptr, *bw = nullptr;
     uint64_t *mem = nullptr;
+    double *rate_cpu = nullptr, *bw_cpu = nullptr;   // host side of offload (zeros without it)
+    uint64_t *mem_cpu = nullptr;
+    int32_t *capg = nullptr;                          // [V][M][2] blocks in device memory
+    int16_t *gpu_layers = nullptr;                    // [P][M] G of the G--C split (offload only)
     double *link_bw = nullptr, *cong = nullptr;
     uint64_t *prof = nullptr;
     double *leaf = nullptr, *tau = nullptr;

@@ -11,10 +11,24 @@ namespace {
 
 constexpr int kBitmapWords = E2_MAX_DEVICES / 32;
 
+// Blocks of a stage that sit in device memory: as many as fit beside the LM
+// head and output layer on the master (which never leave device memory); -1
+// when the head alone does not fit.
+__device__ __forceinline__ long long device_blocks(uint64_t nb, uint64_t bm, uint64_t hm, uint64_t mem)
+{
+    if (hm > mem) return -1;
+    const uint64_t cap = bm ? (mem - hm) / bm : nb;
+    return (long long)(nb < cap ? nb : cap);
+}
+
 // l_d(n, master): the larger of compute time and streaming time of n identical
-// blocks (plus the LM head and output layer on the master), +inf when the
-// resident bytes exceed the device memory (Sec. 3.2).
+// blocks (plus the LM head and output layer on the master), +inf when they do
+// not fit in memory (Sec. 3.2).  With GPU-CPU offload (a device with host
+// memory) the blocks beyond device memory sit in host memory, if they fit,
+// and run there at the host's rate and bandwidth after the device's part:
+// the two times add (the plans' G--C split, Sec. 4.3).
 __global__ void tables_kernel(Dims dm, const double *rate, const double *bw, const uint64_t *mem,
+                              const double *rate_cpu, const double *bw_cpu, const uint64_t *mem_cpu,
                               const uint64_t *prof, double *leaf)
 {
     const size_t total = (size_t)dm.V * dm.M * 2 * dm.LS;
@@ -30,39 +44,64 @@ __global__ void tables_kernel(Dims dm, const double *rate, const double *bw, con
         if (n < dm.N) {
             const uint64_t nb = (uint64_t)n + 1;
             const int V = dm.V;
-            const uint64_t need = nb * prof[kBlkMem * V + v] + (mf ? prof[kHeadMem * V + v] : 0ull);
-            if (need <= mem[d]) {
-                const uint64_t fl = nb * prof[kBlkFlops * V + v] + (mf ? prof[kHeadFlops * V + v] : 0ull);
-                const uint64_t by = nb * prof[kBlkBytes * V + v] + (mf ? prof[kHeadBytes * V + v] : 0ull);
+            const uint64_t bm = prof[kBlkMem * V + v];
+            const long long g = device_blocks(nb, bm, mf ? prof[kHeadMem * V + v] : 0ull, mem[d]);
+            const uint64_t c = g < 0 ? 0ull : nb - (uint64_t)g;        // offloaded blocks
+            if (g >= 0 && (c == 0 || c * bm <= mem_cpu[d])) {
+                const uint64_t gb = (uint64_t)g;
+                const uint64_t fl = gb * prof[kBlkFlops * V + v] + (mf ? prof[kHeadFlops * V + v] : 0ull);
+                const uint64_t by = gb * prof[kBlkBytes * V + v] + (mf ? prof[kHeadBytes * V + v] : 0ull);
                 const double tc = __ull2double_rn(fl) / rate[d];
                 const double tm = __ull2double_rn(by) / bw[d];
                 out = tc >= tm ? tc : tm;
+                if (c > 0) {
+                    const double hc = __ull2double_rn(c * prof[kBlkFlops * V + v]) / rate_cpu[d];
+                    const double hb = __ull2double_rn(c * prof[kBlkBytes * V + v]) / bw_cpu[d];
+                    out = out + (hc >= hb ? hc : hb);
+                }
             }
         }
         leaf[idx] = out;
     }
 }
 
-// Per (variant, device): the most blocks the device can hold, without and with
-// the LM head (the number of finite entries of its two cost rows), and the
-// per-block time max(blk_flops/rate, blk_bytes/bw) rounded down to float, used
-// by the latency bound.
+// Per (variant, device): the most blocks the device can hold in device and
+// host memory together, without and with the LM head (the number of finite
+// entries of its two cost rows), the most of them in device memory (the G of
+// the G--C split; -1 where the head does not fit), and the per-block time
+// rounded down to float, used by the latency bound: max(blk_flops/rate,
+// blk_bytes/bw), or the host's per-block time where that is smaller and the
+// device offloads (a lower bound on every block's time either way).
 __global__ void captab_kernel(Dims dm, const double *rate, const double *bw, const uint64_t *mem,
-                              const uint64_t *prof, int32_t *cap, float *cpb)
+                              const double *rate_cpu, const double *bw_cpu, const uint64_t *mem_cpu,
+                              const uint64_t *prof, int32_t *cap, int32_t *capg, float *cpb)
 {
     const size_t total = (size_t)dm.V * dm.M;
     for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < total;
          idx += (size_t)gridDim.x * blockDim.x) {
         const int v = (int)(idx / dm.M), d = (int)(idx - (size_t)v * dm.M);
         const int V = dm.V;
+        const uint64_t N = (uint64_t)dm.N;
         const uint64_t bm = prof[kBlkMem * V + v], hm = prof[kHeadMem * V + v], mm = mem[d];
-        const uint64_t c0 = bm ? mm / bm : (uint64_t)dm.N;
-        const uint64_t c1 = mm < hm ? 0ull : (bm ? (mm - hm) / bm : (uint64_t)dm.N);
-        cap[idx * 2] = (int32_t)(c0 < (uint64_t)dm.N ? c0 : (uint64_t)dm.N);
-        cap[idx * 2 + 1] = (int32_t)(c1 < (uint64_t)dm.N ? c1 : (uint64_t)dm.N);
+        const uint64_t hc = bm ? mem_cpu[d] / bm : N;                 // blocks host memory holds
+        const uint64_t g0 = bm ? mm / bm : N;
+        const uint64_t c0 = g0 + hc;
+        const uint64_t g1 = mm < hm ? 0ull : (bm ? (mm - hm) / bm : N);
+        const uint64_t c1 = mm < hm ? 0ull : g1 + hc;
+        cap[idx * 2] = (int32_t)(c0 < N ? c0 : N);
+        cap[idx * 2 + 1] = (int32_t)(c1 < N ? c1 : N);
+        capg[idx * 2] = (int32_t)(g0 < N ? g0 : N);
+        capg[idx * 2 + 1] = mm < hm ? -1 : (int32_t)(g1 < N ? g1 : N);
         const double tc = __ull2double_rn(prof[kBlkFlops * V + v]) / rate[d];
         const double tm = __ull2double_rn(prof[kBlkBytes * V + v]) / bw[d];
-        cpb[idx] = __double2float_rd(tc >= tm ? tc : tm);
+        double t = tc >= tm ? tc : tm;
+        if (dm.offload && hc > 0) {
+            const double hc_ = __ull2double_rn(prof[kBlkFlops * V + v]) / rate_cpu[d];
+            const double hb = __ull2double_rn(prof[kBlkBytes * V + v]) / bw_cpu[d];
+            const double th = hc_ >= hb ? hc_ : hb;
+            t = th < t ? th : t;
+        }
+        cpb[idx] = __double2float_rd(t);
     }
 }
 
@@ -466,9 +505,11 @@ inline unsigned grid_for(size_t n, int threads, size_t cap = 152 * 32)
 cudaError_t launch_tables(const e2_ctx *c)
 {
     const size_t total = (size_t)c->dm.V * c->dm.M * 2 * c->dm.LS;
-    tables_kernel<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm, c->rate, c->bw, c->mem, c->prof, c->leaf);
+    tables_kernel<<<grid_for(total, 256), 256, 0, c->stream>>>(c->dm, c->rate, c->bw, c->mem, c->rate_cpu, c->bw_cpu,
+                                                                c->mem_cpu, c->prof, c->leaf);
     const size_t vm = (size_t)c->dm.V * c->dm.M;
-    captab_kernel<<<grid_for(vm, 256), 256, 0, c->stream>>>(c->dm, c->rate, c->bw, c->mem, c->prof, c->cap, c->cpb);
+    captab_kernel<<<grid_for(vm, 256), 256, 0, c->stream>>>(c->dm, c->rate, c->bw, c->mem, c->rate_cpu, c->bw_cpu,
+                                                             c->mem_cpu, c->prof, c->cap, c->capg, c->cpb);
     c->launches += 2;
     return cudaGetLastError();
 }

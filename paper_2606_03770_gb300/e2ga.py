@@ -23,7 +23,8 @@ E2_OK, E2_EINVAL, E2_ENOMEM, E2_ECUDA, E2_ETIMEOUT, E2_EDEVICE, E2_ESTATE = rang
 
 
 class e2_devices(C.Structure):
-    _fields_ = [("M", C.c_int32), ("rate", C.c_void_p), ("bw", C.c_void_p), ("mem", C.c_void_p)]
+    _fields_ = [("M", C.c_int32), ("rate", C.c_void_p), ("bw", C.c_void_p), ("mem", C.c_void_p),
+                ("rate_cpu", C.c_void_p), ("bw_cpu", C.c_void_p), ("mem_cpu", C.c_void_p)]
 
 
 class e2_links(C.Structure):
@@ -49,7 +50,7 @@ class e2_genomes(C.Structure):
 
 class e2_partitions(C.Structure):
     _fields_ = [("layers", C.c_void_p), ("master", C.c_void_p), ("bsel", C.c_void_p), ("T", C.c_void_p),
-                ("lambda_", C.c_void_p)]
+                ("lambda_", C.c_void_p), ("gpu_layers", C.c_void_p)]
 
 
 class e2_stats(C.Structure):
@@ -227,8 +228,11 @@ class Engine:
                           blk_mem=u64(prob.blk_mem), head_flops=u64(prob.head_flops),
                           head_bytes=u64(prob.head_bytes), head_mem=u64(prob.head_mem),
                           act_bytes=u64(prob.act_bytes))
+        if getattr(prob, "mem_cpu", None) is not None:
+            self._host.update(rate_cpu=f64(prob.rate_cpu), bw_cpu=f64(prob.bw_cpu), mem_cpu=u64(prob.mem_cpu))
         h = self._host
-        self.devs = e2_devices(self.M, _ptr(h["rate"]), _ptr(h["bw"]), _ptr(h["mem"]))
+        self.devs = e2_devices(self.M, _ptr(h["rate"]), _ptr(h["bw"]), _ptr(h["mem"]), _ptr(h.get("rate_cpu")),
+                               _ptr(h.get("bw_cpu")), _ptr(h.get("mem_cpu")))
         self.links = e2_links(_ptr(h["lbw"]), _ptr(h["cong"]), prob.cong_lo, prob.cong_hi)
         self.profile = e2_layer_profile(self.N, self.b_max, *[_ptr(h[k]) for k in (
             "blk_flops", "blk_bytes", "blk_mem", "head_flops", "head_bytes", "head_mem", "act_bytes")],
@@ -253,6 +257,7 @@ class Engine:
         self.bsel = torch.empty((self.P, self.K), dtype=torch.int16, device=dev)
         self.T = torch.empty((self.P, self.K), dtype=torch.float64, device=dev)
         self.L = torch.empty((self.P, self.K), dtype=torch.float64, device=dev)
+        self.gpu_layers = torch.empty((self.P, self.M), dtype=torch.int16, device=dev)
 
     # -- population ------------------------------------------------------------
     def genome_struct(self, g):
@@ -279,20 +284,22 @@ class Engine:
         fit = self.fitness if fitness is None else fitness
         ps = None
         if parts is True:
-            ps = e2_partitions(_ptr(self.layers), _ptr(self.master), _ptr(self.bsel), _ptr(self.T), _ptr(self.L))
+            ps = e2_partitions(_ptr(self.layers), _ptr(self.master), _ptr(self.bsel), _ptr(self.T), _ptr(self.L),
+                               _ptr(self.gpu_layers))
         elif isinstance(parts, dict):
-            ps = e2_partitions(*[_ptr(parts.get(k)) for k in ("layers", "master", "bsel", "T", "L")])
+            ps = e2_partitions(*[_ptr(parts.get(k)) for k in ("layers", "master", "bsel", "T", "L", "gpu_layers")])
         _check(e2_eval_population(self.ctx, gs, _ptr(fit), ps), "e2_eval_population", self.ctx)
         return fit
 
     def results(self):
         """The most recent evaluation's results, as numpy arrays."""
-        ps = e2_partitions(_ptr(self.layers), _ptr(self.master), _ptr(self.bsel), _ptr(self.T), _ptr(self.L))
+        ps = e2_partitions(_ptr(self.layers), _ptr(self.master), _ptr(self.bsel), _ptr(self.T), _ptr(self.L),
+                           _ptr(self.gpu_layers))
         _check(e2_get_results(self.ctx, _ptr(self.fitness), ps), "e2_get_results", self.ctx)
         self.torch.cuda.synchronize()
         return dict(fitness=self.fitness.cpu().numpy(), layers=self.layers.cpu().numpy(),
                     master=self.master.cpu().numpy(), bsel=self.bsel.cpu().numpy(), T=self.T.cpu().numpy(),
-                    L=self.L.cpu().numpy())
+                    L=self.L.cpu().numpy(), gpu_layers=self.gpu_layers.cpu().numpy())
 
     def ga_step(self, seed, generation):
         _check(e2_ga_step(self.ctx, seed, generation), "e2_ga_step", self.ctx)

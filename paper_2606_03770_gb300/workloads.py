@@ -72,6 +72,12 @@ class Problem:
     cong_lo: float = 0.2
     cong_hi: float = 1.0
     seed: int = 0
+    # GPU-CPU offload: host compute rate (FLOP/s), host memory bandwidth
+    # (bytes/s) and host memory for offloaded blocks (bytes) per device; None:
+    # no device offloads (0 host memory: a unified-memory device)
+    rate_cpu: np.ndarray | None = None
+    bw_cpu: np.ndarray | None = None
+    mem_cpu: np.ndarray | None = None
 
     @property
     def M(self) -> int:
@@ -163,10 +169,30 @@ CONFIGS = {
 
 DEVICE_BW_GBS = (50.0, 800.0)  # device memory bandwidth, log-uniform (not given by the configs)
 B_MAX = 8
+# Host side of GPU-CPU offload (the paper's fleet mixes discrete GPUs with host
+# RAM and unified-memory devices): half the devices are unified (no host memory
+# for blocks); the others offload to U[16, 128] GB of host RAM, run offloaded
+# blocks at log-U[0.2, 2] TFLOP/s and stream them at log-U[20, 120] GB/s.
+HOST_MEM_GB = (16.0, 128.0)
+HOST_TFLOPS = (0.2, 2.0)
+HOST_BW_GBS = (20.0, 120.0)
 
 
-def make_config(name: str, seed: int = 0, P: int | None = None) -> Problem:
-    """Draw the named workload with a numpy Philox generator keyed by ``seed``."""
+def offload_fleet(M: int, seed: int):
+    """Host rates, bandwidths and memories of an offloading fleet of M devices,
+    from a generator of its own (the fleet's other draws do not move)."""
+    rng = np.random.Generator(np.random.Philox(key=seed + 104729))
+    unified = rng.uniform(0.0, 1.0, M) < 0.5
+    mem = np.array([0 if u else int(round(x * 1e9)) for u, x in zip(unified, rng.uniform(*HOST_MEM_GB, M))],
+                   dtype=np.uint64)
+    rate = _log_uniform(rng, HOST_TFLOPS[0], HOST_TFLOPS[1], M) * 1e12
+    bw = _log_uniform(rng, HOST_BW_GBS[0], HOST_BW_GBS[1], M) * 1e9
+    return rate, bw, mem
+
+
+def make_config(name: str, seed: int = 0, P: int | None = None, offload: bool = False) -> Problem:
+    """Draw the named workload with a numpy Philox generator keyed by ``seed``
+    (with ``offload``, plus the host side of GPU-CPU offload per device)."""
     c = CONFIGS[name]
     rng = np.random.Generator(np.random.Philox(key=seed))
     M = c["M"]
@@ -193,12 +219,13 @@ def make_config(name: str, seed: int = 0, P: int | None = None) -> Problem:
     prof = dense_profile(NP=NP, ND=ND, b_max=B_MAX, **c["model"])
     P_ = int(P if P is not None else c["P"])
     redraw = c.get("redraw")
+    host = dict(zip(("rate_cpu", "bw_cpu", "mem_cpu"), offload_fleet(M, seed))) if offload else {}
     return Problem(
         name=name, rate=rate, bw=bw, mem=mem, link_bw=link_bw, cong=cong,
         N=c["model"]["N"], NP=NP, ND=ND, P=P_, Q=int(math.ceil(P_ / 32)), K_max=c["K_max"],
         G=c["G"], p_mut=c.get("p_mut", 0.3), redraw=redraw is not None,
         cong_lo=(redraw or (0.2, 1.0))[0], cong_hi=(redraw or (0.2, 1.0))[1], seed=seed,
-        **prof)
+        **prof, **host)
 
 
 def make_problem(rate, bw, mem, link_bw, cong, N, blk_flops, blk_bytes, blk_mem, head_flops,
@@ -206,6 +233,9 @@ def make_problem(rate, bw, mem, link_bw, cong, N, blk_flops, blk_bytes, blk_mem,
     """Build a Problem from explicit arrays (hand-made cases, edge cases)."""
     f64 = lambda x: np.ascontiguousarray(np.asarray(x, dtype=np.float64))
     u64 = lambda x: np.ascontiguousarray(np.asarray(x, dtype=np.uint64))
+    for k, conv in (("rate_cpu", f64), ("bw_cpu", f64), ("mem_cpu", u64)):
+        if kw.get(k) is not None:
+            kw[k] = conv(kw[k])
     return Problem(name=name, rate=f64(rate), bw=f64(bw), mem=u64(mem), link_bw=f64(link_bw),
                    cong=f64(cong), N=int(N), blk_flops=u64(blk_flops), blk_bytes=u64(blk_bytes),
                    blk_mem=u64(blk_mem), head_flops=u64(head_flops), head_bytes=u64(head_bytes),

@@ -892,3 +892,148 @@ def test_splitwise_never_beats_the_role_search():
             assert (a[0], a[1]) >= (b[0], b[1])
             worse += (a[0], a[1]) > (b[0], b[1])
         assert worse >= 1
+
+
+# ---------------------------------------------------------------------------
+# GPU-CPU offload in the cost model (Sec. 1; the plans' G--C column, Sec. 4.3)
+# ---------------------------------------------------------------------------
+def _with_host(prob, rng, integer=True):
+    """Give every other device host memory for a few blocks and a slower host."""
+    import dataclasses
+    M = prob.M
+    mem_cpu = np.where(np.arange(M) % 2 == 0, rng.integers(1, 8, M), 0).astype(np.uint64)
+    if integer:
+        rate_cpu = rng.choice([0.25, 0.5], M)
+        bw_cpu = rng.choice([0.5, 1.0], M)
+    else:
+        rate_cpu = rng.uniform(0.1, 0.5, M)
+        bw_cpu = rng.uniform(0.1, 0.5, M)
+    return dataclasses.replace(prob, rate_cpu=rate_cpu, bw_cpu=bw_cpu, mem_cpu=mem_cpu)
+
+
+def test_offload_stage_cost_hand_values():
+    # device: 2 FLOP/s, 4 B/s, 7 B; block: 2 FLOP, 4 B, 2 B resident; head: 1, 1, 1
+    # host: 1 FLOP/s, 1 B/s, 5 B (two blocks)
+    prob = W.make_problem([2.0], [4.0], [7], [[np.inf]], [[1.0]], 8, [2], [4], [2], [1], [1], [1], [0],
+                          NP=1, ND=1, rate_cpu=[1.0], bw_cpu=[1.0], mem_cpu=[5])
+    op = O.OracleProblem(prob)
+    # 3 blocks fit in device memory: max(6/2, 12/4) = 3
+    assert op.stage_cost(0, 0, 3, False) == 3.0 and op.gpu_blocks(0, 0, 3, False) == 3
+    # 5 blocks: 3 on the device (3 s) + 2 on the host, max(4/1, 8/1) = 8 s
+    assert op.stage_cost(0, 0, 5, False) == 11.0 and op.gpu_blocks(0, 0, 5, False) == 3
+    # as master: the head takes 1 B of device memory (still 3 blocks fit):
+    # max(7/2, 13/4) = 3.5, plus 8 on the host
+    assert op.stage_cost(0, 0, 5, True) == 11.5 and op.gpu_blocks(0, 0, 5, True) == 3
+    # 6 blocks: 3 offloaded need 6 B of host memory, 5 available -> infeasible
+    assert op.stage_cost(0, 0, 6, False) == INF
+    # no host memory: the base model (5 blocks need 10 B > 7 B)
+    import dataclasses
+    base = O.OracleProblem(dataclasses.replace(prob, mem_cpu=np.zeros(1, np.uint64)))
+    assert base.stage_cost(0, 0, 5, False) == INF and base.stage_cost(0, 0, 3, False) == 3.0
+    # a head that does not fit in device memory cannot be placed at all
+    big = O.OracleProblem(dataclasses.replace(prob, head_mem=np.array([8], np.uint64)))
+    assert big.stage_cost(0, 0, 1, True) == INF and big.stage_cost(0, 0, 1, False) == 1.0
+
+
+def test_offload_plan_column_example():
+    """The form of the plans' G--C column: a master with device memory for 20
+    of a 24-block model's blocks beside the head runs 20--4 with the rest in
+    host memory; with more KV slots per block (a larger decode batch) fewer
+    blocks fit on the device (the decode replicas' splits shift toward the
+    host)."""
+    bm = [100, 115]                          # block bytes resident: prefill, decode with more slots
+    prob = W.make_problem([1e12], [1e11], [20 * 100 + 50 + 99], [[np.inf]], [[1.0]], 24, [10, 10], [10, 10], bm,
+                          [5, 5], [5, 5], [50, 50], [0, 0], NP=1, ND=1, rate_cpu=[1e11], bw_cpu=[1e10],
+                          mem_cpu=[10 ** 6])
+    op = O.OracleProblem(prob)
+    assert op.gpu_blocks(0, 0, 24, True) == 20          # 20--4
+    assert op.gpu_blocks(1, 0, 24, True) == 18          # 18--6
+    assert op.stage_cost(0, 0, 24, True) < INF
+
+
+def test_offload_without_host_memory_is_the_base_model():
+    import dataclasses
+    for name in ("c1_tiny", "c2"):
+        prob = W.make_config(name, P=64)
+        host = W.make_config(name, P=64, offload=True)
+        none = dataclasses.replace(host, mem_cpu=np.zeros(prob.M, np.uint64))
+        g = W.random_genomes(prob.M, prob.K_max, 64, seed=3)
+        a = O.OracleProblem(prob).eval_population(g, prob.K_max, nthreads=4)
+        b = O.OracleProblem(none).eval_population(g, prob.K_max, nthreads=4)
+        for k in ("fitness", "layers", "master", "bsel", "T", "L"):
+            assert np.array_equal(a[k], b[k]), (name, k)
+        # the fleet's own draws do not move when the host side is drawn
+        for k in ("rate", "bw", "mem", "link_bw", "cong"):
+            assert np.array_equal(getattr(prob, k), getattr(host, k))
+
+
+def test_offload_device_first_split_is_the_fastest():
+    """With the host slower per block than the device, filling device memory
+    first is the fastest of all feasible device/host splits of a stage."""
+    rng = np.random.default_rng(61)
+    for _ in range(30):
+        prob = _with_host(tiny_problem(rng, 4, 9, V=3, integer=False), rng, integer=False)
+        op = O.OracleProblem(prob)
+        for d in range(4):
+            for v in range(3):
+                for n in range(1, 10):
+                    for master in (False, True):
+                        got = op.stage_cost(v, d, n, master)
+                        hm = int(prob.head_mem[v]) if master else 0
+                        bm = int(prob.blk_mem[v])
+                        best = INF
+                        for g in range(0, n + 1):
+                            c = n - g
+                            if g * bm + hm > int(prob.mem[d]) or c * bm > int(prob.mem_cpu[d]):
+                                continue
+                            fl = g * int(prob.blk_flops[v]) + (int(prob.head_flops[v]) if master else 0)
+                            by = g * int(prob.blk_bytes[v]) + (int(prob.head_bytes[v]) if master else 0)
+                            t = max(fl / prob.rate[d], by / prob.bw[d])
+                            if c:
+                                t += max(c * int(prob.blk_flops[v]) / prob.rate_cpu[d],
+                                         c * int(prob.blk_bytes[v]) / prob.bw_cpu[d])
+                            best = min(best, t)
+                        per_dev = max(int(prob.blk_flops[v]) / prob.rate[d], int(prob.blk_bytes[v]) / prob.bw[d])
+                        per_host = max(int(prob.blk_flops[v]) / prob.rate_cpu[d],
+                                       int(prob.blk_bytes[v]) / prob.bw_cpu[d])
+                        if per_host >= per_dev:
+                            assert got == best or (got == INF and best == INF) or abs(got - best) <= 1e-12 * best
+
+
+@pytest.mark.parametrize("seed", range(16))
+def test_offload_dp_matches_brute_force(seed):
+    rng = np.random.default_rng(100 + seed)
+    N = int(rng.integers(1, 11))
+    M = 6
+    prob = _with_host(tiny_problem(rng, M, N, integer=seed % 4 != 3, head=seed % 5 != 0), rng,
+                      integer=seed % 4 != 3)
+    op = O.OracleProblem(prob)
+    for trial in range(4):
+        m = int(rng.integers(1, M + 1))
+        devs = rng.permutation(M)[:m]
+        v = int(rng.integers(0, prob.V))
+        got = op.dp_pipe(v, devs)
+        bf = bf_dp(op, v, devs, N)
+        if bf is None:
+            assert not got["ok"]
+            continue
+        V, mu, layers = bf
+        assert got["ok"] and got["V"] == V and got["mu"] == mu and list(got["layers"]) == layers
+
+
+def test_offload_metamorphic_power_of_two_scaling():
+    prob = W.make_config("c1_tiny", offload=True)
+    import dataclasses
+    fast = dataclasses.replace(prob, rate=prob.rate * 2, bw=prob.bw * 2, link_bw=prob.link_bw * 2,
+                               rate_cpu=prob.rate_cpu * 2, bw_cpu=prob.bw_cpu * 2, t_a=prob.t_a / 2,
+                               min_tps=prob.min_tps * 2)
+    g = W.random_genomes(prob.M, prob.K_max, 64, seed=8)
+    a = O.OracleProblem(prob).eval_population(g, prob.K_max)
+    b = O.OracleProblem(fast).eval_population(g, prob.K_max)
+    for k in ("layers", "master", "bsel"):
+        assert np.array_equal(a[k], b[k])
+    assert np.array_equal(a["T"] / 2, b["T"]) and np.array_equal(a["L"] / 2, b["L"])
+    assert np.array_equal(a["fitness"][:, :2] / 2, b["fitness"][:, :2])
+    # offloading changes plans: more replicas serve than without host memory
+    base = O.OracleProblem(W.make_config("c1_tiny")).eval_population(g, prob.K_max)
+    assert (a["bsel"] >= 0).sum() > (base["bsel"] >= 0).sum()
