@@ -127,8 +127,15 @@ typedef struct {
                             /* replica is evaluated in both roles, the best of  */
                             /* the 2^R assignments (least objective, then       */
                             /* phase, then smallest mask) is taken and written  */
-                            /* back into the genome's role bits.  Needs K_max   */
-                            /* <= E2_MAX_ROLE_SEARCH and b_max <= 63.           */
+                            /* back into the genome's role bits.  Replicas      */
+                            /* whose role is fixed in the winner are not        */
+                            /* enumerated: one that serves neither role         */
+                            /* (bit clear) and, under the waiting time, one     */
+                            /* that cannot decode (it prefills).  A genome with */
+                            /* more than E2_MAX_ROLE_SEARCH other replicas is   */
+                            /* not searched: it keeps its own role bits for     */
+                            /* them, the fixed ones clear, and is counted in    */
+                            /* e2_stats.role_search_capped.  Needs b_max <= 63. */
                             /* 2: the adapted-SplitWise rule of the paper's     */
                             /* comparison (Sec. 4.2 "Baseline chosen"): both    */
                             /* roles evaluated; the n_P strongest replicas      */
@@ -209,6 +216,9 @@ typedef struct {
     uint64_t launches;          /* kernels this context has launched since
                                    e2_create, cumulative (a recorded generation
                                    counts its kernel nodes per replay)          */
+    uint64_t role_search_capped;/* genomes of the last evaluation whose role
+                                   search was not run (more than
+                                   E2_MAX_ROLE_SEARCH replicas to enumerate)    */
 } e2_stats;
 
 typedef struct e2_ctx e2_ctx;
@@ -218,7 +228,7 @@ typedef struct e2_ctx e2_ctx;
 #define E2_MAX_BATCH 64
 #define E2_MAX_CLUSTERS 64
 #define E2_MAX_POP (1 << 22)
-#define E2_MAX_ROLE_SEARCH 20
+#define E2_MAX_ROLE_SEARCH 20   /* most replicas whose roles the role search enumerates */
 
 /* Bytes of device workspace a context with these sizes needs.  Returns 0 on
  * invalid sizes (each within its E2_MAX_* bound, Q <= P, and

@@ -315,12 +315,14 @@ void orc_eval_genome(const orc_problem *p, int K, const uint16_t *perm, const ui
 
 /* Alg. 2 with its role search: every replica is evaluated in both roles
  * (the prefill DP and the decode sweep), then every role assignment (bit c =
- * 1: replica c decodes) is scored with Eq. 3-5, masks in increasing order; the
- * first with the least (w, phase) wins.  The replicas' outputs are those of
- * their chosen roles, and the chosen assignment goes to *roles_out. */
-void orc_eval_genome_roles(const orc_problem *p, int K, const uint16_t *perm, const uint16_t *sizes,
-                           int R, double fit[4], int16_t *layers, int16_t *master, int16_t *bsel,
-                           double *T, double *L, uint64_t *cand, uint64_t *roles_out)
+ * 1: replica c decodes) is scored with the objective, masks in increasing
+ * order; the first with the least (objective, phase) wins.  The replicas'
+ * outputs are those of their chosen roles, and the chosen assignment goes to
+ * *roles_out.  This is the plain enumeration over all 2^R masks; the search
+ * the library runs (orc_eval_genome_roles) is pinned against it. */
+void orc_eval_genome_roles_full(const orc_problem *p, int K, const uint16_t *perm, const uint16_t *sizes,
+                                int R, double fit[4], int16_t *layers, int16_t *master, int16_t *bsel,
+                                double *T, double *L, uint64_t *cand, uint64_t *roles_out)
 {
     double Tr[2][64], Lr[2][64];
     int mur[2][64], br[2][64];
@@ -352,6 +354,88 @@ void orc_eval_genome_roles(const orc_problem *p, int K, const uint16_t *perm, co
         orc_score(p, R, mask, Tm, Lm, bm, f);
         if (!have || f[0] < bw || (f[0] == bw && f[1] < bp)) {
             have = 1; bw = f[0]; bp = f[1]; best = mask;
+        }
+    }
+    off = 0;
+    for (int c = 0; c < R; ++c) {
+        const int role = (int)((best >> c) & 1u);
+        T[c] = Tr[role][c]; L[c] = Lr[role][c]; master[c] = (int16_t)mur[role][c]; bsel[c] = (int16_t)br[role][c];
+        for (int k = 0; k < sizes[c]; ++k) layers[off + k] = lay[role][off + k];
+        off += sizes[c];
+    }
+    orc_score(p, R, best, T, L, bsel, fit);
+    *roles_out = best;
+    free(lay[0]);
+    free(lay[1]);
+}
+
+/* Most replicas that can decode whose roles orc_eval_genome_roles enumerates. */
+#define ORC_MAX_FREE_ROLES 20
+
+/* Alg. 2's role search as the library runs it, for up to 64 replicas.  Some
+ * replicas' roles are fixed in the winning assignment:
+ *  * a replica that serves neither role adds nothing in either, so its bit is
+ *    clear (the smaller mask wins the tie);
+ *  * under the waiting time (objective 0), a replica that cannot decode
+ *    prefills: clearing its decode bit leaves DS as it is and adds its
+ *    prefill rate (if any) to PS at its place in the ascending-order sum,
+ *    which can only raise PS (round-to-nearest addition is monotone), so w
+ *    and the phase do not grow, and the mask gets smaller.  (Under the
+ *    finishing time a slow prefill replica can raise the rate-weighted mean
+ *    latency, so there only the first rule applies.)
+ * So only the F other replicas are enumerated: the 2^F assignments of their
+ * roles, in increasing order of their masks (the order of the full masks),
+ * the first with the least (objective, phase) winning; each is scored as the
+ * full mask with the fixed replicas' bits clear, exactly as the plain
+ * enumeration scores it.  With more than ORC_MAX_FREE_ROLES such replicas the
+ * search is not run: the genome keeps its own role bits for them (the fixed
+ * ones clear), and *capped is set. */
+void orc_eval_genome_roles(const orc_problem *p, int K, const uint16_t *perm, const uint16_t *sizes,
+                           int R, uint64_t roles_in, double fit[4], int16_t *layers, int16_t *master,
+                           int16_t *bsel, double *T, double *L, uint64_t *cand, uint64_t *roles_out, int *capped)
+{
+    double Tr[2][64], Lr[2][64];
+    int mur[2][64], br[2][64];
+    int dok[64], pok[64];
+    int16_t *lay[2];
+    lay[0] = (int16_t *)malloc(sizeof(int16_t) * (size_t)p->M);
+    lay[1] = (int16_t *)malloc(sizeof(int16_t) * (size_t)p->M);
+    int off = 0;
+    for (int c = 0; c < K; ++c) {
+        master[c] = -1; bsel[c] = -1; T[c] = ORC_INF; L[c] = ORC_INF;
+    }
+    for (int c = 0; c < R; ++c) {
+        pok[c] = orc_eval_cluster(p, perm + off, sizes[c], 0, &Tr[0][c], &Lr[0][c], &mur[0][c], &br[0][c],
+                                  lay[0] + off, cand);
+        dok[c] = orc_eval_cluster(p, perm + off, sizes[c], 1, &Tr[1][c], &Lr[1][c], &mur[1][c], &br[1][c],
+                                  lay[1] + off, cand);
+        off += sizes[c];
+    }
+    int free_idx[64], F = 0;
+    uint64_t free_mask = 0;
+    for (int c = 0; c < R; ++c)
+        if (dok[c] || (p->objective == 1 && pok[c])) { free_idx[F++] = c; free_mask |= (uint64_t)1 << c; }
+    uint64_t best = roles_in & free_mask;
+    *capped = F > ORC_MAX_FREE_ROLES;
+    if (!*capped) {
+        double bw = ORC_INF, bp = ORC_INF;
+        int have = 0;
+        for (uint64_t sub = 0; sub < ((uint64_t)1 << F); ++sub) {
+            uint64_t mask = 0;
+            for (int j = 0; j < F; ++j)
+                if ((sub >> j) & 1u) mask |= (uint64_t)1 << free_idx[j];
+            double Tm[64], Lm[64], f[4];
+            int16_t bm[64];
+            for (int c = 0; c < R; ++c) {
+                const int role = (int)((mask >> c) & 1u);
+                Tm[c] = Tr[role][c];
+                Lm[c] = Lr[role][c];
+                bm[c] = (int16_t)br[role][c];
+            }
+            orc_score(p, R, mask, Tm, Lm, bm, f);
+            if (!have || f[0] < bw || (f[0] == bw && f[1] < bp)) {
+                have = 1; bw = f[0]; bp = f[1]; best = mask;
+            }
         }
     }
     off = 0;
@@ -433,28 +517,38 @@ void orc_eval_genome_splitwise(const orc_problem *p, int K, const uint16_t *perm
     free(lay[1]);
 }
 
+/* role_search 3 is the plain 2^R enumeration (test use only: the pin of the
+ * search).  capped_out, if not NULL, receives the genomes whose search was not
+ * run (more than ORC_MAX_FREE_ROLES replicas can decode). */
 void orc_eval_population(const orc_problem *p, int P, int K, const uint16_t *perm,
                          const uint16_t *sizes, const uint8_t *nclus, const uint64_t *roles,
                          double *fitness, int16_t *layers, int16_t *master, int16_t *bsel,
-                         double *T, double *L, uint64_t *cand, int nthreads, uint64_t *roles_out)
+                         double *T, double *L, uint64_t *cand, int nthreads, uint64_t *roles_out,
+                         uint64_t *capped_out)
 {
-    uint64_t total = 0;
+    uint64_t total = 0, capped_total = 0;
     const int M = p->M;
 #ifdef _OPENMP
-#pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads > 0 ? nthreads : 1) reduction(+ : total)
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads > 0 ? nthreads : 1) reduction(+ : total, capped_total)
 #endif
     for (int g = 0; g < P; ++g) {
         uint64_t c = 0;
-        if (p->role_search == 2)
+        int capped = 0;
+        if (p->role_search == 3)
+            orc_eval_genome_roles_full(p, K, perm + (size_t)g * M, sizes + (size_t)g * K, nclus[g],
+                                       fitness + (size_t)g * 4, layers + (size_t)g * M, master + (size_t)g * K,
+                                       bsel + (size_t)g * K, T + (size_t)g * K, L + (size_t)g * K, &c,
+                                       roles_out + g);
+        else if (p->role_search == 2)
             orc_eval_genome_splitwise(p, K, perm + (size_t)g * M, sizes + (size_t)g * K, nclus[g],
                                       fitness + (size_t)g * 4, layers + (size_t)g * M, master + (size_t)g * K,
                                       bsel + (size_t)g * K, T + (size_t)g * K, L + (size_t)g * K, &c,
                                       roles_out + g);
         else if (p->role_search)
-            orc_eval_genome_roles(p, K, perm + (size_t)g * M, sizes + (size_t)g * K, nclus[g],
+            orc_eval_genome_roles(p, K, perm + (size_t)g * M, sizes + (size_t)g * K, nclus[g], roles[g],
                                   fitness + (size_t)g * 4, layers + (size_t)g * M, master + (size_t)g * K,
                                   bsel + (size_t)g * K, T + (size_t)g * K, L + (size_t)g * K, &c,
-                                  roles_out + g);
+                                  roles_out + g, &capped);
         else {
             orc_eval_genome(p, K, perm + (size_t)g * M, sizes + (size_t)g * K, nclus[g], roles[g],
                             fitness + (size_t)g * 4, layers + (size_t)g * M, master + (size_t)g * K,
@@ -462,9 +556,11 @@ void orc_eval_population(const orc_problem *p, int P, int K, const uint16_t *per
             roles_out[g] = roles[g];
         }
         total += c;
+        capped_total += (uint64_t)capped;
     }
     (void)nthreads;
     if (cand) *cand = total;
+    if (capped_out) *capped_out = capped_total;
 }
 
 /* ------------------------------------------------------------------------ */

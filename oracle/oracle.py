@@ -78,6 +78,7 @@ def lib():
         _lib.orc_splitwise_prefill_count.argtypes = [C.c_uint64, C.c_uint64, C.c_int]
         _lib.orc_eval_population.restype = None
         _lib.orc_eval_population.argtypes = [C.c_void_p, C.c_int, C.c_int] + [C.c_void_p] * 11 + [C.c_int,
+                                                                                                   C.c_void_p,
                                                                                                    C.c_void_p]
         _lib.orc_philox4x32_10.restype = None
         _lib.orc_philox4x32_10.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p]
@@ -188,12 +189,13 @@ class OracleProblem:
                    master=np.zeros((P, K), np.int16), bsel=np.zeros((P, K), np.int16),
                    T=np.zeros((P, K), np.float64), L=np.zeros((P, K), np.float64),
                    roles=np.zeros(P, np.uint64))
-        cand = C.c_uint64(0)
+        cand, capped = C.c_uint64(0), C.c_uint64(0)
         lib().orc_eval_population(self.ref, P, K, _p(perm), _p(sizes), _p(nclus), _p(roles),
                                   _p(out["fitness"]), _p(out["layers"]), _p(out["master"]),
                                   _p(out["bsel"]), _p(out["T"]), _p(out["L"]), C.byref(cand),
-                                  int(nthreads), _p(out["roles"]))
+                                  int(nthreads), _p(out["roles"]), C.byref(capped))
         out["cand"] = cand.value
+        out["capped"] = capped.value
         return out
 
 

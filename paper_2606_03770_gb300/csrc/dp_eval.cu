@@ -929,22 +929,38 @@ __global__ void __launch_bounds__(128) finalize_score_kernel(Dims dm, DevPop pop
     atomicAdd(&out.stats[kStGenomes], 1ull);
 }
 
-// Alg. 2's role search, one warp per genome.  Each replica's lane reads its
-// two results: the prefill run (variant bit b_max, run when the memory allows)
-// and the decode sweep's answer (the largest accepted batch).  Every role
-// assignment r (bit c = 1: replica c decodes) is then scored as Eq. 3-5 score a
-// genome (PS and DS summed in ascending replica order over the replicas that
-// serve their role); the least (w, phase, r) wins.  The replicas' outputs are those of their chosen roles,
-// the chosen roles are written into the genome, and the genome is scored.
+// Alg. 2's role search, one warp per genome (or a block, below).  The lead
+// warp reads every replica's two results (lane l: replicas l and l + 32): the
+// prefill run (variant bit b_max, run when the memory allows) and the decode
+// sweep's answer (the largest accepted batch).  Every role assignment r (bit
+// c = 1: replica c decodes) is scored with the objective (PS and DS summed in
+// ascending replica order over the replicas that serve their role); the least
+// (objective, phase, r) wins.  Some replicas' roles are fixed in the winner:
+// one that serves neither role has its bit clear (it adds nothing either way,
+// and the smaller mask wins); under the waiting time, one that cannot decode
+// prefills (clearing its bit keeps DS and can only raise PS, since
+// round-to-nearest addition is monotone, so w and the phase do not grow and
+// the mask shrinks; under the finishing time a slow prefill replica can raise
+// the rate-weighted mean latency, so only the first rule applies).  The
+// search therefore walks the F other ("free") replicas' roles, free replica j
+// being replica fr(j): compact assignments r' over j, in the order of the
+// full masks they stand for.  With more than E2_MAX_ROLE_SEARCH free replicas
+// the search is not run: the genome keeps its own role bits for them (the
+// fixed replicas' bits clear) and is counted in the stats.  The replicas'
+// outputs are those of their chosen roles, the chosen roles are written into
+// the genome, and the genome is scored.
 template <int WPG, bool FT>
 __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop, SlotInfo si, SplitOut so,
                                                              EvalOut out)
 {
-    __shared__ double s_ps[4][E2_MAX_ROLE_SEARCH], s_ds[4][E2_MAX_ROLE_SEARCH];
-    __shared__ double s_pl[4][E2_MAX_ROLE_SEARCH], s_dl[4][E2_MAX_ROLE_SEARCH];   // rate x Lambda (FT)
-    __shared__ int s_pv[4][E2_MAX_ROLE_SEARCH], s_dv[4][E2_MAX_ROLE_SEARCH];
-    __shared__ int s_off[4][E2_MAX_ROLE_SEARCH + 1], s_code[4][E2_MAX_ROLE_SEARCH];
-    __shared__ long long s_qp[4][E2_MAX_ROLE_SEARCH], s_qd[4][E2_MAX_ROLE_SEARCH];
+    constexpr int KC = E2_MAX_CLUSTERS, KF = E2_MAX_ROLE_SEARCH;
+    __shared__ double s_ps[4][KC], s_ds[4][KC];
+    __shared__ double s_pl[4][KC], s_dl[4][KC];        // rate x Lambda (finishing time)
+    __shared__ int s_pv[4][KC], s_dv[4][KC];
+    __shared__ int s_off[4][KC + 1], s_code[4][KC];
+    __shared__ long long s_qp[4][KC], s_qd[4][KC];
+    __shared__ int s_fr[4][KF];                        // full index of free replica j
+    __shared__ uint64_t s_free[4];                     // mask of the free replicas
     __shared__ double s_bw[4], s_bph[4];
     __shared__ unsigned long long s_wmin[4];           // the least w a warp of the genome has scored (bits)
     __shared__ uint64_t s_br[4];
@@ -959,8 +975,8 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     const int K = dm.K, M = dm.M, V = dm.V, bp = dm.b_max;
     const int R = pop.nclus[g];
     const uint64_t roles0 = pop.roles[g];
-    // the objective of assignment r, PS and DS (and, for the finishing time,
-    // the rate-weighted latencies) summed in ascending replica order from
+    // the objective of full assignment r, PS and DS (and, for the finishing
+    // time, the rate-weighted latencies) summed in ascending replica order from
     // replica c0 on, the sums over replicas 0..c0-1 given
     constexpr bool ft = FT;                            // objective 1: the finishing time
     auto score_from = [&](uint64_t r, int c0, const double *pre, double &PS, double &DS, double &w,
@@ -981,48 +997,75 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     auto score = [&](uint64_t r, double &PS, double &DS, double &w, double &phase) {
         score_from(r, 0, zero4, PS, DS, w, phase);
     };
-    // ---- each replica's two results
-    int best = -1, pok = 0, m = 0;
-    if (lead && lane < R) {
-        const int slot = g * K + lane;
-        const uint64_t mask = si.mask[slot];
-        m = pop.sizes[slot];
-        pok = (int)((mask >> bp) & 1ull);
-        best = mask ? si.best[slot] : -1;
-        s_off[gw][lane] = si.off[slot];
-        s_pv[gw][lane] = pok;
-        s_dv[gw][lane] = best >= 0;
-        s_ps[gw][lane] = pok ? (double)dm.NP / so.T[(size_t)slot * V + bp] : 0.0;
-        s_ds[gw][lane] = best >= 0 ? (double)(best + 1) / so.T[(size_t)slot * V + best] : 0.0;
-        s_pl[gw][lane] = pok ? s_ps[gw][lane] * so.L[(size_t)slot * V + bp] : 0.0;
-        s_dl[gw][lane] = best >= 0 ? s_ds[gw][lane] * so.L[(size_t)slot * V + best] : 0.0;
+    // ---- each replica's two results (lane l: replicas l and l + 32)
+    int best[2] = {-1, -1}, pok[2] = {0, 0}, m[2] = {0, 0};
+    if (lead) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int c = lane + 32 * h;
+            if (c >= R) continue;
+            const int slot = g * K + c;
+            const uint64_t mask = si.mask[slot];
+            m[h] = pop.sizes[slot];
+            pok[h] = (int)((mask >> bp) & 1ull);
+            best[h] = mask ? si.best[slot] : -1;
+            s_off[gw][c] = si.off[slot];
+            s_pv[gw][c] = pok[h];
+            s_dv[gw][c] = best[h] >= 0;
+            s_ps[gw][c] = pok[h] ? (double)dm.NP / so.T[(size_t)slot * V + bp] : 0.0;
+            s_ds[gw][c] = best[h] >= 0 ? (double)(best[h] + 1) / so.T[(size_t)slot * V + best[h]] : 0.0;
+            s_pl[gw][c] = pok[h] ? s_ps[gw][c] * so.L[(size_t)slot * V + bp] : 0.0;
+            s_dl[gw][c] = best[h] >= 0 ? s_ds[gw][c] * so.L[(size_t)slot * V + best[h]] : 0.0;
+        }
+        // the free replicas: those that can decode, and under the finishing
+        // time also those that can only prefill
+        const bool f0 = lane < R && (best[0] >= 0 || (ft && pok[0]));
+        const bool f1 = lane + 32 < R && (best[1] >= 0 || (ft && pok[1]));
+        const unsigned b0 = __ballot_sync(0xFFFFFFFFu, f0), b1 = __ballot_sync(0xFFFFFFFFu, f1);
+        const uint64_t fm = (uint64_t)b0 | ((uint64_t)b1 << 32);
+        const uint64_t below = (1ull << lane) - 1ull;
+        if (f0) { const int j = __popcll(fm & below); if (j < KF) s_fr[gw][j] = lane; }
+        if (f1) { const int j = __popcll(fm & (below << 32 | 0xFFFFFFFFull)); if (j < KF) s_fr[gw][j] = lane + 32; }
+        if (lane == 0) { s_off[gw][R] = M; s_free[gw] = fm; }
     }
-    if (lead && lane == 0) s_off[gw][R] = M;
     if (WPG == 1) __syncwarp();
     else __syncthreads();
-    // ---- the best assignment.  Lane l owns the assignments whose first
-    //      low = min(R, 5) replicas' roles are the bits of l, and walks the
-    //      other H = R - low replicas' roles in Gray-code order (one role flips
-    //      per step).  Along the walk PS and DS are kept as exact fixed-point
-    //      sums (each rate rounded to an integer multiple of 2^-s, s per warp
-    //      so that the total stays below 2^62), with the counts of replicas
-    //      serving each role.  Two screens skip assignments that can only
-    //      lose.  (1) Integer compares: a w no larger than the best w needs
-    //      NP/PS <= max(w, T_a) and ND/DS <= T_a + w (the phase exceeds T_a
-    //      by at most w, and w >= NP/PS once it does), i.e. PS and DS above
-    //      thresholds derived from the best, with margins for the fixed-point
-    //      rounding; with a best w of 0, both must stay within the best phase.
-    //      (2) A lower bound on w and the phase from the float values of the
-    //      sums, without a division (relative error below 1e-6, against a 1e-5
-    //      margin), against the best.  The others are scored exactly: PS and DS
-    //      summed in float64 in ascending replica order, then Eq. 3-5, as the
+    const uint64_t freem = s_free[gw];
+    const int F = __popcll(freem);
+    // a compact assignment over the free replicas -> its full mask
+    auto expand = [&](uint64_t r) -> uint64_t {
+        uint64_t full = 0;
+        for (int j = 0; j < F; ++j)
+            if ((r >> j) & 1ull) full |= 1ull << s_fr[gw][j];
+        return full;
+    };
+    double bw = keyd(kInfKey), bph = keyd(kInfKey);
+    uint64_t br = ~0ull;                                // compact
+    bool capped = F > KF;
+    if (!capped) {
+    // ---- the best assignment.  Thread id owns the compact assignments whose
+    //      first low = min(F, 5) free replicas' roles (7 with a block per
+    //      genome) are the bits of id, and walks the other H = F - low free
+    //      replicas' roles in Gray-code order (one role flips per step).  Along
+    //      the walk PS and DS are kept as exact fixed-point sums (each rate
+    //      rounded to an integer multiple of 2^-s, s per genome so that the
+    //      total stays below 2^62), with the counts of replicas serving each
+    //      role; the fixed replicas add constant terms.  Two screens skip
+    //      assignments that can only lose (waiting time only).  (1) Integer
+    //      compares: a w no larger than the best w needs NP/PS <= max(w, T_a)
+    //      and ND/DS <= T_a + w (the phase exceeds T_a by at most w, and
+    //      w >= NP/PS once it does), i.e. PS and DS above thresholds derived
+    //      from the best, with margins for the fixed-point rounding; with a
+    //      best w of 0, both must stay within the best phase.  (2) A lower
+    //      bound on w and the phase from the float values of the sums, without
+    //      a division (relative error below 1e-6, against a 1e-5 margin),
+    //      against the best.  The others are scored exactly: PS and DS summed
+    //      in float64 in ascending replica order, then the objective, as the
     //      oracle does.  The best key is shared over the warp whenever a lane
     //      improves it, so that few steps of the warp take the exact path.
-    //      With at most 8 replicas every assignment is scored exactly.
-    double bw = keyd(kInfKey), bph = keyd(kInfKey);
-    uint64_t br = ~0ull;
-    constexpr int kFixed = WPG == 1 ? 5 : 7;            // replicas whose roles are the bits of id
-    const int low = R < kFixed ? R : kFixed, H = R - low;
+    //      With at most 8 free replicas every assignment is scored exactly.
+    constexpr int kFixed = WPG == 1 ? 5 : 7;            // free replicas whose roles are the bits of id
+    const int low = F < kFixed ? F : kFixed, H = F - low;
     // fixed-point scales: totals below 2^62; the screen needs every serving
     // rate to be at least 2^24 units (else every assignment is scored exactly)
     double totp = 0.0, totd = 0.0;
@@ -1031,30 +1074,37 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
     // the screens bound the waiting time; the finishing time is scored exactly
     bool in_range = !ft && isfinite(totp) && isfinite(totd) && sp_ > -126 + 64 && sp_ < 126 && sd_ > -126 + 64 &&
                     sd_ < 126;
-    if (lane < R) {
-        const long long qp = in_range && s_pv[gw][lane] ? __double2ll_rn(ldexp(s_ps[gw][lane], sp_)) : 0ll;
-        const long long qd = in_range && s_dv[gw][lane] ? __double2ll_rn(ldexp(s_ds[gw][lane], sd_)) : 0ll;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int c = lane + 32 * h;
+        if (c >= R) continue;
+        const long long qp = in_range && s_pv[gw][c] ? __double2ll_rn(ldexp(s_ps[gw][c], sp_)) : 0ll;
+        const long long qd = in_range && s_dv[gw][c] ? __double2ll_rn(ldexp(s_ds[gw][c], sd_)) : 0ll;
         if (lead) {
-            s_qp[gw][lane] = qp;
-            s_qd[gw][lane] = qd;
+            s_qp[gw][c] = qp;
+            s_qd[gw][c] = qd;
         }
-        if ((s_pv[gw][lane] && qp < (1ll << 24)) || (s_dv[gw][lane] && qd < (1ll << 24))) in_range = false;
+        if ((s_pv[gw][c] && qp < (1ll << 24)) || (s_dv[gw][c] && qd < (1ll << 24))) in_range = false;
     }
     in_range = __all_sync(0xFFFFFFFFu, in_range);
     if (lead && lane == 0) s_wmin[gw] = dkey(keyd(kInfKey));
     if (WPG == 1) __syncwarp();
     else __syncthreads();
-    if (R <= 8) {                                               // at most 256 assignments: score them all
-        for (uint64_t r = id; r < (1ull << R); r += 32 * WPG) {
+    if (F <= 8) {                                               // at most 256 assignments: score them all
+        for (uint64_t r = id; r < (1ull << F); r += 32 * WPG) {
             double PS, DS, w, ph;
-            score(r, PS, DS, w, ph);
+            score(expand(r), PS, DS, w, ph);
             if (w < bw || (w == bw && (ph < bph || (ph == bph && r < br)))) { bw = w; bph = ph; br = r; }
         }
     } else {
+        auto fr = [&](int j) { return s_fr[gw][j]; };
         long long P = 0, D = 0;                                 // fixed-point PS and DS
         int np = 0, nd = 0;                                     // replicas serving prefill / decode
-        for (int c = 0; c < R; ++c) {                           // replicas above low start as prefill
-            const bool dec = c < low && ((id >> c) & 1);
+        for (int c = 0; c < R; ++c)                             // the fixed replicas prefill
+            if (!((freem >> c) & 1ull) && s_pv[gw][c]) { P += s_qp[gw][c]; ++np; }
+        for (int j = 0; j < F; ++j) {                           // free replicas above low start as prefill
+            const int c = fr(j);
+            const bool dec = j < low && ((id >> j) & 1);
             if (dec) { if (s_dv[gw][c]) { D += s_qd[gw][c]; ++nd; } }
             else if (s_pv[gw][c]) { P += s_qp[gw][c]; ++np; }
         }
@@ -1072,21 +1122,25 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
         // the screens compare with we = min(own best w, the least w any warp of
         // the genome has scored); the phase screen only with the own best
         double wsh = keyd(kInfKey);                             // the shared least w last taken
-        // start from the genome's own roles: a real assignment, scored exactly
+        // start from the genome's own roles over the free replicas: a real
+        // assignment, scored exactly
         bool own_fin;                                           // the lane's own best w is finite
         {
-            const uint64_t r0 = roles0 & ((2ull << (R - 1)) - 1ull);
+            uint64_t r0 = 0;
+            for (int j = 0; j < F; ++j) r0 |= ((roles0 >> fr(j)) & 1ull) << j;
             double PS, DS, w, ph;
-            score(r0, PS, DS, w, ph);
+            score(expand(r0), PS, DS, w, ph);
             bw = w; bph = ph; br = r0;
             own_fin = w < keyd(kInfKey);
             improved = true;
         }
-        // one assignment: the screens, then the exact score where they cannot decide
-        // with a block per genome the roles of replicas 0..low+U-1 are fixed per
-        // thread and combination: their exact sums are taken once (prefix)
+        // one assignment: the screens, then the exact score where they cannot
+        // decide.  With a block per genome the roles of free replicas
+        // 0..low+1 are fixed per thread and combination: the exact sums over
+        // full replicas 0..fr(low+1) are taken once (prefix)
         double pre[4][4] = {{0.0, 0.0, 0.0, 0.0}, {0.0, 0.0, 0.0, 0.0}, {0.0, 0.0, 0.0, 0.0},
                             {0.0, 0.0, 0.0, 0.0}};     // [combination][PS, DS, PL, DL]
+        const int c_pre = WPG > 1 ? fr(low + 1) + 1 : 0;       // first replica after the prefix
         auto consider = [&](long long P, long long D, int np, int nd, uint64_t r, int j) {
             if (np == 0 || nd == 0) {                              // PS or DS is 0: w = phase = +inf
                 if (!own_fin && r < br) br = r;                    // ties the own best only while it is +inf
@@ -1100,22 +1154,26 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
                 if (w_lo > bw_up || (zero && ph_lo > bph_up)) return;
             }
             double PS, DS, w, ph;
-            if (WPG > 1) score_from(r, low + 2, pre[j], PS, DS, w, ph);
-            else score(r, PS, DS, w, ph);
+            if (WPG > 1) score_from(expand(r), c_pre, pre[j], PS, DS, w, ph);
+            else score(expand(r), PS, DS, w, ph);
             if (w < bw || (w == bw && (ph < bph || (ph == bph && r < br)))) {
                 bw = w; bph = ph; br = r;
                 own_fin = true;                                    // PS, DS > 0: w is finite
                 improved = true;
             }
         };
-        // the first U = min(H, 2) walked replicas are taken in all 2^U
+        // the first U = min(H, 2) walked free replicas are taken in all 2^U
         // combinations at every step (independent work for the lane); the
         // Gray code walks the other H - U
-        const int U = H < 2 ? H : 2;                            // 2 with a block per genome (R >= 9)
+        const int U = H < 2 ? H : 2;                            // 2 with a block per genome (F >= 9)
         if (WPG > 1)
             for (int j = 0; j < 4; ++j)
-                for (int c = 0; c < low + 2; ++c) {
-                    const bool dec = c < low ? ((id >> c) & 1) : ((j >> (c - low)) & 1);
+                for (int c = 0; c < c_pre; ++c) {
+                    bool dec = false;                               // fixed replicas prefill
+                    if ((freem >> c) & 1ull) {
+                        const int jj = __popcll(freem & ((1ull << c) - 1ull));   // its free index (< low + 2)
+                        dec = jj < low ? ((id >> jj) & 1) : ((j >> (jj - low)) & 1);
+                    }
                     if (dec) {
                         if (s_dv[gw][c]) {
                             pre[j][1] = pre[j][1] + s_ds[gw][c];
@@ -1128,8 +1186,8 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
                 }
         long long dP[2] = {0, 0}, dD[2] = {0, 0};
         int dn[2] = {0, 0}, dm_[2] = {0, 0};
-        for (int j = 0; j < U; ++j) {                           // replica low + j: prefill -> decode
-            const int c = low + j;
+        for (int j = 0; j < U; ++j) {                           // free replica low + j: prefill -> decode
+            const int c = fr(low + j);
             dP[j] = -s_qp[gw][c]; dD[j] = s_qd[gw][c];
             dn[j] = -s_pv[gw][c]; dm_[j] = s_dv[gw][c];
         }
@@ -1146,7 +1204,7 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
             }
             // every lane screens against the warp's best: when a lane improved
             // on its own, the best key (w, phase, r) is shared (all 32 lanes
-            // run the same number of steps once R >= 5)
+            // run the same number of steps once F >= 5)
             if (H > 0 && __any_sync(0xFFFFFFFFu, improved)) {
 #pragma unroll
                 for (int o = 16; o; o >>= 1) {
@@ -1186,8 +1244,8 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
                 }
             }
             if (++q == nq) break;
-            // the next Gray code flips bit t: replica low + U + t changes role
-            const int t = __ffsll((long long)q) - 1, c = low + U + t;
+            // the next Gray code flips bit t: free replica low + U + t changes role
+            const int t = __ffsll((long long)q) - 1, c = fr(low + U + t);
             gq ^= 1ull << t;
             const long long qp = s_qp[gw][c], qd = s_qd[gw][c];     // 0 where the role is not served
             const int pv = s_pv[gw][c], dv = s_dv[gw][c];
@@ -1211,13 +1269,21 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
             if (ow < bw || (ow == bw && (op < bph || (op == bph && orr < br)))) { bw = ow; bph = op; br = orr; }
         }
     }
+    }  // !capped
+    else if (!lead) {
+        return;
+    }
     // ---- outputs of the chosen roles (the genome's first warp)
+    const uint64_t brf = capped ? (roles0 & freem) : expand(br);
     unsigned long long n_rep = 0, n_served = 0, n_paper = 0;
-    if (lane < R) {
-        const int slot = g * K + lane;
-        const int role = (int)((br >> lane) & 1ull);
-        const int code = role ? best : (pok ? bp : -1);
-        s_code[gw][lane] = code;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int c = lane + 32 * h;
+        if (c >= R) continue;
+        const int slot = g * K + c;
+        const int role = (int)((brf >> c) & 1ull);
+        const int code = role ? best[h] : (pok[h] ? bp : -1);
+        s_code[gw][c] = code;
         if (code < 0) {
             out.master[slot] = -1; out.bsel[slot] = -1;
             out.T[slot] = keyd(kInfKey); out.L[slot] = keyd(kInfKey);
@@ -1230,9 +1296,9 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
             ++n_served;
         }
         if (si.mask[slot]) {                         // replicas with no work were counted by the pre-pass
-            const unsigned long long ndec = best >= 0 ? (unsigned long long)(bp - best) : (unsigned long long)bp;
+            const unsigned long long ndec = best[h] >= 0 ? (unsigned long long)(bp - best[h]) : (unsigned long long)bp;
             ++n_rep;
-            n_paper += (1 + ndec) * paper_candidates(m, dm.N);
+            n_paper += (1 + ndec) * paper_candidates(m[h], dm.N);
         }
     }
     __syncwarp();
@@ -1269,16 +1335,17 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
         atomicAdd(&out.stats[kStPaper], n_paper);
     }
     if (n_served) atomicAdd(&out.stats[kStServed], n_served);
+    if (capped) atomicAdd(&out.stats[kStRoleCapped], 1ull);
     double PS, DS, w, phase;
-    score(br, PS, DS, w, phase);
+    score(brf, PS, DS, w, phase);
     double *f = out.fit + (size_t)g * 4;
     f[0] = w; f[1] = phase; f[2] = PS; f[3] = DS;
-    pop.roles[g] = br;
+    pop.roles[g] = brf;
     uint64_t h = hl;
     const uint16_t *ss = pop.sizes + (size_t)g * K;
     for (int i = 0; i < R; ++i) h = mix(h, (uint64_t)ss[i] << 16);
     h = mix(h, (uint64_t)R << 40);
-    h = mix(h, br);
+    h = mix(h, brf);
     out.hash[g] = h;
     atomicAdd(&out.stats[kStGenomes], 1ull);
 }

@@ -202,11 +202,7 @@ int validate_inputs(const e2_devices *d, const e2_links *l, const e2_layer_profi
         if (!(q >= 0.0 && q <= 1.0)) { snprintf(msg, n, "probabilities must lie in [0, 1]"); return E2_EINVAL; }
     if (p->tournament < 1) { snprintf(msg, n, "tournament size must be >= 1"); return E2_EINVAL; }
     if (p->role_search < 0 || p->role_search > 2) { snprintf(msg, n, "role_search must be 0, 1 or 2"); return E2_EINVAL; }
-    if (p->role_search == 1 && (p->K_max > E2_MAX_ROLE_SEARCH || pf->b_max > 63)) {
-        snprintf(msg, n, "role_search 1 needs K_max <= %d and b_max <= 63", E2_MAX_ROLE_SEARCH);
-        return E2_EINVAL;
-    }
-    if (p->role_search == 2 && pf->b_max > 63) { snprintf(msg, n, "role_search 2 needs b_max <= 63"); return E2_EINVAL; }
+    if (p->role_search && pf->b_max > 63) { snprintf(msg, n, "role_search 1 and 2 need b_max <= 63"); return E2_EINVAL; }
     if (p->objective != 0 && p->objective != 1) { snprintf(msg, n, "objective must be 0 or 1"); return E2_EINVAL; }
     return E2_OK;
 }
@@ -711,6 +707,7 @@ int e2_get_stats(e2_ctx *c, e2_stats *out)
     out->served = s[kStServed];
     out->tps_pruned = s[kStTpsPruned];
     out->dp_runs_small = s[kStDpRunsSmall];
+    out->role_search_capped = s[kStRoleCapped];
     out->dp_launches = c->dp_grid1 > 0 ? 2 : 1;
     out->dp_ctas = (uint64_t)c->dp_grid;
     out->dp_smem = c->dp_smem;

@@ -69,7 +69,7 @@ __host__ __device__ __forceinline__ unsigned dp_item_bytes(int m, int N, int war
 
 // Stats slots (unsigned long long, atomically accumulated).
 enum StatSlot { kStGenomes = 0, kStReplicas, kStDpRuns, kStCells, kStProbes, kStPaper, kStPrecheck,
-                kStServed, kStTpsPruned, kStDpRunsSmall, kNumStats };
+                kStServed, kStTpsPruned, kStDpRunsSmall, kStRoleCapped, kNumStats };
 
 // Everything a kernel needs, passed by value.
 struct Dims {

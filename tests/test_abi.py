@@ -100,7 +100,7 @@ def _structs(prob):
 BAD = {
     "role search mode": lambda p: setattr(p, "role_search", 3),
     "objective": lambda p: setattr(p, "objective", 2),
-    "role search with many replicas": lambda p: (setattr(p, "role_search", 1), setattr(p, "K_max", 21)),
+    "role search with a large batch": lambda p: (setattr(p, "role_search", 1), setattr(p, "blk_flops", np.ones(70, np.uint64))),
     "negative rate": lambda p: p.rate.__setitem__(0, -1.0),
     "nan bandwidth": lambda p: p.bw.__setitem__(1, np.nan),
     "zero link": lambda p: p.link_bw.__setitem__((0, 1), 0.0),

@@ -1037,3 +1037,67 @@ def test_offload_metamorphic_power_of_two_scaling():
     # offloading changes plans: more replicas serve than without host memory
     base = O.OracleProblem(W.make_config("c1_tiny")).eval_population(g, prob.K_max)
     assert (a["bsel"] >= 0).sum() > (base["bsel"] >= 0).sum()
+
+
+# ---------------------------------------------------------------------------
+# Alg. 2's role search beyond 20 replicas: only replicas that can decode vary
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("objective,t_a", [(0, 1.0), (0, 1e4), (1, 1.0)])
+def test_role_search_matches_the_plain_enumeration(objective, t_a):
+    """The search enumerates the roles of the replicas that can decode only (a
+    replica that cannot decode prefills in the winning assignment).  Against
+    the plain enumeration of all 2^R masks (R <= 14): tie-heavy small-integer
+    fleets, the w = 0 plateau (a large T_a), the finishing time, and the
+    128-device workload's fleet at up to 14 replicas."""
+    import dataclasses
+    rng = np.random.default_rng(71 + objective + int(t_a))
+    cases = []
+    for _ in range(3):
+        M, N = 16, 10
+        prob = tiny_problem(rng, M, N, V=3, integer=True)
+        prob = dataclasses.replace(prob, min_tps=0.02, t_a=t_a, objective=objective)
+        cases.append((prob, W.random_genomes(M, 14, 10, seed=int(rng.integers(1 << 30)), max_clusters=14), 14))
+    c3 = dataclasses.replace(W.make_config("c3"), t_a=t_a, objective=objective)
+    cases.append((c3, W.random_genomes(c3.M, 14, 6, seed=5, max_clusters=14), 14))
+    seen_free = seen_forced = 0
+    for prob, g, K in cases:
+        fast = O.OracleProblem(dataclasses.replace(prob, role_search=1)).eval_population(g, K, nthreads=4)
+        full = O.OracleProblem(dataclasses.replace(prob, role_search=3)).eval_population(g, K, nthreads=4)
+        for k in ("fitness", "layers", "master", "bsel", "T", "L", "roles"):
+            assert np.array_equal(fast[k], full[k]), k
+        assert fast["capped"] == 0
+        dec = O.OracleProblem(dataclasses.replace(prob, role_search=0))
+        for p in range(len(g["nclus"])):
+            off = 0
+            for c in range(int(g["nclus"][p])):
+                m = int(g["sizes"][p, c])
+                can = m <= prob.N and dec.eval_cluster(g["perm"][p, off:off + m], decode=True)["ok"]
+                off += m
+                if objective == 1:
+                    can = can or (m <= prob.N and dec.eval_cluster(g["perm"][p, off - m:off], decode=False)["ok"])
+                if not can:
+                    assert (int(fast["roles"][p]) >> c) & 1 == 0       # forced to prefill
+                    seen_forced += 1
+                else:
+                    seen_free += 1
+    assert seen_free >= 20 and seen_forced >= 20
+
+
+def test_role_search_caps_at_twenty_decoding_replicas():
+    """More than 20 replicas that can decode: the search is not run; the
+    replicas keep the genome's own role bits (those that cannot decode
+    prefill), and the genome is counted as capped."""
+    import dataclasses
+    M = 24
+    prob = dataclasses.replace(_single_device_replicas([1e6 * (1 + i % 5) for i in range(M)]), role_search=1)
+    K = M
+    g = dict(perm=np.arange(M, dtype=np.uint16)[None, :].copy(), sizes=np.ones((1, K), np.uint16),
+             nclus=np.array([M], np.uint8), roles=np.array([0b1010_1100_0011_0101_1100_1010], np.uint64))
+    out = O.OracleProblem(prob).eval_population(g, K)
+    assert out["capped"] == 1 and int(out["roles"][0]) == int(g["roles"][0])
+    fixed = O.OracleProblem(dataclasses.replace(prob, role_search=0)).eval_population(g, K)
+    assert np.array_equal(out["fitness"], fixed["fitness"])
+    # 20 decoding replicas (4 more that cannot serve at all): the search runs
+    prob20 = dataclasses.replace(prob, mem=np.array([10 ** 12] * 20 + [0] * 4, np.uint64))
+    out20 = O.OracleProblem(prob20).eval_population(g, K)
+    assert out20["capped"] == 0 and int(out20["roles"][0]) >> 20 == 0
