@@ -77,6 +77,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-configs", action="store_true", help="skip the other workloads' lines")
+    ap.add_argument("--repeats", action="store_true",
+                    help="instead of timing: how often replicas repeat over the workload's generations")
     ap.add_argument("--clocks-dir", default=tempfile.gettempdir(),
                     help="folder for the raw nvidia-smi samples of the timed region (clocks_rank<i>.csv)")
     ap.add_argument("--roles", default="bits", choices=["bits", "search"],
@@ -536,9 +538,78 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def replica_keys(pop, P, K, N):
+    """(ordered device tuple, role) of every replica of a population, with the
+    size of its DP runs (m x (N - m + 1), 0 when it has more devices than
+    blocks and runs none)."""
+    keys, work = [], []
+    for g in range(P):
+        off = 0
+        R = int(pop["nclus"][g])
+        roles = int(pop["roles"][g])
+        perm = pop["perm"][g]
+        for c in range(R):
+            m = int(pop["sizes"][g][c])
+            keys.append((perm[off:off + m].tobytes(), (roles >> c) & 1))
+            work.append(m * (N - m + 1) if m <= N else 0)
+            off += m
+    return keys, work
+
+
+def run_repeats(args):
+    """How often a replica (its ordered devices and role) that the evaluation
+    meets was already evaluated: within the same generation, and within the
+    last `window` generations (what a per-replica result cache, Sec. 3.4,
+    would serve), over a long run of the search, by count and by DP work."""
+    import torch
+    import __graft_entry__ as ge
+    ge.build()
+    from paper_2606_03770_gb300.e2ga import Engine
+    prob = problem(args)
+    eng = Engine(prob)
+    eng.init_population(args.seed)
+    window, marks = 5, {1, 2, 10, 50, 100, 150, max(prob.G, 2)}
+    keep = {g for m in marks for g in range(max(1, m - window), m + 1)}
+    hist, rows = {}, []
+    for gen in range(1, max(prob.G, 2) + 1):
+        if gen in keep:
+            pop = eng.get_population()
+            hist[gen] = replica_keys(pop, prob.P, prob.K_max, prob.N)
+        if gen in marks:
+            keys, work = hist[gen]
+            seen, within, within_w = set(), 0, 0
+            for k, w in zip(keys, work):
+                if k in seen:
+                    within += 1
+                    within_w += w
+                seen.add(k)
+            past = set()
+            for g2 in range(max(1, gen - window), gen):
+                past.update(hist[g2][0])
+            cache, cache_w = 0, 0
+            seen = set()
+            for k, w in zip(keys, work):
+                if k in seen or k in past:
+                    cache += 1
+                    cache_w += w
+                seen.add(k)
+            tw = max(1, sum(work))
+            rows.append({"generation": gen, "replicas": len(keys),
+                         "repeat_within_generation": within / len(keys),
+                         "repeat_within_generation_work": within_w / tw,
+                         f"hit_cache_last_{window}_generations": cache / len(keys),
+                         f"hit_cache_last_{window}_generations_work": cache_w / tw})
+        eng.run_generation(args.seed, gen)
+    torch.cuda.synchronize()
+    eng.close()
+    print(json.dumps({"workload": workload_label(prob), "generations": max(prob.G, 2), "rates": rows}), flush=True)
+
+
 def main():
     args = parse()
-    if args.impl == "reference":
+    if args.repeats:
+        run_repeats(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)
