@@ -51,8 +51,11 @@ typedef enum {
     E2_EINVAL = 1,    /* invalid argument (null pointer, size, value, genome) */
     E2_ENOMEM = 2,    /* workspace smaller than e2_workspace_bytes()          */
     E2_ECUDA = 3,     /* a CUDA runtime call failed                           */
-    E2_ETIMEOUT = 4,  /* a bounded device wait expired                        */
-    E2_EDEVICE = 5,   /* a device-side check failed (see e2_strerror)         */
+                      /* (4 is not used: no kernel waits on the device)       */
+    E2_EDEVICE = 5,   /* a device-side consistency check failed: an evaluation */
+                      /* met a state its own pre-checks rule out (reported by  */
+                      /* e2_get_stats; the results of that evaluation are not  */
+                      /* to be trusted)                                        */
     E2_ESTATE = 6     /* call order: e.g. e2_ga_step before any evaluation    */
 } e2_status;
 
@@ -89,11 +92,25 @@ typedef struct {
 } e2_links;
 
 /* Layer profile of one model (Sec. 3.1, Alg. 2 inputs l_P, l_D(b)).  N
- * identical blocks; V = 1 + b_max variants: v = 0 prefill (one request of NP
- * tokens), v = b decode with b requests in flight.  The stage time of n
- * blocks on device d is max(flops/rate_d, bytes/bw_d) with
- * flops = n*blk_flops[v] (+ head_flops[v] on the master), likewise bytes;
- * it is +inf when n*blk_mem[v] (+ head_mem[v]) exceeds mem_d. */
+ * blocks; V = 1 + b_max variants: v = 0 prefill (one request of NP tokens),
+ * v = b decode with b requests in flight.  With PF == NULL the blocks are
+ * identical: the stage time of n blocks on device d is max(flops/rate_d,
+ * bytes/bw_d) with flops = n*blk_flops[v] (+ head_flops[v] on the master),
+ * likewise bytes; it is +inf when n*blk_mem[v] (+ head_mem[v]) exceeds mem_d.
+ *
+ * Blocks of several types (Sec. 3.1: blocks of one type, e.g. sliding-window
+ * or full attention, share a latency): PF, PB, PM give per variant the prefix
+ * sums [V][N+1] of the blocks' flops, bytes and resident bytes (PF[v][0] = 0,
+ * non-decreasing).  The stage of blocks j..i then costs PF[v][i+1]-PF[v][j]
+ * flops (+ the head on the master), likewise bytes and memory.  A stage's cost
+ * depends on where it starts, and the best bottleneck of a prefix is no longer
+ * monotone in its length, so these contexts run the plain scan over every
+ * split (Alg. 1's recurrence, with the masters factored through prefix and
+ * suffix tables) instead of the identical-block kernel.  Needs
+ * e2_workspace_bytes_ex(..., E2_WS_LAYERED), N <= E2_MAX_LAYERED_BLOCKS, and
+ * no GPU-CPU offload (mem_cpu NULL or all zero).  blk_* must still hold valid
+ * values (they bound the range checks; the largest block's work is a good
+ * choice). */
 typedef struct {
     int32_t N;                      /* blocks, 1..E2_MAX_BLOCKS               */
     int32_t b_max;                  /* 1..E2_MAX_BATCH                        */
@@ -106,6 +123,9 @@ typedef struct {
     const uint64_t *act_bytes;      /* [V] activation bytes per link crossing */
     uint64_t NP;                    /* mean input tokens per request, >= 1    */
     uint64_t ND;                    /* mean generated tokens per request, >= 1*/
+    const uint64_t *PF;             /* [V][N+1] prefix sums of block flops, or NULL */
+    const uint64_t *PB;             /* [V][N+1] of block bytes (NULL iff PF is)     */
+    const uint64_t *PM;             /* [V][N+1] of block resident bytes             */
 } e2_layer_profile;
 
 /* Search parameters (Alg. 2 inputs P, G, Q, Min_TPS; App. A mutation mix). */
@@ -219,6 +239,12 @@ typedef struct {
     uint64_t role_search_capped;/* genomes of the last evaluation whose role
                                    search was not run (more than
                                    E2_MAX_ROLE_SEARCH replicas to enumerate)    */
+    uint64_t device_errors;     /* consistency checks of the last evaluation
+                                   that failed on the device (a DP run whose
+                                   memory the pre-pass tested exactly found no
+                                   partition, or a traceback found no split
+                                   attaining its cell); nonzero makes
+                                   e2_get_stats return E2_EDEVICE               */
 } e2_stats;
 
 typedef struct e2_ctx e2_ctx;
@@ -229,12 +255,22 @@ typedef struct e2_ctx e2_ctx;
 #define E2_MAX_CLUSTERS 64
 #define E2_MAX_POP (1 << 22)
 #define E2_MAX_ROLE_SEARCH 20   /* most replicas whose roles the role search enumerates */
+#define E2_MAX_LAYERED_BLOCKS 180   /* most blocks of a profile with per-layer sums */
+#define E2_WS_LAYERED 1u        /* e2_workspace_bytes_ex flag: per-layer profile (PF != NULL) */
 
 /* Bytes of device workspace a context with these sizes needs.  Returns 0 on
  * invalid sizes (each within its E2_MAX_* bound, Q <= P, and
  * P * K_max * (b_max + 1) < 2^31).  Reads only M, N, b_max, P, Q, K_max. */
 size_t e2_workspace_bytes(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_t Q,
                           int32_t K_max);
+
+/* The same with flags: E2_WS_LAYERED adds the per-layer stage-cost table of a
+ * profile with prefix sums (V x M x 2 x N x N float64 times: 29 MB for 32
+ * devices and 80 blocks, 1.2 GB for 512 devices and 126 blocks).  Returns 0
+ * on invalid sizes or unknown flags (and with E2_WS_LAYERED for
+ * N > E2_MAX_LAYERED_BLOCKS). */
+size_t e2_workspace_bytes_ex(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_t Q, int32_t K_max,
+                             uint32_t flags);
 
 /* Validate and copy the inputs (host pointers), lay out the workspace, build
  * the stage-cost and link-cost tables on the device (Sec. 3.2 cost model) and
@@ -334,7 +370,8 @@ int e2_run_generation(e2_ctx *ctx, uint64_t seed, uint32_t generation);
 int e2_run_generation_io(e2_ctx *ctx, const e2_genomes *population, uint64_t seed, uint32_t generation,
                          double *fitness_out, const e2_genomes *next_out);
 
-/* Counters of the last evaluation.  Synchronises. */
+/* Counters of the last evaluation.  Synchronises.  Fills *out and returns
+ * E2_EDEVICE (with a message in e2_last_error) when device_errors is nonzero. */
 int e2_get_stats(e2_ctx *ctx, e2_stats *out);
 
 /* Timing hook (no counterpart in the paper; for measurement): two CUDA events

@@ -59,6 +59,9 @@ typedef struct {
     const double *rate_cpu;      /* [M] host FLOP/s of offloaded blocks, or   */
     const double *bw_cpu;        /* [M] host bytes/s; mem_cpu [M] host bytes  */
     const uint64_t *mem_cpu;     /* for blocks; NULL: no offload anywhere     */
+    const uint64_t *PF, *PB, *PM;/* [V][N+1] prefix sums of per-block flops,  */
+                                 /* bytes, resident bytes (blocks of several  */
+                                 /* types, Sec. 3.1); NULL: identical blocks  */
 } orc_problem;
 
 /* ------------------------------------------------------------------------ */
@@ -91,6 +94,28 @@ int orc_gpu_blocks(const orc_problem *p, int v, int d, int n, int master)
  * host memory (mem_cpu) at the host's, one after the other, so their times
  * add.  Without host memory (mem_cpu NULL or 0: unified-memory devices) every
  * block must fit in device memory, as before. */
+double orc_stage_cost(const orc_problem *p, int v, int d, int n, int master);
+
+/* l_k(j,i,m) for blocks of several types (Sec. 3.1: blocks of the same type
+ * share a latency, types such as sliding-window and full attention differ):
+ * the stage of blocks j..j+n-1 costs the sums of its blocks' work, read off
+ * the per-variant prefix sums PF, PB, PM (the head added on the master), the
+ * larger of compute and streaming time, +inf beyond device memory.  Without
+ * prefix sums every block is the same and only n matters. */
+double orc_stage_cost_at(const orc_problem *p, int v, int d, int j, int n, int master)
+{
+    if (!p->PF) return orc_stage_cost(p, v, d, n, master);
+    const uint64_t *pf = p->PF + (size_t)v * (p->N + 1), *pb = p->PB + (size_t)v * (p->N + 1),
+                   *pm = p->PM + (size_t)v * (p->N + 1);
+    uint64_t need = pm[j + n] - pm[j] + (master ? p->head_mem[v] : 0);
+    if (need > p->mem[d]) return ORC_INF;
+    uint64_t fl = pf[j + n] - pf[j] + (master ? p->head_flops[v] : 0);
+    uint64_t by = pb[j + n] - pb[j] + (master ? p->head_bytes[v] : 0);
+    double tc = (double)fl / p->rate[d];
+    double tm = (double)by / p->bw[d];
+    return tc >= tm ? tc : tm;
+}
+
 double orc_stage_cost(const orc_problem *p, int v, int d, int n, int master)
 {
     int g = orc_gpu_blocks(p, v, d, n, master);
@@ -150,7 +175,7 @@ int orc_dp_pipe(const orc_problem *p, int v, const uint16_t *devs, int m,
 
     for (int mu = 1; mu <= m; ++mu) {                    /* master enumeration */
         for (int i = 0; i < N; ++i) {                    /* Eq. 2 (k = 1)      */
-            D[i] = orc_stage_cost(p, v, devs[0], i + 1, mu == 1);
+            D[i] = orc_stage_cost_at(p, v, devs[0], 0, i + 1, mu == 1);
             TB[i] = -1;
             count += 1;
         }
@@ -163,7 +188,7 @@ int orc_dp_pipe(const orc_problem *p, int v, const uint16_t *devs, int m,
                 double bestc = ORC_INF;
                 int bj = -1;
                 for (int j = k - 1; j <= i; ++j) {
-                    double c = dmax(dmax(Dp[j - 1], orc_stage_cost(p, v, devs[k - 1], i - j + 1, mu == k)), tau);
+                    double c = dmax(dmax(Dp[j - 1], orc_stage_cost_at(p, v, devs[k - 1], j, i - j + 1, mu == k)), tau);
                     count += 1;
                     if (c < bestc) { bestc = c; bj = j; }
                 }
@@ -202,10 +227,12 @@ int orc_dp_pipe(const orc_problem *p, int v, const uint16_t *devs, int m,
 double orc_latency(const orc_problem *p, int v, const uint16_t *devs, int m, int mu,
                    const int16_t *layers)
 {
-    double s = orc_stage_cost(p, v, devs[0], layers[0], mu == 0);
+    double s = orc_stage_cost_at(p, v, devs[0], 0, layers[0], mu == 0);
+    int j = layers[0];
     for (int k = 1; k < m; ++k) {
         s = s + orc_link_cost(p, v, devs[k - 1], devs[k]);
-        s = s + orc_stage_cost(p, v, devs[k], layers[k], mu == k);
+        s = s + orc_stage_cost_at(p, v, devs[k], j, layers[k], mu == k);
+        j += layers[k];
     }
     return s;
 }

@@ -44,7 +44,7 @@ class _Problem(C.Structure):
                 ("act_bytes", C.c_void_p), ("NP", C.c_uint64), ("ND", C.c_uint64),
                 ("min_tps", C.c_double), ("t_a", C.c_double), ("role_search", C.c_int),
                 ("objective", C.c_int), ("rate_cpu", C.c_void_p), ("bw_cpu", C.c_void_p),
-                ("mem_cpu", C.c_void_p)]
+                ("mem_cpu", C.c_void_p), ("PF", C.c_void_p), ("PB", C.c_void_p), ("PM", C.c_void_p)]
 
 
 class _GA(C.Structure):
@@ -59,6 +59,8 @@ def lib():
         _lib = C.CDLL(build())
         _lib.orc_stage_cost.restype = C.c_double
         _lib.orc_stage_cost.argtypes = [C.c_void_p, C.c_int, C.c_int, C.c_int, C.c_int]
+        _lib.orc_stage_cost_at.restype = C.c_double
+        _lib.orc_stage_cost_at.argtypes = [C.c_void_p, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int]
         _lib.orc_gpu_blocks.restype = C.c_int
         _lib.orc_gpu_blocks.argtypes = [C.c_void_p, C.c_int, C.c_int, C.c_int, C.c_int]
         _lib.orc_link_cost.restype = C.c_double
@@ -121,13 +123,17 @@ class OracleProblem:
         off = getattr(prob, "mem_cpu", None) is not None
         if off:
             self.arrays.update(rate_cpu=f64(prob.rate_cpu), bw_cpu=f64(prob.bw_cpu), mem_cpu=u64(prob.mem_cpu))
+        layered = getattr(prob, "PF", None) is not None
+        if layered:
+            self.arrays.update(PF=u64(prob.PF), PB=u64(prob.PB), PM=u64(prob.PM))
         a = self.arrays
         self.s = _Problem(prob.M, prob.N, prob.V, *[_p(a[k]) for k in
                           ("rate", "bw", "mem", "link_bw", "cong", "blk_flops", "blk_bytes",
                            "blk_mem", "head_flops", "head_bytes", "head_mem", "act_bytes")],
                           prob.NP, prob.ND, prob.min_tps, prob.t_a, int(getattr(prob, "role_search", 0)),
                           int(getattr(prob, "objective", 0)),
-                          *([_p(a[k]) for k in ("rate_cpu", "bw_cpu", "mem_cpu")] if off else [None] * 3))
+                          *([_p(a[k]) for k in ("rate_cpu", "bw_cpu", "mem_cpu")] if off else [None] * 3),
+                          *([_p(a[k]) for k in ("PF", "PB", "PM")] if layered else [None] * 3))
 
     def set_cong(self, cong):
         self.arrays["cong"] = np.ascontiguousarray(cong, dtype=np.float64)
@@ -139,6 +145,9 @@ class OracleProblem:
 
     def stage_cost(self, v, d, n, master):
         return lib().orc_stage_cost(self.ref, v, d, n, int(master))
+
+    def stage_cost_at(self, v, d, j, n, master):
+        return lib().orc_stage_cost_at(self.ref, v, d, j, n, int(master))
 
     def gpu_blocks(self, v, d, n, master):
         return lib().orc_gpu_blocks(self.ref, v, d, n, int(master))

@@ -286,6 +286,11 @@ __global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop
             for (int pass = 0; pass < npass; ++pass) {
                 const int prole = dm.role_search ? (pass == 0) : role;
                 const int nvar = prole ? dm.b_max : 1;
+                if (dm.layered) {                           // per-layer profiles: every variant runs (the
+                    if (dm.role_search && !prole) mask |= 1ull << dm.b_max;   // tests assume identical blocks)
+                    else mask |= nvar >= 64 ? ~0ull : ((1ull << nvar) - 1ull);
+                    continue;
+                }
                 const bool bound = prole && dm.min_tps > 0.0;
                 // When the costs grow with the batch both verdicts are monotone,
                 // so each is found by a search over the variants: the largest
@@ -674,7 +679,14 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
             __syncthreads();
             const uint32_t V = s_V;
             const int mus = s_mu;
-            if (V == kInf) continue;   // cannot happen: the pre-pass checked memory
+            if (V == kInf) {
+                // the pre-pass tested this variant's memory exactly, unless the
+                // profile's costs do not grow with the batch: then the batches
+                // below the largest that passed run untested, and may have no
+                // partition.  Otherwise this cannot happen.
+                if (tid == 0 && (dm.grows || !role)) atomicAdd(&out.stats[kStDeviceErrors], 1ull);
+                continue;
+            }
             for (int r = tid; r < W; r += blockDim.x)
                 row1s[r] = (Key)tb.leaf_rank[((vM + devs[mus - 1]) * 2 + 1) * dm.LS + r];
             __syncthreads();
@@ -765,6 +777,250 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
     }
     if (tid == 0 && st_runs) atomicAdd(&out.stats[cls ? kStDpRunsSmall : kStDpRuns], st_runs);
   }
+}
+
+// ---------------------------------------------------------------------------
+// Blocks of several types (per-layer prefix sums): the plain-scan DP.
+//
+// A stage's cost now depends on where it starts, and the best bottleneck of a
+// prefix is no longer monotone in its length (a heavy block can make fewer
+// blocks cost more), so the crossover bisection of dp_eval_body does not
+// apply.  Each cell takes the full minimum over its splits, as Eq. 1 writes
+// it, on the float64 times themselves (their bit patterns, which order like
+// the values), read from the per-layer cost table:
+//   F_k[r] = min_s max(F_{k-1}[s], l_k(s+k-1 .. r+k-1), tau_k)     devices 1..k, no master
+//   G_k[b] = min_t max(l_k(first t+1 of its range), G_{k+1}[b-t], tau_{k+1})   devices k..m
+//   V_mu   = min_{a,b} max(F_{mu-1}[a], l^head_mu(the W-a-b blocks between), G_{mu+1}[b], tau_mu, tau_mu+1)
+// mu* = the smallest mu with the least V_mu; its prefix columns (the head at
+// mu*) are recomputed from column mu* on, and the traceback takes the smallest
+// split attaining each cell's value.  Every value and tie is the oracle's.
+// ---------------------------------------------------------------------------
+__host__ __device__ __forceinline__ unsigned dp_layered_item_bytes(int m, int N)
+{
+    const unsigned W = (unsigned)(N - m + 1);
+    const unsigned bytes = 8u * (2u * (unsigned)m * W + 2u * (unsigned)m) + 4u * (unsigned)m + 2u * (unsigned)m;
+    return (bytes + 15u) & ~15u;
+}
+
+size_t dp_layered_smem_bytes(int M, int N)
+{
+    size_t best = 0;
+    const int mmax = M < N ? M : N;
+    for (int m = 1; m <= mmax; ++m) {
+        const size_t b = dp_layered_item_bytes(m, N);
+        if (b > best) best = b;
+    }
+    return best;
+}
+
+__global__ void __launch_bounds__(128) dp_layered_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out, WorkList wl,
+                                                         SlotInfo si, SplitOut so)
+{
+    extern __shared__ __align__(16) unsigned char lsm[];
+    __shared__ unsigned s_item;
+    __shared__ int s_done, s_mu;
+    __shared__ double s_T, s_L;
+    const int K = dm.K, M = dm.M, N = dm.N;
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
+    const uint64_t INF = kInfKey;
+    const unsigned n_items = wl.ctrl[kCtrlEnd];
+    const size_t NN = (size_t)N * N;
+    for (;;) {
+        if (tid == 0) s_item = atomicAdd(&wl.ctrl[kCtrlNext], 1u);
+        __syncthreads();
+        const unsigned idx = s_item;
+        __syncthreads();
+        if (idx >= n_items) break;
+        const uint64_t item = wl.items[idx];
+        const int slot = (int)(item >> 8), code = (int)(item & 0x3Fu);
+        if (tid == 0) s_done = *(volatile const int32_t *)&si.best[slot] > code;   // a larger batch won
+        __syncthreads();
+        if (s_done) continue;
+        const int g = slot / K, c = slot - g * K;
+        const size_t gk = (size_t)g * K + c;
+        const int off = si.off[slot], m = pop.sizes[gk];
+        const int role = (int)((item >> 7) & 1u);
+        const bool sweep = (item >> 6) & 1u;
+        const int v = role ? code + 1 : 0;
+        const int W = N - m + 1;
+        uint64_t *F = reinterpret_cast<uint64_t *>(lsm);          // [m][W] prefix (then mu*'s) columns
+        uint64_t *G = F + (size_t)m * W;                          // [m][W] suffix columns
+        uint64_t *Vmu = G + (size_t)m * W;                        // [m]
+        uint64_t *tk = Vmu + m;                                   // [m] tk[k] = link k-1 -> k (0-based)
+        int *nk = reinterpret_cast<int *>(tk + m);                // [m]
+        uint16_t *devs = reinterpret_cast<uint16_t *>(nk + m);    // [m]
+        const double *lc = tb.lcost + (size_t)v * M * 2 * NN;
+        for (int k = tid; k < m; k += blockDim.x) devs[k] = pop.perm[(size_t)g * M + off + k];
+        __syncthreads();
+        for (int k = tid; k < m; k += blockDim.x)
+            tk[k] = k ? dkey(tb.tau[((size_t)v * M + devs[k - 1]) * M + devs[k]]) : 0ull;
+        // l_k(j .. j+n-1) (k 0-based), with the head when mf
+        auto cost = [&](int k, int j, int n, int mf) -> uint64_t {
+            return dkey(lc[((size_t)devs[k] * 2 + mf) * NN + (size_t)j * N + (n - 1)]);
+        };
+        __syncthreads();
+        unsigned long long probes = 0;
+        // ---- prefix columns F_1..F_m (no master)
+        for (int r = tid; r < W; r += blockDim.x) F[r] = cost(0, 0, r + 1, 0);
+        __syncthreads();
+        for (int k = 2; k <= m; ++k) {
+            const uint64_t *prev = F + (size_t)(k - 2) * W;
+            uint64_t *cur = F + (size_t)(k - 1) * W;
+            const uint64_t t = tk[k - 1];
+            for (int r = tid; r < W; r += blockDim.x) {
+                uint64_t best = INF;
+                for (int s2 = 0; s2 <= r; ++s2)
+                    best = umin64(best, umax64(umax64(prev[s2], cost(k - 1, s2 + k - 1, r - s2 + 1, 0)), t));
+                cur[r] = best;
+                probes += (unsigned long long)(r + 1);
+            }
+            __syncthreads();
+        }
+        // ---- suffix columns G_m..G_2: devices k..m hold the last b + m - k + 1 blocks
+        for (int b = tid; b < W; b += blockDim.x) G[(size_t)(m - 1) * W + b] = cost(m - 1, N - 1 - b, b + 1, 0);
+        __syncthreads();
+        for (int k = m - 1; k >= 2; --k) {
+            const uint64_t *nxt = G + (size_t)k * W;
+            uint64_t *cur = G + (size_t)(k - 1) * W;
+            const uint64_t t = tk[k];
+            for (int b = tid; b < W; b += blockDim.x) {
+                const int j0 = N - (b + m - k + 1);
+                uint64_t best = INF;
+                for (int t2 = 0; t2 <= b; ++t2)
+                    best = umin64(best, umax64(umax64(cost(k - 1, j0, t2 + 1, 0), nxt[b - t2]), t));
+                cur[b] = best;
+                probes += (unsigned long long)(b + 1);
+            }
+            __syncthreads();
+        }
+        // ---- masters: a warp per master, lanes over the (a, b) splits
+        for (int mu = wid + 1; mu <= m; mu += NW) {
+            const uint64_t *Fp = mu >= 2 ? F + (size_t)(mu - 2) * W : nullptr;
+            const uint64_t *Gs = mu <= m - 1 ? G + (size_t)mu * W : nullptr;
+            uint64_t lk = 0;
+            if (mu >= 2) lk = umax64(lk, tk[mu - 1]);
+            if (mu <= m - 1) lk = umax64(lk, tk[mu]);
+            uint64_t best = INF;
+            const int amax = mu >= 2 ? W - 1 : 0;
+            for (int a = 0; a <= amax; ++a) {
+                const uint64_t fa = Fp ? Fp[a] : 0ull;
+                if (fa >= best) continue;                       // cannot lower the minimum
+                const int bmax = mu <= m - 1 ? W - 1 - a : 0;
+                for (int b = lane; b <= bmax; b += 32) {
+                    const uint64_t gb = Gs ? Gs[b] : 0ull;
+                    const uint64_t h = cost(mu - 1, (mu - 1) + a, W - a - b, 1);
+                    best = umin64(best, umax64(umax64(fa, gb), umax64(h, lk)));
+                }
+                probes += (unsigned long long)((bmax + 1 + 31 - lane) / 32);
+#pragma unroll
+                for (int o = 16; o; o >>= 1) best = umin64(best, __shfl_xor_sync(0xFFFFFFFFu, best, o));
+            }
+            if (lane == 0) Vmu[mu - 1] = best;
+        }
+        __syncthreads();
+        if (tid == 0) {                                           // the smallest master with the least value
+            int mus = 1;
+            for (int mu = 2; mu <= m; ++mu)
+                if (Vmu[mu - 1] < Vmu[mus - 1]) mus = mu;
+            s_mu = mus;
+        }
+        __syncthreads();
+        const int mus = s_mu;
+        const uint64_t V = Vmu[mus - 1];
+        if (V == INF) {                                           // no partition (memory)
+            if (tid == 0 && !role) {                              // a prefill result that does not exist
+                const size_t sv = gk * dm.V + code;
+                so.T[sv] = keyd(kInfKey);
+                so.L[sv] = keyd(kInfKey);
+            }
+            if (lane == 0) atomicAdd(&out.stats[kStProbes], probes);
+            if (tid == 0) atomicAdd(&out.stats[kStDpRuns], 1ull);
+            __syncthreads();
+            continue;
+        }
+        // ---- mu*'s prefix columns from column mu* on (the head at mu*)
+        for (int k = mus; k <= m; ++k) {
+            uint64_t *cur = F + (size_t)(k - 1) * W;
+            const int mf = k == mus;
+            if (k == 1) {
+                for (int r = tid; r < W; r += blockDim.x) cur[r] = cost(0, 0, r + 1, 1);
+            } else {
+                const uint64_t *prev = F + (size_t)(k - 2) * W;
+                const uint64_t t = tk[k - 1];
+                for (int r = tid; r < W; r += blockDim.x) {
+                    uint64_t best = INF;
+                    for (int s2 = 0; s2 <= r; ++s2)
+                        best = umin64(best, umax64(umax64(prev[s2], cost(k - 1, s2 + k - 1, r - s2 + 1, mf)), t));
+                    cur[r] = best;
+                    probes += (unsigned long long)(r + 1);
+                }
+            }
+            __syncthreads();
+        }
+        // ---- traceback (warp 0): the smallest split attaining each cell's value
+        if (wid == 0) {
+            int r = W - 1;
+            for (int k = m; k >= 2; --k) {
+                const uint64_t D = F[(size_t)(k - 1) * W + r];
+                const uint64_t *prev = F + (size_t)(k - 2) * W;
+                const uint64_t t = tk[k - 1];
+                const int mf = k == mus;
+                int sp = -1;
+                for (int base = 0; base <= r && sp < 0; base += 32) {
+                    const int s2 = base + lane;
+                    const bool hit = s2 <= r && umax64(umax64(prev[s2], cost(k - 1, s2 + k - 1, r - s2 + 1, mf)), t) == D;
+                    const unsigned bal = __ballot_sync(0xFFFFFFFFu, hit);
+                    if (bal) sp = base + __ffs(bal) - 1;
+                }
+                if (sp < 0) {                                     // cannot happen: D is attained
+                    sp = 0;
+                    if (lane == 0) atomicAdd(&out.stats[kStDeviceErrors], 1ull);
+                }
+                if (lane == 0) nk[k - 1] = r - sp + 1;
+                r = sp;
+            }
+            if (lane == 0) nk[0] = r + 1;
+            __syncwarp();
+            // stage and link times of the partition in pipeline order
+            if (lane == 0) {
+                double lam = 0.0;
+                uint64_t tmax = 0;
+                int j = 0;
+                for (int k = 0; k < m; ++k) {
+                    const double lk = keyd(cost(k, j, nk[k], k == mus - 1));
+                    const double tl = k ? keyd(tk[k]) : 0.0;
+                    if (k == 0) lam = lk;
+                    else { lam = lam + tl; lam = lam + lk; }
+                    tmax = umax64(tmax, umax64(dkey(lk), dkey(tl)));
+                    j += nk[k];
+                }
+                s_L = lam;
+                s_T = keyd(tmax);
+                s_done = (!role) || lam <= dm.lam_max;            // 1.0 / lam >= Min_TPS
+            }
+        }
+        __syncthreads();
+        const size_t sv = gk * dm.V + code;
+        if (s_done) {
+            int16_t *lay_out = so.layers + ((size_t)g * dm.V + code) * M + off;
+            for (int k = tid; k < m; k += blockDim.x) lay_out[k] = (int16_t)nk[k];
+            if (tid == 0) {
+                so.mu[sv] = (int16_t)(mus - 1);
+                so.T[sv] = s_T;
+                so.L[sv] = s_L;
+                __threadfence();
+                if (sweep) atomicMax(&si.best[slot], code);
+            }
+        } else if (tid == 0 && !role) {
+            so.T[sv] = keyd(kInfKey);
+        }
+        if (lane == 0) atomicAdd(&out.stats[kStProbes], probes);
+        if (tid == 0) {
+            atomicAdd(&out.stats[kStDpRuns], 1ull);
+            atomicAdd(&out.stats[kStCells], (unsigned long long)(2 * m + (m - mus + 1)) * W + m);
+        }
+        __syncthreads();
+    }
 }
 
 // One launch per DP class (cls): the same code over the class's items, with
@@ -1008,6 +1264,7 @@ __global__ void __launch_bounds__(128) finalize_roles_kernel(Dims dm, DevPop pop
             const uint64_t mask = si.mask[slot];
             m[h] = pop.sizes[slot];
             pok[h] = (int)((mask >> bp) & 1ull);
+            if (pok[h] && dm.layered) pok[h] = so.T[(size_t)slot * V + bp] < keyd(kInfKey);   // the run found none
             best[h] = mask ? si.best[slot] : -1;
             s_off[gw][c] = si.off[slot];
             s_pv[gw][c] = pok[h];
@@ -1384,6 +1641,7 @@ __global__ void __launch_bounds__(128) finalize_splitwise_kernel(Dims dm, DevPop
             const uint64_t mask = si.mask[slot];
             m[h] = pop.sizes[slot];
             pok[h] = (int)((mask >> bp) & 1ull);
+            if (pok[h] && dm.layered) pok[h] = so.T[(size_t)slot * V + bp] < keyd(kInfKey);   // the run found none
             best[h] = mask ? si.best[slot] : -1;
             s_off[wl][c] = si.off[slot];
             if (pok[h]) strength[h] = (double)dm.NP / so.T[(size_t)slot * V + bp];
@@ -1575,9 +1833,25 @@ static cudaError_t load_span_probes()
 
 cudaError_t configure_eval(e2_ctx *c)
 {
-    const void *kernel = reinterpret_cast<const void *>(dp_eval_kernel);
     cudaError_t e = load_span_probes();
     if (e != cudaSuccess) return e;
+    if (c->dm.layered) {                         // the plain-scan path: one launch, one class
+        const void *lk = reinterpret_cast<const void *>(dp_layered_kernel);
+        e = cudaFuncSetAttribute(lk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c->dp_smem);
+        if (e != cudaSuccess) return e;
+        int per_sm = 0, sms = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, lk, c->dp_threads, c->dp_smem);
+        if (e != cudaSuccess) return e;
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
+        if (e != cudaSuccess) return e;
+        c->dp_grid = (per_sm > 0 ? per_sm : 1) * (sms > 0 ? sms : 1);
+        c->dm.dp_warps = c->dp_threads / 32;
+        c->dm.dp_small = 0;
+        c->dp_grid1 = 0;
+        c->dp_smem1 = 0;
+        return cudaSuccess;
+    }
+    const void *kernel = reinterpret_cast<const void *>(dp_eval_kernel);
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c->dp_smem);
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
@@ -1614,7 +1888,7 @@ cudaError_t configure_eval(e2_ctx *c)
 cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
 {
     Tables tb{c->rate, c->bw, c->mem, c->rate_cpu, c->bw_cpu, c->mem_cpu, c->prof, c->leaf, c->tau, c->cap,
-              c->capg, c->cpb, c->tau_lb, c->leaf_rank, c->tau_rank};
+              c->capg, c->cpb, c->tau_lb, c->leaf_rank, c->tau_rank, c->lcost};
     EvalOut out{c->fit, c->layers, c->master, c->bsel, c->T, c->L, c->hash, c->stats, c->gpu_layers};
     SlotInfo si{c->slot_off, c->slot_mask, c->slot_size, c->slot_best};
     WorkList wl{c->items, c->order_bins};
@@ -1638,7 +1912,10 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
         if ((e = cudaEventRecord(c->ev_dp_fork, c->stream)) != cudaSuccess) return e;
         if ((e = cudaStreamWaitEvent(c->side, c->ev_dp_fork, 0)) != cudaSuccess) return e;
     }
-    dp_eval_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so, 0);
+    if (c->dm.layered)
+        dp_layered_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so);
+    else
+        dp_eval_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so, 0);
     if (c->dp_grid1 > 0) {
         dp_eval_kernel<<<(unsigned)c->dp_grid1, c->dp_threads, c->dp_smem1, c->side>>>(c->dm, tb, p, out, wl, si, so,
                                                                                       1);

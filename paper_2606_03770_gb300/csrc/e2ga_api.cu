@@ -21,7 +21,7 @@ size_t align_up(size_t x, size_t a = 256) { return (x + a - 1) / a * a; }
 
 struct Layout {
     size_t rate, bw, mem, rate_cpu, bw_cpu, mem_cpu, link_bw, cong, prof, leaf, tau, tau_lb, cap, capg, cpb,
-        leaf_sorted, beff_sorted, tau_sorted, leaf_rank, tau_rank, gpu_layers;
+        leaf_sorted, beff_sorted, tau_sorted, leaf_rank, tau_rank, gpu_layers, psum, lcost;
     size_t perm[2], sizes[2], nclus[2], roles[2];
     size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, stats, err, order_bins, items, slot_off, slot_mask, slot_size, slot_best,
         split_T, split_L, split_mu, split_layers, total;
@@ -37,7 +37,7 @@ bool dims_ok(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_t Q, int32_t 
            K <= E2_MAX_CLUSTERS && (uint64_t)P * (uint64_t)K * (uint64_t)(b_max + 1) < (1ull << 31);
 }
 
-Layout layout(int M, int N, int b_max, int P, int Q, int K)
+Layout layout(int M, int N, int b_max, int P, int Q, int K, bool layered = false)
 {
     Layout l{};
     const size_t V = (size_t)b_max + 1, MM = (size_t)M * M;
@@ -93,6 +93,10 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K)
     l.split_L = take(8 * (size_t)P * K * V);                 // and bit b_max = prefill when roles are searched
     l.split_mu = take(2 * (size_t)P * K * V);
     l.split_layers = take(2 * (size_t)P * V * M);
+    if (layered) {
+        l.psum = take(8 * 3 * V * ((size_t)N + 1));
+        l.lcost = take(8 * V * M * 2 * (size_t)N * N);
+    }
     l.total = o;
     return l;
 }
@@ -189,6 +193,28 @@ int validate_inputs(const e2_devices *d, const e2_links *l, const e2_layer_profi
         }
         if (pf->act_bytes[v] >= kTwo53) { snprintf(msg, n, "activation bytes reach 2^53"); return E2_EINVAL; }
     }
+    if (pf->PF || pf->PB || pf->PM) {                 // blocks of several types: per-layer prefix sums
+        if (!pf->PF || !pf->PB || !pf->PM) { snprintf(msg, n, "PF, PB and PM must be given together"); return E2_EINVAL; }
+        if (pf->N > E2_MAX_LAYERED_BLOCKS) {
+            snprintf(msg, n, "per-layer profiles take at most %d blocks", E2_MAX_LAYERED_BLOCKS);
+            return E2_EINVAL;
+        }
+        const uint64_t *ps[3] = {pf->PF, pf->PB, pf->PM};
+        for (int a = 0; a < 3; ++a)
+            for (int v = 0; v < V; ++v) {
+                const uint64_t *row = ps[a] + (size_t)v * (pf->N + 1);
+                if (row[0] != 0) { snprintf(msg, n, "prefix sums must start at 0"); return E2_EINVAL; }
+                for (int i = 0; i < pf->N; ++i)
+                    if (row[i + 1] < row[i]) { snprintf(msg, n, "prefix sums must not decrease"); return E2_EINVAL; }
+                if (row[pf->N] >= kTwo53 || arr[a + 3][v] >= kTwo53 - row[pf->N]) {
+                    snprintf(msg, n, "profile variant %d: a stage's sum plus the head reaches 2^53", v);
+                    return E2_EINVAL;
+                }
+            }
+        if (d->mem_cpu)
+            for (int i = 0; i < M; ++i)
+                if (d->mem_cpu[i]) { snprintf(msg, n, "per-layer profiles do not take GPU-CPU offload"); return E2_EINVAL; }
+    }
     if (pf->NP < 1 || pf->ND < 1 || pf->NP >= kTwo53 || pf->ND >= kTwo53) {
         snprintf(msg, n, "NP and ND must be in [1, 2^53)");
         return E2_EINVAL;
@@ -274,8 +300,16 @@ extern "C" {
 
 size_t e2_workspace_bytes(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_t Q, int32_t K_max)
 {
-    if (!dims_ok(M, N, b_max, P, Q, K_max)) return 0;
-    return layout(M, N, b_max, P, Q, K_max).total;
+    return e2_workspace_bytes_ex(M, N, b_max, P, Q, K_max, 0u);
+}
+
+size_t e2_workspace_bytes_ex(int32_t M, int32_t N, int32_t b_max, int32_t P, int32_t Q, int32_t K_max,
+                             uint32_t flags)
+{
+    if (!dims_ok(M, N, b_max, P, Q, K_max) || (flags & ~E2_WS_LAYERED)) return 0;
+    const bool layered = (flags & E2_WS_LAYERED) != 0;
+    if (layered && N > E2_MAX_LAYERED_BLOCKS) return 0;
+    return layout(M, N, b_max, P, Q, K_max, layered).total;
 }
 
 // Whether the decode variants' costs never shrink as the batch grows: block
@@ -332,7 +366,8 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     int st = validate_inputs(devs, links, prof, prm, msg, sizeof msg);
     if (st) return reject(st, msg);
     const int M = devs->M, N = prof->N, b_max = prof->b_max, P = prm->P, Q = prm->Q, K = prm->K_max;
-    const Layout l = layout(M, N, b_max, P, Q, K);
+    const bool layered = prof->PF != nullptr;
+    const Layout l = layout(M, N, b_max, P, Q, K, layered);
     if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255))
         return reject(E2_EINVAL, "workspace must be non-null and 256-byte aligned");
     if (workspace_bytes < l.total) return reject(E2_ENOMEM, "workspace smaller than e2_workspace_bytes()");
@@ -343,6 +378,7 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->dm = Dims{M, N, b_max + 1, b_max, P, Q, K, l.LS, prm->tournament, prof->NP, prof->ND,
                  prm->min_tps, prm->t_a, latency_ceiling(prm->min_tps), prm->role_search, 0.0f, 0u, 4,
                  costs_grow_with_batch(prof, b_max), prm->objective};
+    c->dm.layered = layered ? 1 : 0;
     c->dm.offload = 0;
     if (devs->mem_cpu)
         for (int i = 0; i < M; ++i) c->dm.offload |= devs->mem_cpu[i] != 0;
@@ -376,7 +412,7 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, c->device) != cudaSuccess)
         return fail_free(E2_ECUDA, "cudaDeviceGetAttribute failed");
     c->dp_threads = 128;
-    c->dp_smem = dp_smem_bytes(M, N, c->dp_threads, 4);
+    c->dp_smem = layered ? dp_layered_smem_bytes(M, N) : dp_smem_bytes(M, N, c->dp_threads, 4);
     if ((M < N ? M : N) > kMaxReplicaDevices)
         return fail_free(E2_EINVAL, "replicas could exceed 256 devices (min(M, N) > 256)");
     if (c->dp_smem + 1024 > (size_t)smem_optin)
@@ -398,6 +434,10 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->mem_cpu = reinterpret_cast<uint64_t *>(ws + l.mem_cpu);
     c->capg = reinterpret_cast<int32_t *>(ws + l.capg);
     c->gpu_layers = reinterpret_cast<int16_t *>(ws + l.gpu_layers);
+    if (layered) {
+        c->psum = reinterpret_cast<uint64_t *>(ws + l.psum);
+        c->lcost = reinterpret_cast<double *>(ws + l.lcost);
+    }
     c->link_bw = reinterpret_cast<double *>(ws + l.link_bw);
     c->cong = reinterpret_cast<double *>(ws + l.cong);
     c->prof = reinterpret_cast<uint64_t *>(ws + l.prof);
@@ -455,6 +495,12 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     chk(cudaMemcpyAsync(c->link_bw, links->bw, 8 * MM, cudaMemcpyHostToDevice, c->stream));
     chk(cudaMemcpyAsync(c->cong, links->cong, 8 * MM, cudaMemcpyHostToDevice, c->stream));
     chk(cudaMemcpyAsync(c->prof, prof_h, 8 * kNumProf * V, cudaMemcpyHostToDevice, c->stream));
+    if (layered) {
+        const size_t row = 8 * V * ((size_t)N + 1);
+        chk(cudaMemcpyAsync(c->psum, prof->PF, row, cudaMemcpyHostToDevice, c->stream));
+        chk(cudaMemcpyAsync(c->psum + V * ((size_t)N + 1), prof->PB, row, cudaMemcpyHostToDevice, c->stream));
+        chk(cudaMemcpyAsync(c->psum + 2 * V * ((size_t)N + 1), prof->PM, row, cudaMemcpyHostToDevice, c->stream));
+    }
     if (e == cudaSuccess) e = launch_tables(c);
     if (e == cudaSuccess) e = launch_tau(c);
     if (e == cudaSuccess) e = build_leaf_sorted(c);
@@ -708,12 +754,15 @@ int e2_get_stats(e2_ctx *c, e2_stats *out)
     out->tps_pruned = s[kStTpsPruned];
     out->dp_runs_small = s[kStDpRunsSmall];
     out->role_search_capped = s[kStRoleCapped];
+    out->device_errors = s[kStDeviceErrors];
     out->dp_launches = c->dp_grid1 > 0 ? 2 : 1;
     out->dp_ctas = (uint64_t)c->dp_grid;
     out->dp_smem = c->dp_smem;
     out->dp_ctas_small = (uint64_t)c->dp_grid1;
     out->dp_smem_small = c->dp_smem1;
     out->launches = c->launches;
+    if (out->device_errors)
+        return fail(c, E2_EDEVICE, "a device-side consistency check of the last evaluation failed");
     return E2_OK;
 }
 
@@ -732,7 +781,6 @@ const char *e2_strerror(int s)
     case E2_EINVAL: return "invalid argument";
     case E2_ENOMEM: return "workspace too small";
     case E2_ECUDA: return "CUDA runtime error";
-    case E2_ETIMEOUT: return "bounded device wait expired";
     case E2_EDEVICE: return "device-side check failed";
     case E2_ESTATE: return "call out of order";
     default: return "unknown status";

@@ -69,7 +69,7 @@ __host__ __device__ __forceinline__ unsigned dp_item_bytes(int m, int N, int war
 
 // Stats slots (unsigned long long, atomically accumulated).
 enum StatSlot { kStGenomes = 0, kStReplicas, kStDpRuns, kStCells, kStProbes, kStPaper, kStPrecheck,
-                kStServed, kStTpsPruned, kStDpRunsSmall, kStRoleCapped, kNumStats };
+                kStServed, kStTpsPruned, kStDpRunsSmall, kStRoleCapped, kStDeviceErrors, kNumStats };
 
 // Everything a kernel needs, passed by value.
 struct Dims {
@@ -89,6 +89,7 @@ struct Dims {
                          // shrink from one decode batch to the next (the pre-pass tests are then monotone)
     int objective;       // 0: waiting time w (Eq. 3-5); 1: per-request finishing time FT
     int offload;         // 1: some device has host memory for offloaded blocks
+    int layered;         // 1: blocks of several types (per-layer prefix sums): the plain-scan DP path
 };
 
 struct Tables {
@@ -106,6 +107,8 @@ struct Tables {
     const float *tau_lb;       // [V][M][M]: tau rounded down
     const uint32_t *leaf_rank; // [V][M][2][LS]: order key of leaf within its variant's value set
     const uint32_t *tau_rank;  // [V][M][M]
+    const double *lcost;       // [V][M][2][N][N] (per-layer profiles only): lcost[((v*M+d)*2+mf)*N*N + j*N + n-1]
+                               // = time of blocks j..j+n-1 on device d (+inf beyond the model or memory)
 };
 
 // Per (genome, replica slot) results of the evaluation pre-pass.
@@ -205,6 +208,8 @@ struct e2_ctx {
     double *rate_cpu = nullptr, *bw_cpu = nullptr;   // host side of offload (zeros without it)
     uint64_t *mem_cpu = nullptr;
     int32_t *capg = nullptr;                          // [V][M][2] blocks in device memory
+    uint64_t *psum = nullptr;                         // [3][V][N+1] per-layer prefix sums PF, PB, PM (layered)
+    double *lcost = nullptr;                          // [V][M][2][N][N] per-layer stage times (layered)
     int16_t *gpu_layers = nullptr;                    // [P][M] G of the G--C split (offload only)
     double *link_bw = nullptr, *cong = nullptr;
     uint64_t *prof = nullptr;
@@ -261,7 +266,7 @@ struct e2_ctx {
 
 namespace e2 {
 // launchers (defined in the .cu files); return cudaGetLastError()
-cudaError_t launch_tables(const e2_ctx *c);   // leaf, cap and cpb tables
+cudaError_t launch_tables(const e2_ctx *c);   // leaf, cap and cpb tables (and lcost for per-layer profiles)
 cudaError_t launch_tau(const e2_ctx *c);
 cudaError_t launch_redraw(const e2_ctx *c, uint64_t seed, uint32_t gen);
 cudaError_t launch_validate(const e2_ctx *c, const DevPop &p);
@@ -277,6 +282,7 @@ cudaError_t find_ga_node(cudaGraph_t graph, cudaGraphNode_t *node);
 cudaError_t set_ga_node(const e2_ctx *c, cudaGraphExec_t exec, cudaGraphNode_t node, const DevPop &src,
                         const DevPop &dst, uint64_t seed, uint32_t gen);
 size_t dp_smem_bytes(int M, int N, int threads, int key_bytes);
+size_t dp_layered_smem_bytes(int M, int N);   // the plain-scan DP's shared memory for the largest replica
 cudaError_t configure_eval(e2_ctx *c);   // shared memory limit and persistent grid size
 size_t rank_pow2(size_t n);
 cudaError_t build_leaf_sorted(const e2_ctx *c);   // once per context

@@ -65,6 +65,42 @@ __global__ void tables_kernel(Dims dm, const double *rate, const double *bw, con
     }
 }
 
+// Per-layer profiles (blocks of several types): the time of blocks j..j+n-1 on
+// device d, with and without the head, from the prefix sums PF, PB, PM
+// (psum[a][v][N+1]): the larger of compute and streaming time, +inf beyond
+// device memory or past the last block.
+__global__ void layered_tables_kernel(Dims dm, const double *rate, const double *bw, const uint64_t *mem,
+                                      const uint64_t *prof, const uint64_t *psum, double *lcost)
+{
+    const size_t NN = (size_t)dm.N * dm.N, total = (size_t)dm.V * dm.M * 2 * NN;
+    const size_t row = (size_t)dm.N + 1, plane = (size_t)dm.V * row;
+    for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < total;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        const int n = (int)(idx % dm.N) + 1;
+        const int j = (int)((idx / dm.N) % dm.N);
+        size_t rest = idx / NN;
+        const int mf = (int)(rest & 1);
+        rest >>= 1;
+        const int d = (int)(rest % dm.M);
+        const int v = (int)(rest / dm.M);
+        double out = keyd(kInfKey);
+        if (j + n <= dm.N) {
+            const int V = dm.V;
+            const uint64_t *pf = psum + (size_t)v * row, *pb = psum + plane + (size_t)v * row,
+                           *pm = psum + 2 * plane + (size_t)v * row;
+            const uint64_t need = pm[j + n] - pm[j] + (mf ? prof[kHeadMem * V + v] : 0ull);
+            if (need <= mem[d]) {
+                const uint64_t fl = pf[j + n] - pf[j] + (mf ? prof[kHeadFlops * V + v] : 0ull);
+                const uint64_t by = pb[j + n] - pb[j] + (mf ? prof[kHeadBytes * V + v] : 0ull);
+                const double tc = __ull2double_rn(fl) / rate[d];
+                const double tm = __ull2double_rn(by) / bw[d];
+                out = tc >= tm ? tc : tm;
+            }
+        }
+        lcost[idx] = out;
+    }
+}
+
 // Per (variant, device): the most blocks the device can hold in device and
 // host memory together, without and with the LM head (the number of finite
 // entries of its two cost rows), the most of them in device memory (the G of
@@ -511,6 +547,12 @@ cudaError_t launch_tables(const e2_ctx *c)
     captab_kernel<<<grid_for(vm, 256), 256, 0, c->stream>>>(c->dm, c->rate, c->bw, c->mem, c->rate_cpu, c->bw_cpu,
                                                              c->mem_cpu, c->prof, c->cap, c->capg, c->cpb);
     c->launches += 2;
+    if (c->dm.layered) {
+        const size_t lt = (size_t)c->dm.V * c->dm.M * 2 * c->dm.N * c->dm.N;
+        layered_tables_kernel<<<grid_for(lt, 256), 256, 0, c->stream>>>(c->dm, c->rate, c->bw, c->mem, c->prof,
+                                                                         c->psum, c->lcost);
+        ++c->launches;
+    }
     return cudaGetLastError();
 }
 

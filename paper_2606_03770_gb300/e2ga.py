@@ -19,7 +19,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_build", "libe2ga.so")
 _lib = None
 
-E2_OK, E2_EINVAL, E2_ENOMEM, E2_ECUDA, E2_ETIMEOUT, E2_EDEVICE, E2_ESTATE = range(7)
+E2_OK, E2_EINVAL, E2_ENOMEM, E2_ECUDA, E2_EDEVICE, E2_ESTATE = 0, 1, 2, 3, 5, 6
 
 
 class e2_devices(C.Structure):
@@ -34,7 +34,8 @@ class e2_links(C.Structure):
 class e2_layer_profile(C.Structure):
     _fields_ = [("N", C.c_int32), ("b_max", C.c_int32), ("blk_flops", C.c_void_p), ("blk_bytes", C.c_void_p),
                 ("blk_mem", C.c_void_p), ("head_flops", C.c_void_p), ("head_bytes", C.c_void_p),
-                ("head_mem", C.c_void_p), ("act_bytes", C.c_void_p), ("NP", C.c_uint64), ("ND", C.c_uint64)]
+                ("head_mem", C.c_void_p), ("act_bytes", C.c_void_p), ("NP", C.c_uint64), ("ND", C.c_uint64),
+                ("PF", C.c_void_p), ("PB", C.c_void_p), ("PM", C.c_void_p)]
 
 
 class e2_params(C.Structure):
@@ -57,12 +58,13 @@ class e2_stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in ("genomes", "replicas", "dp_runs", "dp_cells", "dp_probes",
                                          "paper_candidates", "prechecked", "served", "tps_pruned",
                                          "dp_runs_small", "dp_launches", "dp_ctas", "dp_smem", "dp_ctas_small",
-                                         "dp_smem_small", "launches", "role_search_capped")]
+                                         "dp_smem_small", "launches", "role_search_capped", "device_errors")]
 
 
 # name -> (restype, argtypes); the exported surface of include/e2ga.h
 SIGNATURES = {
     "e2_workspace_bytes": (C.c_size_t, [C.c_int32] * 6),
+    "e2_workspace_bytes_ex": (C.c_size_t, [C.c_int32] * 6 + [C.c_uint32]),
     "e2_create": (C.c_int, [C.c_void_p] * 5 + [C.c_size_t, C.c_void_p, C.c_void_p]),
     "e2_destroy": (C.c_int, [C.c_void_p]),
     "e2_set_population": (C.c_int, [C.c_void_p, C.c_void_p]),
@@ -109,8 +111,15 @@ class E2Error(RuntimeError):
 
 
 # ---- same-named thin wrappers ------------------------------------------------
+E2_WS_LAYERED = 1
+
+
 def e2_workspace_bytes(M, N, b_max, P, Q, K_max):
     return load().e2_workspace_bytes(M, N, b_max, P, Q, K_max)
+
+
+def e2_workspace_bytes_ex(M, N, b_max, P, Q, K_max, flags):
+    return load().e2_workspace_bytes_ex(M, N, b_max, P, Q, K_max, flags)
 
 
 def e2_create(devs, links, prof, prm, workspace_ptr, workspace_bytes, stream_ptr):
@@ -234,14 +243,18 @@ class Engine:
         self.devs = e2_devices(self.M, _ptr(h["rate"]), _ptr(h["bw"]), _ptr(h["mem"]), _ptr(h.get("rate_cpu")),
                                _ptr(h.get("bw_cpu")), _ptr(h.get("mem_cpu")))
         self.links = e2_links(_ptr(h["lbw"]), _ptr(h["cong"]), prob.cong_lo, prob.cong_hi)
+        layered = getattr(prob, "PF", None) is not None
+        if layered:
+            self._host.update(PF=u64(prob.PF), PB=u64(prob.PB), PM=u64(prob.PM))
         self.profile = e2_layer_profile(self.N, self.b_max, *[_ptr(h[k]) for k in (
             "blk_flops", "blk_bytes", "blk_mem", "head_flops", "head_bytes", "head_mem", "act_bytes")],
-            prob.NP, prob.ND)
+            prob.NP, prob.ND, *[_ptr(h.get(k)) for k in ("PF", "PB", "PM")])
         pk = prob.p_kind
         self.params = e2_params(self.P, self.Q, self.K, prob.tournament, prob.min_tps, prob.t_a, prob.p_cx,
                                 prob.p_mut, pk[0], pk[1], pk[2], int(getattr(prob, "role_search", 0)),
                                 int(getattr(prob, "objective", 0)))
-        self.ws_bytes = e2_workspace_bytes(self.M, self.N, self.b_max, self.P, self.Q, self.K)
+        self.ws_bytes = e2_workspace_bytes_ex(self.M, self.N, self.b_max, self.P, self.Q, self.K,
+                                              E2_WS_LAYERED if layered else 0)
         if self.ws_bytes == 0:
             raise E2Error(E2_EINVAL, "e2_workspace_bytes")
         self.workspace = torch.empty(self.ws_bytes, dtype=torch.uint8, device="cuda")

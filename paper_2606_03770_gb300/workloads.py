@@ -78,6 +78,11 @@ class Problem:
     rate_cpu: np.ndarray | None = None
     bw_cpu: np.ndarray | None = None
     mem_cpu: np.ndarray | None = None
+    # blocks of several types: per-variant prefix sums [V][N+1] of the blocks'
+    # flops, bytes and resident bytes (None: N identical blocks, blk_*)
+    PF: np.ndarray | None = None
+    PB: np.ndarray | None = None
+    PM: np.ndarray | None = None
 
     @property
     def M(self) -> int:
@@ -145,6 +150,50 @@ def dense_profile(N, d, ffn, kv_heads, vocab, NP, ND, b_max, wbits=16):
                 head_mem=hs, act_bytes=a)
 
 
+def layered_profile(N, d, ffn, kv_heads, vocab, NP, ND, b_max, wbits=16, window=128, pattern="alternate"):
+    """Blocks of two types, as in a model that alternates sliding-window and
+    full attention: a sliding-window block attends to (and keeps the KV cache
+    of) at most ``window`` positions, a full-attention block to the whole
+    context.  Returns the identical-block fields (each the largest block, so
+    that range checks stay conservative) plus the per-variant prefix sums
+    PF, PB, PM [V][N+1] of the blocks' flops, bytes and resident bytes.
+    ``pattern``: "alternate" (sliding on even blocks) or "tail" (the last
+    N // 4 blocks full, the rest sliding)."""
+    d_kv = d if kv_heads is None else kv_heads * HEAD_DIM
+    P_l = 2 * d * d + 2 * d * d_kv + 3 * d * ffn
+    wbytes = P_l * wbits // 8
+    assert wbytes * 8 == P_l * wbits
+    ctx = NP + ND
+    V = 1 + b_max
+    base = dense_profile(N, d, ffn, kv_heads, vocab, NP, ND, b_max, wbits)
+    PF = np.zeros((V, N + 1), np.uint64)
+    PB = np.zeros((V, N + 1), np.uint64)
+    PM = np.zeros((V, N + 1), np.uint64)
+    for v in range(V):
+        f, y, s_ = [], [], []
+        for l in range(N):
+            sliding = (l % 2 == 0) if pattern == "alternate" else (l < N - N // 4)
+            if v == 0:
+                seen = min(NP, window) if sliding else NP
+                f.append(2 * P_l * NP + 4 * NP * seen * d)
+                kv = min(NP, window) if sliding else NP
+                y.append(wbytes + kv * 2 * d_kv * 2)
+                s_.append(wbytes + kv * 2 * d_kv * 2)
+            else:
+                seen = min(ctx, window) if sliding else ctx
+                f.append(2 * P_l * v + 4 * v * seen * d)
+                y.append(wbytes + v * seen * 2 * d_kv * 2)
+                s_.append(wbytes + v * seen * 2 * d_kv * 2)
+        PF[v, 1:] = np.cumsum(np.array(f, dtype=np.uint64))
+        PB[v, 1:] = np.cumsum(np.array(y, dtype=np.uint64))
+        PM[v, 1:] = np.cumsum(np.array(s_, dtype=np.uint64))
+        base["blk_flops"][v] = max(f)
+        base["blk_bytes"][v] = max(y)
+        base["blk_mem"][v] = max(s_)
+    base.update(PF=PF, PB=PB, PM=PM)
+    return base
+
+
 # Fleet and model shapes of the five workloads the planner is measured on.  The
 # 32-block model keeps fp16 weights; the 80- and 126-block models carry 4-bit
 # weights, the precision of the models the paper deploys (Q4_K_M, MXFP4), without
@@ -190,9 +239,12 @@ def offload_fleet(M: int, seed: int):
     return rate, bw, mem
 
 
-def make_config(name: str, seed: int = 0, P: int | None = None, offload: bool = False) -> Problem:
+def make_config(name: str, seed: int = 0, P: int | None = None, offload: bool = False,
+                layered: str | None = None) -> Problem:
     """Draw the named workload with a numpy Philox generator keyed by ``seed``
-    (with ``offload``, plus the host side of GPU-CPU offload per device)."""
+    (with ``offload``, plus the host side of GPU-CPU offload per device; with
+    ``layered`` = "alternate" or "tail", the model's blocks are of two types,
+    sliding-window and full attention, given as per-layer prefix sums)."""
     c = CONFIGS[name]
     rng = np.random.Generator(np.random.Philox(key=seed))
     M = c["M"]
@@ -216,7 +268,10 @@ def make_config(name: str, seed: int = 0, P: int | None = None, offload: bool = 
     else:
         NP = int(round(float(np.mean(rng.integers(pk[1], pk[2] + 1, 1000)))))
     ND = NP  # generated tokens: input/generated ratios of 0.77-1.65 are reported, take 1
-    prof = dense_profile(NP=NP, ND=ND, b_max=B_MAX, **c["model"])
+    if layered:
+        prof = layered_profile(NP=NP, ND=ND, b_max=B_MAX, pattern=layered, **c["model"])
+    else:
+        prof = dense_profile(NP=NP, ND=ND, b_max=B_MAX, **c["model"])
     P_ = int(P if P is not None else c["P"])
     redraw = c.get("redraw")
     host = dict(zip(("rate_cpu", "bw_cpu", "mem_cpu"), offload_fleet(M, seed))) if offload else {}
@@ -233,7 +288,7 @@ def make_problem(rate, bw, mem, link_bw, cong, N, blk_flops, blk_bytes, blk_mem,
     """Build a Problem from explicit arrays (hand-made cases, edge cases)."""
     f64 = lambda x: np.ascontiguousarray(np.asarray(x, dtype=np.float64))
     u64 = lambda x: np.ascontiguousarray(np.asarray(x, dtype=np.uint64))
-    for k, conv in (("rate_cpu", f64), ("bw_cpu", f64), ("mem_cpu", u64)):
+    for k, conv in (("rate_cpu", f64), ("bw_cpu", f64), ("mem_cpu", u64), ("PF", u64), ("PB", u64), ("PM", u64)):
         if kw.get(k) is not None:
             kw[k] = conv(kw[k])
     return Problem(name=name, rate=f64(rate), bw=f64(bw), mem=u64(mem), link_bw=f64(link_bw),

@@ -43,7 +43,8 @@ def declared_struct_fields(name):
     return [(t, n) for t, n in re.findall(r"(\w+)\s*\*?\s*(\w+)\s*;", body)]
 
 
-@pytest.mark.parametrize("name", ["e2_devices", "e2_params", "e2_stats", "e2_genomes", "e2_partitions"])
+@pytest.mark.parametrize("name", ["e2_devices", "e2_layer_profile", "e2_params", "e2_stats", "e2_genomes",
+                                  "e2_partitions"])
 def test_binding_structs_follow_the_header(name):
     """The ctypes mirrors of the header's structs: same fields in the same
     order, with the same widths."""

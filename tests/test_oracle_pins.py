@@ -1101,3 +1101,120 @@ def test_role_search_caps_at_twenty_decoding_replicas():
     prob20 = dataclasses.replace(prob, mem=np.array([10 ** 12] * 20 + [0] * 4, np.uint64))
     out20 = O.OracleProblem(prob20).eval_population(g, K)
     assert out20["capped"] == 0 and int(out20["roles"][0]) >> 20 == 0
+
+
+# ---------------------------------------------------------------------------
+# blocks of several types: per-layer prefix sums PF, PB, PM (Sec. 3.1)
+# ---------------------------------------------------------------------------
+def _layered(prob, rng, integer=True):
+    """Per-layer work for a tiny problem: block l's flops, bytes and resident
+    bytes drawn per variant (small integers: heavy and light blocks, ties)."""
+    import dataclasses
+    V, N = prob.V, prob.N
+    f = rng.integers(1, 6, (V, N)) if integer else rng.integers(1, 1000, (V, N))
+    b = rng.integers(0, 6, (V, N)) if integer else rng.integers(0, 1000, (V, N))
+    m = rng.integers(1, 3, (V, N))
+    cum = lambda x: np.concatenate([np.zeros((V, 1), np.uint64), np.cumsum(x, axis=1).astype(np.uint64)], axis=1)
+    return dataclasses.replace(prob, PF=cum(f), PB=cum(b), PM=cum(m), blk_flops=f.max(1).astype(np.uint64),
+                               blk_bytes=b.max(1).astype(np.uint64), blk_mem=m.max(1).astype(np.uint64))
+
+
+def bf_value_at(op, v, devs, total, k, mu):
+    """min over compositions of blocks 0..total-1 on devs[0..k) of the largest
+    stage or link time, with per-layer costs (a stage's cost depends on where
+    it starts)."""
+    best = INF
+    for comp in compositions(total, k):
+        worst, j = 0.0, 0
+        for t in range(k):
+            worst = max(worst, op.stage_cost_at(v, int(devs[t]), j, comp[t], t == mu))
+            if t >= 1:
+                worst = max(worst, op.link_cost(v, int(devs[t - 1]), int(devs[t])))
+            j += comp[t]
+        best = min(best, worst)
+    return best
+
+
+def bf_dp_at(op, v, devs, N):
+    m = len(devs)
+    if m > N:
+        return None
+    vals = [bf_value_at(op, v, devs, N, m, mu) for mu in range(m)]
+    V = min(vals)
+    if V == INF:
+        return None
+    mu = vals.index(V)
+    layers = [0] * m
+    i = N - 1
+    for k in range(m, 1, -1):
+        target = bf_value_at(op, v, devs, i + 1, k, mu)
+        tau = op.link_cost(v, int(devs[k - 2]), int(devs[k - 1]))
+        for j in range(k - 1, i + 1):
+            prev = bf_value_at(op, v, devs, j, k - 1, mu)
+            c = max(prev, op.stage_cost_at(v, int(devs[k - 1]), j, i - j + 1, mu == k - 1), tau)
+            if c == target:
+                break
+        layers[k - 1] = i - j + 1
+        i = j - 1
+    layers[0] = i + 1
+    return V, mu, layers
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_layered_dp_matches_brute_force(seed):
+    rng = np.random.default_rng(300 + seed)
+    N = int(rng.integers(1, 10))
+    M = 6
+    prob = _layered(tiny_problem(rng, M, N, integer=seed % 4 != 3, head=seed % 5 != 0), rng, integer=seed % 4 != 3)
+    op = O.OracleProblem(prob)
+    for trial in range(4):
+        m = int(rng.integers(1, M + 1))
+        devs = rng.permutation(M)[:m]
+        v = int(rng.integers(0, prob.V))
+        got = op.dp_pipe(v, devs)
+        bf = bf_dp_at(op, v, devs, N)
+        if bf is None:
+            assert not got["ok"]
+            continue
+        V, mu, layers = bf
+        assert got["ok"] and got["V"] == V and got["mu"] == mu and list(got["layers"]) == layers, (devs, v)
+
+
+def test_layered_with_uniform_sums_is_the_identical_block_model():
+    import dataclasses
+    for name in ("c1_tiny", "c2"):
+        prob = W.make_config(name, P=64)
+        V, N = prob.V, prob.N
+        ramp = np.arange(N + 1, dtype=np.uint64)[None, :]
+        lay = dataclasses.replace(prob, PF=prob.blk_flops[:, None] * ramp, PB=prob.blk_bytes[:, None] * ramp,
+                                  PM=prob.blk_mem[:, None] * ramp)
+        g = W.random_genomes(prob.M, prob.K_max, 64, seed=4)
+        a = O.OracleProblem(prob).eval_population(g, prob.K_max, nthreads=4)
+        b = O.OracleProblem(lay).eval_population(g, prob.K_max, nthreads=4)
+        for k in ("fitness", "layers", "master", "bsel", "T", "L"):
+            assert np.array_equal(a[k], b[k]), (name, k)
+
+
+def test_layered_prefix_optimum_is_not_monotone():
+    """Why blocks of several types need the plain scan: with blocks (light,
+    heavy, light) on a fast then a slow device, two blocks cost more than
+    three (the slow device must take the heavy block when only two are
+    placed).  D(1, 2) = 100 > D(2, 2) = 11; the partition of three blocks
+    puts the heavy block on the fast device."""
+    # device 0: 1 FLOP/s, device 1: 0.1 FLOP/s; blocks' flops 1, 10, 1
+    PF = np.array([[0, 1, 11, 12]], np.uint64)
+    zero = np.zeros((1, 4), np.uint64)
+    prob = W.make_problem([1.0, 0.1], [1.0, 1.0], [100, 100], np.full((2, 2), np.inf), np.ones((2, 2)), 3,
+                          [10], [0], [0], [0], [0], [0], [0], NP=1, ND=1, PF=PF, PB=zero, PM=zero)
+    op = O.OracleProblem(prob)
+    full = op.dp_pipe(0, [0, 1])
+    assert full["ok"] and full["V"] == 11.0 and list(full["layers"]) == [2, 1]
+    two = O.OracleProblem(dataclasses_replace(prob, N=2, PF=PF[:, :3], PB=zero[:, :3], PM=zero[:, :3])).dp_pipe(0, [0, 1])
+    assert two["V"] == 100.0 and list(two["layers"]) == [1, 1]
+    # the per-request latency walks the blocks in order: 11 + 1/0.1
+    assert op.latency(0, [0, 1], full["mu"], full["layers"]) == 11.0 + 10.0
+
+
+def dataclasses_replace(p, **kw):
+    import dataclasses
+    return dataclasses.replace(p, **kw)
