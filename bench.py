@@ -79,6 +79,8 @@ def parse():
     ap.add_argument("--no-configs", action="store_true", help="skip the other workloads' lines")
     ap.add_argument("--repeats", action="store_true",
                     help="instead of timing: how often replicas repeat over the workload's generations")
+    ap.add_argument("--cpu-only", action="store_true",
+                    help="instead of timing the GPU: the oracle's CPU baseline of the workload (all cores, one core)")
     ap.add_argument("--clocks-dir", default=tempfile.gettempdir(),
                     help="folder for the raw nvidia-smi samples of the timed region (clocks_rank<i>.csv)")
     ap.add_argument("--roles", default="bits", choices=["bits", "search"],
@@ -607,7 +609,11 @@ def run_repeats(args):
 
 def main():
     args = parse()
-    if args.repeats:
+    if args.cpu_only:
+        prob = problem(args)
+        print(json.dumps({"workload": workload_label(prob), "cpu_baseline": cpu_baseline(prob, args.seed)}),
+              flush=True)
+    elif args.repeats:
         run_repeats(args)
     elif args.impl == "reference":
         run_reference(args)
