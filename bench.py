@@ -58,11 +58,11 @@ OPS_PER_PROBE = 5
 OPS_PER_CELL = 5
 INT32_LANES_PER_SM = 128
 # dram__bytes_read.sum + dram__bytes_write.sum of the two DP launches of one
-# generation at the default workload (class 0: 26.90 + 5.11 MB, class 1:
-# 26.91 + 6.99 MB), from the ncu capture in profiles/; cold (ncu flushes the
+# generation at the default workload (class 0: 30.21 + 9.29 MB, class 1:
+# 24.55 + 5.46 MB), from the ncu capture in profiles/; cold (ncu flushes the
 # caches before each launch), so it counts the L2-resident order-key rows
 # again
-DP_TRAFFIC_BYTES = 65_907_968
+DP_TRAFFIC_BYTES = 69_509_632
 DP_TRAFFIC_SOURCE = "profiles/dp_eval_c4_gen2.md (dram read+write, both DP launches of one generation, cold)"
 
 

@@ -98,6 +98,7 @@ __device__ __forceinline__ void cp_async4(void *smem_dst, const void *gmem_src)
 
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
+
 __device__ __forceinline__ int warp_sum(int x)
 {
 #pragma unroll
@@ -124,12 +125,12 @@ __constant__ uint16_t c_span_probes[3][E2_MAX_BLOCKS + 1];
 
 // Shared-memory bytes for the largest replica the problem allows, with keys of
 // key_bytes bytes.
-size_t dp_smem_bytes(int M, int N, int threads, int key_bytes)
+size_t dp_smem_bytes(int M, int N, int threads, int key_bytes, bool spill)
 {
     size_t best = 0;
     const int mmax = M < N ? M : N;
     for (int m = 1; m <= mmax; ++m) {
-        const size_t bytes = dp_item_bytes(m, N, threads / 32, key_bytes);
+        const size_t bytes = dp_item_bytes(m, N, threads / 32, key_bytes, spill);
         if (bytes > best) best = bytes;
     }
     return best;
@@ -350,7 +351,7 @@ __global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop
             } else {
                 const int W = N - m + 1;
                 const int lg = (int)(1.0f * __log2f(1.0f + (float)m * (float)W));
-                const int cls = dp_item_bytes(m, N, dm.dp_warps, 4) <= dm.dp_small;
+                const int cls = dp_item_bytes(m, N, dm.dp_warps, 4, false) <= dm.dp_small;   // class 1 never spills
                 const int size = (lg < kSizeBins - 1 ? lg : kSizeBins - 1) | cls << 4;
                 si.size[slot] = (uint8_t)size;
                 const int nv = __popcll(mask);
@@ -493,7 +494,7 @@ template <> struct HeadRow<uint32_t> {
 // Every comparison is between ranks of the same stage and link times the
 // oracle compares, so V, mu*, the partition, T and Lambda are bit-identical to
 // Alg. 1.
-template <typename Key>
+template <typename Key, bool SPILL>
 __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, const DevPop &pop, const EvalOut &out,
                                              const WorkList &wl, const SlotInfo &si, const SplitOut &so, int cls)
 {
@@ -510,6 +511,9 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, NW = blockDim.x >> 5;
     constexpr Key kInf = (Key)~(Key)0;
     const unsigned n_items = wl.ctrl[kCtrlEnd + cls];         // this class's items end here
+    constexpr bool spill = SPILL;
+    // this CTA's suffix-column scratch (only the first launch's CTAs spill)
+    uint32_t *gsp = spill ? wl.gspill + (size_t)blockIdx.x * wl.spill_stride : nullptr;
     if (tid == 0) s_next = ~0u;
   for (;;) {
     // ---- next work item of the class (heaviest first); warp 1 claims it
@@ -546,10 +550,11 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
         int *nk = cnt1 + m;                                     // [m]
         Key *leaf0 = reinterpret_cast<Key *>(nk + m);           // [m][W] l_k(n)
         Key *Fst = leaf0 + (size_t)m * W;                       // [m][W] prefix / traceback columns
-        Key *Gst = Fst + (size_t)m * W;                         // [m][W] suffix columns
-        Key *Hb = Gst + (size_t)m * W;                          // [NW][W] per-warp convolution
+        Key *Gst = Fst + (size_t)m * W;                         // [m][W] suffix columns ([2][W] spilled)
+        Key *Hb = Gst + (size_t)(spill ? 2 : m) * W;            // [NW][W] per-warp convolution
         Key *Lb = Hb + (size_t)NW * W;                          // [NW][W] per-warp head row
-        Key *row1s = Lb + (size_t)NW * W;                       // [W] head row of mu*
+        Key *Sb = Lb + (size_t)NW * W;                          // [NW][W] per-warp suffix column (spilled)
+        Key *row1s = Sb + (spill ? (size_t)NW * W : 0);         // [W] head row of mu*
         Key *delta = row1s + W;                                 // [W] the empty stage
         Key *tauk = delta + W;                                  // [m] tauk[k] = link (k-1) -> k
         Key *lbm = tauk + m;                                    // [m] l^head_k(1)
@@ -564,8 +569,11 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
         auto colF = [&](int k) -> const Key * {
             return k == 0 ? delta : k == 1 ? leaf0 : Fst + (size_t)(k - 1) * W;
         };
+        // suffix column G_k: in shared memory (two of them, alternating, when spilled;
+        // the others then live in this CTA's global scratch, gsp)
         auto colG = [&](int k) -> const Key * {
-            return k == m + 1 ? delta : k == m ? leaf0 + (size_t)(m - 1) * W : Gst + (size_t)(k - 1) * W;
+            return k == m + 1 ? delta : k == m ? leaf0 + (size_t)(m - 1) * W
+                                               : Gst + (size_t)(spill ? (k & 1) : k - 1) * W;
         };
 
         const unsigned long long lprobe = 32 - __clz(W);
@@ -627,9 +635,12 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                 for (int k = m - 1; k >= 2; --k) {
                     const Key *prev = colG(k + 1), *row = leaf0 + (size_t)(k - 1) * W;
                     const Key t = tauk[k];
-                    Key *cur = Gst + (size_t)(k - 1) * W;
+                    Key *cur = Gst + (size_t)(spill ? (k & 1) : k - 1) * W;
                     const int per = (W + 63) >> 6;
-                    dp_span(prev, row, t, cur, (tid - 64) * per, min(W, (tid - 63) * per));
+                    const int r0 = (tid - 64) * per, r1 = min(W, (tid - 63) * per);
+                    dp_span(prev, row, t, cur, r0, r1);
+                    if (spill)                                      // the thread's own cells, to the scratch
+                        for (int r = r0; r < r1; ++r) __stcg(gsp + (size_t)(k - 1) * W + r, (uint32_t)cur[r]);
                     bar_named(2, 64);
                 }
             }
@@ -654,9 +665,15 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                 const uint32_t bv = (uint32_t)(bk >> 32);
                 if (lb > bv || (lb == bv && (unsigned)mu > (unsigned)(bk & 0xFFFFFFFFu))) continue;
                 const uint32_t *hrow = tb.leaf_rank + ((vM + devs[mu - 1]) * 2 + 1) * dm.LS;
+                const Key *P = colF(mu - 1), *S = colG(mu + 1);
                 HeadRow<Key> hr;
                 hr.start(L1, hrow, W, lane);                          // in flight while H is built
-                const Key *P = colF(mu - 1), *S = colG(mu + 1);
+                if (spill && mu + 1 <= m - 1) {                       // the suffix column from the scratch
+                    Key *sb = Sb + (size_t)wid * W;                   // (L2: written by this CTA's other warps)
+                    for (int r = lane; r < W; r += 32) sb[r] = (Key)__ldcg(gsp + (size_t)mu * W + r);
+                    __syncwarp();
+                    S = sb;
+                }
                 const int per = (W + 31) >> 5;
                 dp_span(P, S, (Key)0, H, lane * per, min(W, (lane + 1) * per));
                 hr.finish(L1, hrow, W, lane);
@@ -1025,10 +1042,13 @@ __global__ void __launch_bounds__(128) dp_layered_kernel(Dims dm, Tables tb, Dev
 
 // One launch per DP class (cls): the same code over the class's items, with
 // the class's shared-memory allocation.
+// SPILL: the suffix columns live in the global scratch (dm.g_spill), a
+// separate instance so that the other contexts keep their register count.
+template <bool SPILL>
 __global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out, WorkList wl,
                                                       SlotInfo si, SplitOut so, int cls)
 {
-    dp_eval_body<uint32_t>(dm, tb, pop, out, wl, si, so, cls);
+    dp_eval_body<uint32_t, SPILL>(dm, tb, pop, out, wl, si, so, cls);
 }
 
 // The genome's objective from the role sums (PS, DS; PL, DL the rate-weighted
@@ -1851,7 +1871,12 @@ cudaError_t configure_eval(e2_ctx *c)
         c->dp_smem1 = 0;
         return cudaSuccess;
     }
-    const void *kernel = reinterpret_cast<const void *>(dp_eval_kernel);
+    // class 0 runs every replica size (spilling its suffix columns where that
+    // raises its occupancy); class 1, where it raises the occupancy of the
+    // sizes it takes, runs the small ones without spilling
+    const void *kernel = c->dm.g_spill ? reinterpret_cast<const void *>(dp_eval_kernel<true>)
+                                       : reinterpret_cast<const void *>(dp_eval_kernel<false>);
+    const void *kernel1 = reinterpret_cast<const void *>(dp_eval_kernel<false>);
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c->dp_smem);
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
@@ -1865,16 +1890,38 @@ cudaError_t configure_eval(e2_ctx *c)
     c->dp_grid = (per_sm > 0 ? per_sm : 1) * sms;
     const int warps = c->dp_threads / 32, mmax = c->dm.M < c->dm.N ? c->dm.M : c->dm.N;
     size_t small = 0;
-    for (int m = 1; m <= mmax; ++m) {
-        const size_t b = dp_item_bytes(m, c->dm.N, warps, 4);
-        if (2 * b <= c->dp_smem && b > small) small = b;
+    if (!c->dm.g_spill) {
+        // the sizes whose run fits in half the largest one's shared memory
+        for (int m = 1; m <= mmax; ++m) {
+            const size_t b = dp_item_bytes(m, c->dm.N, warps, 4, false);
+            if (2 * b <= c->dp_smem && b > small) small = b;
+        }
+    } else {
+        // the non-spilling kernel's best occupancy (its registers' limit), and the
+        // largest size that keeps it
+        e = cudaFuncSetAttribute(kernel1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c->dp_smem);
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(kernel1, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 cudaSharedmemCarveoutMaxShared);
+        if (e != cudaSuccess) return e;
+        int best1 = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&best1, kernel1, c->dp_threads, 16);
+        if (e != cudaSuccess) return e;
+        for (int m = 1; m <= mmax; ++m) {
+            const size_t b = dp_item_bytes(m, c->dm.N, warps, 4, false);
+            if (b <= small || b > c->dp_smem) continue;
+            int occ = 0;
+            e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kernel1, c->dp_threads, b);
+            if (e != cudaSuccess) return e;
+            if (occ >= best1) small = b;
+        }
     }
     c->dm.dp_warps = warps;
     c->dm.dp_small = 0;
     c->dp_grid1 = 0;
     c->dp_smem1 = 0;
     if (small > 0) {
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm1, kernel, c->dp_threads, small);
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm1, kernel1, c->dp_threads, small);
         if (e != cudaSuccess) return e;
         if (per_sm1 > per_sm) {
             c->dm.dp_small = (unsigned)small;
@@ -1882,6 +1929,8 @@ cudaError_t configure_eval(e2_ctx *c)
             c->dp_smem1 = small;
         }
     }
+    if (c->dm.g_spill && c->dp_grid > kSpillCtas) c->dp_grid = kSpillCtas;   // the scratch holds kSpillCtas CTAs
+    c->dm.dp_grid0 = c->dp_grid;
     return cudaSuccess;
 }
 
@@ -1891,7 +1940,7 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
               c->capg, c->cpb, c->tau_lb, c->leaf_rank, c->tau_rank, c->lcost};
     EvalOut out{c->fit, c->layers, c->master, c->bsel, c->T, c->L, c->hash, c->stats, c->gpu_layers};
     SlotInfo si{c->slot_off, c->slot_mask, c->slot_size, c->slot_best};
-    WorkList wl{c->items, c->order_bins};
+    WorkList wl{c->items, c->order_bins, c->gspill, (unsigned)c->spill_stride};
     SplitOut so{c->split_T, c->split_L, c->split_mu, c->split_layers};
     const long long slots = (long long)c->dm.P * c->dm.K;
     cudaError_t e = cudaMemsetAsync(c->order_bins, 0, sizeof(unsigned) * kCtrlWords, c->stream);
@@ -1914,11 +1963,15 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     }
     if (c->dm.layered)
         dp_layered_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so);
+    else if (c->dm.g_spill)
+        dp_eval_kernel<true><<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si,
+                                                                                           so, 0);
     else
-        dp_eval_kernel<<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si, so, 0);
-    if (c->dp_grid1 > 0) {
-        dp_eval_kernel<<<(unsigned)c->dp_grid1, c->dp_threads, c->dp_smem1, c->side>>>(c->dm, tb, p, out, wl, si, so,
-                                                                                      1);
+        dp_eval_kernel<false><<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si,
+                                                                                            so, 0);
+    if (c->dp_grid1 > 0) {                       // class 1: the small sizes, never spilling
+        dp_eval_kernel<false><<<(unsigned)c->dp_grid1, c->dp_threads, c->dp_smem1, c->side>>>(c->dm, tb, p, out, wl,
+                                                                                            si, so, 1);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
         if ((e = cudaEventRecord(c->ev_dp_join, c->side)) != cudaSuccess) return e;
         if ((e = cudaStreamWaitEvent(c->stream, c->ev_dp_join, 0)) != cudaSuccess) return e;

@@ -21,7 +21,7 @@ size_t align_up(size_t x, size_t a = 256) { return (x + a - 1) / a * a; }
 
 struct Layout {
     size_t rate, bw, mem, rate_cpu, bw_cpu, mem_cpu, link_bw, cong, prof, leaf, tau, tau_lb, cap, capg, cpb,
-        leaf_sorted, beff_sorted, tau_sorted, leaf_rank, tau_rank, gpu_layers, psum, lcost;
+        leaf_sorted, beff_sorted, tau_sorted, leaf_rank, tau_rank, gpu_layers, psum, lcost, gspill;
     size_t perm[2], sizes[2], nclus[2], roles[2];
     size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, stats, err, order_bins, items, slot_off, slot_mask, slot_size, slot_best,
         split_T, split_L, split_mu, split_layers, total;
@@ -96,6 +96,8 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K, bool layered = false
     if (layered) {
         l.psum = take(8 * 3 * V * ((size_t)N + 1));
         l.lcost = take(8 * V * M * 2 * (size_t)N * N);
+    } else if (dp_spills(M, N, 4)) {
+        l.gspill = take(4 * (size_t)kSpillCtas * dp_spill_stride(M, N));
     }
     l.total = o;
     return l;
@@ -412,7 +414,8 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     if (cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, c->device) != cudaSuccess)
         return fail_free(E2_ECUDA, "cudaDeviceGetAttribute failed");
     c->dp_threads = 128;
-    c->dp_smem = layered ? dp_layered_smem_bytes(M, N) : dp_smem_bytes(M, N, c->dp_threads, 4);
+    c->dm.g_spill = !layered && dp_spills(M, N, c->dp_threads / 32);
+    c->dp_smem = layered ? dp_layered_smem_bytes(M, N) : dp_smem_bytes(M, N, c->dp_threads, 4, c->dm.g_spill);
     if ((M < N ? M : N) > kMaxReplicaDevices)
         return fail_free(E2_EINVAL, "replicas could exceed 256 devices (min(M, N) > 256)");
     if (c->dp_smem + 1024 > (size_t)smem_optin)
@@ -437,6 +440,10 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     if (layered) {
         c->psum = reinterpret_cast<uint64_t *>(ws + l.psum);
         c->lcost = reinterpret_cast<double *>(ws + l.lcost);
+    }
+    if (c->dm.g_spill) {
+        c->gspill = reinterpret_cast<uint32_t *>(ws + l.gspill);
+        c->spill_stride = dp_spill_stride(M, N);
     }
     c->link_bw = reinterpret_cast<double *>(ws + l.link_bw);
     c->cong = reinterpret_cast<double *>(ws + l.cong);

@@ -59,12 +59,48 @@ enum CtrlWord { kCtrlEnd = kAllBins, kCtrlNext = kCtrlEnd + kDpClasses, kCtrlTic
 // the device ids (rounded up to 16 bytes).  No slack: a few bytes more per CTA
 // can cost a CTA per SM (the 80-block model's largest DP, 22,208 B, fits 10
 // per SM; 16 B more fit 9).
-__host__ __device__ __forceinline__ unsigned dp_item_bytes(int m, int N, int warps, int key_bytes)
+//
+// With `spill` the suffix columns live in a global scratch (L2) and shared
+// memory keeps two of them (the chain's previous and current column) plus a
+// per-warp buffer the master combine stages its suffix column into: about a
+// third less shared memory for the large replicas, and more CTAs per SM.
+__host__ __device__ __forceinline__ unsigned dp_item_bytes(int m, int N, int warps, int key_bytes, bool spill = false)
 {
     const unsigned W = (unsigned)(N - m + 1);
-    const unsigned keys = 3u * (unsigned)m * W + (unsigned)(2 * warps + 2) * W + 2u * (unsigned)m;
+    const unsigned gcols = spill ? 2u : (unsigned)m;
+    const unsigned keys = 2u * (unsigned)m * W + gcols * W + (unsigned)((spill ? 3 : 2) * warps + 2) * W +
+                          2u * (unsigned)m;
     const unsigned bytes = (unsigned)m * 12u + keys * (unsigned)key_bytes + (unsigned)m * 2u;
     return (bytes + 15u) & ~15u;
+}
+
+// Whether the DP spills its suffix columns (see dp_item_bytes): when the
+// largest replica's run would otherwise need more than kSpillAbove bytes of
+// shared memory (fewer than five CTAs per SM), as with the 126-block model.
+// A function of the sizes alone, so that the workspace size can include the
+// scratch: kSpillCtas persistent CTAs at most, each with room for the largest
+// run's suffix columns.
+constexpr unsigned kSpillAbove = 40u * 1024u;
+constexpr int kSpillCtas = 4096;
+__host__ __forceinline__ bool dp_spills(int M, int N, int warps)
+{
+    const int mmax = M < N ? M : N;
+    unsigned best = 0;
+    for (int m = 1; m <= mmax; ++m) {
+        const unsigned b = dp_item_bytes(m, N, warps, 4, false);
+        if (b > best) best = b;
+    }
+    return best > kSpillAbove;
+}
+__host__ __forceinline__ size_t dp_spill_stride(int M, int N)   // keys per CTA: max over m of m * W
+{
+    const int mmax = M < N ? M : N;
+    size_t best = 0;
+    for (int m = 1; m <= mmax; ++m) {
+        const size_t k = (size_t)m * (size_t)(N - m + 1);
+        if (k > best) best = k;
+    }
+    return (best + 3) & ~(size_t)3;
 }
 
 // Stats slots (unsigned long long, atomically accumulated).
@@ -83,13 +119,15 @@ struct Dims {
                          // 2: both roles per replica, the adapted-SplitWise rule picks the roles
     float lam_max_up;    // lam_max rounded up to float (the float latency bound is compared with it)
     unsigned dp_small;   // shared-memory bytes of DP class 1 (0: one class); m is in class 1 iff
-                         // dp_item_bytes(m, N, dp_warps, 4) <= dp_small
+                         // dp_item_bytes(m, N, dp_warps, 4, false) <= dp_small (class 1 never spills)
     int dp_warps;        // warps per DP CTA
     int grows;           // 1: block memory, head memory, block flops and bytes and activation bytes never
                          // shrink from one decode batch to the next (the pre-pass tests are then monotone)
     int objective;       // 0: waiting time w (Eq. 3-5); 1: per-request finishing time FT
     int offload;         // 1: some device has host memory for offloaded blocks
     int layered;         // 1: blocks of several types (per-layer prefix sums): the plain-scan DP path
+    int g_spill;         // 1: the DP keeps its suffix columns in the global scratch (dp_item_bytes)
+    int dp_grid0;        // CTAs of the first DP launch (the ones with a suffix-column scratch)
 };
 
 struct Tables {
@@ -123,6 +161,8 @@ struct SlotInfo {
 struct WorkList {
     uint64_t *items;           // [P*K*(b_max+1)] (slot << 8) | role << 7 | sweep << 6 | variant bit
     unsigned *ctrl;            // [kAllBins] bins/cursors, then the CtrlWord words
+    uint32_t *gspill;          // [kSpillCtas][spill_stride] suffix columns of each persistent DP CTA
+    unsigned spill_stride;     // keys per CTA
 };
 
 // Results of the DP runs, per (slot, variant bit).
@@ -234,6 +274,8 @@ struct e2_ctx {
     int32_t *err = nullptr;
     unsigned *order_bins = nullptr;   // [kCtrlWords]
     uint64_t *items = nullptr;        // [P*K*b_max] DP work items, heaviest first
+    uint32_t *gspill = nullptr;       // suffix-column scratch of the DP CTAs (dm.g_spill only)
+    size_t spill_stride = 0;          // its keys per CTA
     int32_t *slot_off = nullptr;      // [P*K]
     uint64_t *slot_mask = nullptr;    // [P*K]
     uint8_t *slot_size = nullptr;     // [P*K]
@@ -281,7 +323,7 @@ cudaError_t launch_step(const e2_ctx *c, const DevPop &src, const DevPop &dst, u
 cudaError_t find_ga_node(cudaGraph_t graph, cudaGraphNode_t *node);
 cudaError_t set_ga_node(const e2_ctx *c, cudaGraphExec_t exec, cudaGraphNode_t node, const DevPop &src,
                         const DevPop &dst, uint64_t seed, uint32_t gen);
-size_t dp_smem_bytes(int M, int N, int threads, int key_bytes);
+size_t dp_smem_bytes(int M, int N, int threads, int key_bytes, bool spill = false);
 size_t dp_layered_smem_bytes(int M, int N);   // the plain-scan DP's shared memory for the largest replica
 cudaError_t configure_eval(e2_ctx *c);   // shared memory limit and persistent grid size
 size_t rank_pow2(size_t n);

@@ -74,15 +74,16 @@ def test_eval_parity_full_size_sampled(name, P, sample):
     idx = np.sort(np.random.default_rng(5).choice(P, sample, replace=False))
     ora = O.OracleProblem(prob).eval_population(take(g, idx), prob.K_max, nthreads=O.num_threads())
     assert_eval_equal(gpu, ora, rows=idx)
-    # the 126-block model's largest DP leaves room for 4 CTAs per SM: the
-    # replica sizes that need half of it run in a second launch with more
+    # the 126-block model's largest DP spills its suffix columns to a global
+    # scratch (6 CTAs per SM instead of 4); the small replica sizes run in a
+    # second launch that does not spill, at that kernel's best occupancy
     st = eng.stats()
     assert st["dp_launches"] == (2 if st["dp_ctas_small"] else 1)
     assert st["dp_runs_small"] < st["dp_runs"]
     assert (st["dp_runs_small"] > 0) == (st["dp_launches"] == 2), st
     if name == "c4":
-        assert st["dp_launches"] == 2 and st["dp_ctas_small"] >= 2 * st["dp_ctas"], st
-        assert 2 * st["dp_smem_small"] <= st["dp_smem"], st
+        assert st["dp_launches"] == 2 and st["dp_ctas_small"] > st["dp_ctas"], st
+        assert st["dp_smem_small"] < st["dp_smem"] <= 40 * 1024, st
     eng.close()
 
 
