@@ -270,6 +270,8 @@ struct e2_ctx {
     uint64_t *hash = nullptr;
     int32_t *dup = nullptr, *elite = nullptr;
     double *elite_fit = nullptr;
+    unsigned long long *elite_ctl = nullptr;   // [8]: threshold key of the elite selection, counts, path flag
+    int32_t *elite_cand = nullptr;             // [P] its candidates
     unsigned long long *stats = nullptr;
     int32_t *err = nullptr;
     unsigned *order_bins = nullptr;   // [kCtrlWords]

@@ -328,10 +328,12 @@ __global__ void __launch_bounds__(256) dup_kernel(Dims dm, DevPop p, const doubl
 // w, phase, index); the first Q ranks are the elites, and the warp of an elite
 // copies it into slot rank(g) of the next population.
 __global__ void __launch_bounds__(256) rank_kernel(Dims dm, const double *fit, const int32_t *dup,
-                                                   int32_t *elite, double *elite_fit, DevPop src, DevPop dst)
+                                                   int32_t *elite, double *elite_fit, DevPop src, DevPop dst,
+                                                   const unsigned long long *ctl)
 {
     __shared__ uint64_t s_w[kEliteTile], s_p[kEliteTile];
     __shared__ int s_d[kEliteTile];
+    if (ctl[2] != 0) return;                       // the candidate ranking took the elites
     const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
     const int g = blockIdx.x * (blockDim.x >> 5) + wl;
     const bool live = g < dm.P;
@@ -362,6 +364,151 @@ __global__ void __launch_bounds__(256) rank_kernel(Dims dm, const double *fit, c
             dst.roles[rank] = src.roles[g];
             elite[rank] = g;
             for (int q = 0; q < 4; ++q) elite_fit[(size_t)rank * 4 + q] = fit[(size_t)g * 4 + q];
+        }
+    }
+}
+
+// Elite selection without ranking every genome.  When at least Q genomes are
+// distinct, the elites are the Q first distinct genomes in the order (w,
+// phase, index), and each has w <= w_Q, the Q-th smallest w among the
+// distinct genomes (a genome with a larger w has at least Q distinct genomes
+// before it).  One CTA finds w_Q exactly by a radix select over the bit
+// patterns of w (8 passes of 8 bits, highest first) and lists the distinct
+// genomes with w <= w_Q; only they are ranked against the population.  When
+// w_Q is +inf (fewer than Q genomes have a finite w, as early in a search on
+// a large fleet) the finite ones are ranked and the rest of the elites are
+// the first distinct genomes of the (+inf, +inf) group in index order.  With
+// fewer than Q distinct genomes (duplicates then fill the elite slots) the
+// full ranking runs instead.  ctl: [0] w_Q bits, [1] candidates to rank,
+// [2] 1 = the selection applies (0: full ranking), [3] elites listed after
+// the candidates whose rank is their place in the list.
+constexpr int kSelThreads = 1024;
+
+__global__ void __launch_bounds__(kSelThreads) elite_select_kernel(int P, int Q, const double *fit, const int32_t *dup,
+                                                                   unsigned long long *ctl, int32_t *cand)
+{
+    __shared__ unsigned hist[256];
+    __shared__ unsigned long long s_prefix;
+    __shared__ unsigned s_need, s_distinct, s_ncand;
+    const uint64_t *fk = reinterpret_cast<const uint64_t *>(fit);
+    const int tid = threadIdx.x;
+    if (tid == 0) { s_prefix = 0; s_need = (unsigned)Q; s_distinct = 0; s_ncand = 0; }
+    __syncthreads();
+    unsigned nd = 0;
+    for (int g = tid; g < P; g += kSelThreads) nd += dup[g] == 0;
+    atomicAdd(&s_distinct, nd);
+    __syncthreads();
+    const bool apply = Q > 0 && s_distinct >= (unsigned)Q;
+    for (int pass = 0; apply && pass < 8; ++pass) {
+        const int shift = 56 - 8 * pass;
+        const uint64_t hi_mask = pass ? ~0ull << (shift + 8) : 0ull;
+        for (int b = tid; b < 256; b += kSelThreads) hist[b] = 0;
+        __syncthreads();
+        const uint64_t prefix = s_prefix;
+        for (int g = tid; g < P; g += kSelThreads) {
+            if (dup[g]) continue;
+            const uint64_t w = fk[(size_t)g * 4];
+            if ((w & hi_mask) == prefix) atomicAdd(&hist[(w >> shift) & 0xFFu], 1u);
+        }
+        __syncthreads();
+        if (tid == 0) {                                   // the bucket holding the need-th smallest
+            unsigned need = s_need, b = 0;
+            while (hist[b] < need) { need -= hist[b]; ++b; }
+            s_need = need;
+            s_prefix = prefix | ((uint64_t)b << shift);
+        }
+        __syncthreads();
+    }
+    __shared__ unsigned s_bad, s_wsum[kSelThreads / 32], s_run;
+    unsigned direct = 0;                                  // elites whose rank is their place in the list
+    bool use = apply;
+    if (apply) {
+        const uint64_t wq = s_prefix;
+        if (wq != kInfKey) {                              // rank every distinct genome with w <= w_Q
+            for (int g = tid; g < P; g += kSelThreads)
+                if (!dup[g] && fk[(size_t)g * 4] <= wq) cand[atomicAdd(&s_ncand, 1u)] = g;
+            __syncthreads();
+        } else {
+            // fewer than Q distinct genomes with a finite w: those are ranked; the
+            // rest of the elites are the first distinct genomes of the (+inf, +inf)
+            // group, in index order (an infinite w comes with an infinite phase;
+            // anything else takes the full ranking)
+            if (tid == 0) s_bad = 0;
+            __syncthreads();
+            for (int g = tid; g < P; g += kSelThreads) {
+                if (dup[g]) continue;
+                if (fk[(size_t)g * 4] != kInfKey) cand[atomicAdd(&s_ncand, 1u)] = g;
+                else if (fk[(size_t)g * 4 + 1] != kInfKey) s_bad = 1;
+            }
+            __syncthreads();
+            use = s_bad == 0;
+            const unsigned F = s_ncand, need = (unsigned)Q - F;
+            if (use) {
+                const int lane = tid & 31, wl = tid >> 5;
+                if (tid == 0) s_run = 0;
+                __syncthreads();
+                for (int base = 0; base < P && s_run < need; base += kSelThreads) {
+                    const int g = base + tid;
+                    const bool f = g < P && !dup[g] && fk[(size_t)g * 4] == kInfKey;
+                    const unsigned bal = __ballot_sync(0xFFFFFFFFu, f);
+                    if (lane == 0) s_wsum[wl] = __popc(bal);
+                    __syncthreads();
+                    unsigned before = 0;
+                    for (int w2 = 0; w2 < wl; ++w2) before += s_wsum[w2];
+                    const unsigned ord = s_run + before + __popc(bal & ((1u << lane) - 1u));
+                    if (f && ord < need) cand[F + ord] = g;
+                    __syncthreads();
+                    if (tid == 0) {
+                        unsigned t = 0;
+                        for (int w2 = 0; w2 < kSelThreads / 32; ++w2) t += s_wsum[w2];
+                        s_run += t;
+                    }
+                    __syncthreads();
+                }
+                direct = need;
+            }
+        }
+    }
+    if (tid == 0) {
+        ctl[0] = s_prefix;
+        ctl[1] = use ? s_ncand : 0;
+        ctl[2] = use ? 1ull : 0ull;
+        ctl[3] = use ? direct : 0;
+    }
+}
+
+// rank(g) for the candidates (one warp each, the whole population scanned from
+// L2); an elite (rank < Q) is copied into slot rank of the next population.
+__global__ void __launch_bounds__(256) elite_cand_rank_kernel(Dims dm, const double *fit, const int32_t *dup,
+                                                              const unsigned long long *ctl, const int32_t *cand,
+                                                              int32_t *elite, double *elite_fit, DevPop src, DevPop dst)
+{
+    if (ctl[2] == 0) return;
+    const unsigned ncand = (unsigned)ctl[1], total = ncand + (unsigned)ctl[3];
+    const int lane = threadIdx.x & 31;
+    const unsigned warps = gridDim.x * (blockDim.x >> 5);
+    const uint64_t *fk = reinterpret_cast<const uint64_t *>(fit);
+    for (unsigned i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); i < total; i += warps) {
+        const int g = cand[i];
+        int rank = (int)i;                               // entries past ncand: rank = place in the list
+        if (i < ncand) {
+            const uint64_t w = fk[(size_t)g * 4], ph = fk[(size_t)g * 4 + 1];
+            rank = 0;
+            for (int h = lane; h < dm.P; h += 32)
+                rank += elite_before(dup[h], fk[(size_t)h * 4], fk[(size_t)h * 4 + 1], h, 0, w, ph, g);
+#pragma unroll
+            for (int x = 16; x; x >>= 1) rank += __shfl_xor_sync(0xFFFFFFFFu, rank, x);
+        }
+        if (rank < dm.Q) {
+            const int M = dm.M, K = dm.K;
+            for (int j = lane; j < M; j += 32) dst.perm[(size_t)rank * M + j] = src.perm[(size_t)g * M + j];
+            for (int j = lane; j < K; j += 32) dst.sizes[(size_t)rank * K + j] = src.sizes[(size_t)g * K + j];
+            if (lane == 0) {
+                dst.nclus[rank] = src.nclus[g];
+                dst.roles[rank] = src.roles[g];
+                elite[rank] = g;
+                for (int q = 0; q < 4; ++q) elite_fit[(size_t)rank * 4 + q] = fit[(size_t)g * 4 + q];
+            }
         }
     }
 }
@@ -591,9 +738,15 @@ cudaError_t launch_elites(const e2_ctx *c, const DevPop &p, const DevPop &dst)
 {
     const unsigned blocks = (unsigned)(((size_t)c->dm.P * 32 + 255) / 256);
     dup_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, p, c->fit, c->hash, c->dup);
-    if (c->dm.Q > 0)
-        rank_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, c->fit, c->dup, c->elite, c->elite_fit, p, dst);
-    c->launches += c->dm.Q > 0 ? 2 : 1;
+    if (c->dm.Q > 0) {
+        elite_select_kernel<<<1, kSelThreads, 0, c->stream>>>(c->dm.P, c->dm.Q, c->fit, c->dup, c->elite_ctl,
+                                                              c->elite_cand);
+        elite_cand_rank_kernel<<<152 * 4, 256, 0, c->stream>>>(c->dm, c->fit, c->dup, c->elite_ctl, c->elite_cand,
+                                                               c->elite, c->elite_fit, p, dst);
+        rank_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, c->fit, c->dup, c->elite, c->elite_fit, p, dst,
+                                                   c->elite_ctl);
+    }
+    c->launches += c->dm.Q > 0 ? 4 : 1;
     return cudaGetLastError();
 }
 
