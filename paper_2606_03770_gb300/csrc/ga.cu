@@ -411,11 +411,24 @@ __global__ void __launch_bounds__(kSelThreads) elite_select_kernel(int P, int Q,
             if ((w & hi_mask) == prefix) atomicAdd(&hist[(w >> shift) & 0xFFu], 1u);
         }
         __syncthreads();
-        if (tid == 0) {                                   // the bucket holding the need-th smallest
-            unsigned need = s_need, b = 0;
-            while (hist[b] < need) { need -= hist[b]; ++b; }
-            s_need = need;
-            s_prefix = prefix | ((uint64_t)b << shift);
+        if (tid < 32) {                                   // the bucket holding the need-th smallest:
+            const unsigned need = s_need;                 // a warp scan of eight-bin sums, then the
+            unsigned c = 0;                               // lane whose sums cross need scans its bins
+#pragma unroll
+            for (int j = 0; j < 8; ++j) c += hist[tid * 8 + j];
+            unsigned incl = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const unsigned y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+                if (tid >= o) incl += y;
+            }
+            const unsigned crossed = __ballot_sync(0xFFFFFFFFu, incl >= need);
+            if (tid == __ffs(crossed) - 1) {
+                unsigned left = need - (incl - c), b = (unsigned)tid * 8;
+                while (hist[b] < left) { left -= hist[b]; ++b; }
+                s_need = left;
+                s_prefix = prefix | ((uint64_t)b << shift);
+            }
         }
         __syncthreads();
     }
@@ -477,29 +490,49 @@ __global__ void __launch_bounds__(kSelThreads) elite_select_kernel(int P, int Q,
     }
 }
 
-// rank(g) for the candidates (one warp each, the whole population scanned from
-// L2); an elite (rank < Q) is copied into slot rank of the next population.
-__global__ void __launch_bounds__(256) elite_cand_rank_kernel(Dims dm, const double *fit, const int32_t *dup,
+// rank(g) for the candidates, one warp each.  Every genome before a candidate
+// in the elite order is distinct with a w no larger, so it is a candidate
+// itself: a candidate's rank is its count of candidates before it, taken
+// over tiles of the candidate list staged in shared memory.  An elite (rank
+// < Q) is copied into slot rank of the next population.
+__global__ void __launch_bounds__(256) elite_cand_rank_kernel(Dims dm, const double *fit,
                                                               const unsigned long long *ctl, const int32_t *cand,
                                                               int32_t *elite, double *elite_fit, DevPop src, DevPop dst)
 {
+    __shared__ uint64_t s_w[kEliteTile], s_p[kEliteTile];
+    __shared__ int s_g[kEliteTile];
     if (ctl[2] == 0) return;
     const unsigned ncand = (unsigned)ctl[1], total = ncand + (unsigned)ctl[3];
-    const int lane = threadIdx.x & 31;
-    const unsigned warps = gridDim.x * (blockDim.x >> 5);
+    const int lane = threadIdx.x & 31, NWB = blockDim.x >> 5;
     const uint64_t *fk = reinterpret_cast<const uint64_t *>(fit);
-    for (unsigned i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); i < total; i += warps) {
-        const int g = cand[i];
+    for (unsigned i0 = blockIdx.x * NWB; i0 < total; i0 += gridDim.x * NWB) {   // uniform over the block
+        const unsigned i = i0 + (threadIdx.x >> 5);
+        const bool live = i < total, ranked = i < ncand;
+        const int g = live ? cand[i] : 0;
+        const uint64_t w = ranked ? fk[(size_t)g * 4] : 0, ph = ranked ? fk[(size_t)g * 4 + 1] : 0;
         int rank = (int)i;                               // entries past ncand: rank = place in the list
-        if (i < ncand) {
-            const uint64_t w = fk[(size_t)g * 4], ph = fk[(size_t)g * 4 + 1];
-            rank = 0;
-            for (int h = lane; h < dm.P; h += 32)
-                rank += elite_before(dup[h], fk[(size_t)h * 4], fk[(size_t)h * 4 + 1], h, 0, w, ph, g);
+        if (i0 < ncand) {
+            int cnt = 0;
+            for (unsigned base = 0; base < ncand; base += kEliteTile) {
+                __syncthreads();
+                for (unsigned t = threadIdx.x; t < kEliteTile && base + t < ncand; t += blockDim.x) {
+                    const int h = cand[base + t];
+                    s_g[t] = h;
+                    s_w[t] = fk[(size_t)h * 4];
+                    s_p[t] = fk[(size_t)h * 4 + 1];
+                }
+                __syncthreads();
+                if (ranked) {
+                    const unsigned lim = min((unsigned)kEliteTile, ncand - base);
+                    for (unsigned t = lane; t < lim; t += 32)
+                        cnt += elite_before(0, s_w[t], s_p[t], s_g[t], 0, w, ph, g);
+                }
+            }
 #pragma unroll
-            for (int x = 16; x; x >>= 1) rank += __shfl_xor_sync(0xFFFFFFFFu, rank, x);
+            for (int x = 16; x; x >>= 1) cnt += __shfl_xor_sync(0xFFFFFFFFu, cnt, x);
+            if (ranked) rank = cnt;
         }
-        if (rank < dm.Q) {
+        if (live && rank < dm.Q) {
             const int M = dm.M, K = dm.K;
             for (int j = lane; j < M; j += 32) dst.perm[(size_t)rank * M + j] = src.perm[(size_t)g * M + j];
             for (int j = lane; j < K; j += 32) dst.sizes[(size_t)rank * K + j] = src.sizes[(size_t)g * K + j];
@@ -741,7 +774,7 @@ cudaError_t launch_elites(const e2_ctx *c, const DevPop &p, const DevPop &dst)
     if (c->dm.Q > 0) {
         elite_select_kernel<<<1, kSelThreads, 0, c->stream>>>(c->dm.P, c->dm.Q, c->fit, c->dup, c->elite_ctl,
                                                               c->elite_cand);
-        elite_cand_rank_kernel<<<152 * 4, 256, 0, c->stream>>>(c->dm, c->fit, c->dup, c->elite_ctl, c->elite_cand,
+        elite_cand_rank_kernel<<<152 * 4, 256, 0, c->stream>>>(c->dm, c->fit, c->elite_ctl, c->elite_cand,
                                                                c->elite, c->elite_fit, p, dst);
         rank_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, c->fit, c->dup, c->elite, c->elite_fit, p, dst,
                                                    c->elite_ctl);
