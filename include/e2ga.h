@@ -223,16 +223,16 @@ typedef struct {
     uint64_t tps_pruned;        /* decode variants a latency lower bound proved
                                    to miss Min_TPS (their DP is skipped)        */
     uint64_t dp_runs_small;     /* of dp_runs, those of the second DP launch:
-                                   replica sizes whose DP needs at most half the
-                                   largest one's shared memory, run with more
-                                   CTAs per SM (0 where that raises no
-                                   occupancy and one launch runs them all)      */
+                                   the small replica sizes, run with
+                                   more runs in flight per SM, four warps per
+                                   run or one (0 where that raises no occupancy
+                                   and one launch runs them all)                */
     uint64_t dp_launches;       /* DP kernel launches per evaluation (1 or 2;
                                    fixed at e2_create)                          */
     uint64_t dp_ctas;           /* persistent CTAs of the first DP launch       */
     uint64_t dp_smem;           /* and its dynamic shared memory per CTA (B)    */
     uint64_t dp_ctas_small;     /* the same for the second launch (0: none)     */
-    uint64_t dp_smem_small;
+    uint64_t dp_smem_small;     /* (per run: per warp when a warp runs one)     */
     uint64_t launches;          /* kernels this context has launched since
                                    e2_create, cumulative (a recorded generation
                                    counts its kernel nodes per replay)          */
@@ -245,6 +245,9 @@ typedef struct {
                                    partition, or a traceback found no split
                                    attaining its cell); nonzero makes
                                    e2_get_stats return E2_EDEVICE               */
+    uint64_t dp_runs_per_cta_small; /* runs in flight per CTA of the second launch:
+                                   1 (four warps per run) or 4 (a warp each; 0:
+                                   no second launch)                            */
 } e2_stats;
 
 typedef struct e2_ctx e2_ctx;

@@ -42,69 +42,11 @@
 // step 4).  mu* = the smallest mu with the least bottleneck (the oracle's
 // first-wins argmin); its columns are recomputed for the traceback.
 #include "e2ga_internal.cuh"
+#include "dp_span.cuh"
 
 namespace e2 {
 
 namespace {
-
-// D_k[r] for one cell (see the header comment), on order keys (the largest
-// value is +inf).
-template <typename Key>
-__device__ __forceinline__ Key dp_cell(const Key *__restrict__ prev, const Key *__restrict__ row, Key tau, int r)
-{
-    int lo = 0, hi = r + 1;
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (prev[mid] >= row[r - mid]) hi = mid;
-        else lo = mid + 1;
-    }
-    Key h = (Key)~(Key)0;
-    if (lo <= r) h = prev[lo];
-    if (lo >= 1) h = min(h, row[r - lo + 1]);
-    return max(h, tau);
-}
-
-// D_k[r] for the cells r0 <= r < r1 of one column: the first crossover by
-// bisection, then each next one from the last.  With both operands
-// non-decreasing, the crossover of r + 1 is that of r or one more (if
-// prev[s] >= row[r-s] then prev[s+1] >= row[(r+1)-(s+1)]), so every cell after
-// the first costs one probe.
-template <typename Key>
-__device__ __forceinline__ void dp_span(const Key *__restrict__ prev, const Key *__restrict__ row, Key tau,
-                                        Key *__restrict__ cur, int r0, int r1)
-{
-    if (r0 >= r1) return;
-    int r = r0, lo = 0, hi = r0 + 1;
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (prev[mid] >= row[r - mid]) hi = mid;
-        else lo = mid + 1;
-    }
-    for (;;) {
-        Key h = (Key)~(Key)0;
-        if (lo <= r) h = prev[lo];
-        if (lo >= 1) h = min(h, row[r - lo + 1]);
-        cur[r] = max(h, tau);
-        if (++r >= r1) break;
-        if (!(prev[lo] >= row[r - lo])) ++lo;                // lo <= r: the crossover moves by at most one
-    }
-}
-
-__device__ __forceinline__ void cp_async4(void *smem_dst, const void *gmem_src)
-{
-    const unsigned sa = (unsigned)__cvta_generic_to_shared(smem_dst);
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(sa), "l"(gmem_src) : "memory");
-}
-
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
-
-
-__device__ __forceinline__ int warp_sum(int x)
-{
-#pragma unroll
-    for (int o = 16; o; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
-    return x;
-}
 
 // Candidates (mu, k, i, j) the plain recurrence examines for one DP run:
 // m * (N + sum_{k=2..m} (N-k+1)(N-k+2)/2).
@@ -450,23 +392,6 @@ __global__ void order_scatter_kernel(Dims dm, DevPop pop, SlotInfo si, WorkList 
         }
     }
 }
-
-// A row of order keys from the rank table into shared memory, copied
-// asynchronously.
-__device__ __forceinline__ void stage_row(uint32_t *dst, const uint32_t *src, int W, int lane)
-{
-    for (int n = lane; n < W; n += 32) cp_async4(dst + n, src + n);
-}
-
-// The head row of a master, fetched asynchronously while the warp builds H.
-template <typename Key> struct HeadRow;
-template <> struct HeadRow<uint32_t> {
-    __device__ __forceinline__ void start(uint32_t *dst, const uint32_t *src, int W, int lane)
-    {
-        for (int r = lane; r < W; r += 32) cp_async4(dst + r, src + r);
-    }
-    __device__ __forceinline__ void finish(uint32_t *, const uint32_t *, int, int) { cp_async_wait_all(); }
-};
 
 // Persistent CTAs; each work item is one (genome, replica slot, variant) the
 // pre-pass kept, skipped if a larger batch of its replica was already
@@ -1867,6 +1792,7 @@ cudaError_t configure_eval(e2_ctx *c)
         c->dp_grid = (per_sm > 0 ? per_sm : 1) * (sms > 0 ? sms : 1);
         c->dm.dp_warps = c->dp_threads / 32;
         c->dm.dp_small = 0;
+        c->dp_warp1 = 0;
         c->dp_grid1 = 0;
         c->dp_smem1 = 0;
         return cudaSuccess;
@@ -1929,6 +1855,35 @@ cudaError_t configure_eval(e2_ctx *c)
             c->dp_smem1 = small;
         }
     }
+    // without a four-warp class 1, the small sizes may run one per warp: the
+    // largest per-warp slice whose runs in flight per SM are at least twice
+    // class 0's (its CTAs per SM).  A warp's run takes longer than a CTA's, so
+    // this pays only with many runs per warp: the population's slots at least
+    // eight times the class's runs in flight on the GPU.
+    c->dp_warp1 = 0;
+    if (c->dm.dp_small == 0) {
+        size_t wslice = 0;
+        int wocc = 0;
+        for (int m = 1; m <= mmax; ++m) {
+            const size_t b = dp_item_bytes(m, c->dm.N, 1, 4, false);
+            if (b <= wslice || b > c->dp_smem) continue;
+            int occ = 0;
+            e = dp_warp_occupancy((unsigned)b, &occ);
+            if (e != cudaSuccess) return e;
+            if (occ * kDpWarpRuns >= 2 * per_sm) { wslice = b; wocc = occ; }
+        }
+        const long long slots = (long long)c->dm.P * c->dm.K;
+        if (wslice > 0 && slots < 8LL * kDpWarpRuns * wocc * sms) wslice = 0;
+        if (wslice > 0) {
+            e = dp_warp_occupancy((unsigned)wslice, &wocc);
+            if (e != cudaSuccess) return e;
+            c->dm.dp_small = (unsigned)wslice;
+            c->dm.dp_warps = 1;
+            c->dp_warp1 = 1;
+            c->dp_grid1 = wocc * sms;
+            c->dp_smem1 = wslice;
+        }
+    }
     if (c->dm.g_spill && c->dp_grid > kSpillCtas) c->dp_grid = kSpillCtas;   // the scratch holds kSpillCtas CTAs
     c->dm.dp_grid0 = c->dp_grid;
     return cudaSuccess;
@@ -1970,9 +1925,13 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
         dp_eval_kernel<false><<<(unsigned)c->dp_grid, c->dp_threads, c->dp_smem, c->stream>>>(c->dm, tb, p, out, wl, si,
                                                                                             so, 0);
     if (c->dp_grid1 > 0) {                       // class 1: the small sizes, never spilling
-        dp_eval_kernel<false><<<(unsigned)c->dp_grid1, c->dp_threads, c->dp_smem1, c->side>>>(c->dm, tb, p, out, wl,
-                                                                                            si, so, 1);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        if (c->dp_warp1)
+            e = dp_warp_launch(c->dp_grid1, (unsigned)c->dp_smem1, c->side, c->dm, tb, p, out, wl, si, so);
+        else
+            dp_eval_kernel<false><<<(unsigned)c->dp_grid1, c->dp_threads, c->dp_smem1, c->side>>>(c->dm, tb, p, out,
+                                                                                                wl, si, so, 1);
+        if (e == cudaSuccess) e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
         if ((e = cudaEventRecord(c->ev_dp_join, c->side)) != cudaSuccess) return e;
         if ((e = cudaStreamWaitEvent(c->stream, c->ev_dp_join, 0)) != cudaSuccess) return e;
     }

@@ -771,6 +771,7 @@ int e2_get_stats(e2_ctx *c, e2_stats *out)
     out->dp_smem = c->dp_smem;
     out->dp_ctas_small = (uint64_t)c->dp_grid1;
     out->dp_smem_small = c->dp_smem1;
+    out->dp_runs_per_cta_small = c->dp_grid1 > 0 ? (c->dp_warp1 ? (uint64_t)kDpWarpRuns : 1u) : 0u;
     out->launches = c->launches;
     if (out->device_errors)
         return fail(c, E2_EDEVICE, "a device-side consistency check of the last evaluation failed");

@@ -120,7 +120,7 @@ struct Dims {
     float lam_max_up;    // lam_max rounded up to float (the float latency bound is compared with it)
     unsigned dp_small;   // shared-memory bytes of DP class 1 (0: one class); m is in class 1 iff
                          // dp_item_bytes(m, N, dp_warps, 4, false) <= dp_small (class 1 never spills)
-    int dp_warps;        // warps per DP CTA
+    int dp_warps;        // warps of a class-1 run's layout: 1 when class 1 runs one run per warp
     int grows;           // 1: block memory, head memory, block flops and bytes and activation bytes never
                          // shrink from one decode batch to the next (the pre-pass tests are then monotone)
     int objective;       // 0: waiting time w (Eq. 3-5); 1: per-request finishing time FT
@@ -289,7 +289,8 @@ struct e2_ctx {
     unsigned long long gen_kernels[2] = {0, 0}; // kernel nodes of each recorded generation
     int dp_grid = 0;                  // persistent DP CTAs of class 0
     int dp_grid1 = 0;                 // persistent DP CTAs of class 1 (0: one class)
-    size_t dp_smem1 = 0;              // their shared memory
+    size_t dp_smem1 = 0;              // their shared memory (per warp with dp_warp1)
+    int dp_warp1 = 0;                 // 1: class 1 runs one DP run per warp (dp_warp.cu)
     cudaEvent_t ev_dp_fork = nullptr, ev_dp_join = nullptr;   // class 1 runs on the side stream
     cudaEvent_t ev_dp_start = nullptr, ev_dp_stop = nullptr;   // optional timing hook
     // recorded generation (e2_run_generation), one per population buffer
@@ -326,6 +327,14 @@ cudaError_t find_ga_node(cudaGraph_t graph, cudaGraphNode_t *node);
 cudaError_t set_ga_node(const e2_ctx *c, cudaGraphExec_t exec, cudaGraphNode_t node, const DevPop &src,
                         const DevPop &dst, uint64_t seed, uint32_t gen);
 size_t dp_smem_bytes(int M, int N, int threads, int key_bytes, bool spill = false);
+// The warp-per-run DP kernel of the small replica sizes (dp_warp.cu): its CTA
+// size, its CTAs per SM with `slice` bytes of shared memory per warp, and its
+// launch on `stream` over class 1 of the work list.
+constexpr int kDpWarpRuns = 4;
+cudaError_t dp_warp_occupancy(unsigned slice, int *per_sm);
+cudaError_t dp_warp_launch(int grid, unsigned slice, cudaStream_t stream, const Dims &dm, const Tables &tb,
+                           const DevPop &pop, const EvalOut &out, const WorkList &wl, const SlotInfo &si,
+                           const SplitOut &so);
 size_t dp_layered_smem_bytes(int M, int N);   // the plain-scan DP's shared memory for the largest replica
 cudaError_t configure_eval(e2_ctx *c);   // shared memory limit and persistent grid size
 size_t rank_pow2(size_t n);

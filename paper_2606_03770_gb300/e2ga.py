@@ -58,7 +58,8 @@ class e2_stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in ("genomes", "replicas", "dp_runs", "dp_cells", "dp_probes",
                                          "paper_candidates", "prechecked", "served", "tps_pruned",
                                          "dp_runs_small", "dp_launches", "dp_ctas", "dp_smem", "dp_ctas_small",
-                                         "dp_smem_small", "launches", "role_search_capped", "device_errors")]
+                                         "dp_smem_small", "launches", "role_search_capped", "device_errors",
+                                         "dp_runs_per_cta_small")]
 
 
 # name -> (restype, argtypes); the exported surface of include/e2ga.h

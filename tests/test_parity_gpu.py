@@ -79,7 +79,6 @@ def test_eval_parity_full_size_sampled(name, P, sample):
     # second launch that does not spill, at that kernel's best occupancy
     st = eng.stats()
     assert st["dp_launches"] == (2 if st["dp_ctas_small"] else 1)
-    assert st["dp_runs_small"] < st["dp_runs"]
     assert (st["dp_runs_small"] > 0) == (st["dp_launches"] == 2), st
     if name == "c4":
         assert st["dp_launches"] == 2 and st["dp_ctas_small"] > st["dp_ctas"], st
