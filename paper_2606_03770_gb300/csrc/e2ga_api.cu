@@ -23,7 +23,7 @@ struct Layout {
     size_t rate, bw, mem, rate_cpu, bw_cpu, mem_cpu, link_bw, cong, prof, leaf, tau, tau_lb, cap, capg, cpb,
         leaf_sorted, beff_sorted, tau_sorted, leaf_rank, tau_rank, gpu_layers, psum, lcost, gspill;
     size_t perm[2], sizes[2], nclus[2], roles[2];
-    size_t fit, layers, master, bsel, T, L, hash, dup, elite, elite_fit, elite_ctl, elite_cand, stats, err, order_bins, items, slot_off, slot_mask, slot_size, slot_best,
+    size_t fit, layers, master, bsel, T, L, hash, dup, dup_key, dup_idx, elite, elite_fit, elite_ctl, elite_cand, stats, err, order_bins, items, slot_off, slot_mask, slot_size, slot_best,
         split_T, split_L, split_mu, split_layers, total;
     int LS;
 };
@@ -79,6 +79,8 @@ Layout layout(int M, int N, int b_max, int P, int Q, int K, bool layered = false
     l.L = take(8 * (size_t)P * K);
     l.hash = take(8 * (size_t)P);
     l.dup = take(4 * (size_t)P);
+    l.dup_key = take(8 * (size_t)dup_table_size(P));         // fingerprint table of the duplicate test
+    l.dup_idx = take(4 * (size_t)dup_table_size(P));
     l.elite = take(4 * (size_t)(Q > 0 ? Q : 1));
     l.elite_fit = take(32 * (size_t)(Q > 0 ? Q : 1));
     l.elite_ctl = take(64);                                   // the elite selection's threshold and counts
@@ -469,6 +471,8 @@ int e2_create(const e2_devices *devs, const e2_links *links, const e2_layer_prof
     c->L = reinterpret_cast<double *>(ws + l.L);
     c->hash = reinterpret_cast<uint64_t *>(ws + l.hash);
     c->dup = reinterpret_cast<int32_t *>(ws + l.dup);
+    c->dup_key = reinterpret_cast<uint64_t *>(ws + l.dup_key);
+    c->dup_idx = reinterpret_cast<int32_t *>(ws + l.dup_idx);
     c->elite = reinterpret_cast<int32_t *>(ws + l.elite);
     c->elite_fit = reinterpret_cast<double *>(ws + l.elite_fit);
     c->elite_ctl = reinterpret_cast<unsigned long long *>(ws + l.elite_ctl);

@@ -81,6 +81,13 @@ __host__ __device__ __forceinline__ unsigned dp_item_bytes(int m, int N, int war
 // scratch: kSpillCtas persistent CTAs at most, each with room for the largest
 // run's suffix columns.
 constexpr unsigned kSpillAbove = 40u * 1024u;
+// Slots of the duplicate test's fingerprint table: the power of two >= 2P.
+__host__ __device__ __forceinline__ unsigned dup_table_size(int P)
+{
+    unsigned t = 2;
+    while (t < 2u * (unsigned)P) t <<= 1;
+    return t;
+}
 constexpr int kSpillCtas = 4096;
 __host__ __forceinline__ bool dp_spills(int M, int N, int warps)
 {
@@ -269,6 +276,8 @@ struct e2_ctx {
     double *T = nullptr, *L = nullptr;
     uint64_t *hash = nullptr;
     int32_t *dup = nullptr, *elite = nullptr;
+    uint64_t *dup_key = nullptr;      // [dup_table_size(P)] fingerprint table of the duplicate test
+    int32_t *dup_idx = nullptr;       //   and the smallest genome index of each fingerprint
     double *elite_fit = nullptr;
     unsigned long long *elite_ctl = nullptr;   // [8]: threshold key of the elite selection, counts, path flag
     int32_t *elite_cand = nullptr;             // [P] its candidates

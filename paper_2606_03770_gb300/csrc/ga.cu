@@ -283,8 +283,83 @@ __device__ __forceinline__ bool elite_before(int da, uint64_t wa, uint64_t pa, i
 constexpr int kEliteTile = 1024;
 
 // A genome equal to a lower-indexed one is a duplicate.  Equal genomes have
-// equal fitness (the evaluation is deterministic) and equal fingerprints, so
-// only those pairs are compared in full.
+// equal fingerprints (the finaliser's hash of the ordering, the replica sizes,
+// their count and the roles), so a genome is compared in full only with
+// genomes of its fingerprint: first with the lowest-indexed one, found in an
+// open-addressing table (dup_table_size(P) >= 2P slots, linear probing, so
+// never full; a slot keeps its fingerprint and the smallest index that carries
+// it); if the two differ -- a 64-bit collision, or genomes that differ only
+// in sizes or role bits past their replica count, which the fingerprint does
+// not cover -- with every lower-indexed genome of its fingerprint.
+// From kDupTableFrom genomes on (below, the table's fill and extra launch cost
+// more than the quadratic test: 1,024 genomes +2% per generation, 4,096 -1.8%).
+constexpr int kDupTableFrom = 4096;
+constexpr uint64_t kNoKey = ~0ull;                       // an empty slot
+__device__ __forceinline__ uint64_t table_key(uint64_t h) { return h == kNoKey ? kNoKey - 1 : h; }
+__device__ __forceinline__ unsigned table_start(uint64_t k, unsigned mask) { return (unsigned)(k ^ (k >> 32)) & mask; }
+
+// (the table is filled with kNoKey and INT32_MAX beforehand)
+__global__ void __launch_bounds__(256) dup_insert_kernel(int P, const uint64_t *hash, unsigned long long *tkey,
+                                                         int32_t *tidx, unsigned mask)
+{
+    for (int g = blockIdx.x * blockDim.x + threadIdx.x; g < P; g += gridDim.x * blockDim.x) {
+        const uint64_t k = table_key(hash[g]);
+        unsigned s = table_start(k, mask);
+        for (unsigned i = 0; i <= mask; ++i, s = (s + 1) & mask) {   // (a free slot is always found)
+            const unsigned long long prev = atomicCAS(&tkey[s], (unsigned long long)kNoKey, (unsigned long long)k);
+            if (prev == kNoKey || prev == k) {
+                atomicMin(&tidx[s], g);
+                break;
+            }
+        }
+    }
+}
+
+// Whether genomes a and b are equal (ordering, sizes, replica count, roles); a warp.
+__device__ __forceinline__ bool same_genome(const DevPop &p, int a, int b, int M, int K, int lane)
+{
+    bool diff = p.nclus[a] != p.nclus[b] || p.roles[a] != p.roles[b];
+    for (int i = lane; i < M && !diff; i += 32) diff = p.perm[(size_t)a * M + i] != p.perm[(size_t)b * M + i];
+    for (int i = lane; i < K && !diff; i += 32) diff = p.sizes[(size_t)a * K + i] != p.sizes[(size_t)b * K + i];
+    return __ballot_sync(0xFFFFFFFFu, diff) == 0u;
+}
+
+// One warp per genome.
+__global__ void __launch_bounds__(256) dup_lookup_kernel(Dims dm, DevPop p, const uint64_t *hash,
+                                                         const unsigned long long *tkey, const int32_t *tidx,
+                                                         unsigned mask, int32_t *dup)
+{
+    const int lane = threadIdx.x & 31;
+    const int g = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (g >= dm.P) return;
+    const uint64_t hr = hash[g], k = table_key(hr);
+    int first = g;
+    if (lane == 0) {                                              // (present: g itself was inserted)
+        unsigned s = table_start(k, mask);
+        for (unsigned i = 0; i < mask && tkey[s] != k; ++i) s = (s + 1) & mask;
+        if (tkey[s] == k) first = tidx[s];
+    }
+    first = __shfl_sync(0xFFFFFFFFu, first, 0);
+    bool d = false;
+    if (first < g) {
+        d = same_genome(p, first, g, dm.M, dm.K, lane);
+        for (int base = first + 1; base < g && !d; base += 32) {  // a fingerprint shared by different genomes
+            const int o = base + lane;
+            unsigned b = __ballot_sync(0xFFFFFFFFu, o < g && hash[o] == hr);
+            while (b && !d) {
+                const int oo = base + __ffs(b) - 1;
+                b &= b - 1;
+                d = same_genome(p, oo, g, dm.M, dm.K, lane);
+            }
+        }
+    }
+    if (lane == 0) dup[g] = d;
+}
+
+// Below kDupTableFrom genomes, the duplicate test compares each genome with
+// every lower-indexed one: equal genomes have equal fitness (the evaluation is
+// deterministic) and equal fingerprints, so only those pairs are compared in
+// full.
 __global__ void __launch_bounds__(256) dup_kernel(Dims dm, DevPop p, const double *fit,
                                                   const uint64_t *hash, int32_t *dup)
 {
@@ -770,7 +845,20 @@ cudaError_t launch_init(const e2_ctx *c, const DevPop &p, uint64_t seed)
 cudaError_t launch_elites(const e2_ctx *c, const DevPop &p, const DevPop &dst)
 {
     const unsigned blocks = (unsigned)(((size_t)c->dm.P * 32 + 255) / 256);
-    dup_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, p, c->fit, c->hash, c->dup);
+    const bool table = c->dm.P >= kDupTableFrom;
+    if (table) {
+        const unsigned tsize = dup_table_size(c->dm.P);
+        cudaError_t e = cudaMemsetAsync(c->dup_key, 0xFF, sizeof(uint64_t) * tsize, c->stream);
+        if (e == cudaSuccess) e = cudaMemsetAsync(c->dup_idx, 0x7F, sizeof(int32_t) * tsize, c->stream);
+        if (e != cudaSuccess) return e;
+        dup_insert_kernel<<<(unsigned)((c->dm.P + 255) / 256), 256, 0, c->stream>>>(
+            c->dm.P, c->hash, reinterpret_cast<unsigned long long *>(c->dup_key), c->dup_idx, tsize - 1);
+        dup_lookup_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, p, c->hash,
+                                                         reinterpret_cast<const unsigned long long *>(c->dup_key),
+                                                         c->dup_idx, tsize - 1, c->dup);
+    } else {
+        dup_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, p, c->fit, c->hash, c->dup);
+    }
     if (c->dm.Q > 0) {
         elite_select_kernel<<<1, kSelThreads, 0, c->stream>>>(c->dm.P, c->dm.Q, c->fit, c->dup, c->elite_ctl,
                                                               c->elite_cand);
@@ -779,7 +867,7 @@ cudaError_t launch_elites(const e2_ctx *c, const DevPop &p, const DevPop &dst)
         rank_kernel<<<blocks, 256, 0, c->stream>>>(c->dm, c->fit, c->dup, c->elite, c->elite_fit, p, dst,
                                                    c->elite_ctl);
     }
-    c->launches += c->dm.Q > 0 ? 4 : 1;
+    c->launches += (table ? 2 : 1) + (c->dm.Q > 0 ? 3 : 0);
     return cudaGetLastError();
 }
 

@@ -358,7 +358,7 @@ def test_min_tps_boundary_exact():
     assert served[0] == ora["bsel"][p, c] and served[1] != served[0]
 
 
-@pytest.mark.parametrize("name,P,gens", [("c1_tiny", 64, 5), ("c2", 1024, 5), ("c4", 1024, 4)])
+@pytest.mark.parametrize("name,P,gens", [("c1_tiny", 64, 5), ("c2", 1024, 5), ("c4", 1024, 4), ("c5", 4096, 3)])
 def test_recorded_generation_matches_separate_calls(name, P, gens):
     """e2_run_generation (one recorded graph per population buffer) gives the
     populations and fitness of e2_eval_population + e2_ga_step, also when
@@ -388,10 +388,12 @@ def test_recorded_generation_matches_separate_calls(name, P, gens):
         assert np.array_equal(fa, fb), gen
         assert_genomes_equal(a.get_population(), b.get_population())
         # a replay counts the recorded kernel nodes: as many as the separate calls launch
-        # (pre-pass, scatter, DP launches, finaliser, duplicates, elite selection,
-        # candidate ranks, full ranks, children)
+        # (pre-pass, scatter, DP launches, finaliser, duplicates -- from 4,096 genomes
+        # a fingerprint table and a lookup --, elite selection, candidate ranks, full
+        # ranks, children)
         sa, sb = a.stats(), b.stats()
-        assert sa["launches"] - la == sb["launches"] - lb == 8 + sa["dp_launches"], gen
+        expected = 8 + sa["dp_launches"] + (1 if P >= 4096 else 0)
+        assert sa["launches"] - la == sb["launches"] - lb == expected, gen
     torch.cuda.synchronize()
     assert x.elapsed_time(y) > 0
     b.set_timing_events()
