@@ -429,7 +429,7 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
     __shared__ double s_L, s_T;
     __shared__ unsigned s_item, s_next;           // s_next: an item claimed during the last traceback
     __shared__ unsigned long long s_bestkey;     // (V << 32) | mu of the best master so far
-    __shared__ uint32_t s_V0;
+    __shared__ uint32_t s_V0, s_V1;
     __shared__ unsigned s_prb[3];                // probes of a column over 32, 64, 128 threads
 
     const int K = dm.K, M = dm.M, N = dm.N;
@@ -518,6 +518,8 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
             }
             for (int k = wid; k < m; k += NW)                       // the loads of a row overlap
                 stage_row(leaf0 + (size_t)k * W, tb.leaf_rank + (vM + devs[k]) * 2 * dm.LS, W, lane);
+            if (SPILL && wid == NW - 1)                             // device 1's head row (step 3)
+                stage_row(row1s, tb.leaf_rank + ((vM + devs[0]) * 2 + 1) * dm.LS, W, lane);
             cp_async_wait_all();
             __syncthreads();
             // ---- 2. masters the memory allows (the pre-pass guarantees one)
@@ -534,27 +536,46 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                 return (Z - (cnt0[k] == 0)) == 0 && cnt1[k] >= 1 && S0 - cnt0[k] + cnt1[k] >= N;
             };
             ++st_runs;
-            // ---- 3. prefix columns (warps 0-1) and suffix columns (warps 2-3)
-            if (wid < 2) {
+            // ---- 3. prefix columns (warps 0-1) and suffix columns (warps 2-3).
+            //      With the spilled layout (the largest replicas) the prefix chain
+            //      runs first with the head on device 1: if then V_1 (its last
+            //      cell) equals V0 (the master-free optimum, from the suffix
+            //      side), every V_mu >= V0 = V_1, so mu* = 1 and these are the
+            //      columns step 5 would recompute; steps 4 and 5 are skipped.
+            //      Otherwise the chain runs again without the head.
+            auto prefix_chain = [&](bool head1) {
                 for (int k = 2; k <= m - 1; ++k) {
-                    const Key *prev = colF(k - 1), *row = leaf0 + (size_t)(k - 1) * W;
+                    const Key *prev = (head1 && k == 2) ? row1s : colF(k - 1), *row = leaf0 + (size_t)(k - 1) * W;
                     const Key t = tauk[k - 1];
                     Key *cur = Fst + (size_t)(k - 1) * W;
                     const int per = (W + 63) >> 6;                 // cells per thread
                     dp_span(prev, row, t, cur, tid * per, min(W, (tid + 1) * per));
                     bar_named(1, 64);
                 }
-                if (wid == 0) {                                   // V0 = F_m[W-1], the master-free optimum:
-                    uint32_t v0 = 0;                              // the minimum over every split, by the lanes
-                    if (m >= 2) {
-                        const Key *prev = colF(m - 1), *row = leaf0 + (size_t)(m - 1) * W;
-                        v0 = kInf;
-                        for (int q = lane; q < W; q += 32) v0 = min(v0, (uint32_t)max(prev[q], row[W - 1 - q]));
+            };
+            // the last cell of a chain, its minimum over every split taken by a warp's lanes
+            auto top_cell = [&](const Key *a, const Key *b, Key t) -> uint32_t {
+                uint32_t x = kInf;
+                for (int q = lane; q < W; q += 32) x = min(x, (uint32_t)max(a[q], b[W - 1 - q]));
 #pragma unroll
-                        for (int o = 16; o; o >>= 1) v0 = min(v0, __shfl_xor_sync(0xFFFFFFFFu, v0, o));
-                        v0 = max(v0, (uint32_t)tauk[m - 1]);
+                for (int o = 16; o; o >>= 1) x = min(x, __shfl_xor_sync(0xFFFFFFFFu, x, o));
+                return max(x, (uint32_t)t);
+            };
+            if (wid < 2) {
+                prefix_chain(SPILL);
+                if (wid == 0) {                                   // V0 = F_m[W-1] (V_1 when spilled)
+                    uint32_t v = 0;
+                    if (m >= 2)
+                        v = top_cell((SPILL && m == 2) ? row1s : colF(m - 1), leaf0 + (size_t)(m - 1) * W, tauk[m - 1]);
+                    if (lane == 0) {
+                        if (SPILL) {                              // (V_1, 1) seeds the best master
+                            s_V1 = v;
+                            s_bestkey = (m >= 2 && v != (uint32_t)kInf) ? ((unsigned long long)v << 32) | 1u : ~0ull;
+                        } else {
+                            s_V0 = v;
+                            s_bestkey = ~0ull;
+                        }
                     }
-                    if (lane == 0) { s_V0 = v0; s_bestkey = ~0ull; }
                 }
             } else {
                 for (int k = m - 1; k >= 2; --k) {
@@ -568,6 +589,10 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                         for (int r = r0; r < r1; ++r) __stcg(gsp + (size_t)(k - 1) * W + r, (uint32_t)cur[r]);
                     bar_named(2, 64);
                 }
+                if (SPILL && wid == 2) {                          // V0 = G_1[W-1]
+                    const uint32_t v = m >= 2 ? top_cell(leaf0, colG(2), tauk[1]) : 0u;
+                    if (lane == 0) s_V0 = v;
+                }
             }
             if (tid == 0 && m >= 3) {
                 st_cells += 2ull * (m - 2) * W;
@@ -579,12 +604,25 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
             //      optimum F_m[W-1]: the head only adds) exceeds the best V found
             //      so far, or ties it with a larger index
             const uint32_t V0 = s_V0;
+            bool spec = false;                                    // mu* = 1 proved (the spilled layout)
+            if (SPILL) {
+                spec = m >= 2 && s_V1 == V0 && V0 != (uint32_t)kInf;
+                if (tid == 0 && m >= 2) { st_cells += 1; st_probes += lprobe; }
+                if (!spec && m >= 3) {                            // the combine needs the master-free columns
+                    if (wid < 2) prefix_chain(false);
+                    if (tid == 0) {
+                        st_cells += (unsigned long long)(m - 2) * W;
+                        st_probes += (unsigned long long)(m - 2) * s_prb[1];
+                    }
+                    __syncthreads();
+                }
+            }
             auto bound = [&](int k) -> uint32_t { return mu_ok(k + 1) ? max(V0, (uint32_t)lbm[k]) : (uint32_t)kInf; };
 
             unsigned long long w_cells = 0, w_probes = 0;
             Key *H = Hb + (size_t)wid * W, *L1 = Lb + (size_t)wid * W;
-            for (int mu = wid + 1; mu <= m; mu += NW) {
-                if (!mu_ok(mu)) continue;
+            for (int mu = wid + 1; mu <= m && !spec; mu += NW) {
+                if (!mu_ok(mu) || (SPILL && m >= 2 && mu == 1)) continue;   // (V_1 is known when spilled)
                 const uint32_t lb = bound(mu - 1);
                 const unsigned long long bk = *reinterpret_cast<volatile unsigned long long *>(&s_bestkey);
                 const uint32_t bv = (uint32_t)(bk >> 32);
@@ -629,16 +667,18 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                 if (tid == 0 && (dm.grows || !role)) atomicAdd(&out.stats[kStDeviceErrors], 1ull);
                 continue;
             }
-            for (int r = tid; r < W; r += blockDim.x)
-                row1s[r] = (Key)tb.leaf_rank[((vM + devs[mus - 1]) * 2 + 1) * dm.LS + r];
-            __syncthreads();
-            // ---- 5. mu*'s prefix columns, for the traceback
+            if (!spec) {
+                for (int r = tid; r < W; r += blockDim.x)
+                    row1s[r] = (Key)tb.leaf_rank[((vM + devs[mus - 1]) * 2 + 1) * dm.LS + r];
+                __syncthreads();
+            }
+            // ---- 5. mu*'s prefix columns, for the traceback (already there when spec)
             auto rowk = [&](int k) -> const Key * { return k == mus ? row1s : leaf0 + (size_t)(k - 1) * W; };
             auto colD = [&](int k) -> const Key * {
                 if (k == 1) return mus == 1 ? row1s : leaf0;
                 return Fst + (size_t)(k - 1) * W;
             };
-            for (int k = (mus > 2 ? mus : 2); k <= m - 1; ++k) {
+            for (int k = (mus > 2 ? mus : 2); k <= m - 1 && !spec; ++k) {
                 const Key *prev = colD(k - 1), *row = rowk(k);
                 const Key t = tauk[k - 1];
                 Key *cur = Fst + (size_t)(k - 1) * W;
@@ -970,7 +1010,7 @@ __global__ void __launch_bounds__(128) dp_layered_kernel(Dims dm, Tables tb, Dev
 // SPILL: the suffix columns live in the global scratch (dm.g_spill), a
 // separate instance so that the other contexts keep their register count.
 template <bool SPILL>
-__global__ void __launch_bounds__(128) dp_eval_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out, WorkList wl,
+__global__ void __launch_bounds__(128, SPILL ? 6 : 0) dp_eval_kernel(Dims dm, Tables tb, DevPop pop, EvalOut out, WorkList wl,
                                                       SlotInfo si, SplitOut so, int cls)
 {
     dp_eval_body<uint32_t, SPILL>(dm, tb, pop, out, wl, si, so, cls);
