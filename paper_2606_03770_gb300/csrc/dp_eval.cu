@@ -132,12 +132,12 @@ __device__ __forceinline__ int item_bin(int level, int size)
 // too; rounding can only keep a variant the exact bound would drop, which
 // costs a DP run and changes no result.  Other profiles test every batch from
 // the largest down, and the first that passes keeps the smaller ones.
-// The surviving variants form the slot's mask.  A slot with nothing to run
-// (empty, more devices than blocks, no variant left) gets its outputs here;
-// the others count their work items into the ordering bins.  The last warp to
-// finish (a ticket taken after a fence where the warp counted, no waiting)
-// scans the bins into starting offsets, class 0 first and heaviest first
-// within a class, and stores the item total and where class 1 starts.
+// The surviving variants form the slot's mask.  A replica with nothing to run
+// (more devices than blocks, no variant left) gets its outputs here, and the
+// genome's last replica writes those of its empty slots (a warp on an empty
+// slot does nothing else); the others count their work items into the
+// ordering bins, which bins_kernel then scans into starting offsets, class 0
+// first and heaviest first within a class.
 __global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop pop, SlotInfo si, EvalOut out,
                                                   unsigned *ctrl)
 {
@@ -147,7 +147,6 @@ __global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop
     const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
     const int K = dm.K, M = dm.M, N = dm.N;
     const long long slot = (long long)blockIdx.x * (blockDim.x >> 5) + wl;
-    bool counted = false;                                     // this warp added to the bins
     if (slot < (long long)dm.P * K) {
         const int g = (int)(slot / K), c = (int)(slot - (long long)g * K);
         // the genome's replica count, sizes and roles, loaded together (all in bounds)
@@ -274,10 +273,17 @@ __global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop
                 }
             }
         }
-        // ---- the slot's outputs or its work count
+        // ---- the slot's outputs or its work count (the genome's last replica
+        //      also writes those of its slots past R)
         if (c < R && !mask)                                          // a replica that cannot serve
             for (int k = lane; k < m; k += 32) out.layers[(size_t)g * M + off + k] = -1;
-        if (lane == 0) {
+        if (c == R - 1)
+            for (int e = R + lane; e < K; e += 32) {
+                const size_t es = (size_t)g * K + e;
+                out.master[es] = -1; out.bsel[es] = -1;
+                out.T[es] = keyd(kInfKey); out.L[es] = keyd(kInfKey);
+            }
+        if (lane == 0 && c < R) {
             si.mask[slot] = mask;
             si.best[slot] = -1;
             if (n_pre) atomicAdd(&out.stats[kStPrecheck], n_pre);
@@ -298,22 +304,18 @@ __global__ void __launch_bounds__(64, 20) slot_kernel(Dims dm, Tables tb, DevPop
                 si.size[slot] = (uint8_t)size;
                 const int nv = __popcll(mask);
                 for (int lv = 0; lv < nv; ++lv) atomicAdd(&ctrl[item_bin(lv, size)], 1u);
-                counted = true;
             }
         }
     }
-    // ---- the last warp to finish scans the bins: with nb bins in use (class
-    //      1's only where that class exists), lane t owns positions
-    //      [t nb/32, (t+1) nb/32) of the descending bin order (class 0's bins,
-    //      then class 1's), read eight at a time
-    unsigned ticket = 0;
-    if (lane == 0) {
-        if (counted) __threadfence();                         // publish the bin counts (only they are read)
-        ticket = atomicAdd(&ctrl[kCtrlTicket], 1u);
-    }
-    ticket = __shfl_sync(0xFFFFFFFFu, ticket, 0);
-    if (ticket != gridDim.x * (blockDim.x >> 5) - 1) return;
-    __threadfence();
+}
+
+// The ordering bins' scan, after the pre-pass: with nb bins in use (class
+// 1's only where that class exists), lane t owns positions [t nb/32,
+// (t+1) nb/32) of the descending bin order (class 0's bins, then class 1's),
+// read eight at a time.  One warp.
+__global__ void bins_kernel(Dims dm, unsigned *ctrl)
+{
+    const int lane = threadIdx.x & 31;
     const int per = (dm.dp_small ? kAllBins : kOrderBins) / 32;
     unsigned *own = ctrl + kAllBins - 1 - lane * per;              // own[-j] = position per lane + j
     unsigned sum = 0;
@@ -1944,6 +1946,7 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
     const int mcap = c->dm.M < c->dm.N ? c->dm.M : c->dm.N;
     slot_kernel<<<(unsigned)((slots + 1) / 2), 64, 2 * variant_stride(mcap), c->stream>>>(c->dm, tb, p, si, out,
                                                                                       c->order_bins);
+    bins_kernel<<<1, 32, 0, c->stream>>>(c->dm, c->order_bins);
     order_scatter_kernel<<<gb, 256, 0, c->stream>>>(c->dm, p, si, wl);
     // while a launch sequence is being recorded, the timing events become
     // event-record nodes of the graph (an ordinary record would only mark a
@@ -1993,7 +1996,7 @@ cudaError_t launch_eval(const e2_ctx *c, const DevPop &p)
         else finalize_roles_kernel<1, false><<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
     }
     else finalize_score_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, si, so, out);
-    c->launches += c->dp_grid1 > 0 ? 5 : 4;
+    c->launches += c->dp_grid1 > 0 ? 6 : 5;
     if (c->dm.offload) {
         gc_split_kernel<<<fb, 128, 0, c->stream>>>(c->dm, p, c->capg, out);
         ++c->launches;

@@ -388,11 +388,11 @@ def test_recorded_generation_matches_separate_calls(name, P, gens):
         assert np.array_equal(fa, fb), gen
         assert_genomes_equal(a.get_population(), b.get_population())
         # a replay counts the recorded kernel nodes: as many as the separate calls launch
-        # (pre-pass, scatter, DP launches, finaliser, duplicates -- from 4,096 genomes
-        # a fingerprint table and a lookup --, elite selection, candidate ranks, full
-        # ranks, children)
+        # (pre-pass, bin scan, scatter, DP launches, finaliser, duplicates -- from 4,096
+        # genomes a fingerprint table and a lookup --, elite selection, candidate ranks,
+        # full ranks, children)
         sa, sb = a.stats(), b.stats()
-        expected = 8 + sa["dp_launches"] + (1 if P >= 4096 else 0)
+        expected = 9 + sa["dp_launches"] + (1 if P >= 4096 else 0)
         assert sa["launches"] - la == sb["launches"] - lb == expected, gen
     torch.cuda.synchronize()
     assert x.elapsed_time(y) > 0
