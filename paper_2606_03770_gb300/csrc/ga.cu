@@ -689,10 +689,11 @@ __global__ void __launch_bounds__(256) ga_kernel(Dims dm, DevPop src, DevPop dst
         // ---- uniform crossover and repair
         const uint16_t *pa = src.perm + (size_t)par[0] * M, *pb = src.perm + (size_t)par[1] * M;
         Stream cx(seed, gen, (uint32_t)s, kCross);
-        for (int i = lane; i < M; i += 32) {
-            child[i] = (uint64_t)cx.word((uint32_t)i) < thr.cx ? pb[i] : pa[i];
-            first[i] = 0x7FFFFFFF;
-        }
+        for (int q = lane; 4 * q < M; q += 32)                  // a lane takes the 4 positions of one
+            for (int i = 4 * q; i < 4 * q + 4 && i < M; ++i) {  // block of the stream (one Philox call)
+                child[i] = (uint64_t)cx.word((uint32_t)i) < thr.cx ? pb[i] : pa[i];
+                first[i] = 0x7FFFFFFF;
+            }
         __syncwarp();
         for (int i = lane; i < M; i += 32) atomicMin(&first[child[i]], i);
         __syncwarp();
@@ -733,7 +734,8 @@ __global__ void __launch_bounds__(256) ga_kernel(Dims dm, DevPop src, DevPop dst
                     r = (int)below(mt.word(2), (uint32_t)R);
                 } else if (kind >= thr.k3) {                       // regenerate both chromosomes
                     Stream sp(seed, gen, (uint32_t)s, kMutPerm);
-                    for (int t = lane; t < M - 1; t += 32) words[t] = sp.word((uint32_t)t);
+                    for (int q = lane; 4 * q < M - 1; q += 32)
+                        for (int t = 4 * q; t < 4 * q + 4 && t < M - 1; ++t) words[t] = sp.word((uint32_t)t);
                     for (int i = lane; i < M; i += 32) child[i] = (uint32_t)i;
                     __syncwarp();
                     if (lane == 0)
@@ -749,7 +751,8 @@ __global__ void __launch_bounds__(256) ga_kernel(Dims dm, DevPop src, DevPop dst
                 for (int c = 0; c < r; ++c) kept += (int)ssz[c];
                 const int Mr = M - kept, Kr = K - r;
                 Stream sg(seed, gen, (uint32_t)s, kMutGroup), sr(seed, gen, (uint32_t)s, kMutRoles);
-                for (int t = lane; t < Mr; t += 32) words[t] = sg.word((uint32_t)t);
+                for (int q = lane; 4 * q < Mr; q += 32)
+                    for (int t = 4 * q; t < 4 * q + 4 && t < Mr; ++t) words[t] = sg.word((uint32_t)t);
                 const uint64_t bits = (uint64_t)sr.word(0) | ((uint64_t)sr.word(1) << 32);
                 __syncwarp();
                 if (lane == 0) {
