@@ -189,6 +189,28 @@ def test_eval_parity_edge_cases(case):
     eng.close()
 
 
+@pytest.mark.parametrize("min_tps", [0.0, 0.02])
+def test_spilled_layout_tie_heavy(min_tps):
+    """Replicas of ~20 devices over a 126-block model run in the spilled layout,
+    where the prefix chain speculates on the head on device 1: small-integer
+    costs make the master-free optimum, V_1 and the other masters tie often, so
+    both the proof of mu* = 1 and its fallback (the chain again without the
+    head, the combine seeded with master 1) meet exact ties."""
+    rng = np.random.default_rng(606)
+    M, N, K, P = 64, 126, 3, 64
+    prob = _edge_problem(rng, M, N, P, K, integer=True, Q=4, min_tps=min_tps)
+    g = W.random_genomes(M, K, P, seed=66)
+    eng = engine(prob)
+    eng.eval(g)
+    gpu = eng.results()
+    ora = O.OracleProblem(prob).eval_population(g, K, nthreads=O.num_threads())
+    assert_eval_equal(gpu, ora)
+    st = eng.stats()
+    assert st["dp_smem"] <= 40 * 1024 and st["device_errors"] == 0, st   # the spilled layout
+    assert st["served"] == int((ora["bsel"] >= 0).sum()) > 20
+    eng.close()
+
+
 @pytest.mark.parametrize("case", range(6))
 def test_eval_parity_costs_growing_with_batch(case):
     """The small-integer edge problems with each decode cost row sorted, so
