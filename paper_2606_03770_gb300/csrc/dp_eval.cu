@@ -430,6 +430,10 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
     __shared__ uint32_t s_V;
     __shared__ double s_L, s_T;
     __shared__ unsigned s_item, s_next;           // s_next: an item claimed during the last traceback
+    // (spilled layout) s_next's item word, replica size and offset, and where its device ids,
+    // capacities and keys wait in shared memory (-1: not fetched)
+    __shared__ unsigned long long s_pre_item;
+    __shared__ int s_pre_m, s_pre_off, s_pre_at, s_pre_use;
     __shared__ unsigned long long s_bestkey;     // (V << 32) | mu of the best master so far
     __shared__ uint32_t s_V0, s_V1;
     __shared__ unsigned s_prb[3];                // probes of a column over 32, 64, 128 threads
@@ -441,7 +445,7 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
     constexpr bool spill = SPILL;
     // this CTA's suffix-column scratch (only the first launch's CTAs spill)
     uint32_t *gsp = spill ? wl.gspill + (size_t)blockIdx.x * wl.spill_stride : nullptr;
-    if (tid == 0) s_next = ~0u;
+    if (tid == 0) { s_next = ~0u; s_pre_at = -1; }
   for (;;) {
     // ---- next work item of the class (heaviest first); warp 1 claims it
     //      while warp 0 traces the last one back
@@ -449,19 +453,22 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
         const unsigned nx = s_next;
         s_next = ~0u;
         s_item = nx != ~0u ? nx : atomicAdd(&wl.ctrl[kCtrlNext + cls], 1u);
+        s_pre_use = nx != ~0u ? s_pre_at : -1;
+        s_pre_at = -1;
     }
     __syncthreads();
     const unsigned idx = s_item;
+    const int pre_at = SPILL ? s_pre_use : -1;                  // the item's data fetched already
     __syncthreads();
     if (idx >= n_items) break;
-    const uint64_t item = wl.items[idx];
+    const uint64_t item = pre_at >= 0 ? s_pre_item : wl.items[idx];
     const int slot = (int)(item >> 8), code = (int)(item & 0x3Fu);
     if (tid == 0) s_done = *(volatile const int32_t *)&si.best[slot] > code;   // a larger batch won
     __syncthreads();
     if (s_done) continue;
     const int g = slot / K, c = slot - g * K;
     const size_t gk = (size_t)g * K + c;
-    const int off = si.off[slot], m = pop.sizes[gk];
+    const int off = pre_at >= 0 ? s_pre_off : si.off[slot], m = pre_at >= 0 ? s_pre_m : pop.sizes[gk];
     const int role = (int)((item >> 7) & 1u);                   // decode
     const bool sweep = (item >> 6) & 1u;                        // the result advances the decode sweep
     uint64_t vmask = 1ull << code;
@@ -487,7 +494,19 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
         Key *lbm = tauk + m;                                    // [m] l^head_k(1)
         uint16_t *devs = reinterpret_cast<uint16_t *>(lbm + m);   // [m]
 
-        for (int k = tid; k < m; k += blockDim.x) devs[k] = pop.perm[(size_t)g * M + off + k];
+        int p_c0 = 0, p_c1 = 0;                                 // this thread's device's fetched
+        Key p_t = 0, p_l = 0;                                   // capacities and keys (pre_at >= 0)
+        if (pre_at >= 0) {                                      // read them all before any is overwritten
+            const int *q0 = reinterpret_cast<const int *>(smem + pre_at), *q1 = q0 + m;
+            const Key *qt = reinterpret_cast<const Key *>(q1 + m), *ql = qt + m;
+            const uint16_t *qd = reinterpret_cast<const uint16_t *>(ql + m);
+            int d = 0;
+            if (tid < m) { d = qd[tid]; p_c0 = q0[tid]; p_c1 = q1[tid]; p_t = qt[tid]; p_l = ql[tid]; }
+            __syncthreads();
+            if (tid < m) devs[tid] = (uint16_t)d;
+        } else {
+            for (int k = tid; k < m; k += blockDim.x) devs[k] = pop.perm[(size_t)g * M + off + k];
+        }
         if (tid < 3) s_prb[tid] = c_span_probes[tid][W];
         for (int r = tid; r < W; r += blockDim.x) delta[r] = r ? kInf : (Key)0;
         __syncthreads();
@@ -510,13 +529,17 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
             const int v = role ? bit + 1 : 0;
             const size_t vM = (size_t)v * M;
             // ---- 1. capacities, link ranks and master-free cost rows
-            for (int k = tid; k < m; k += blockDim.x) {
-                const size_t vd = vM + devs[k];
-                const int c0 = tb.cap[vd * 2], c1 = tb.cap[vd * 2 + 1];
-                cnt0[k] = c0 < W ? c0 : W;
-                cnt1[k] = c1 < W ? c1 : W;
-                tauk[k] = k ? (Key)tb.tau_rank[(vM + devs[k - 1]) * M + devs[k]] : (Key)0;
-                lbm[k] = (Key)tb.leaf_rank[((vM + devs[k]) * 2 + 1) * dm.LS];   // l^head_k(1)
+            if (pre_at >= 0) {
+                if (tid < m) { cnt0[tid] = p_c0; cnt1[tid] = p_c1; tauk[tid] = p_t; lbm[tid] = p_l; }
+            } else {
+                for (int k = tid; k < m; k += blockDim.x) {
+                    const size_t vd = vM + devs[k];
+                    const int c0 = tb.cap[vd * 2], c1 = tb.cap[vd * 2 + 1];
+                    cnt0[k] = c0 < W ? c0 : W;
+                    cnt1[k] = c1 < W ? c1 : W;
+                    tauk[k] = k ? (Key)tb.tau_rank[(vM + devs[k - 1]) * M + devs[k]] : (Key)0;
+                    lbm[k] = (Key)tb.leaf_rank[((vM + devs[k]) * 2 + 1) * dm.LS];   // l^head_k(1)
+                }
             }
             for (int k = wid; k < m; k += NW)                       // the loads of a row overlap
                 stage_row(leaf0 + (size_t)k * W, tb.leaf_rank + (vM + devs[k]) * 2 * dm.LS, W, lane);
@@ -735,8 +758,41 @@ __device__ __forceinline__ void dp_eval_body(const Dims &dm, const Tables &tb, c
                     s_T = keyd(tmax);
                     s_done = (!role) || lam <= dm.lam_max;       // 1.0 / lam >= Min_TPS
                 }
-            } else if (wid == 1 && lane == 0) {
-                s_next = atomicAdd(&wl.ctrl[kCtrlNext + cls], 1u);
+            } else if (wid == 1) {
+                unsigned nx = 0;
+                if (lane == 0) nx = atomicAdd(&wl.ctrl[kCtrlNext + cls], 1u);
+                nx = __shfl_sync(0xFFFFFFFFu, nx, 0);
+                if (lane == 0) s_next = nx;
+                if (SPILL && nx < n_items) {
+                    // (spilled layout) the next item's header, device ids, capacities
+                    // and keys, into this run's suffix-column and per-warp buffers,
+                    // which nothing reads from here to the next item
+                    const uint64_t it2 = wl.items[nx];
+                    const int slot2 = (int)(it2 >> 8), code2 = (int)(it2 & 0x3Fu);
+                    const int g2 = slot2 / K, c2 = slot2 - g2 * K;
+                    const int off2 = si.off[slot2], m2 = pop.sizes[(size_t)g2 * K + c2];
+                    const int at = (int)(reinterpret_cast<unsigned char *>(Gst) - smem);
+                    const long room = reinterpret_cast<unsigned char *>(row1s) - reinterpret_cast<unsigned char *>(Gst);
+                    if (m2 <= N && m2 <= (int)blockDim.x && 18L * m2 <= room) {
+                        const int W2 = N - m2 + 1;
+                        const size_t vM2 = (size_t)(((it2 >> 7) & 1u) ? code2 + 1 : 0) * M;
+                        int *q0 = reinterpret_cast<int *>(smem + at), *q1 = q0 + m2;
+                        Key *qt = reinterpret_cast<Key *>(q1 + m2), *ql = qt + m2;
+                        uint16_t *qd = reinterpret_cast<uint16_t *>(ql + m2);
+                        for (int k = lane; k < m2; k += 32) {
+                            const int d = pop.perm[(size_t)g2 * M + off2 + k];
+                            qd[k] = (uint16_t)d;
+                            const int a0 = tb.cap[(vM2 + d) * 2], a1 = tb.cap[(vM2 + d) * 2 + 1];
+                            q0[k] = a0 < W2 ? a0 : W2;
+                            q1[k] = a1 < W2 ? a1 : W2;
+                            ql[k] = (Key)tb.leaf_rank[((vM2 + d) * 2 + 1) * dm.LS];
+                        }
+                        __syncwarp();
+                        for (int k = lane; k < m2; k += 32)
+                            qt[k] = k ? (Key)tb.tau_rank[(vM2 + qd[k - 1]) * M + qd[k]] : (Key)0;
+                        if (lane == 0) { s_pre_item = it2; s_pre_m = m2; s_pre_off = off2; s_pre_at = at; }
+                    }
+                }
             }
             __syncthreads();
             if (s_done) {
