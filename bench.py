@@ -62,7 +62,7 @@ INT32_LANES_PER_SM = 128
 # 24.55 + 5.46 MB), from the ncu capture in profiles/; cold (ncu flushes the
 # caches before each launch), so it counts the L2-resident order-key rows
 # again
-DP_TRAFFIC_BYTES = 68_998_144
+DP_TRAFFIC_BYTES = 69_413_632
 DP_TRAFFIC_SOURCE = "profiles/dp_eval_c4_gen2.md (dram read+write, both DP launches of one generation, cold)"
 
 
