@@ -192,6 +192,38 @@ def test_dp_matches_brute_force(seed):
         assert list(got["layers"]) == layers
 
 
+def test_head_only_adds_and_a_free_head_on_device_1_decides_the_master():
+    """The facts the spilled DP layout's speculation rests on (Sec. 3.2, Alg. 1),
+    by enumeration: every master's optimum V_mu is at least the master-free
+    optimum V0 (the head only adds cost); so when the head on device 1 leaves
+    the optimum unchanged (V_1 == V0), the first-wins argmin over masters is
+    device 1 and the DP's value is V0.  Small-integer costs make both cases
+    (V_1 == V0 and V_1 > V0) frequent."""
+    rng = np.random.default_rng(2718)
+    hits = misses = 0
+    for trial in range(60):
+        N = int(rng.integers(2, 9))
+        M = 5
+        prob = tiny_problem(rng, M, N, integer=True, head=True)
+        op = O.OracleProblem(prob)
+        m = int(rng.integers(2, min(M, N) + 1))
+        devs = rng.permutation(M)[:m]
+        v = int(rng.integers(0, prob.V))
+        V0 = bf_value(op, v, devs, N, m, m)                     # no device holds the head
+        Vmu = [bf_value(op, v, devs, N, m, mu) for mu in range(m)]
+        assert all(x >= V0 for x in Vmu), (Vmu, V0)
+        if V0 == INF:
+            continue
+        got = op.dp_pipe(v, devs)
+        if Vmu[0] == V0:
+            hits += 1
+            assert got["ok"] and got["mu"] == 0 and got["V"] == V0
+        elif got["ok"]:
+            misses += 1
+            assert got["V"] == min(Vmu) >= V0
+    assert hits >= 10 and misses >= 5, (hits, misses)
+
+
 def test_dp_more_devices_than_blocks_is_infeasible():
     rng = np.random.default_rng(0)
     prob = tiny_problem(rng, 6, 4, tight_mem=False)
